@@ -1,0 +1,497 @@
+"""Benchmark of the SMem reader hot path on GB300.
+
+Default workload (one GPU): 410M-shaped batched decode -- L = 24 reader
+layers, H = 16 heads, d_h = 64, blocks of b = R = 64, 64 sequences with
+contexts uniform in [64, 256] memory blocks and in-block offsets uniform in
+[0, 63], pool slots in a seeded shuffled order. A step is one decode token
+for all 64 sequences through all 24 layers (24 decode launches); whenever a
+sequence's in-block offset wraps 63 -> 0 the finished block is appended to
+its memory (synthetic rows) inside the step. The pool (~66 GB) is far
+larger than L2, so no flush is needed between steps.
+
+Prints one JSON line. ``--impl reference`` times the fp64 CPU oracle on the
+same workload (a bounded sample) instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "decode tok/s + cross-attn HBM GB/s (% peak); one-block cached-serve latency ms"
+WORKLOAD = dict(name="410M-shaped batched decode", L=24, H=16, D=64, seqs=64, ctx_lo=64, ctx_hi=256, seed=0)
+R = 64
+B_TOK = 64
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--seqs", type=int, default=WORKLOAD["seqs"])
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------------------- helpers
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def source_sha(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def profiled_traffic(profile_name, kernel_src, units_now):
+    """DRAM bytes per launch from a committed ncu summary, scaled to this
+    launch's units, or None if the kernel source changed since the capture."""
+    path = os.path.join(ROOT, "profiles", profile_name)
+    if not os.path.exists(path):
+        return None
+    kv = {}
+    for line in open(path):
+        if ":" in line and not line.startswith("#"):
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    try:
+        if kv.get("kernel_source_sha256") != source_sha(kernel_src):
+            return None
+        per_unit = float(kv["dram_bytes_per_launch"]) / float(kv["units_per_launch"])
+        return per_unit * units_now
+    except (KeyError, ValueError):
+        return None
+
+
+# ----------------------------------------------------------------------------- decode workload
+class DecodeWorkload:
+    """Device state of the 410M-shaped batched-decode workload."""
+
+    def __init__(self, seqs, steps_total, seed, device, rank=0):
+        import torch
+
+        import synth
+        from paper_2609_32395_gb300 import smem
+
+        W = WORKLOAD
+        self.L, self.H, self.D = W["L"], W["H"], W["D"]
+        self.S = seqs
+        self.seed = seed + 1000 * rank
+        self.device = device
+        self.nblk = synth.ragged_contexts(self.seed, seqs, W["ctx_lo"], W["ctx_hi"]).astype(np.int64)
+        self.pos = synth.inblock_positions(self.seed, seqs, B_TOK).astype(np.int64)
+        # appends each sequence will need over all steps
+        self.n_new = [(int(p) + steps_total) // B_TOK + 1 for p in self.pos]
+        capacity = int(self.nblk.sum()) + sum(self.n_new)
+        max_blocks = int(self.nblk.max()) + max(self.n_new) + 1
+        perm = synth.slot_permutation(self.seed, capacity)
+        self.cfg = smem.make_config(self.L, self.H, self.D, seqs, max_blocks, capacity, free_order=perm)
+        self.cache = smem.SmemCache(self.cfg, device=device)
+        self.h = self.cache.h
+        torch.cuda.synchronize()
+        # memory blocks 0..nblk-1 of every sequence
+        chunk = 16
+        for s in range(seqs):
+            n = int(self.nblk[s])
+            for b0 in range(0, n, chunk):
+                ids = list(range(b0, min(n, b0 + chunk)))
+                K, V = synth.block_rows_torch(self.seed, s, ids, self.L, self.H, R, self.D, device)
+                for i, j in enumerate(ids):
+                    smem.smem_append_block(self.h, s, j, K[i], V[i])
+                del K, V
+        # blocks that will be appended when a sequence's block completes
+        self.new_K, self.new_V = [], []
+        for s in range(seqs):
+            ids = [int(self.nblk[s]) + k for k in range(self.n_new[s])]
+            K, V = synth.block_rows_torch(self.seed, s, ids, self.L, self.H, R, self.D, device)
+            self.new_K.append(K)
+            self.new_V.append(V)
+        self.new_used = [0] * seqs
+        # in-block rows 0..p-1 of every sequence and layer
+        for s in range(seqs):
+            p = int(self.pos[s])
+            for layer in range(self.L):
+                if p:
+                    Kb = synth.tensor_torch(self.seed, synth.KIND_KIN, (p, self.H, self.D), s, layer, 0,
+                                            device=device)
+                    Vb = synth.tensor_torch(self.seed, synth.KIND_VIN, (p, self.H, self.D), s, layer, 0,
+                                            device=device)
+                    smem.smem_write_inblock(self.h, s, layer, p, Kb, Vb)
+        # per-layer decode inputs (a few distinct sets, cycled)
+        self.n_sets = 2
+        shape = (seqs, self.H, self.D)
+        self.inputs = []
+        for k in range(self.n_sets):
+            per_layer = []
+            for layer in range(self.L):
+                per_layer.append([synth.tensor_torch(self.seed, kind, shape, layer, k, device=device)
+                                  for kind in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW,
+                                               synth.KIND_QDEC_C)])
+            self.inputs.append(per_layer)
+        self.osa = torch.empty(shape, dtype=torch.bfloat16, device=device)
+        self.oca = torch.empty(shape, dtype=torch.bfloat16, device=device)
+        self.seq_ids = np.arange(seqs, dtype=np.int32)
+        self.step_no = 0
+        torch.cuda.synchronize()
+
+    def rows_read(self):
+        """Memory rows + in-block rows one decode launch reads (all sequences)."""
+        return int(self.nblk.sum()) * R + int((self.pos + 1).sum())
+
+    def step(self, events=None, host_inputs=None, host_outputs=None, host_blocks=None):
+        """One decode token for every sequence through all layers. Returns the
+        number of this library's kernel launches."""
+        import torch
+
+        from paper_2609_32395_gb300 import smem
+
+        launches = 0
+        st = torch.cuda.current_stream()
+        k = self.step_no % self.n_sets
+        for layer in range(self.L):
+            qs, kn, vn, qc = self.inputs[k][layer]
+            if host_inputs is not None:
+                hq = host_inputs[k][layer]
+                for dst, src in zip((qs, kn, vn, qc), hq):
+                    dst.copy_(src, non_blocking=True)
+            if events is not None:
+                events[0][layer].record(st)
+            smem.smem_decode(self.h, layer, self.seq_ids, self.pos.astype(np.int32), self.nblk.astype(np.int32),
+                             qs, kn, vn, qc, self.osa, self.oca)
+            if events is not None:
+                events[1][layer].record(st)
+            launches += 1
+            if host_outputs is not None:
+                host_outputs[0][layer].copy_(self.osa, non_blocking=True)
+                host_outputs[1][layer].copy_(self.oca, non_blocking=True)
+        self.pos += 1
+        for s in np.nonzero(self.pos == B_TOK)[0]:
+            u = self.new_used[s]
+            K, V = self.new_K[s][u], self.new_V[s][u]
+            if host_blocks is not None:
+                K.copy_(host_blocks[0], non_blocking=True)
+                V.copy_(host_blocks[1], non_blocking=True)
+            smem.smem_append_block(self.h, int(s), int(self.nblk[s]), K, V)
+            launches += 1
+            self.new_used[s] += 1
+            self.nblk[s] += 1
+            self.pos[s] = 0
+        self.step_no += 1
+        return launches
+
+
+# ----------------------------------------------------------------------------- oracle (cpu) timing
+class OracleDecodeSample:
+    """A bounded sample of the default workload for the fp64 CPU oracle: the
+    first `n_seqs` sequences at `layers`, inputs generated once. `call(i)`
+    runs and times one (sequence, layer) decode call of the oracle."""
+
+    def __init__(self, seqs, n_seqs=3, layers=(0, 13), rank=0):
+        import oracle
+        import synth
+
+        W = WORKLOAD
+        self.L, self.H, self.D = W["L"], W["H"], W["D"]
+        s_seed = W["seed"] + 1000 * rank
+        nblk = synth.ragged_contexts(s_seed, seqs, W["ctx_lo"], W["ctx_hi"])
+        pos = synth.inblock_positions(s_seed, seqs, B_TOK)
+        self.mean_rows = float(nblk.mean()) * R + float(pos.mean()) + 1
+        f = oracle.bf16_bits_to_f64
+        H, D = self.H, self.D
+        self.calls = []
+        for s in range(min(n_seqs, seqs)):
+            n, p = int(nblk[s]), int(pos[s])
+            for layer in layers:
+                keys = np.array([synth.stream_key(s_seed, 1, s, j, layer, kind)
+                                 for kind in (synth.KIND_K, synth.KIND_V) for j in range(n)], dtype=np.int64)
+                rows = synth.normal_bf16_np(keys, H * R * D).reshape(2, n, H, R, D)
+                kin = synth.tensor_np(s_seed, synth.KIND_KIN, (B_TOK, H, D), s, layer, 0)[:p]
+                vin = synth.tensor_np(s_seed, synth.KIND_VIN, (B_TOK, H, D), s, layer, 0)[:p]
+                q = [synth.tensor_np(s_seed, kind, (seqs, H, D), layer, 0)[s]
+                     for kind in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
+                self.calls.append(dict(idx=np.arange(n), mk=f(rows[0]), mv=f(rows[1]), n=n, p=p, kin=f(kin),
+                                       vin=f(vin), q=[f(x) for x in q], rows=n * R + p + 1))
+        self.desc = (f"fp64 C oracle, single thread: decode calls (all {H} heads, full contexts) of sequences "
+                     f"0..{min(n_seqs, seqs) - 1} at layers {list(layers)}, repeated; time per memory row "
+                     f"extrapolated to the workload's mean context and {self.L} layers per token")
+
+    def call(self, i):
+        import oracle
+
+        c = self.calls[i % len(self.calls)]
+        t0 = time.perf_counter()
+        oracle.reader_decode(c["idx"], c["mk"], c["mv"], c["n"], c["p"], c["kin"], c["vin"], *c["q"])
+        return time.perf_counter() - t0, c["rows"]
+
+    def tok_per_s(self, secs, rows):
+        """Tokens/s of the oracle on the workload, from time spent on rows."""
+        per_row = secs / rows
+        return 1.0 / (per_row * self.mean_rows * self.L)
+
+
+def oracle_baseline(seqs, budget_s=12.0):
+    samp = OracleDecodeSample(seqs)
+    secs = rows = 0.0
+    n = 0
+    while secs < budget_s or n < len(samp.calls):
+        t, r = samp.call(n)
+        secs += t
+        rows += r
+        n += 1
+    return {"value": samp.tok_per_s(secs, rows), "unit": "tok/s", "cores": 1, "kind": "oracle",
+            "sample": f"{samp.desc}; {n} calls, {secs:.1f} s"}
+
+
+# ----------------------------------------------------------------------------- arms
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    W = WORKLOAD
+    samp = OracleDecodeSample(args.seqs)
+    secs = rows = 0.0
+    for i in range(args.warmup + args.steps):
+        t, r = samp.call(i)
+        if i >= args.warmup:
+            secs += t
+            rows += r
+    value = samp.tok_per_s(secs, rows)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": W["name"], "layers": W["L"], "heads": W["H"], "head_dim": W["D"],
+                   "sequences": args.seqs, "context_blocks": [W["ctx_lo"], W["ctx_hi"]], "block": B_TOK},
+        "cpu_baseline": {"value": value, "unit": "tok/s", "cores": 1, "kind": "oracle",
+                         "sample": f"each step one call; {samp.desc}"},
+        "e2e": {"value": value, "unit": "tok/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+
+    from paper_2609_32395_gb300 import smem
+
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    smem.lib()  # fails loudly without the CUDA library
+
+    e2e_steps = 0 if args.no_e2e else min(args.steps, 64)
+    wl = DecodeWorkload(args.seqs, args.warmup + args.steps + e2e_steps + 2, WORKLOAD["seed"], device, rank)
+
+    def barrier():
+        if ws > 1:
+            import torch.distributed as dist
+
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        wl.step()
+    barrier()
+
+    # --- timed region (device-resident inputs)
+    rows, bytes_alg = [], []
+    st = torch.cuda.current_stream()
+    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(wl.L)] for _ in range(2)]
+          for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches = 0
+    with ClockSampler(local) as clk:
+        barrier()
+        start.record(st)
+        for i in range(args.steps):
+            r = wl.rows_read()
+            rows.append(r)
+            launches += wl.step(events=ev[i])
+        end.record(st)
+        barrier()
+    elapsed = start.elapsed_time(end) / 1e3
+    # per-launch durations of the decode kernel
+    kern_ms = [ev[i][0][l].elapsed_time(ev[i][1][l]) for i in range(args.steps) for l in range(wl.L)]
+    row_bytes = 4 * wl.H * wl.D  # K + V bf16 per row per layer
+    alg_bytes = [r * row_bytes for r in rows for _ in range(wl.L)]
+    achieved = sum(alg_bytes) / (sum(kern_ms) / 1e3) / 1e9
+
+    tokens = args.steps * args.seqs
+    if ws > 1:
+        import torch.distributed as dist
+
+        t = torch.tensor([elapsed], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+    value = tokens * ws / elapsed
+
+    # --- end to end: host inputs / outputs / appended rows through the C ABI
+    e2e = None
+    if e2e_steps:
+        pin = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True).copy_(t.cpu())  # noqa: E731
+        host_in = [[[pin(x) for x in wl.inputs[k][l]] for l in range(wl.L)] for k in range(wl.n_sets)]
+        host_out = [[torch.empty(wl.osa.shape, dtype=torch.bfloat16, pin_memory=True) for _ in range(wl.L)]
+                    for _ in range(2)]
+        host_blk = (pin(wl.new_K[0][0]), pin(wl.new_V[0][0]))
+        appends_before = sum(wl.new_used)
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            wl.step(host_inputs=host_in, host_outputs=host_out, host_blocks=host_blk)
+            torch.cuda.current_stream().synchronize()  # the step's outputs are on the host
+        barrier()
+        e2e_el = time.perf_counter() - t0
+        n_app = sum(wl.new_used) - appends_before
+        h2d = wl.L * 4 * args.seqs * wl.H * wl.D * 2 + n_app / e2e_steps * 2 * host_blk[0].numel() * 2
+        d2h = wl.L * 2 * args.seqs * wl.H * wl.D * 2
+        if ws > 1:
+            import torch.distributed as dist
+
+            t = torch.tensor([e2e_el], device=device, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_el = float(t.item())
+        e2e = {"value": e2e_steps * args.seqs * ws / e2e_el, "unit": "tok/s",
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+    err = smem.smem_check_device_error(wl.h)
+    if err != smem.OK:
+        raise RuntimeError("device error recorded during the benchmark")
+
+    if rank != 0:
+        if ws > 1:
+            import torch.distributed as dist
+
+            dist.destroy_process_group()
+        return
+
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    units_launch = float(np.mean(rows))
+    traffic = profiled_traffic("decode_410m.txt", os.path.join(ROOT, "paper_2609_32395_gb300", "csrc",
+                                                                   "smem_decode.cu"), units_launch)
+    cpu = None if args.no_cpu_baseline else oracle_baseline(args.seqs)
+    line = {
+        "metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD["name"], "layers": wl.L, "heads": wl.H, "head_dim": wl.D,
+                   "sequences": args.seqs, "context_blocks": [WORKLOAD["ctx_lo"], WORKLOAD["ctx_hi"]],
+                   "block": B_TOK, "rows_per_block": R, "pool_bytes": int(wl.cache.nbytes),
+                   "l2": "inputs larger than L2 (pool of memory rows >> 129 MB); no flush",
+                   "parallelism": f"independent sequences per GPU x{ws}"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "kernel": "decode_kernel<64> (split-K paged cross-attention + in-block self-attention)",
+                     "peak_source": f"{peak_src} hbm_gbs", "kernel_ms_mean": float(np.mean(kern_ms)),
+                     "alg_bytes_per_launch": float(np.mean(alg_bytes))},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+    }
+    if e2e:
+        line["e2e"] = e2e
+    if cpu:
+        line["cpu_baseline"] = cpu
+    print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

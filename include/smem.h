@@ -1,0 +1,205 @@
+/*
+ * smem.h -- C ABI of the SMem reader hot path on one GB300 (sm_103a).
+ *
+ * SMem (arXiv 2609.32395) keeps a context as a static memory: every block of
+ * b tokens is encoded once, on its own, into b memory rows, and a reader
+ * attends within the current block (block-local causal self-attention) and
+ * then across the rows of all strictly earlier blocks (block-causal
+ * cross-attention, with an optional learned null row); Sec. 2 "Model" and
+ * App. A "Reader". This library serves that reader's attention over a
+ * block-paged cache of the per-layer cross-attention K/V of the memory rows
+ * (the "materialized cross-attention K/V" of Sec. 3.1):
+ *
+ *   - a pool of slots, one slot per memory block, each holding the block's
+ *     K and V rows for every layer and head (bf16);
+ *   - per sequence, a block table sorted by block index (the canonical order
+ *     of Sec. 2) mapping block index -> slot, and one FIFO of free slots;
+ *   - in-block self-attention K/V rows of the block being decoded.
+ *
+ * Deleting a block is a table edit plus a slot free (no row moves, O(b) as
+ * in Theorem 1's editing cost); reads depend only on the block set, and the
+ * kernels reduce in an order fixed by the number of blocks read, so the same
+ * block set gives bitwise-identical outputs whatever the edit path.
+ *
+ * Conventions
+ *   - Element type "bf16" is IEEE bfloat16 (passed as void pointers).
+ *   - Device pointers are CUDA device addresses of the current device; every
+ *     device pointer must be 16-byte aligned (SMEM_ERR_ALIGN otherwise).
+ *   - `stream` is a cudaStream_t cast to void* (NULL = legacy default
+ *     stream). All device work is enqueued on it; no call blocks except
+ *     where stated. Host bookkeeping is updated synchronously, so calls on
+ *     one cache must be issued from one thread and, when they touch device
+ *     state, on one stream (or streams the caller orders).
+ *   - Return value: SMEM_OK (0) or a negative SMEM_ERR_* code. A failing
+ *     call leaves the cache's state (tables, free list, device contents)
+ *     as it was. No C++ exception crosses this interface.
+ *   - The library allocates no device memory: the caller passes one device
+ *     buffer of smem_cache_required_bytes() bytes to smem_cache_create and
+ *     owns it; it must outlive the cache.
+ *   - Supported shapes: block_tokens == rows_per_block == 64,
+ *     head_dim 64 or 128 (SMEM_ERR_UNSUPPORTED otherwise).
+ */
+#ifndef SMEM_H
+#define SMEM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SMEM_ABI_VERSION 1
+
+enum {
+    SMEM_OK = 0,
+    SMEM_ERR_INVALID_ARG = -1,     /* bad argument value, shape or id      */
+    SMEM_ERR_ALIGN = -2,           /* pointer not 16-byte aligned          */
+    SMEM_ERR_NO_SUCH_SEQ = -3,     /* sequence id out of range             */
+    SMEM_ERR_DUPLICATE_BLOCK = -4, /* block index already in the table    */
+    SMEM_ERR_NO_SUCH_BLOCK = -5,   /* block index not in the table         */
+    SMEM_ERR_POOL_FULL = -6,       /* no free slot                         */
+    SMEM_ERR_TABLE_FULL = -7,      /* sequence holds max_blocks_per_seq    */
+    SMEM_ERR_CUDA = -8,            /* a CUDA runtime call failed           */
+    SMEM_ERR_DEVICE_FAULT = -9,    /* a kernel recorded an error           */
+    SMEM_ERR_UNSUPPORTED = -10,    /* shape outside the supported set      */
+    SMEM_ERR_NO_DEVICE = -11       /* bookkeeping-only cache: no device op */
+};
+
+/* Cache geometry. Notation of the paper: L reader layers, H heads of
+ * dimension d_h, blocks of b tokens, R memory rows per block (R = b). */
+typedef struct smem_config {
+    int32_t n_layers;           /* L >= 1                                      */
+    int32_t n_heads;            /* H >= 1                                      */
+    int32_t head_dim;           /* d_h: 64 or 128                              */
+    int32_t block_tokens;       /* b: 64                                       */
+    int32_t rows_per_block;     /* R: 64                                       */
+    int32_t max_seqs;           /* sequence ids are 0 .. max_seqs-1            */
+    int32_t max_blocks_per_seq; /* table capacity per sequence                 */
+    int32_t capacity_slots;     /* C: pool slots (memory blocks held at once)  */
+    int32_t has_null_row;       /* 1: prepend a per-layer learned null row     */
+    int32_t max_decode_batch;   /* largest nb of smem_decode, <= max_seqs      */
+    const int32_t *free_order;  /* host, C entries: initial FIFO order, a
+                                   permutation of 0..C-1; NULL = ascending.
+                                   Copied at create time.                      */
+} smem_config;
+
+typedef struct smem_cache smem_cache;
+
+/* Size in bytes of the device buffer a cache with this geometry needs
+ * (pool, in-block K/V, null rows, device block tables, split-K workspace).
+ * Returns 0 for an invalid or unsupported geometry. */
+size_t smem_cache_required_bytes(const smem_config *cfg);
+
+/* Creates a cache. dev_buf: device buffer of at least
+ * smem_cache_required_bytes(cfg) bytes, 256-byte aligned, owned by the
+ * caller; dev_buf == NULL with dev_bytes == 0 creates a bookkeeping-only
+ * cache (tables and free list, no device state, no CUDA call; device
+ * operations then return SMEM_ERR_NO_DEVICE). Device creation zeroes the
+ * tables and the workspace counters on the legacy default stream and waits
+ * for it. *out receives the handle. */
+int smem_cache_create(const smem_config *cfg, void *dev_buf, size_t dev_bytes, smem_cache **out);
+
+/* Frees the host state. The device buffer stays the caller's. The caller
+ * must ensure no enqueued work on the cache is still pending. */
+int smem_cache_destroy(smem_cache *c);
+
+/* Sets the learned null row (App. A "Positions and memory": one d-vector
+ * prepended to the memory, projected by each layer's key/value maps):
+ * k_null, v_null: device bf16 [L][H][d_h]. Requires has_null_row. Until it
+ * is set the null row's k and v are zero. */
+int smem_set_null_row(smem_cache *c, const void *k_null, const void *v_null, void *stream);
+
+/* Appends memory block `block_idx` of sequence `seq` (Sec. 2: a block's rows
+ * are written once, at its frozen index, and never change): takes the slot
+ * at the front of the free FIFO, copies K and V (device bf16
+ * [L][H][R][d_h], the block's cross-attention keys/values for every layer)
+ * into it and inserts (block_idx, slot) into the sorted table. block_idx
+ * >= 0 and unique within the sequence. *slot_out (may be NULL) receives the
+ * slot. On a bookkeeping-only cache K and V must be NULL. */
+int smem_append_block(smem_cache *c, int32_t seq, int32_t block_idx, const void *K, const void *V,
+                      void *stream, int32_t *slot_out);
+
+/* Deletes block `block_idx` of `seq` (Theorem 1: the result is exactly the
+ * memory in which the block was never encoded; other blocks keep their
+ * indices): removes the table entry and puts the slot at the back of the
+ * free FIFO. No memory row moves. */
+int smem_delete_block(smem_cache *c, int32_t seq, int32_t block_idx, void *stream);
+
+/* Deletes every block of `seq`; slots go to the back of the free FIFO in
+ * ascending block order. */
+int smem_release_seq(smem_cache *c, int32_t seq, void *stream);
+
+/* Writes in-block self-attention rows 0..n_rows-1 of (seq, layer) for a
+ * later smem_decode (e.g. the K/V a one-block prefill computed for the first
+ * n_rows tokens of the current block). K, V: device bf16 [n_rows][H][d_h],
+ * 0 <= n_rows <= b. */
+int smem_write_inblock(smem_cache *c, int32_t seq, int32_t layer, int32_t n_rows, const void *K,
+                       const void *V, void *stream);
+
+/* One-block reader attention for one layer (block-skip serving, Sec. 3.1):
+ * the b query tokens of block `q_block_idx` of `seq`
+ *   Osa[t] = softmax_{u<=t}(Qs[t].Ks[u] / sqrt(d_h)) Vs      (in-block causal)
+ *   Oca[t] = softmax_r(Qc[t].k_r / sqrt(d_h)) v_r           (cross-attention)
+ * where r runs over the null row (if any) and the rows of every table
+ * block with index < q_block_idx, in ascending block index. An empty row
+ * set gives Oca = 0. Qs, Ks, Vs, Qc, Osa, Oca: device bf16 [b][H][d_h];
+ * fp32 accumulation, bf16 round-to-nearest-even outputs. */
+int smem_prefill_block(smem_cache *c, int32_t seq, int32_t layer, int32_t q_block_idx, const void *Qs,
+                       const void *Ks, const void *Vs, const void *Qc, void *Osa, void *Oca, void *stream);
+
+/* One decode step of one layer for nb sequences (KV-cached decode,
+ * Sec. 3.1): item i is sequence seq_ids[i] (distinct), whose new token sits
+ * at in-block offset pos[i] in [0, b) of block q_block_idx[i]. The step
+ * writes k_new[i], v_new[i] into in-block row pos[i] of (seq, layer), then
+ *   osa[i] = softmax over in-block rows 0..pos[i] (the new one included)
+ *   oca[i] = cross-attention over the null row (if any) and the rows of the
+ *            table blocks with index < q_block_idx[i], ascending.
+ * seq_ids, pos, q_block_idx: HOST arrays [nb]; qs, k_new, v_new, qc, osa,
+ * oca: device bf16 [nb][H][d_h]. 1 <= nb <= max_decode_batch. */
+int smem_decode(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids, const int32_t *pos,
+                const int32_t *q_block_idx, const void *qs, const void *k_new, const void *v_new,
+                const void *qc, void *osa, void *oca, void *stream);
+
+/* Introspection for bit-exact bookkeeping checks (host state, no CUDA).
+ * smem_get_table: the table of `seq` in ascending block index; up to `cap`
+ * entries into idx_out / slot_out (either may be NULL); *n_out = length.
+ * smem_get_free_fifo: the free FIFO front to back. */
+int smem_get_table(const smem_cache *c, int32_t seq, int32_t *idx_out, int32_t *slot_out, int32_t cap,
+                   int32_t *n_out);
+int smem_get_free_fifo(const smem_cache *c, int32_t *slots_out, int32_t cap, int32_t *n_out);
+
+/* Copies the device copy of `seq`'s slot table (host int32, up to `cap`
+ * entries, *n_out = length) after the work enqueued on `stream`. Blocks
+ * until that stream has drained. */
+int smem_get_device_table(smem_cache *c, int32_t seq, int32_t *slot_out, int32_t cap, int32_t *n_out,
+                          void *stream);
+
+/* Reads the device error word after the work enqueued on `stream` (blocks
+ * until it drains): SMEM_OK, or SMEM_ERR_DEVICE_FAULT if a kernel gave up a
+ * bounded wait; the word is then cleared. */
+int smem_check_device_error(smem_cache *c, void *stream);
+
+/* Number of pool slots currently free. */
+int smem_free_slots(const smem_cache *c, int32_t *n_out);
+
+/* Text describing the last SMEM_ERR_CUDA / SMEM_ERR_DEVICE_FAULT of the
+ * calling thread (static storage, overwritten by the next failure). */
+const char *smem_last_error_detail(void);
+
+/* Testing hook (failure injection on the host): the n-th next device launch
+ * of this cache fails with SMEM_ERR_CUDA before anything is enqueued, so
+ * callers can check that a failing call leaves the state unchanged.
+ * n = 0 disables it. */
+int smem_debug_fail_after(smem_cache *c, int32_t n);
+
+/* Static text of an error code. */
+const char *smem_strerror(int code);
+
+/* SMEM_ABI_VERSION of the loaded library. */
+int smem_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SMEM_H */

@@ -1,0 +1,150 @@
+// smem_copy.cu -- writes into the block-paged cache: block append (rows into
+// a slot plus the sorted-table insert), table removal on delete, in-block
+// self-attention rows, null row, zero fill.
+//
+// A memory block's rows are written once, when the block is appended, and
+// never change afterwards (arXiv 2609.32395, Sec. 2 "Model"); deleting a
+// block edits only its table entry (Theorem 1's O(b) edit), so no kernel here
+// ever moves another block's rows. Table edits run in one CTA that shifts the
+// suffix of one sequence's row in chunks: every chunk is read into registers
+// before any thread writes, and chunks go in the direction that never
+// overwrites an unread entry.
+#include <cuda_runtime.h>
+
+#include "smem_internal.h"
+
+namespace smem {
+
+constexpr int kCopyThreads = 256;
+
+// Shift entries [pos, n) of `row` one place up and store `value` at pos.
+__device__ void table_insert_cta(int* row, int pos, int n, int value) {
+  for (int hi = n; hi > pos; hi -= blockDim.x) {
+    const int lo = hi - (int)blockDim.x > pos ? hi - (int)blockDim.x : pos;
+    const int i = lo + (int)threadIdx.x;
+    const int v = i < hi ? row[i] : 0;
+    __syncthreads();
+    if (i < hi) row[i + 1] = v;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) row[pos] = value;
+}
+
+// Remove entry pos of a row holding n entries; the freed tail entry is -1.
+__device__ void table_remove_cta(int* row, int pos, int n) {
+  for (int lo = pos + 1; lo < n; lo += blockDim.x) {
+    const int hi = lo + (int)blockDim.x < n ? lo + (int)blockDim.x : n;
+    const int i = lo + (int)threadIdx.x;
+    const int v = i < hi ? row[i] : 0;
+    __syncthreads();
+    if (i < hi) row[i - 1] = v;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) row[n - 1] = -1;
+}
+
+// Grid: n_copy CTAs copy K and V [L][H][R][D] into the slot laid out as
+// [L][H][2][R][D]; one extra CTA edits the table.
+__global__ void __launch_bounds__(kCopyThreads) append_kernel(uint4* slot_base, const uint4* K, const uint4* V,
+                                                              long long heads, int chunks_per_head, int* table_row,
+                                                              int pos, int n_old, int slot, int n_copy) {
+  if ((int)blockIdx.x == n_copy) {
+    table_insert_cta(table_row, pos, n_old, slot);
+    return;
+  }
+  const long long per_kv = heads * chunks_per_head;
+  const long long total = 2 * per_kv;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (long long)n_copy * blockDim.x) {
+    const int kv = i >= per_kv;
+    const long long j = kv ? i - per_kv : i;
+    const long long lh = j / chunks_per_head;
+    const int off = (int)(j - lh * chunks_per_head);
+    const uint4 v = kv ? V[j] : K[j];
+    slot_base[(lh * 2 + kv) * chunks_per_head + off] = v;
+  }
+}
+
+__global__ void __launch_bounds__(kCopyThreads) table_remove_kernel(int* row, int pos, int n) {
+  table_remove_cta(row, pos, n);
+}
+
+// rows [n][H][D] (K and V) -> in-block layout [H][2][b][D] of one layer
+__global__ void inblock_write_kernel(uint4* ib, const uint4* K, const uint4* V, int n, int H, int cpr) {
+  const int total = 2 * n * H * cpr;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    const int kv = i >= n * H * cpr;
+    const int j = kv ? i - n * H * cpr : i;
+    const int t = j / (H * cpr);
+    const int h = (j / cpr) % H;
+    const int c = j % cpr;
+    ib[((h * 2 + kv) * kBlockTok + t) * cpr + c] = kv ? V[j] : K[j];
+  }
+}
+
+// k, v [L][H][D] -> null_kv [L][H][2][D]
+__global__ void null_write_kernel(uint4* dst, const uint4* k, const uint4* v, int LH, int cpr) {
+  const int total = 2 * LH * cpr;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    const int kv = i >= LH * cpr;
+    const int j = kv ? i - LH * cpr : i;
+    const int lh = j / cpr, c = j % cpr;
+    dst[(lh * 2 + kv) * cpr + c] = kv ? v[j] : k[j];
+  }
+}
+
+__global__ void zero_kernel(uint4* p, long long n16) {
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += (long long)gridDim.x * blockDim.x)
+    p[i] = make_uint4(0, 0, 0, 0);
+}
+
+cudaError_t launch_append(uint16_t* slot_base, const uint16_t* K, const uint16_t* V, int L, int H, int D,
+                          int* table_row, int pos, int n_old, int slot, cudaStream_t st) {
+  const int chunks_per_head = kRows * D * 2 / 16;
+  const long long heads = (long long)L * H;
+  const long long total = 2 * heads * chunks_per_head;
+  long long n_copy = (total + kCopyThreads * 4 - 1) / (kCopyThreads * 4);
+  if (n_copy > 1184) n_copy = 1184;
+  append_kernel<<<(int)n_copy + 1, kCopyThreads, 0, st>>>(
+      reinterpret_cast<uint4*>(slot_base), reinterpret_cast<const uint4*>(K), reinterpret_cast<const uint4*>(V),
+      heads, chunks_per_head, table_row, pos, n_old, slot, (int)n_copy);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_table_remove(int* table_row, int pos, int n_old, cudaStream_t st) {
+  table_remove_kernel<<<1, kCopyThreads, 0, st>>>(table_row, pos, n_old);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
+                                 int D, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  const int cpr = D * 2 / 16;
+  const int total = 2 * n * H * cpr;
+  const int blocks = (total + 255) / 256;
+  inblock_write_kernel<<<blocks, 256, 0, st>>>(reinterpret_cast<uint4*>(ib_layer_base),
+                                               reinterpret_cast<const uint4*>(K),
+                                               reinterpret_cast<const uint4*>(V), n, H, cpr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
+                              cudaStream_t st) {
+  const int cpr = D * 2 / 16;
+  const int total = 2 * L * H * cpr;
+  null_write_kernel<<<(total + 255) / 256, 256, 0, st>>>(
+      reinterpret_cast<uint4*>(null_kv), reinterpret_cast<const uint4*>(k), reinterpret_cast<const uint4*>(v), L * H,
+      cpr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st) {
+  const long long n16 = (long long)(bytes / 16);
+  if (n16 == 0) return cudaSuccess;
+  long long blocks = (n16 + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  zero_kernel<<<(int)blocks, 256, 0, st>>>(reinterpret_cast<uint4*>(p), n16);
+  return cudaGetLastError();
+}
+
+}  // namespace smem

@@ -1,0 +1,125 @@
+// smem_internal.h -- launch parameters and launchers shared by the C ABI
+// (smem_capi.cpp) and the kernels (*.cu). Not part of the public ABI.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime_api.h>
+
+#ifdef __CUDACC__
+#define SMEM_HD __host__ __device__
+#else
+#define SMEM_HD
+#endif
+
+namespace smem {
+
+constexpr int kRows = 64;     // R: memory rows per block (one K/V tile)
+constexpr int kBlockTok = 64; // b: query tokens per block
+
+// ---------------------------------------------------------------------------
+// device-buffer geometry (all offsets in bytes from dev_buf)
+// ---------------------------------------------------------------------------
+struct Layout {
+  int L, H, D, max_seqs, max_blocks, capacity, has_null, max_batch;
+  int dec_max_splits;  // split-K partial slots per (decode item, head)
+  int pf_max_splits;   // split-K partial slots per prefill head
+  size_t slot_elems;   // bf16 elements per pool slot = L*H*2*R*D
+  size_t off_pool, off_inblock, off_null, off_table, off_dec_part, off_dec_cnt, off_pf_part, off_pf_cnt,
+      off_err, total;
+};
+
+// Split-K plan of the decode cross-attention: the number of memory blocks a
+// split reads, a function of the sequence's block count alone (so the same
+// block set always reduces in the same order).
+SMEM_HD inline int decode_split_blocks(int nblk) {
+  int sb = (nblk + 31) / 32;
+  return sb < 4 ? 4 : (sb > 16 ? 16 : sb);
+}
+SMEM_HD inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+// Split plan of the one-block prefill cross-attention, again a function of
+// the block count (and the cache's fixed head count) alone.
+constexpr int kPrefillTargetUnits = 296;  // about two work units per SM of a GB300
+constexpr int kPrefillMaxSplits = 64;
+SMEM_HD inline int prefill_split_blocks(int nblk, int H) {
+  int per_head = ceil_div(kPrefillTargetUnits, H);
+  int sb = ceil_div(nblk, per_head);
+  if (sb < 2) sb = 2;
+  int ns = ceil_div(nblk, sb);
+  if (ns > kPrefillMaxSplits) sb = ceil_div(nblk, kPrefillMaxSplits);
+  return sb;
+}
+
+// ---------------------------------------------------------------------------
+// decode
+// ---------------------------------------------------------------------------
+constexpr int kMaxDecodeItems = 512;  // items per launch (kernel parameter space)
+
+struct DecodeItem {
+  int seq;         // sequence id (row of the device table)
+  int nblk;        // memory blocks read (table prefix with index < q_block_idx)
+  int pos;         // in-block offset p of the new token
+  int pair_begin;  // first (item, split) pair of this item
+};
+
+struct DecodeParams {
+  const uint16_t* pool;      // [C][L][H][2][R][D]
+  uint16_t* inblock;         // [max_seqs][L][H][2][b][D]
+  const int* table;          // [max_seqs][max_blocks] slots, ascending block index
+  const uint16_t* null_kv;   // [L][H][2][D] or nullptr
+  float* part;               // [pair][H][D + 2]: m, l, acc[D]
+  unsigned* counters;        // [max_batch][H], zero between launches
+  int* err;                  // device error word
+  const uint16_t* qs;        // [nb][H][D]
+  const uint16_t* k_new;
+  const uint16_t* v_new;
+  const uint16_t* qc;
+  uint16_t* osa;
+  uint16_t* oca;
+  long long slot_elems;      // elements per pool slot
+  int L, H, layer, max_blocks, capacity;
+  int n_items, n_pairs;      // items and CA (item, split) pairs in this launch
+  float scale_log2;          // log2(e) / sqrt(D)
+  DecodeItem items[kMaxDecodeItems];
+};
+
+cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st);
+int decode_max_grid(int D, int num_sms);
+
+// ---------------------------------------------------------------------------
+// copies and table edits
+// ---------------------------------------------------------------------------
+// Appends: copy K, V [L][H][R][D] into a pool slot and insert `slot` at
+// table position `pos` of `seq` (n_old entries before the insert).
+cudaError_t launch_append(uint16_t* slot_base, const uint16_t* K, const uint16_t* V, int L, int H, int D,
+                          int* table_row, int pos, int n_old, int slot, cudaStream_t st);
+// Removes table position `pos` of a row holding n_old entries.
+cudaError_t launch_table_remove(int* table_row, int pos, int n_old, cudaStream_t st);
+// In-block write: rows [n][H][D] -> inblock[seq][layer][h][2][b][D].
+cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
+                                 int D, cudaStream_t st);
+// Null row: k,v [L][H][D] -> null_kv [L][H][2][D].
+cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
+                              cudaStream_t st);
+cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st);
+
+// ---------------------------------------------------------------------------
+// prefill
+// ---------------------------------------------------------------------------
+struct PrefillArgs {
+  const uint16_t* pool;
+  const int* table_row;       // slots of this sequence, ascending block index
+  const uint16_t* null_kv;    // [L][H][2][D] or nullptr
+  const uint16_t *qs, *ks, *vs, *qc;  // [b][H][D]
+  uint16_t *osa, *oca;
+  float* part;                // [H][pf_max_splits][b][D + 2]
+  unsigned* counters;         // [H]
+  int* err;
+  long long slot_elems;
+  int L, H, D, layer, nblk, split_blks, n_splits, capacity;
+  float scale_log2;
+};
+cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);
+
+}  // namespace smem

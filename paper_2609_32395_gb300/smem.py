@@ -1,0 +1,271 @@
+"""Python binding of the C ABI in include/smem.h (argument marshalling only).
+
+Every function keeps the C name and forwards to ``libsmem.so``; all work of
+the reader path runs in the library's CUDA kernels. Device buffers are torch
+tensors (bf16, contiguous, on the cache's device); the stream is torch's
+current CUDA stream unless one is given. A negative return code raises
+:class:`SmemError`. There is no CPU fallback: if the library is missing or
+fails to load, :func:`lib` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import _build
+
+OK = 0
+ERR_INVALID_ARG = -1
+ERR_ALIGN = -2
+ERR_NO_SUCH_SEQ = -3
+ERR_DUPLICATE_BLOCK = -4
+ERR_NO_SUCH_BLOCK = -5
+ERR_POOL_FULL = -6
+ERR_TABLE_FULL = -7
+ERR_CUDA = -8
+ERR_DEVICE_FAULT = -9
+ERR_UNSUPPORTED = -10
+ERR_NO_DEVICE = -11
+
+EXPORTED = [
+    "smem_cache_required_bytes", "smem_cache_create", "smem_cache_destroy", "smem_set_null_row",
+    "smem_append_block", "smem_delete_block", "smem_release_seq", "smem_write_inblock", "smem_prefill_block",
+    "smem_decode", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table", "smem_check_device_error",
+    "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
+]
+
+
+class SmemError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        detail = ""
+        if code in (ERR_CUDA, ERR_DEVICE_FAULT):
+            detail = " (" + lib().smem_last_error_detail().decode() + ")"
+        super().__init__(f"{where}: {lib().smem_strerror(code).decode()} [{code}]{detail}")
+
+
+class SmemConfig(ctypes.Structure):
+    _fields_ = [
+        ("n_layers", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+        ("block_tokens", ctypes.c_int32), ("rows_per_block", ctypes.c_int32), ("max_seqs", ctypes.c_int32),
+        ("max_blocks_per_seq", ctypes.c_int32), ("capacity_slots", ctypes.c_int32),
+        ("has_null_row", ctypes.c_int32), ("max_decode_batch", ctypes.c_int32),
+        ("free_order", ctypes.POINTER(ctypes.c_int32)),
+    ]
+
+
+_lib = None
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int32
+_i32p = ctypes.POINTER(ctypes.c_int32)
+
+
+def lib():
+    """The loaded libsmem.so (built in-tree on first use)."""
+    global _lib
+    if _lib is None:
+        import torch  # noqa: F401  (load PyTorch's CUDA runtime first, so both share it)
+
+        path = _build.build()
+        L = ctypes.CDLL(path, mode=ctypes.RTLD_GLOBAL)
+        cfgp = ctypes.POINTER(SmemConfig)
+        sig = {
+            "smem_cache_required_bytes": (ctypes.c_size_t, [cfgp]),
+            "smem_cache_create": (ctypes.c_int, [cfgp, _vp, ctypes.c_size_t, ctypes.POINTER(_vp)]),
+            "smem_cache_destroy": (ctypes.c_int, [_vp]),
+            "smem_set_null_row": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
+            "smem_append_block": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _vp, _i32p]),
+            "smem_delete_block": (ctypes.c_int, [_vp, _i32, _i32, _vp]),
+            "smem_release_seq": (ctypes.c_int, [_vp, _i32, _vp]),
+            "smem_write_inblock": (ctypes.c_int, [_vp, _i32, _i32, _i32, _vp, _vp, _vp]),
+            "smem_prefill_block": (ctypes.c_int, [_vp, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
+            "smem_decode": (ctypes.c_int, [_vp, _i32, _i32, _i32p, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
+            "smem_get_table": (ctypes.c_int, [_vp, _i32, _i32p, _i32p, _i32, _i32p]),
+            "smem_get_free_fifo": (ctypes.c_int, [_vp, _i32p, _i32, _i32p]),
+            "smem_get_device_table": (ctypes.c_int, [_vp, _i32, _i32p, _i32, _i32p, _vp]),
+            "smem_check_device_error": (ctypes.c_int, [_vp, _vp]),
+            "smem_free_slots": (ctypes.c_int, [_vp, _i32p]),
+            "smem_last_error_detail": (ctypes.c_char_p, []),
+            "smem_debug_fail_after": (ctypes.c_int, [_vp, _i32]),
+            "smem_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+            "smem_abi_version": (ctypes.c_int, []),
+        }
+        for name, (res, args) in sig.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(rc: int, where: str) -> int:
+    if rc != OK:
+        raise SmemError(rc, where)
+    return rc
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+
+        if not torch.cuda.is_available():
+            return None
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _i32arr(a):
+    arr = np.ascontiguousarray(a, dtype=np.int32)
+    return arr, arr.ctypes.data_as(_i32p)
+
+
+def make_config(n_layers, n_heads, head_dim, max_seqs, max_blocks_per_seq, capacity_slots, has_null_row=False,
+                max_decode_batch=None, free_order=None, block_tokens=64, rows_per_block=64) -> SmemConfig:
+    cfg = SmemConfig(n_layers, n_heads, head_dim, block_tokens, rows_per_block, max_seqs, max_blocks_per_seq,
+                     capacity_slots, int(bool(has_null_row)),
+                     max_seqs if max_decode_batch is None else max_decode_batch, None)
+    if free_order is not None:
+        arr, p = _i32arr(free_order)
+        cfg._free_order_keep = arr
+        cfg.free_order = p
+    return cfg
+
+
+def smem_cache_required_bytes(cfg: SmemConfig) -> int:
+    return int(lib().smem_cache_required_bytes(ctypes.byref(cfg)))
+
+
+def smem_cache_create(cfg: SmemConfig, dev_buf=None):
+    """dev_buf: a torch uint8 CUDA tensor of >= required bytes, or None for a
+    bookkeeping-only cache. Returns the opaque handle (c_void_p)."""
+    h = ctypes.c_void_p()
+    nbytes = 0 if dev_buf is None else dev_buf.numel() * dev_buf.element_size()
+    _check(lib().smem_cache_create(ctypes.byref(cfg), _ptr(dev_buf), nbytes, ctypes.byref(h)), "smem_cache_create")
+    return h
+
+
+def smem_cache_destroy(h):
+    return _check(lib().smem_cache_destroy(h), "smem_cache_destroy")
+
+
+def smem_set_null_row(h, k_null, v_null, stream=None):
+    return _check(lib().smem_set_null_row(h, _ptr(k_null), _ptr(v_null), _stream(stream)), "smem_set_null_row")
+
+
+def smem_append_block(h, seq, block_idx, K=None, V=None, stream=None) -> int:
+    slot = ctypes.c_int32(-1)
+    st = _stream(stream) if K is not None else None
+    _check(lib().smem_append_block(h, seq, block_idx, _ptr(K), _ptr(V), st, ctypes.byref(slot)), "smem_append_block")
+    return slot.value
+
+
+def smem_delete_block(h, seq, block_idx, stream=None, device=True):
+    st = _stream(stream) if device else None
+    return _check(lib().smem_delete_block(h, seq, block_idx, st), "smem_delete_block")
+
+
+def smem_release_seq(h, seq, stream=None):
+    return _check(lib().smem_release_seq(h, seq, None), "smem_release_seq")
+
+
+def smem_write_inblock(h, seq, layer, n_rows, K, V, stream=None):
+    return _check(lib().smem_write_inblock(h, seq, layer, n_rows, _ptr(K), _ptr(V), _stream(stream)),
+                  "smem_write_inblock")
+
+
+def smem_prefill_block(h, seq, layer, q_block_idx, Qs, Ks, Vs, Qc, Osa, Oca, stream=None):
+    return _check(lib().smem_prefill_block(h, seq, layer, q_block_idx, _ptr(Qs), _ptr(Ks), _ptr(Vs), _ptr(Qc),
+                                           _ptr(Osa), _ptr(Oca), _stream(stream)), "smem_prefill_block")
+
+
+def smem_decode(h, layer, seq_ids, pos, q_block_idx, qs, k_new, v_new, qc, osa, oca, stream=None):
+    s, sp = _i32arr(seq_ids)
+    p, pp = _i32arr(pos)
+    q, qp = _i32arr(q_block_idx)
+    return _check(lib().smem_decode(h, layer, len(s), sp, pp, qp, _ptr(qs), _ptr(k_new), _ptr(v_new), _ptr(qc),
+                                    _ptr(osa), _ptr(oca), _stream(stream)), "smem_decode")
+
+
+def smem_get_table(h, seq):
+    n = ctypes.c_int32(0)
+    _check(lib().smem_get_table(h, seq, None, None, 0, ctypes.byref(n)), "smem_get_table")
+    idx = np.zeros(max(n.value, 1), dtype=np.int32)
+    slot = np.zeros(max(n.value, 1), dtype=np.int32)
+    _check(lib().smem_get_table(h, seq, idx.ctypes.data_as(_i32p), slot.ctypes.data_as(_i32p), n.value,
+                                ctypes.byref(n)), "smem_get_table")
+    return idx[: n.value].tolist(), slot[: n.value].tolist()
+
+
+def smem_get_free_fifo(h):
+    n = ctypes.c_int32(0)
+    _check(lib().smem_get_free_fifo(h, None, 0, ctypes.byref(n)), "smem_get_free_fifo")
+    out = np.zeros(max(n.value, 1), dtype=np.int32)
+    _check(lib().smem_get_free_fifo(h, out.ctypes.data_as(_i32p), n.value, ctypes.byref(n)), "smem_get_free_fifo")
+    return out[: n.value].tolist()
+
+
+def smem_get_device_table(h, seq, cap, stream=None):
+    n = ctypes.c_int32(0)
+    out = np.zeros(max(cap, 1), dtype=np.int32)
+    _check(lib().smem_get_device_table(h, seq, out.ctypes.data_as(_i32p), cap, ctypes.byref(n), _stream(stream)),
+           "smem_get_device_table")
+    return out[: min(n.value, cap)].tolist()
+
+
+def smem_check_device_error(h, stream=None) -> int:
+    """Returns OK or ERR_DEVICE_FAULT (does not raise for the latter)."""
+    rc = lib().smem_check_device_error(h, _stream(stream))
+    if rc not in (OK, ERR_DEVICE_FAULT):
+        raise SmemError(rc, "smem_check_device_error")
+    return rc
+
+
+def smem_free_slots(h) -> int:
+    n = ctypes.c_int32(0)
+    _check(lib().smem_free_slots(h, ctypes.byref(n)), "smem_free_slots")
+    return n.value
+
+
+def smem_debug_fail_after(h, n: int):
+    return _check(lib().smem_debug_fail_after(h, n), "smem_debug_fail_after")
+
+
+def smem_abi_version() -> int:
+    return int(lib().smem_abi_version())
+
+
+class SmemCache:
+    """Owns a cache handle and (for device caches) its device buffer."""
+
+    def __init__(self, cfg: SmemConfig, device=None):
+        import torch
+
+        self.cfg = cfg
+        self.nbytes = smem_cache_required_bytes(cfg)
+        if self.nbytes == 0:
+            raise SmemError(ERR_INVALID_ARG, "smem_cache_required_bytes")
+        self.buf = None
+        if device is not None:
+            self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        self.h = smem_cache_create(cfg, self.buf)
+
+    def close(self):
+        if self.h is not None:
+            smem_cache_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
