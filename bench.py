@@ -45,6 +45,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--seqs", type=int, default=WORKLOAD["seqs"])
+    ap.add_argument("--layers", type=int, default=WORKLOAD["L"],
+                    help="fewer layers: same per-launch work, smaller pool (profiling captures)")
     return ap.parse_args()
 
 
@@ -150,14 +152,14 @@ def profiled_traffic(profile_name, kernel_src, units_now):
 class DecodeWorkload:
     """Device state of the 410M-shaped batched-decode workload."""
 
-    def __init__(self, seqs, steps_total, seed, device, rank=0):
+    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None):
         import torch
 
         import synth
         from paper_2609_32395_gb300 import smem
 
         W = WORKLOAD
-        self.L, self.H, self.D = W["L"], W["H"], W["D"]
+        self.L, self.H, self.D = (layers or W["L"]), W["H"], W["D"]
         self.S = seqs
         self.seed = seed + 1000 * rank
         self.device = device
@@ -367,7 +369,8 @@ def run_ours(args):
     smem.lib()  # fails loudly without the CUDA library
 
     e2e_steps = 0 if args.no_e2e else min(args.steps, 64)
-    wl = DecodeWorkload(args.seqs, args.warmup + args.steps + e2e_steps + 2, WORKLOAD["seed"], device, rank)
+    wl = DecodeWorkload(args.seqs, args.warmup + args.steps + e2e_steps + 2, WORKLOAD["seed"], device, rank,
+                        layers=args.layers)
 
     def barrier():
         if ws > 1:
@@ -389,12 +392,14 @@ def run_ours(args):
     launches = 0
     with ClockSampler(local) as clk:
         barrier()
+        torch.cuda.nvtx.range_push("timed")
         start.record(st)
         for i in range(args.steps):
             r = wl.rows_read()
             rows.append(r)
             launches += wl.step(events=ev[i])
         end.record(st)
+        torch.cuda.nvtx.range_pop()
         barrier()
     elapsed = start.elapsed_time(end) / 1e3
     # per-launch durations of the decode kernel

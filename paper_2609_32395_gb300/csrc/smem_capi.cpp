@@ -24,6 +24,7 @@
 using smem::Layout;
 
 struct smem_cache {
+  CUtensorMap pool_map{};  // decode kernel's view of the pool (device caches)
   smem_config cfg{};
   Layout lay{};
   uint8_t* dev = nullptr;  // nullptr: bookkeeping-only
@@ -87,9 +88,9 @@ int make_layout(const smem_config* c, Layout* L) {
   L->off_table = off;
   off = align_up(off + (size_t)L->max_seqs * L->max_blocks * 4, A);
   L->off_dec_part = off;
-  off = align_up(off + (size_t)L->max_batch * L->H * L->dec_max_splits * (D + 2) * 4, A);
+  off = align_up(off + (size_t)L->max_batch * L->H * L->dec_max_splits * (D + 4) * 4, A);
   L->off_dec_cnt = off;
-  off = align_up(off + (size_t)L->max_batch * L->H * 4, A);
+  off = align_up(off + (size_t)L->max_batch * L->H * 4 + 64, A);  // + unit scheduler words
   L->off_pf_part = off;
   off = align_up(off + (size_t)L->H * L->pf_max_splits * smem::kBlockTok * (D + 2) * 4, A);
   L->off_pf_cnt = off;
@@ -192,12 +193,19 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
     c->dev = static_cast<uint8_t*>(dev_buf);
     cudaError_t e = cudaGetDevice(&c->device);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
-    // zero everything after the in-block rows: null rows, tables, workspace,
-    // counters and the error word
-    if (e == cudaSuccess) e = smem::launch_zero(c->dev + L.off_null, L.total - L.off_null, nullptr);
+    // zero everything but the pool: in-block rows, null rows, tables,
+    // workspace, counters and the error word
+    if (e == cudaSuccess) e = smem::launch_zero(c->dev + L.off_inblock, L.total - L.off_inblock, nullptr);
     if (e == cudaSuccess) e = cudaStreamSynchronize(nullptr);
     if (e != cudaSuccess) {
       set_detail("create", e);
+      delete c;
+      return SMEM_ERR_CUDA;
+    }
+    const int er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity,
+                                         smem::decode_stage_rows(L.D));
+    if (er != 0) {
+      std::snprintf(g_detail, sizeof(g_detail), "tensor map encode failed (%d)", er);
       delete c;
       return SMEM_ERR_CUDA;
     }
@@ -382,12 +390,15 @@ int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids
   static thread_local smem::DecodeParams P;
   for (int i0 = 0; i0 < nb; i0 += smem::kMaxDecodeItems) {
     const int n = std::min(nb - i0, smem::kMaxDecodeItems);
+    P.tmap = c->pool_map;
     P.pool = reinterpret_cast<const uint16_t*>(c->dev + L.off_pool);
     P.inblock = reinterpret_cast<uint16_t*>(c->dev + L.off_inblock);
     P.table = reinterpret_cast<const int*>(c->dev + L.off_table);
     P.null_kv = null_kv(c);
     P.part = reinterpret_cast<float*>(c->dev + L.off_dec_part);
     P.counters = reinterpret_cast<unsigned*>(c->dev + L.off_dec_cnt);
+    P.sched = reinterpret_cast<unsigned long long*>(c->dev + L.off_dec_cnt +
+                                                    ((size_t)L.max_batch * L.H * 4 + 15) / 16 * 16);
     P.err = reinterpret_cast<int*>(c->dev + L.off_err);
     P.qs = static_cast<const uint16_t*>(qs) + i0 * tok;
     P.k_new = static_cast<const uint16_t*>(k_new) + i0 * tok;
@@ -416,7 +427,8 @@ int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids
     }
     P.n_pairs = pairs;
     const long long units = (long long)(pairs + n) * L.H;
-    const int grid = (int)std::min<long long>(units, smem::decode_max_grid(L.D, c->num_sms));
+    const long long wpc = smem::decode_warps_per_cta();
+    const int grid = (int)std::min<long long>((units + wpc - 1) / wpc, smem::decode_max_grid(L.D, c->num_sms));
     if (injected_failure(c)) return SMEM_ERR_CUDA;
     const int rc = check_launch(c, smem::launch_decode(P, L.D, grid, as_stream(stream)), "decode");
     if (rc) return rc;

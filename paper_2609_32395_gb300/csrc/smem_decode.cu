@@ -9,44 +9,53 @@
 //
 // Work decomposition. A work unit is (item, split, head) for CA -- a split is
 // a run of consecutive table blocks whose length depends only on the block
-// count -- or (item, head) for SA. Units are dealt round-robin to persistent
-// CTAs. Each CTA has one producer warp that streams the units' K/V tiles
-// (one memory block = R rows of K and of V for one head, 2 x 8 KB at
-// d_h = 64) from the paged pool into a ring of shared-memory stages with bulk
-// TMA copies completing on mbarriers, and four consumer warps that each own a
-// quarter of every tile's rows: 16-byte shared loads, fp32 dot products
-// reduced across the lanes of a row, warp-level online softmax in base 2,
-// fp32 accumulation of P.V. At the end of a unit the four warps merge in warp
-// order; a CA unit writes its split partial (m, l, acc[d_h]) and the CTA
-// that completes the last split of an (item, head) merges all splits in split
-// order (null row first) and writes bf16 oca. No CTA ever waits for another.
-// Every reduction order is fixed by the block count, so the same block set
-// gives the same bits whatever the slots or the edit history.
+// count -- or (item, head) for SA. Units are dealt round-robin to worker
+// warps; every warp of a CTA is an independent worker with its own ring of
+// shared-memory stages. A stage holds 32 rows (d_h = 64) or 16 rows
+// (d_h = 128) of K and of V of one head -- 8 KB -- loaded by tensor TMA with
+// the 128-byte swizzle, so that a lane can read a whole K row without bank
+// conflicts. Lane 0 keeps the ring three stages ahead of the warp, across
+// unit boundaries. Scores are lane-per-row fp32 dot products (no shuffles),
+// the online softmax runs in base 2 with one warp maximum per stage, and P.V
+// accumulates in fp32 with each lane owning 8 columns of a quarter of the
+// rows. A CA unit writes its split partial (m, l, acc[d_h]); the warp that
+// completes the last split of an (item, head) merges all splits in split
+// order (null row first). SA units read their <= 64 in-block rows straight
+// from global memory. No warp ever waits for another warp; every reduction
+// order is fixed by the block count, so the same block set gives the same
+// bits whatever the slots or the edit history.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cudaTypedefs.h>
 
 #include "smem_device.cuh"
 #include "smem_internal.h"
 
 namespace smem {
 
+constexpr int kUnitQueue = 8;  // fetched-but-unconsumed units of a warp (<= NS + 1 used)
+
 template <int D>
-struct DecCfg {
+struct Dec {
   static constexpr int R = kRows;
-  static constexpr int TILE_BYTES = R * D * 2;  // K or V of one block and head
-  static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
-  static constexpr int NSTAGE = D == 64 ? 6 : 3;
-  static constexpr int NCW = 4;                     // consumer warps
-  static constexpr int THREADS = (NCW + 1) * 32;    // + one producer warp
-  static constexpr int LPR = D / 8;                 // lanes per row (16 B each)
-  static constexpr int RPI = 32 / LPR;              // rows per warp load
-  static constexpr int ROWS_PER_WARP = R / NCW;
-  static constexpr int ITERS = ROWS_PER_WARP / RPI;
-  static constexpr int OFF_BARS = NSTAGE * STAGE_BYTES;
-  static constexpr int OFF_COMB = OFF_BARS + 2 * NSTAGE * 8;
-  static constexpr int OFF_MISC = OFF_COMB + NCW * (D + 2) * 4;
-  static constexpr int SMEM = OFF_MISC + 64;
+  static constexpr int SROWS = D == 64 ? 32 : 16;  // rows per stage
+  static constexpr int CHUNKS = R / SROWS;         // stages per memory block
+  static constexpr int HALF = SROWS * D * 2;       // K (or V) bytes of a stage
+  static constexpr int STAGE = 2 * HALF;           // 8 KB
+  static constexpr int BOXES = D / 64;             // 128-byte-wide TMA boxes per row
+  static constexpr int BOX_BYTES = SROWS * 128;
+  static constexpr int NW = 8;                     // worker warps per CTA
+  static constexpr int NS = 3;                     // stages per warp
+  static constexpr int THREADS = NW * 32;
+  static constexpr int LPR = D / 64;               // lanes per row in the score phase
+  static constexpr int OFF_BAR = NW * NS * STAGE;
+  static constexpr int OFF_P = OFF_BAR + NW * NS * 8;
+  static constexpr int OFF_Q = OFF_P + NW * 64 * 4;            // per stage: the unit's query
+  static constexpr int OFF_UQ = OFF_Q + NW * NS * D * 2;         // per warp: unit queue
+  static constexpr int OFF_END = OFF_UQ + NW * kUnitQueue * 4;
+  static constexpr int SMEM = OFF_END + 1024;      // + slack to align the base to 1 KB
 };
 
 struct Unit {
@@ -55,7 +64,7 @@ struct Unit {
   int h;
   int split;  // CA only
   int b0;     // first table position (CA)
-  int nt;     // tiles
+  int nt;     // memory blocks (CA)
 };
 
 __device__ __forceinline__ Unit unit_of(const DecodeParams& p, int u) {
@@ -83,318 +92,499 @@ __device__ __forceinline__ Unit unit_of(const DecodeParams& p, int u) {
     U.h = v - U.item * p.H;
     U.split = 0;
     U.b0 = 0;
-    U.nt = 1;
+    U.nt = 0;
   }
   return U;
 }
 
-__device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
-  uint32_t r;
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
   asm volatile(
-      "{\n\t.reg .pred pi, po;\n\t"
-      "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.or.pred po, %2, %3, pi;\n\t"
-      "selp.u32 %0, 1, 0, po;\n\t}"
-      : "=r"(r)
-      : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+      "[%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
-  return r != 0;
+}
+
+__device__ __forceinline__ uint4 ld_nc16(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ void store_bf16x8(uint16_t* dst, const float* v, float scale) {
+  uint4 o;
+  o.x = pack_bf16x2(v[0] * scale, v[1] * scale);
+  o.y = pack_bf16x2(v[2] * scale, v[3] * scale);
+  o.z = pack_bf16x2(v[4] * scale, v[5] * scale);
+  o.w = pack_bf16x2(v[6] * scale, v[7] * scale);
+  *reinterpret_cast<uint4*>(dst) = o;
+}
+
+// Issue side of one warp's chunk stream over dynamically fetched CA units.
+// Lane 0 only. Units come from a launch-wide atomic counter, one unit ahead
+// of the unit being issued; each fetched unit is pushed on the warp's unit
+// queue together with the stage that holds its first chunk.
+struct Issue {
+  int u;       // unit being issued (< 0: exhausted)
+  int c;       // next chunk of that unit
+  int nc;      // chunks of that unit
+  int item, h, b0;
+  int next_u;  // unit fetched for after this one
+  int pushed;  // queue entries pushed
+};
+
+__device__ __forceinline__ int fetch_unit(const DecodeParams& p) {
+  const unsigned long long u = atomicAdd(p.sched, 1ull);
+  const int nca = p.n_pairs * p.H;
+  return u < (unsigned long long)nca ? (int)u : -1;
 }
 
 template <int D>
-__global__ void __launch_bounds__(DecCfg<D>::THREADS, 2)
-    decode_kernel(const __grid_constant__ DecodeParams p) {
-  using C = DecCfg<D>;
-  extern __shared__ __align__(128) uint8_t smem_raw[];
-  uint8_t* stages = smem_raw;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + C::OFF_BARS);
-  uint64_t* empty = full + C::NSTAGE;
-  float* comb = reinterpret_cast<float*>(smem_raw + C::OFF_COMB);  // [NCW][D+2]
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem_raw + C::OFF_MISC);
-  volatile unsigned* ticket = reinterpret_cast<volatile unsigned*>(smem_raw + C::OFF_MISC + 4);
-  volatile float* null_score = reinterpret_cast<volatile float*>(smem_raw + C::OFF_MISC + 8);
+__device__ __forceinline__ void issue_begin_unit(const DecodeParams& p, Issue& is, int u, int* uq) {
+  is.u = u;
+  is.c = 0;
+  if (u >= 0) {
+    const Unit U = unit_of(p, u);
+    is.nc = U.nt * Dec<D>::CHUNKS;
+    is.item = U.item;
+    is.h = U.h;
+    is.b0 = U.b0;
+    is.next_u = fetch_unit(p);
+  } else {
+    is.nc = 0;
+  }
+  uq[is.pushed % kUnitQueue] = u;  // -1 marks the end of the stream
+  ++is.pushed;
+}
 
-  const int tid = threadIdx.x;
-  const int warp = tid >> 5;
-  const int lane = tid & 31;
-  const int total = (p.n_pairs + p.n_items) * p.H;
-
-  if (tid == 0) {
-    for (int s = 0; s < C::NSTAGE; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], C::NCW);
+// Loads the next chunk of the stream into `stage` (and the unit's query into
+// `qslot` with its first chunk); returns false when the stream is exhausted.
+template <int D>
+__device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uint8_t* stage, uint16_t* qslot,
+                                           uint64_t* bar, int* uq) {
+  using C = Dec<D>;
+  if (is.u < 0) return false;
+  const int blk = is.b0 + is.c / C::CHUNKS;
+  const int row0 = (is.c % C::CHUNKS) * C::SROWS;
+  const int slot = p.table[(size_t)p.items[is.item].seq * p.max_blocks + blk];
+  const uint32_t qbytes = is.c == 0 ? D * 2 : 0;
+  if (slot < 0 || slot >= p.capacity) {
+    record_error(p.err, kDevErrBounds);
+    mbar_arrive(bar);  // the stage keeps stale rows; the error is flagged
+  } else {
+    const int y = ((p.layer * p.H + is.h) * 2) * C::R + row0;
+    mbar_arrive_expect_tx(bar, C::STAGE + qbytes);
+#pragma unroll
+    for (int bx = 0; bx < C::BOXES; ++bx) {
+      tma_load_3d(stage + bx * C::BOX_BYTES, &p.tmap, bx * 64, y, slot, bar);
+      tma_load_3d(stage + C::HALF + bx * C::BOX_BYTES, &p.tmap, bx * 64, y + C::R, slot, bar);
     }
-    *abort_flag = 0;
+    if (qbytes) bulk_g2s(qslot, p.qc + ((size_t)is.item * p.H + is.h) * D, qbytes, bar);
+  }
+  if (++is.c == is.nc) issue_begin_unit<D>(p, is, is.next_u, uq);
+  return true;
+}
+
+// Self-attention unit: in-block rows 0..p-1 and the new token's row, read
+// directly from global memory. Writes osa, stores the new row, and writes
+// oca for a sequence that has no readable memory block.
+template <int D>
+__device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int lane) {
+  constexpr int LPR = Dec<D>::LPR;
+  constexpr int RPP = 32 / LPR;  // rows per pass
+  const DecodeItem& it = p.items[U.item];
+  const int n = it.pos + 1;
+  const size_t qoff = ((size_t)U.item * p.H + U.h) * D;
+  const uint16_t* ib = p.inblock + (((size_t)it.seq * p.L + p.layer) * p.H + U.h) * (size_t)2 * kBlockTok * D;
+  const int hh = lane % LPR;  // which 64 columns of the row
+  float q[64];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    float t[8];
+    unpack8(ld_nc16(p.qs + qoff + hh * 64 + j * 8), t);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
+  }
+  // scores of rows lane/LPR + k*RPP
+  float s[kBlockTok / RPP];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int k = 0; k < kBlockTok / RPP; ++k) {
+    const int r = k * RPP + lane / LPR;
+    float dot = 0.f;
+    if (r < n) {
+      const uint16_t* row = r == it.pos ? p.k_new + qoff : ib + (size_t)r * D;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        float t[8];
+        unpack8(ld_nc16(row + hh * 64 + j * 8), t);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
+      }
+    }
+    if (LPR == 2) dot += __shfl_xor_sync(0xffffffffu, dot, 1);
+    s[k] = r < n ? dot : -INFINITY;
+    mx = fmaxf(mx, s[k]);
+  }
+#pragma unroll
+  for (int o = LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  float l = 0.f;
+#pragma unroll
+  for (int k = 0; k < kBlockTok / RPP; ++k) {
+    const int r = k * RPP + lane / LPR;
+    const float pr = r < n ? exp2f(s[k] - mx) : 0.f;
+    if (hh == 0) {
+      l += pr;
+      pbuf[r] = pr;
+    }
+  }
+  __syncwarp();
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+  // P.V: lane (g, c) owns column chunk c of rows g*RG .. g*RG+RG-1
+  constexpr int CPL = D / 8;        // column chunks
+  constexpr int G = 32 / CPL;       // row groups
+  constexpr int RG = kBlockTok / G; // rows per group
+  const int g = lane / CPL, c = lane % CPL;
+  float acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+  for (int i = 0; i < RG; ++i) {
+    const int r = g * RG + i;
+    if (r < n) {
+      const float pr = pbuf[r];
+      const uint16_t* row = r == it.pos ? p.v_new + qoff : ib + (size_t)kBlockTok * D + (size_t)r * D;
+      float t[8];
+      unpack8(ld_nc16(row + c * 8), t);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] = fmaf(pr, t[e], acc[e]);
+    }
+  }
+#pragma unroll
+  for (int o = CPL; o < 32; o <<= 1)
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+  if (g == 0) store_bf16x8(p.osa + qoff + c * 8, acc, 1.f / l);
+  // the new token's k and v become in-block row p for later steps
+  if (lane < 2 * CPL) {
+    const int kv = lane / CPL, cc = lane % CPL;
+    uint16_t* dst = (uint16_t*)ib + (size_t)kv * kBlockTok * D + (size_t)it.pos * D + cc * 8;
+    *reinterpret_cast<uint4*>(dst) = ld_nc16((kv ? p.v_new : p.k_new) + qoff + cc * 8);
+  }
+  // no readable memory block: oca is the null row's value or zero
+  if (it.nblk == 0 && lane < CPL) {
+    float v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = 0.f;
+    if (p.null_kv) unpack8(ld_nc16(p.null_kv + ((size_t)p.layer * p.H + U.h) * 2 * D + D + lane * 8), v);
+    store_bf16x8(p.oca + qoff + lane * 8, v, 1.f);
+  }
+  __syncwarp();
+}
+
+// Split partials a warp has written but not yet announced (pend1), or
+// announced with a ticket still in flight (pend2): the fence and the atomic of
+// a unit are issued one unit later and their result read two units later,
+// so neither stalls the warp while the ring keeps streaming.
+struct Pending {
+  int valid, item, h, nsplit, pair_begin;
+  unsigned ticket;  // lane 0
+};
+
+template <int D>
+__device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane) {
+  constexpr int CPT = D / 32;  // columns per lane
+  const size_t qoff = ((size_t)pd.item * p.H + pd.h) * D;
+  float nscore = -INFINITY;
+  if (p.null_kv) {
+    // null-row score with the same scaled-query dot product as the rows
+    const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + pd.h) * 2 * D;
+    float dot = 0.f;
+#pragma unroll
+    for (int e = 0; e < CPT; ++e)
+      dot = fmaf(bf16lo(p.qc[qoff + lane * CPT + e]) * p.scale_log2, bf16lo(kn[lane * CPT + e]), dot);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+    nscore = dot;
+  }
+  const float* pb = p.part + ((size_t)pd.pair_begin * p.H + pd.h) * (D + 4);
+  const size_t ps = (size_t)p.H * (D + 4);
+  float M = nscore;
+  for (int s2 = 0; s2 < pd.nsplit; ++s2) M = fmaxf(M, __ldcg(pb + s2 * ps));
+  float Lsum = 0.f, A[CPT];
+#pragma unroll
+  for (int e = 0; e < CPT; ++e) A[e] = 0.f;
+  if (p.null_kv) {
+    const float f = exp2f(nscore - M);
+    Lsum = f;
+    const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.H + pd.h) * 2 * D + D;
+#pragma unroll
+    for (int e = 0; e < CPT; ++e) A[e] = f * bf16lo(vn[lane * CPT + e]);
+  }
+  for (int s2 = 0; s2 < pd.nsplit; ++s2) {
+    const float* ps2 = pb + s2 * ps;
+    const float f = exp2f(__ldcg(ps2) - M);
+    Lsum = fmaf(f, __ldcg(ps2 + 1), Lsum);
+#pragma unroll
+    for (int e = 0; e < CPT; ++e) A[e] = fmaf(f, __ldcg(ps2 + 4 + lane * CPT + e), A[e]);
+  }
+  const float inv = 1.f / Lsum;
+  uint32_t* o32 = reinterpret_cast<uint32_t*>(p.oca + qoff) + lane * (CPT / 2);
+#pragma unroll
+  for (int e = 0; e < CPT; e += 2) o32[e / 2] = pack_bf16x2(A[e] * inv, A[e + 1] * inv);
+  if (lane == 0) p.counters[pd.item * p.H + pd.h] = 0u;
+}
+
+// pend2: read its ticket; the warp that completed the last split merges.
+template <int D>
+__device__ __forceinline__ void settle(const DecodeParams& p, Pending& pd, int lane) {
+  if (!pd.valid) return;
+  const unsigned t = __shfl_sync(0xffffffffu, pd.ticket, 0);
+  if (t == (unsigned)(pd.nsplit - 1)) {
+    __threadfence();
+    merge_splits<D>(p, pd, lane);
+  }
+  pd.valid = 0;
+}
+
+// pend1 -> pend2: make its partial visible, then take a ticket.
+__device__ __forceinline__ void announce(const DecodeParams& p, Pending& from, Pending& to, int lane) {
+  if (!from.valid) return;
+  __threadfence();
+  if (lane == 0) from.ticket = atomicAdd(&p.counters[from.item * p.H + from.h], 1u);
+  to = from;
+  from.valid = 0;
+}
+
+template <int D>
+__global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid_constant__ DecodeParams p) {
+  using C = Dec<D>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  uint8_t* ring = base + warp * C::NS * C::STAGE;
+  uint64_t* full = reinterpret_cast<uint64_t*>(base + C::OFF_BAR) + warp * C::NS;
+  float* pbuf = reinterpret_cast<float*>(base + C::OFF_P) + warp * 64;
+  uint16_t* qarea = reinterpret_cast<uint16_t*>(base + C::OFF_Q) + warp * C::NS * D;
+  int* uq = reinterpret_cast<int*>(base + C::OFF_UQ) + warp * kUnitQueue;
+
+  if (lane == 0) {
+    for (int s = 0; s < C::NS; ++s) mbar_init(&full[s], 1);
     fence_mbar_init();
   }
   __syncthreads();
 
-  const size_t head_elems = (size_t)2 * C::R * D;  // K and V rows of one head
+  const int wid = blockIdx.x * C::NW + warp;
+  const int stride = gridDim.x * C::NW;
 
-  // ------------------------------------------------------------------ producer
-  if (warp == C::NCW) {
-    if (lane != 0) return;
-    uint32_t fill = 0;
-    uint32_t last_round[C::NSTAGE];
-    bool issued[C::NSTAGE];
-#pragma unroll
-    for (int s = 0; s < C::NSTAGE; ++s) { issued[s] = false; last_round[s] = 0; }
-    bool ok = true;
-    for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
-      const Unit U = unit_of(p, u);
-      const DecodeItem& it = p.items[U.item];
-      for (int t = 0; t < U.nt; ++t, ++fill) {
-        const int st = fill % C::NSTAGE;
-        const uint32_t round = fill / C::NSTAGE;
-        if (round > 0 && !mbar_wait_bounded(&empty[st], (round - 1) & 1, abort_flag)) {
-          if (!*abort_flag) record_error(p.err, kDevErrWaitEmpty);
-          *abort_flag = 1;
-          ok = false;
-          break;
-        }
-        uint8_t* kdst = stages + st * C::STAGE_BYTES;
-        uint8_t* vdst = kdst + C::TILE_BYTES;
-        if (!U.sa) {
-          const int slot = p.table[(size_t)it.seq * p.max_blocks + U.b0 + t];
-          if (slot < 0 || slot >= p.capacity) {
-            record_error(p.err, kDevErrBounds);
-            mbar_arrive(&full[st]);  // stale stage contents; the error is flagged
-          } else {
-            const uint16_t* src =
-                p.pool + (size_t)slot * p.slot_elems + ((size_t)p.layer * p.H + U.h) * head_elems;
-            mbar_arrive_expect_tx(&full[st], C::STAGE_BYTES);
-            bulk_g2s(kdst, src, C::TILE_BYTES, &full[st]);
-            bulk_g2s(vdst, src + C::R * D, C::TILE_BYTES, &full[st]);
-          }
-        } else {
-          const int pos = it.pos;
-          const uint32_t row_bytes = D * 2;
-          const uint16_t* ib =
-              p.inblock + (((size_t)it.seq * p.L + p.layer) * p.H + U.h) * (size_t)2 * kBlockTok * D;
-          const size_t qoff = ((size_t)U.item * p.H + U.h) * D;
-          mbar_arrive_expect_tx(&full[st], 2u * (uint32_t)(pos + 1) * row_bytes);
-          if (pos > 0) {
-            bulk_g2s(kdst, ib, (uint32_t)pos * row_bytes, &full[st]);
-            bulk_g2s(vdst, ib + (size_t)kBlockTok * D, (uint32_t)pos * row_bytes, &full[st]);
-          }
-          bulk_g2s(kdst + pos * row_bytes, p.k_new + qoff, row_bytes, &full[st]);
-          bulk_g2s(vdst + pos * row_bytes, p.v_new + qoff, row_bytes, &full[st]);
-        }
-        issued[st] = true;
-        last_round[st] = round;
-      }
-    }
-    if (!ok) {
-      // give copies already in flight (bounded) time to land before exit
-#pragma unroll
-      for (int s = 0; s < C::NSTAGE; ++s)
-        if (issued[s]) mbar_wait_bounded(&full[s], last_round[s] & 1, nullptr);
-    }
-    return;
+  // prologue: start streaming the first CA units
+  Issue is;
+  int issued = 0;
+  if (lane == 0) {
+    is.pushed = 0;
+    issue_begin_unit<D>(p, is, fetch_unit(p), uq);
+    for (int s = 0; s < C::NS; ++s)
+      if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * D, &full[s], uq)) ++issued;
   }
 
-  // ----------------------------------------------------------------- consumers
-  const int w = warp;
-  const int g = lane / C::LPR;  // row group within a warp load
-  const int c = lane % C::LPR;  // 16-byte column chunk
-  constexpr unsigned FULL = 0xffffffffu;
-  uint32_t fill = 0;
+  // self-attention units (static, while the first tiles are in flight)
+  for (int u = wid; u < p.n_items * p.H; u += stride) {
+    Unit U;
+    U.sa = 1;
+    U.item = u / p.H;
+    U.h = u - U.item * p.H;
+    sa_unit<D>(p, U, pbuf, lane);
+  }
+  __syncwarp();
 
-  for (int u = blockIdx.x; u < total; u += gridDim.x) {
+  constexpr int CPL = D / 8;             // P.V column chunks
+  constexpr int G = 32 / CPL;            // P.V row groups per stage
+  constexpr int RG = C::SROWS / G;       // rows per group per stage (8)
+  const int g = lane / CPL, c = lane % CPL;
+  const int hh = lane % C::LPR;          // score phase: which 64 columns
+  const int rr = lane / C::LPR;          // score phase: row within the stage
+  int k = 0;                             // chunks consumed
+  int popped = 0;
+  bool failed = false;
+  Pending pend1, pend2;
+  pend1.valid = pend2.valid = 0;
+
+  while (!failed) {
+    const int u = uq[popped % kUnitQueue];
+    ++popped;
+    if (u < 0) break;
     const Unit U = unit_of(p, u);
     const DecodeItem& it = p.items[U.item];
     const size_t qoff = ((size_t)U.item * p.H + U.h) * D;
-    const int n_valid = U.sa ? it.pos + 1 : C::R;
-
-    float q[8];
-    {
-      const uint4 qv = *reinterpret_cast<const uint4*>((U.sa ? p.qs : p.qc) + qoff + c * 8);
-      unpack8(qv, q);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) q[j] *= p.scale_log2;
-    }
+    float q[64];
     float m = -INFINITY, l = 0.f, acc[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) acc[j] = 0.f;
-    bool failed = false;
+    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
 
-    for (int t = 0; t < U.nt; ++t, ++fill) {
-      const int st = fill % C::NSTAGE;
-      const uint32_t round = fill / C::NSTAGE;
-      if (!failed && !mbar_wait_bounded(&full[st], round & 1, abort_flag)) {
-        if (!*abort_flag) record_error(p.err, kDevErrWaitFull);
-        *abort_flag = 1;
+    const int nch = U.nt * C::CHUNKS;
+    for (int ch = 0; ch < nch; ++ch, ++k) {
+      const int s = k % C::NS;
+      const uint32_t par = (k / C::NS) & 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(&full[s], par, nullptr));
+      if (!ok) {
+        if (lane == 0) record_error(p.err, kDevErrWaitFull);
         failed = true;
+        break;
       }
-      if (failed) continue;
-      const uint8_t* kt = stages + st * C::STAGE_BYTES;
-      const uint8_t* vt = kt + C::TILE_BYTES;
-
-      float s[C::ITERS];
-      float tmax = -INFINITY;
+      if (ch == 0) {
+        const uint16_t* qs = qarea + s * D + hh * 64;
 #pragma unroll
-      for (int i = 0; i < C::ITERS; ++i) {
-        const int r = w * C::ROWS_PER_WARP + i * C::RPI + g;
-        float dot = 0.f;
-        if (r < n_valid) {
-          const uint4 kv = *reinterpret_cast<const uint4*>(kt + r * (D * 2) + c * 16);
-          float kf[8];
-          unpack8(kv, kf);
+        for (int j = 0; j < 8; ++j) {
+          float t[8];
+          unpack8(*reinterpret_cast<const uint4*>(qs + j * 8), t);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) dot = fmaf(q[j], kf[j], dot);
+          for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
         }
-#pragma unroll
-        for (int o = 1; o < C::LPR; o <<= 1) dot += __shfl_xor_sync(FULL, dot, o);
-        s[i] = r < n_valid ? dot : -INFINITY;
-        tmax = fmaxf(tmax, s[i]);
       }
+      const uint8_t* kb = ring + s * C::STAGE;
+      const uint8_t* vb = kb + C::HALF;
+      // scores: lane-per-row (two lanes per row at d_h = 128)
+      float dot0 = 0.f, dot1 = 0.f;
+      const uint8_t* krow = kb + hh * C::BOX_BYTES + rr * 128;
 #pragma unroll
-      for (int o = C::LPR; o < 32; o <<= 1) tmax = fmaxf(tmax, __shfl_xor_sync(FULL, tmax, o));
-      const float m_new = fmaxf(m, tmax);
-      if (m_new != -INFINITY) {
-        const float alpha = exp2f(m - m_new);
-        l *= alpha;
+      for (int j = 0; j < 8; j += 2) {
+        float t0[8], t1[8];
+        unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
+        unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[j] *= alpha;
-#pragma unroll
-        for (int i = 0; i < C::ITERS; ++i) {
-          const int r = w * C::ROWS_PER_WARP + i * C::RPI + g;
-          if (r < n_valid) {
-            const float pr = exp2f(s[i] - m_new);
-            l += pr;
-            const uint4 vv = *reinterpret_cast<const uint4*>(vt + r * (D * 2) + c * 16);
-            float vf[8];
-            unpack8(vv, vf);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) acc[j] = fmaf(pr, vf[j], acc[j]);
-          }
+        for (int e = 0; e < 8; ++e) {
+          dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
+          dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
         }
-        m = m_new;
+      }
+      float sc = dot0 + dot1;
+      if (C::LPR == 2) sc += __shfl_xor_sync(0xffffffffu, sc, 1);
+      float mx = sc;
+#pragma unroll
+      for (int o = C::LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      const float m_new = fmaxf(m, mx);
+      const float alpha = exp2f(m - m_new);
+      const float pr = exp2f(sc - m_new);
+      l = l * alpha + (hh == 0 ? pr : 0.f);
+      if (hh == 0) pbuf[rr] = pr;
+      m = m_new;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] *= alpha;
+      __syncwarp();
+      // P.V: lane (g, c), rows g*RG .. g*RG+RG-1, columns c*8 .. c*8+7
+      const uint8_t* vcol = vb + (c >> 3) * C::BOX_BYTES;
+      const int cc = c & 7;
+      const float4 p0 = *reinterpret_cast<const float4*>(pbuf + g * RG);
+      const float4 p1 = *reinterpret_cast<const float4*>(pbuf + g * RG + 4);
+      const float pv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+#pragma unroll
+      for (int i = 0; i < RG; ++i) {
+        const int r = g * RG + i;
+        float t[8];
+        unpack8(*reinterpret_cast<const uint4*>(vcol + r * 128 + ((cc ^ (r & 7)) << 4)), t);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] = fmaf(pv[i], t[e], acc[e]);
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[st]);
+      // refill this stage with the chunk NS ahead
+      if (lane == 0) {
+        fence_proxy_async_smem();
+        if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * D, &full[s], uq)) ++issued;
+      }
+      __syncwarp();
     }
+    if (failed) break;
 
-    // merge the row groups of this warp (fixed butterfly)
+    // merge the row groups and the lanes of the warp (fixed butterflies)
 #pragma unroll
-    for (int o = C::LPR; o < 32; o <<= 1) {
-      l += __shfl_xor_sync(FULL, l, o);
+    for (int o = 1; o < 32; o <<= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) acc[j] += __shfl_xor_sync(FULL, acc[j], o);
+    for (int o = CPL; o < 32; o <<= 1)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+
+    const int nsplit = ceil_div(it.nblk, decode_split_blocks(it.nblk));
+    if (nsplit == 1 && !p.null_kv) {
+      if (g == 0) store_bf16x8(p.oca + qoff + c * 8, acc, 1.f / l);
+      continue;
     }
+    settle<D>(p, pend2, lane);
+    announce(p, pend1, pend2, lane);
+    float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h) * (D + 4);
     if (g == 0) {
-      float* cw = comb + w * (D + 2);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) cw[2 + c * 8 + j] = acc[j];
-      if (c == 0) { cw[0] = m; cw[1] = l; }
+      *reinterpret_cast<float4*>(pp + 4 + c * 8) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+      *reinterpret_cast<float4*>(pp + 8 + c * 8) = make_float4(acc[4], acc[5], acc[6], acc[7]);
     }
-    if (bar_any(1, C::NCW * 32, failed)) break;  // uniform across consumer warps
-
-    // merge the four warps in warp order; thread j owns column j
-    const int nsplit = U.sa ? 1 : ceil_div(it.nblk, decode_split_blocks(it.nblk));
-    const bool direct = U.sa || (nsplit == 1 && !p.null_kv);
-    if (tid < D) {
-      float M = -INFINITY;
-#pragma unroll
-      for (int ww = 0; ww < C::NCW; ++ww) M = fmaxf(M, comb[ww * (D + 2)]);
-      float Lsum = 0.f, A = 0.f;
-#pragma unroll
-      for (int ww = 0; ww < C::NCW; ++ww) {
-        const float f = exp2f(comb[ww * (D + 2)] - M);
-        Lsum = fmaf(f, comb[ww * (D + 2) + 1], Lsum);
-        A = fmaf(f, comb[ww * (D + 2) + 2 + tid], A);
-      }
-      if (direct) {
-        uint16_t* out = U.sa ? p.osa : p.oca;
-        const __nv_bfloat16 o = __float2bfloat16_rn(A / Lsum);
-        out[qoff + tid] = *reinterpret_cast<const uint16_t*>(&o);
-      } else {
-        float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h) * (D + 2);
-        pp[2 + tid] = A;
-        if (tid == 0) { pp[0] = M; pp[1] = Lsum; }
-      }
+    if (lane == 0) {
+      pp[0] = m;
+      pp[1] = l;
     }
-    if (U.sa) {
-      // store the new token's k, v as in-block row p for the next steps
-      if (w == 0 && lane < 2 * C::LPR) {
-        const int kv = lane / C::LPR, cc = lane % C::LPR;
-        uint16_t* ib = p.inblock + (((size_t)it.seq * p.L + p.layer) * p.H + U.h) * (size_t)2 * kBlockTok * D +
-                       (size_t)kv * kBlockTok * D + (size_t)it.pos * D;
-        const uint16_t* src = (kv ? p.v_new : p.k_new) + qoff;
-        *reinterpret_cast<uint4*>(ib + cc * 8) = *reinterpret_cast<const uint4*>(src + cc * 8);
-      }
-      // a sequence with no readable memory block: oca is the null row's
-      // value (a softmax over one row) or zero
-      if (it.nblk == 0 && tid < D) {
-        float val = 0.f;
-        if (p.null_kv) val = bf16lo(p.null_kv[((size_t)p.layer * p.H + U.h) * 2 * D + D + tid]);
-        const __nv_bfloat16 o = __float2bfloat16_rn(val);
-        p.oca[qoff + tid] = *reinterpret_cast<const uint16_t*>(&o);
-      }
-    } else if (!direct) {
-      __threadfence();
-      named_bar_sync(1, C::NCW * 32);
-      if (tid == 0) *ticket = atomicAdd(&p.counters[U.item * p.H + U.h], 1u);
-      named_bar_sync(1, C::NCW * 32);
-      if (*ticket == (unsigned)(nsplit - 1)) {
-        __threadfence();
-        if (p.null_kv && w == 0) {
-          // null-row score with the same scaled-q dot product as the rows
-          const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + U.h) * 2 * D;
-          float dot = 0.f;
-          if (lane < C::LPR) {
-            const uint4 kv = *reinterpret_cast<const uint4*>(kn + lane * 8);
-            float kf[8];
-            unpack8(kv, kf);
-            float qq[8];
-            unpack8(*reinterpret_cast<const uint4*>(p.qc + qoff + lane * 8), qq);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) dot = fmaf(qq[j] * p.scale_log2, kf[j], dot);
-          }
-#pragma unroll
-          for (int o = 1; o < C::LPR; o <<= 1) dot += __shfl_xor_sync(FULL, dot, o);
-          if (lane == 0) *null_score = dot;
-        }
-        named_bar_sync(1, C::NCW * 32);
-        if (tid < D) {
-          const float* pb = p.part + ((size_t)it.pair_begin * p.H + U.h) * (D + 2);
-          const size_t ps = (size_t)p.H * (D + 2);
-          float M = p.null_kv ? *null_score : -INFINITY;
-          for (int s = 0; s < nsplit; ++s) M = fmaxf(M, __ldcg(pb + s * ps));
-          float Lsum = 0.f, A = 0.f;
-          if (p.null_kv) {
-            const float f = exp2f(*null_score - M);
-            Lsum = f;
-            A = f * bf16lo(p.null_kv[((size_t)p.layer * p.H + U.h) * 2 * D + D + tid]);
-          }
-          for (int s = 0; s < nsplit; ++s) {
-            const float f = exp2f(__ldcg(pb + s * ps) - M);
-            Lsum = fmaf(f, __ldcg(pb + s * ps + 1), Lsum);
-            A = fmaf(f, __ldcg(pb + s * ps + 2 + tid), A);
-          }
-          const __nv_bfloat16 o = __float2bfloat16_rn(A / Lsum);
-          p.oca[qoff + tid] = *reinterpret_cast<const uint16_t*>(&o);
-        }
-        if (tid == 0) p.counters[U.item * p.H + U.h] = 0u;
-      }
-    }
-    named_bar_sync(1, C::NCW * 32);  // comb[] and the ticket are reused next unit
+    pend1.valid = 1;
+    pend1.item = U.item;
+    pend1.h = U.h;
+    pend1.nsplit = nsplit;
+    pend1.pair_begin = it.pair_begin;
   }
+
+  if (!failed) {
+    settle<D>(p, pend2, lane);
+    announce(p, pend1, pend2, lane);
+    settle<D>(p, pend2, lane);
+  }
+  if (lane == 0) {
+    if (failed) {
+      // let copies already in flight land (bounded) before the warp exits
+      for (int j = k; j < issued; ++j) mbar_wait_bounded(&full[j % C::NS], (j / C::NS) & 1, nullptr);
+    }
+    // the last warp out resets the unit counter for the next launch
+    const unsigned long long done = atomicAdd(p.sched + 1, 1ull);
+    if (done == (unsigned long long)gridDim.x * C::NW - 1) {
+      p.sched[0] = 0ull;
+      p.sched[1] = 0ull;
+    }
+  }
+}
+
+int decode_stage_rows(int D) { return D == 64 ? Dec<64>::SROWS : Dec<128>::SROWS; }
+
+int encode_pool_map(CUtensorMap* map, void* pool, int L, int H, int D, int capacity, int rows_per_box) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  if (!encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return -1;
+    encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)L * H * 2 * kRows, (cuuint64_t)capacity};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)D * 2 * L * H * 2 * kRows};
+  const cuuint32_t box[3] = {64, (cuuint32_t)rows_per_box, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, pool, dims, strides, box, estr,
+                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : (int)r;
 }
 
 int decode_max_grid(int D, int num_sms) {
   (void)D;
-  return 2 * num_sms;
+  return num_sms;
 }
+
+int decode_warps_per_cta() { return Dec<64>::NW; }
 
 cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st) {
   if (D == 64) {
-    using C = DecCfg<64>;
+    using C = Dec<64>;
     cudaError_t e = cudaFuncSetAttribute(decode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     decode_kernel<64><<<grid, C::THREADS, C::SMEM, st>>>(p);
   } else if (D == 128) {
-    using C = DecCfg<128>;
+    using C = Dec<128>;
     cudaError_t e = cudaFuncSetAttribute(decode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     decode_kernel<128><<<grid, C::THREADS, C::SMEM, st>>>(p);

@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime_api.h>
 
 #ifdef __CUDACC__
@@ -64,12 +65,14 @@ struct DecodeItem {
 };
 
 struct DecodeParams {
+  CUtensorMap tmap;          // pool viewed as [C][L*H*2*R][D] bf16, 128-byte swizzle
   const uint16_t* pool;      // [C][L][H][2][R][D]
   uint16_t* inblock;         // [max_seqs][L][H][2][b][D]
   const int* table;          // [max_seqs][max_blocks] slots, ascending block index
   const uint16_t* null_kv;   // [L][H][2][D] or nullptr
-  float* part;               // [pair][H][D + 2]: m, l, acc[D]
-  unsigned* counters;        // [max_batch][H], zero between launches
+  float* part;               // [pair][H][D + 4]: m, l, pad, pad, acc[D]
+  unsigned* counters;        // [max_batch][H] split tickets, zero between launches
+  unsigned long long* sched; // [2]: next CA unit, warps finished; zero between launches
   int* err;                  // device error word
   const uint16_t* qs;        // [nb][H][D]
   const uint16_t* k_new;
@@ -86,6 +89,11 @@ struct DecodeParams {
 
 cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st);
 int decode_max_grid(int D, int num_sms);
+int decode_warps_per_cta();
+// Encodes the tensor map of the pool for the decode kernel (rows of D bf16,
+// boxes of 64 columns x rows_per_box rows).
+int encode_pool_map(CUtensorMap* map, void* pool, int L, int H, int D, int capacity, int rows_per_box);
+int decode_stage_rows(int D);
 
 // ---------------------------------------------------------------------------
 // copies and table edits
