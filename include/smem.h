@@ -63,7 +63,9 @@ enum {
     SMEM_ERR_CUDA = -8,            /* a CUDA runtime call failed           */
     SMEM_ERR_DEVICE_FAULT = -9,    /* a kernel recorded an error           */
     SMEM_ERR_UNSUPPORTED = -10,    /* shape outside the supported set      */
-    SMEM_ERR_NO_DEVICE = -11       /* bookkeeping-only cache: no device op */
+    SMEM_ERR_NO_DEVICE = -11,      /* bookkeeping-only cache: no device op */
+    SMEM_ERR_SCRATCH_LIMIT = -12   /* request needs more than the library's
+                                      fixed scratch (smem_decode_static_scratch) */
 };
 
 /* Cache geometry. Notation of the paper: L reader layers, H heads of
@@ -160,6 +162,38 @@ int smem_prefill_block(smem_cache *c, int32_t seq, int32_t layer, int32_t q_bloc
 int smem_decode(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids, const int32_t *pos,
                 const int32_t *q_block_idx, const void *qs, const void *k_new, const void *v_new,
                 const void *qc, void *osa, void *oca, void *stream);
+
+/* Bytes of the library's fixed device scratch used by
+ * smem_decode_static_scratch (16 MiB; held on every GPU that loads the
+ * library, for the life of the process). */
+#define SMEM_STATIC_SCRATCH_BYTES (16u << 20)
+
+/* Same decode step, arguments and results as smem_decode, but its split-K
+ * scratch (per-split partial softmax states, split tickets and the unit
+ * scheduler's counters) lives in a fixed array inside the library instead
+ * of in the cache's device buffer, and the call allocates nothing. It is for
+ * callers that must not allocate device memory on the serving path: a plugin
+ * inside an engine or graph runtime that owns every device allocation and
+ * hands out only inputs and outputs, or a latency-critical loop where an
+ * allocation's implicit device-wide synchronisation is not acceptable.
+ * (The paper has no counterpart; this is an interface choice of this
+ * library.)
+ *   - Scratch needed: 256 + 4*H*min(nb, 512) rounded up to 256, plus
+ *     4*H*(d_h + 4) per (item, split) pair of the largest 512-item chunk;
+ *     a request above SMEM_STATIC_SCRATCH_BYTES returns
+ *     SMEM_ERR_SCRATCH_LIMIT before anything is enqueued.
+ *   - The first call on each device looks up the array's device address
+ *     with that device current; make that first call before any stream
+ *     capture on the device.
+ *   - Every call on every cache of the process shares the one array, and it
+ *     keeps the last call's contents: each call first clears the counters it
+ *     needs at zero. Calls whose work overlaps on the GPU (different streams
+ *     without ordering) race on the array and give wrong results; order
+ *     them. */
+int smem_decode_static_scratch(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids,
+                               const int32_t *pos, const int32_t *q_block_idx, const void *qs,
+                               const void *k_new, const void *v_new, const void *qc, void *osa,
+                               void *oca, void *stream);
 
 /* Introspection for bit-exact bookkeeping checks (host state, no CUDA).
  * smem_get_table: the table of `seq` in ascending block index; up to `cap`

@@ -436,6 +436,105 @@ int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids
   return SMEM_OK;
 }
 
+int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,
+                               const int32_t* q_block_idx, const void* qs, const void* k_new, const void* v_new,
+                               const void* qc, void* osa, void* oca, void* stream) {
+  // Same validation as smem_decode; the split-K scratch comes from the
+  // library's fixed array instead of the cache's workspace.
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  const Layout& L = c->lay;
+  if (layer < 0 || layer >= L.L || nb < 1 || nb > L.max_batch) return SMEM_ERR_INVALID_ARG;
+  if (!seq_ids || !pos || !q_block_idx) return SMEM_ERR_INVALID_ARG;
+  const void* ptrs[6] = {qs, k_new, v_new, qc, osa, oca};
+  for (const void* p : ptrs) {
+    if (!p) return SMEM_ERR_INVALID_ARG;
+    if (!aligned16(p)) return SMEM_ERR_ALIGN;
+  }
+  if (++c->seen_epoch == 0) {
+    std::fill(c->seen.begin(), c->seen.end(), 0u);
+    c->seen_epoch = 1;
+  }
+  std::vector<int> nblk(nb);
+  for (int i = 0; i < nb; ++i) {
+    const int s = seq_ids[i];
+    if (s < 0 || s >= L.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
+    if (c->seen[s] == c->seen_epoch) return SMEM_ERR_INVALID_ARG;
+    c->seen[s] = c->seen_epoch;
+    if (pos[i] < 0 || pos[i] >= smem::kBlockTok || q_block_idx[i] < 0) return SMEM_ERR_INVALID_ARG;
+    const std::vector<int32_t>& ix = c->idx[s];
+    nblk[i] = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx[i]) - ix.begin());
+  }
+  // scratch layout per launch: [256 B scheduler words][tickets][partials]
+  const size_t ticket_bytes = align_up((size_t)std::min(nb, smem::kMaxDecodeItems) * L.H * 4, 256);
+  size_t need = 0;
+  for (int i0 = 0; i0 < nb; i0 += smem::kMaxDecodeItems) {
+    const int n = std::min(nb - i0, smem::kMaxDecodeItems);
+    size_t pairs = 0;
+    for (int i = 0; i < n; ++i)
+      if (nblk[i0 + i]) pairs += smem::ceil_div(nblk[i0 + i], smem::decode_split_blocks(nblk[i0 + i]));
+    need = std::max(need, 256 + ticket_bytes + pairs * L.H * (L.D + 4) * 4);
+  }
+  if (need > SMEM_STATIC_SCRATCH_BYTES) {
+    std::snprintf(g_detail, sizeof(g_detail), "decode needs %zu bytes of scratch, the fixed array holds %u", need,
+                  SMEM_STATIC_SCRATCH_BYTES);
+    return SMEM_ERR_SCRATCH_LIMIT;
+  }
+  DeviceGuard g(c->device);
+  void* scratch = nullptr;
+  const int se = smem::static_scratch_address(&scratch);
+  if (se != 0) return check_launch(c, (cudaError_t)se, "static scratch address");
+  uint8_t* sb = static_cast<uint8_t*>(scratch);
+  const size_t tok = (size_t)L.H * L.D;
+  static thread_local smem::DecodeParams P;
+  for (int i0 = 0; i0 < nb; i0 += smem::kMaxDecodeItems) {
+    const int n = std::min(nb - i0, smem::kMaxDecodeItems);
+    P.tmap = c->pool_map;
+    P.pool = reinterpret_cast<const uint16_t*>(c->dev + L.off_pool);
+    P.inblock = reinterpret_cast<uint16_t*>(c->dev + L.off_inblock);
+    P.table = reinterpret_cast<const int*>(c->dev + L.off_table);
+    P.null_kv = null_kv(c);
+    P.sched = reinterpret_cast<unsigned long long*>(sb);
+    P.counters = reinterpret_cast<unsigned*>(sb + 256);
+    P.part = reinterpret_cast<float*>(sb + 256 + ticket_bytes);
+    P.err = reinterpret_cast<int*>(c->dev + L.off_err);
+    P.qs = static_cast<const uint16_t*>(qs) + i0 * tok;
+    P.k_new = static_cast<const uint16_t*>(k_new) + i0 * tok;
+    P.v_new = static_cast<const uint16_t*>(v_new) + i0 * tok;
+    P.qc = static_cast<const uint16_t*>(qc) + i0 * tok;
+    P.osa = static_cast<uint16_t*>(osa) + i0 * tok;
+    P.oca = static_cast<uint16_t*>(oca) + i0 * tok;
+    P.slot_elems = (long long)L.slot_elems;
+    P.L = L.L;
+    P.H = L.H;
+    P.layer = layer;
+    P.max_blocks = L.max_blocks;
+    P.capacity = L.capacity;
+    P.n_items = n;
+    P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
+    int pairs = 0;
+    for (int i = 0; i < n; ++i) {
+      P.items[i].seq = seq_ids[i0 + i];
+      P.items[i].nblk = nblk[i0 + i];
+      P.items[i].pos = pos[i0 + i];
+      P.items[i].pair_begin = pairs;
+      if (nblk[i0 + i]) pairs += smem::ceil_div(nblk[i0 + i], smem::decode_split_blocks(nblk[i0 + i]));
+    }
+    P.n_pairs = pairs;
+    const long long units = (long long)(pairs + n) * L.H;
+    const long long wpc = smem::decode_warps_per_cta();
+    const int grid = (int)std::min<long long>((units + wpc - 1) / wpc, smem::decode_max_grid(L.D, c->num_sms));
+    if (injected_failure(c)) return SMEM_ERR_CUDA;
+    // the array keeps the previous call's contents: clear the scheduler
+    // words and tickets this launch needs at zero
+    int rc = check_launch(c, smem::launch_zero(sb, 256 + ticket_bytes, as_stream(stream)), "static scratch clear");
+    if (rc) return rc;
+    rc = check_launch(c, smem::launch_decode(P, L.D, grid, as_stream(stream)), "decode (static scratch)");
+    if (rc) return rc;
+  }
+  return SMEM_OK;
+}
+
 int smem_get_table(const smem_cache* c, int32_t seq, int32_t* idx_out, int32_t* slot_out, int32_t cap,
                    int32_t* n_out) {
   if (!c || !n_out || cap < 0) return SMEM_ERR_INVALID_ARG;
@@ -527,6 +626,7 @@ const char* smem_strerror(int code) {
     case SMEM_ERR_DEVICE_FAULT: return "device error recorded";
     case SMEM_ERR_UNSUPPORTED: return "unsupported shape";
     case SMEM_ERR_NO_DEVICE: return "bookkeeping-only cache";
+    case SMEM_ERR_SCRATCH_LIMIT: return "request exceeds the fixed scratch array";
     default: return "unknown error";
   }
 }

@@ -29,6 +29,9 @@
 
 #include <cmath>
 #include <cudaTypedefs.h>
+#include <mutex>
+
+#include "../../include/smem.h"
 
 #include "smem_device.cuh"
 #include "smem_internal.h"
@@ -546,6 +549,31 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       p.sched[1] = 0ull;
     }
   }
+}
+
+// Fixed scratch of smem_decode_static_scratch: split partials, tickets and
+// scheduler words for callers that cannot allocate. Host code sees only a
+// stand-in symbol; the device address comes from cudaGetSymbolAddress.
+static __device__ __align__(256) unsigned char g_decode_static_scratch[SMEM_STATIC_SCRATCH_BYTES];
+
+int static_scratch_address(void** out) {
+  constexpr int kMaxDevices = 64;
+  static std::mutex mu;
+  static void* addr[kMaxDevices] = {};
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return (int)e;
+  if (dev < 0 || dev >= kMaxDevices) return (int)cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_decode_static_scratch);  // this device is current
+    if (e != cudaSuccess) return (int)e;
+    if (!p) return (int)cudaErrorInvalidSymbol;
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return 0;
 }
 
 int decode_stage_rows(int D) { return D == 64 ? Dec<64>::SROWS : Dec<128>::SROWS; }

@@ -88,6 +88,9 @@ struct DecodeParams {
 };
 
 cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st);
+// Device address of the fixed scratch array of smem_decode_static_scratch on
+// the current device (looked up once per device). Returns a cudaError_t.
+int static_scratch_address(void** out);
 int decode_max_grid(int D, int num_sms);
 int decode_warps_per_cta();
 // Encodes the tensor map of the pool for the decode kernel (rows of D bf16,

@@ -28,11 +28,13 @@ ERR_CUDA = -8
 ERR_DEVICE_FAULT = -9
 ERR_UNSUPPORTED = -10
 ERR_NO_DEVICE = -11
+ERR_SCRATCH_LIMIT = -12
+STATIC_SCRATCH_BYTES = 16 << 20
 
 EXPORTED = [
     "smem_cache_required_bytes", "smem_cache_create", "smem_cache_destroy", "smem_set_null_row",
     "smem_append_block", "smem_delete_block", "smem_release_seq", "smem_write_inblock", "smem_prefill_block",
-    "smem_decode", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table", "smem_check_device_error",
+    "smem_decode", "smem_decode_static_scratch", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table", "smem_check_device_error",
     "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
 ]
 
@@ -82,6 +84,8 @@ def lib():
             "smem_write_inblock": (ctypes.c_int, [_vp, _i32, _i32, _i32, _vp, _vp, _vp]),
             "smem_prefill_block": (ctypes.c_int, [_vp, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
             "smem_decode": (ctypes.c_int, [_vp, _i32, _i32, _i32p, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
+            "smem_decode_static_scratch": (ctypes.c_int, [_vp, _i32, _i32, _i32p, _i32p, _i32p, _vp, _vp, _vp, _vp,
+                                                          _vp, _vp, _vp]),
             "smem_get_table": (ctypes.c_int, [_vp, _i32, _i32p, _i32p, _i32, _i32p]),
             "smem_get_free_fifo": (ctypes.c_int, [_vp, _i32p, _i32, _i32p]),
             "smem_get_device_table": (ctypes.c_int, [_vp, _i32, _i32p, _i32, _i32p, _vp]),
@@ -194,6 +198,16 @@ def smem_decode(h, layer, seq_ids, pos, q_block_idx, qs, k_new, v_new, qc, osa, 
     q, qp = _i32arr(q_block_idx)
     return _check(lib().smem_decode(h, layer, len(s), sp, pp, qp, _ptr(qs), _ptr(k_new), _ptr(v_new), _ptr(qc),
                                     _ptr(osa), _ptr(oca), _stream(stream)), "smem_decode")
+
+
+def smem_decode_static_scratch(h, layer, seq_ids, pos, q_block_idx, qs, k_new, v_new, qc, osa, oca, stream=None):
+    """smem_decode with the library's fixed scratch array (allocates nothing)."""
+    s, sp = _i32arr(seq_ids)
+    p, pp = _i32arr(pos)
+    q, qp = _i32arr(q_block_idx)
+    return _check(lib().smem_decode_static_scratch(h, layer, len(s), sp, pp, qp, _ptr(qs), _ptr(k_new), _ptr(v_new),
+                                                   _ptr(qc), _ptr(osa), _ptr(oca), _stream(stream)),
+                  "smem_decode_static_scratch")
 
 
 def smem_get_table(h, seq):
