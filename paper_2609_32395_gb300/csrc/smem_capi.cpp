@@ -24,7 +24,8 @@
 using smem::Layout;
 
 struct smem_cache {
-  CUtensorMap pool_map{};  // decode kernel's view of the pool (device caches)
+  CUtensorMap pool_map{};     // decode kernel's view of the pool (device caches)
+  CUtensorMap pool_map_pf{};  // prefill kernel's view (whole 64-row tiles)
   smem_config cfg{};
   Layout lay{};
   uint8_t* dev = nullptr;  // nullptr: bookkeeping-only
@@ -92,7 +93,7 @@ int make_layout(const smem_config* c, Layout* L) {
   L->off_dec_cnt = off;
   off = align_up(off + (size_t)L->max_batch * L->H * 4 + 64, A);  // + unit scheduler words
   L->off_pf_part = off;
-  off = align_up(off + (size_t)L->H * L->pf_max_splits * smem::kBlockTok * (D + 2) * 4, A);
+  off = align_up(off + (size_t)L->H * L->pf_max_splits * smem::kBlockTok * (D + 4) * 4, A);
   L->off_pf_cnt = off;
   off = align_up(off + (size_t)L->H * 4, A);
   L->off_err = off;
@@ -202,8 +203,10 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
       delete c;
       return SMEM_ERR_CUDA;
     }
-    const int er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity,
-                                         smem::decode_stage_rows(L.D));
+    int er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity,
+                                   smem::decode_stage_rows(L.D));
+    if (er == 0)
+      er = smem::encode_pool_map(&c->pool_map_pf, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity, smem::kRows);
     if (er != 0) {
       std::snprintf(g_detail, sizeof(g_detail), "tensor map encode failed (%d)", er);
       delete c;
@@ -334,6 +337,7 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
   const std::vector<int32_t>& ix = c->idx[seq];
   const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx) - ix.begin());
   smem::PrefillArgs a{};
+  a.pool_map = &c->pool_map_pf;
   a.pool = reinterpret_cast<const uint16_t*>(c->dev + c->lay.off_pool);
   a.table_row = table_row(c, seq);
   a.null_kv = null_kv(c);

@@ -119,12 +119,13 @@ cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st);
 // prefill
 // ---------------------------------------------------------------------------
 struct PrefillArgs {
+  const CUtensorMap* pool_map;  // pool viewed as [C][L*H*2*R][D], boxes of 64 columns x 64 rows
   const uint16_t* pool;
   const int* table_row;       // slots of this sequence, ascending block index
   const uint16_t* null_kv;    // [L][H][2][D] or nullptr
   const uint16_t *qs, *ks, *vs, *qc;  // [b][H][D]
   uint16_t *osa, *oca;
-  float* part;                // [H][pf_max_splits][b][D + 2]
+  float* part;                // [H][pf_max_splits][b][D + 4]: m, l, pad, pad, O[D]
   unsigned* counters;         // [H]
   int* err;
   long long slot_elems;

@@ -1,9 +1,476 @@
-// smem_prefill.cu -- one-block reader pass (placeholder until the tensor-core
-// kernel lands).
+// smem_prefill.cu -- one-block reader pass for one layer (block-skip serving).
+//
+// For the b = 64 query tokens of the final block (arXiv 2609.32395, Sec. 3.1
+// "Reuse": a fully cached context is served by running the reader on the
+// final block alone; Sec. 2 "Model" and App. A "Reader" for the attention):
+//   Osa[t] = softmax_{u<=t}(s Qs[t].Ks[u]) Vs        block-local causal SA
+//   Oca[t] = softmax_r(s Qc[t].k_r) v_r               block-causal CA
+// where r runs over the null row and the rows of every table block with index
+// below the query block, in ascending block index.
+//
+// The CA scores and P.V form a dense (64 x N.R) x (N.R x d_h) contraction, so
+// they run on the 5th-generation tensor cores: per CTA, one (head, split)
+// work unit. A producer warp streams the split's K and V tiles (64 rows x
+// d_h, 128-byte swizzle) into a ring with tensor TMA; an MMA warp issues
+// S = Q.K^T (M = 64 queries, N = 64 keys) into one of two TMEM buffers and
+// O += P.V (N = d_h, V read MN-major) into a TMEM accumulator; four softmax
+// warps read S rows from TMEM (row 16w + t%16, half t/16 of the keys), run a
+// base-2 online softmax, and write P as bf16 into a swizzled smem tile. The
+// running maximum is raised only when a row's maximum grows by more than 2^8
+// (then that row of O is rescaled in TMEM); otherwise the stale maximum keeps
+// every P <= 256, and O and l stay consistent with it. QK^T of tile j+1
+// overlaps the softmax of tile j. A split writes its partial (m, l, O) and the
+// CTA that completes the last split of a head merges all splits in split
+// order (null row first). The in-block SA is one masked tile per head on the
+// same machinery. Reduction orders depend only on the block count.
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
+#include <cmath>
+
+#include "smem_device.cuh"
 #include "smem_internal.h"
+#include "smem_tc.cuh"
 
 namespace smem {
-cudaError_t launch_prefill(const PrefillArgs&, cudaStream_t) { return cudaErrorNotSupported; }
+
+template <int D>
+struct Pf {
+  static constexpr int R = kRows;
+  static constexpr int B = kBlockTok;
+  static constexpr int BOXES = D / 64;            // 128-byte-wide column boxes
+  static constexpr int BOX = 64 * 128;            // one [64 rows][128 B] box
+  static constexpr int TILE = BOXES * BOX;        // K or V of one block and head
+  static constexpr int STAGE = 2 * TILE;
+  static constexpr int NS = D == 64 ? 4 : 3;
+  static constexpr int PBYTES = 64 * 64 * 2;      // P tile [64 queries][64 keys] bf16
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_RING = TILE;
+  static constexpr int OFF_P = OFF_RING + NS * STAGE;
+  static constexpr int OFF_BAR = OFF_P + 2 * PBYTES;
+  // barriers: q_full | full[NS] | empty[NS] | s_full[2] | s_free[2] | p_full[2] | o_done[2] | drain
+  static constexpr int NBARS = 1 + 2 * NS + 9;
+  static constexpr int OFF_MISC = OFF_BAR + NBARS * 8;
+  static constexpr int SMEM = OFF_MISC + 64 + 1024;
+  static constexpr int THREADS = 192;             // 4 softmax warps, producer, MMA
+  static constexpr uint32_t TMEM_COLS = 256;      // S0 | S1 | O
+  static constexpr uint32_t COL_O = 128;
+  static constexpr uint32_t ID_QK = tc::idesc_bf16(64, 64, 0, 0);
+  static constexpr uint32_t ID_PV = tc::idesc_bf16(64, D, 0, 1);
+};
+
+constexpr float kRescaleLog2 = 8.0f;  // raise the running max when it grows by more than 2^8
+
+struct PrefillParams {
+  CUtensorMap pool;          // [C][L*H*2*R][D], box 64 x 64 rows
+  CUtensorMap qs, ks, vs, qc;  // [b][H][D], box 64 x 1 x 64
+  const int* table_row;
+  const uint16_t* null_kv;
+  const uint16_t* qc_ptr;
+  uint16_t* osa;
+  uint16_t* oca;
+  float* part;
+  unsigned* counters;
+  int* err;
+  int L, H, layer, nblk, split_blks, n_splits, capacity, max_splits;
+  float scale_log2;
+};
+
+template <int D>
+__global__ void __launch_bounds__(Pf<D>::THREADS, 1) prefill_kernel(const __grid_constant__ PrefillParams p) {
+  using C = Pf<D>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint8_t* qt = base + C::OFF_Q;
+  uint8_t* ring = base + C::OFF_RING;
+  uint8_t* pt = base + C::OFF_P;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::OFF_BAR);
+  uint64_t* q_full = bars;
+  uint64_t* full = bars + 1;
+  uint64_t* empty = full + C::NS;
+  uint64_t* s_full = empty + C::NS;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* o_done = p_full + 2;
+  uint64_t* drain = o_done + 2;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(base + C::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::OFF_MISC + 4);
+  volatile unsigned* ticket = reinterpret_cast<volatile unsigned*>(base + C::OFF_MISC + 8);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int n_ca = p.n_splits * p.H;
+  const bool sa = (int)blockIdx.x >= n_ca;
+  const int h = sa ? (int)blockIdx.x - n_ca : (int)blockIdx.x % p.H;
+  const int split = sa ? 0 : (int)blockIdx.x / p.H;
+  const int b0 = split * p.split_blks;
+  const int nt = sa ? 1 : min(p.split_blks, p.nblk - b0);
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < C::NS; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_free[b], 4);
+      mbar_init(&p_full[b], 4);
+      mbar_init(&o_done[b], 1);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 4) tc::alloc(tslot, C::TMEM_COLS);
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = *tslot;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      const CUtensorMap* qmap = sa ? &p.qs : &p.qc;
+      mbar_arrive_expect_tx(q_full, C::TILE);
+#pragma unroll
+      for (int bx = 0; bx < C::BOXES; ++bx) tc::tma_load_3d(qt + bx * C::BOX, qmap, bx * 64, h, 0, q_full);
+      int issued = 0;
+      for (int j = 0; j < nt; ++j) {
+        const int st = j % C::NS;
+        if (j >= C::NS && !mbar_wait_bounded(&empty[st], ((j / C::NS) - 1) & 1, abort_flag)) {
+          if (!*abort_flag) record_error(p.err, kDevErrWaitEmpty);
+          *abort_flag = 1;
+          break;
+        }
+        uint8_t* kd = ring + st * C::STAGE;
+        uint8_t* vd = kd + C::TILE;
+        if (sa) {
+          mbar_arrive_expect_tx(&full[st], C::STAGE);
+#pragma unroll
+          for (int bx = 0; bx < C::BOXES; ++bx) {
+            tc::tma_load_3d(kd + bx * C::BOX, &p.ks, bx * 64, h, 0, &full[st]);
+            tc::tma_load_3d(vd + bx * C::BOX, &p.vs, bx * 64, h, 0, &full[st]);
+          }
+        } else {
+          const int slot = p.table_row[b0 + j];
+          if (slot < 0 || slot >= p.capacity) {
+            record_error(p.err, kDevErrBounds);
+            mbar_arrive(&full[st]);
+          } else {
+            mbar_arrive_expect_tx(&full[st], C::STAGE);
+            const int y = ((p.layer * p.H + h) * 2) * C::R;
+#pragma unroll
+            for (int bx = 0; bx < C::BOXES; ++bx) {
+              tc::tma_load_3d(kd + bx * C::BOX, &p.pool, bx * 64, y, slot, &full[st]);
+              tc::tma_load_3d(vd + bx * C::BOX, &p.pool, bx * 64, y + C::R, slot, &full[st]);
+            }
+          }
+        }
+        ++issued;
+      }
+      if (*abort_flag) {
+        mbar_wait_bounded(q_full, 0, nullptr);
+        for (int j = 0; j < issued; ++j) mbar_wait_bounded(&full[j % C::NS], (j / C::NS) & 1, nullptr);
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait_bounded(q_full, 0, abort_flag);
+      tc::fence_after();
+      const uint32_t qa = smem_u32(qt);
+      for (int jj = 0; ok && jj <= nt; ++jj) {
+        if (jj < nt) {  // S[jj%2] = Q . K^T
+          const int st = jj % C::NS, sb = jj & 1;
+          ok = mbar_wait_bounded(&full[st], (jj / C::NS) & 1, abort_flag);
+          if (ok && jj >= 2) ok = mbar_wait_bounded(&s_free[sb], ((jj >> 1) - 1) & 1, abort_flag);
+          if (!ok) break;
+          tc::fence_after();
+          const uint32_t ka = smem_u32(ring + st * C::STAGE);
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) {
+            const uint32_t off = (k >> 2) * C::BOX + (k & 3) * 32;
+            tc::mma_bf16(tmem + 64 * sb, tc::sdesc_sw128(qa + off, 16, 1024), tc::sdesc_sw128(ka + off, 16, 1024),
+                         C::ID_QK, k > 0);
+          }
+          tc::commit(&s_full[sb]);
+        }
+        if (jj >= 1) {  // O += P . V for tile jj-1
+          const int j = jj - 1, st = j % C::NS, pb = j & 1;
+          ok = mbar_wait_bounded(&p_full[pb], (j >> 1) & 1, abort_flag);
+          if (!ok) break;
+          tc::fence_after();
+          const uint32_t pa = smem_u32(pt + pb * C::PBYTES);
+          const uint32_t va = smem_u32(ring + st * C::STAGE + C::TILE);
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024),
+                         tc::sdesc_sw128(va + k * 2048, C::BOX, 1024), C::ID_PV, (j > 0 || k > 0));
+          tc::commit(&empty[st]);
+          tc::commit(&o_done[pb]);
+        }
+      }
+      if (!ok) {
+        if (!*abort_flag) record_error(p.err, kDevErrWaitMma);
+        *abort_flag = 1;
+      }
+      // all issued MMAs complete before the CTA can release TMEM
+      tc::commit(drain);
+      mbar_wait_bounded(drain, 0, nullptr);
+    }
+  } else {
+    // ---------------------------------------------------------- softmax warps
+    const int r = 16 * warp + (lane & 15);  // query row
+    const int hf = lane >> 4;               // key half of the S tile
+    const uint32_t trow = tmem + ((uint32_t)(32 * warp) << 16);
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nt && ok; ++j) {
+      const int sb = j & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait_bounded(&s_full[sb], (j >> 1) & 1, abort_flag));
+      if (!ok) break;
+      tc::fence_after();
+      uint32_t sr[32];
+      tc::ld_16x32bx2_x32<32>(trow + 64 * sb, sr);
+      tc::wait_ld();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);
+      float x[32];
+      float tmax = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 32; ++c) {
+        const int u = hf * 32 + c;
+        x[c] = (!sa || u <= r) ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
+        tmax = fmaxf(tmax, x[c]);
+      }
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
+      const float m_new = fmaxf(m_used, tmax);
+      const bool need = m_new > m_used + kRescaleLog2;
+      if (j > 0 && __any_sync(0xffffffffu, need)) {
+        // rescale this warp's rows of O once the previous P.V has landed
+        ok = __all_sync(0xffffffffu, mbar_wait_bounded(&o_done[(j - 1) & 1], ((j - 1) >> 1) & 1, abort_flag));
+        if (!ok) break;
+        tc::fence_after();
+        const float alpha = need ? exp2f(m_used - m_new) : 1.f;
+#pragma unroll
+        for (int cb = 0; cb < D / 64; ++cb) {
+          uint32_t o[32];
+          tc::ld_16x32bx2_x32<D / 2>(trow + C::COL_O + 32 * cb, o);
+          tc::wait_ld();
+#pragma unroll
+          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+          tc::st_16x32bx2_x32<D / 2>(trow + C::COL_O + 32 * cb, o);
+        }
+        tc::wait_st();
+      }
+      if (need) {
+        l *= exp2f(m_used - m_new);
+        m_used = m_new;
+      }
+      uint32_t pk[16];
+#pragma unroll
+      for (int c = 0; c < 32; c += 2) {
+        const float p0 = exp2f(x[c] - m_used), p1 = exp2f(x[c + 1] - m_used);
+        l += p0 + p1;
+        pk[c >> 1] = pack_bf16x2(p0, p1);
+      }
+      // P buffer sb was last read by P.V of tile j-2
+      if (j >= 2) {
+        ok = __all_sync(0xffffffffu, mbar_wait_bounded(&o_done[sb], ((j - 2) >> 1) & 1, abort_flag));
+        if (!ok) break;
+      }
+      uint8_t* prow = pt + sb * C::PBYTES + r * 128;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int chunk = hf * 4 + q;
+        *reinterpret_cast<uint4*>(prow + ((chunk ^ (r & 7)) << 4)) =
+            make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+      }
+      fence_proxy_async_smem();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[sb]);
+    }
+    if (!ok) {
+      if (lane == 0 && !*abort_flag) record_error(p.err, kDevErrWaitFull);
+      *abort_flag = 1;
+    }
+    // ---------------------------------------------------------- epilogue
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait_bounded(&o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, abort_flag));
+    float o[D / 2];
+    if (ok) {
+      tc::fence_after();
+#pragma unroll
+      for (int cb = 0; cb < D / 64; ++cb) {
+        uint32_t t[32];
+        tc::ld_16x32bx2_x32<D / 2>(trow + C::COL_O + 32 * cb, t);
+        tc::wait_ld();
+#pragma unroll
+        for (int c = 0; c < 32; ++c) o[cb * 32 + c] = __uint_as_float(t[c]);
+      }
+    }
+    const float lrow = l + __shfl_xor_sync(0xffffffffu, l, 16);
+    const int col0 = hf * (D / 2);  // this thread's columns of O
+    const bool direct = sa || (p.n_splits == 1 && !p.null_kv);
+    if (ok && direct) {
+      uint16_t* out = (sa ? p.osa : p.oca) + ((size_t)r * p.H + h) * D + col0;
+      const float inv = 1.f / lrow;
+#pragma unroll
+      for (int c = 0; c < D / 2; c += 8) {
+        uint4 w;
+        w.x = pack_bf16x2(o[c] * inv, o[c + 1] * inv);
+        w.y = pack_bf16x2(o[c + 2] * inv, o[c + 3] * inv);
+        w.z = pack_bf16x2(o[c + 4] * inv, o[c + 5] * inv);
+        w.w = pack_bf16x2(o[c + 6] * inv, o[c + 7] * inv);
+        *reinterpret_cast<uint4*>(out + c) = w;
+      }
+    }
+    if (ok && sa && p.nblk == 0) {
+      // no readable memory block: oca is the null row's value or zero
+      uint16_t* out = p.oca + ((size_t)r * p.H + h) * D + col0;
+      const uint16_t* vn = p.null_kv ? p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D + D + col0 : nullptr;
+#pragma unroll
+      for (int c = 0; c < D / 2; c += 8)
+        *reinterpret_cast<uint4*>(out + c) = vn ? *reinterpret_cast<const uint4*>(vn + c) : make_uint4(0, 0, 0, 0);
+    }
+    if (ok && !direct) {
+      float* pp = p.part + (((size_t)h * p.max_splits + split) * C::B + r) * (D + 4);
+#pragma unroll
+      for (int c = 0; c < D / 2; c += 4)
+        *reinterpret_cast<float4*>(pp + 4 + col0 + c) = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+      if (hf == 0) {
+        pp[0] = m_used;
+        pp[1] = lrow;
+      }
+      __threadfence();
+    }
+    // the four softmax warps agree on the outcome before the ticket
+    const bool all_ok = bar_all(1, 128, ok);
+    if (all_ok && !direct) {
+      if (threadIdx.x == 0) *ticket = atomicAdd(&p.counters[h], 1u);
+      named_bar_sync(1, 128);
+      if (*ticket == (unsigned)(p.n_splits - 1)) {
+        __threadfence();
+        // merge all splits of this head for row r, columns col0.., in split order
+        const size_t qoff = ((size_t)r * p.H + h) * D;
+        float nscore = -INFINITY;
+        if (p.null_kv) {
+          const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
+          float dot = 0.f;
+          for (int c = 0; c < D / 2; ++c)
+            dot = fmaf(bf16lo(p.qc_ptr[qoff + col0 + c]), bf16lo(kn[col0 + c]), dot);
+          dot += __shfl_xor_sync(0xffffffffu, dot, 16);
+          nscore = dot * p.scale_log2;
+        }
+        const float* pb = p.part + ((size_t)h * p.max_splits * C::B + r) * (D + 4);
+        const size_t ps = (size_t)C::B * (D + 4);
+        float M = nscore;
+        for (int s2 = 0; s2 < p.n_splits; ++s2) M = fmaxf(M, __ldcg(pb + s2 * ps));
+        float Lsum = 0.f, A[D / 2];
+#pragma unroll
+        for (int c = 0; c < D / 2; ++c) A[c] = 0.f;
+        if (p.null_kv) {
+          const float f = exp2f(nscore - M);
+          Lsum = f;
+          const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D + D + col0;
+#pragma unroll
+          for (int c = 0; c < D / 2; ++c) A[c] = f * bf16lo(vn[c]);
+        }
+        for (int s2 = 0; s2 < p.n_splits; ++s2) {
+          const float* ps2 = pb + s2 * ps;
+          const float f = exp2f(__ldcg(ps2) - M);
+          Lsum = fmaf(f, __ldcg(ps2 + 1), Lsum);
+#pragma unroll
+          for (int c = 0; c < D / 2; c += 4) {
+            const float4 v = __ldcg(reinterpret_cast<const float4*>(ps2 + 4 + col0 + c));
+            A[c] = fmaf(f, v.x, A[c]);
+            A[c + 1] = fmaf(f, v.y, A[c + 1]);
+            A[c + 2] = fmaf(f, v.z, A[c + 2]);
+            A[c + 3] = fmaf(f, v.w, A[c + 3]);
+          }
+        }
+        const float inv = 1.f / Lsum;
+        uint16_t* out = p.oca + qoff + col0;
+#pragma unroll
+        for (int c = 0; c < D / 2; c += 8) {
+          uint4 w;
+          w.x = pack_bf16x2(A[c] * inv, A[c + 1] * inv);
+          w.y = pack_bf16x2(A[c + 2] * inv, A[c + 3] * inv);
+          w.z = pack_bf16x2(A[c + 4] * inv, A[c + 5] * inv);
+          w.w = pack_bf16x2(A[c + 6] * inv, A[c + 7] * inv);
+          *reinterpret_cast<uint4*>(out + c) = w;
+        }
+        if (threadIdx.x == 0) p.counters[h] = 0u;
+      }
+    }
+  }
+  tc::fence_before();
+  __syncthreads();
+  if (warp == 4) {
+    tc::fence_after();
+    tc::dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int D>
+static cudaError_t launch_prefill_d(const PrefillParams& p, int grid, cudaStream_t st) {
+  using C = Pf<D>;
+  cudaError_t e = cudaFuncSetAttribute(prefill_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  prefill_kernel<D><<<grid, C::THREADS, C::SMEM, st>>>(p);
+  return cudaGetLastError();
+}
+
+static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  if (!encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return -1;
+    encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)kBlockTok};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2};
+  const cuuint32_t box[3] = {64, 1, (cuuint32_t)kBlockTok};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
+                            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : (int)r;
+}
+
+cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
+  static thread_local PrefillParams P;
+  P.pool = *a.pool_map;
+  if (encode_bhd(&P.qs, a.qs, a.H, a.D) || encode_bhd(&P.ks, a.ks, a.H, a.D) || encode_bhd(&P.vs, a.vs, a.H, a.D) ||
+      encode_bhd(&P.qc, a.qc, a.H, a.D))
+    return cudaErrorInvalidValue;
+  P.table_row = a.table_row;
+  P.null_kv = a.null_kv;
+  P.qc_ptr = a.qc;
+  P.osa = a.osa;
+  P.oca = a.oca;
+  P.part = a.part;
+  P.counters = a.counters;
+  P.err = a.err;
+  P.L = a.L;
+  P.H = a.H;
+  P.layer = a.layer;
+  P.nblk = a.nblk;
+  P.split_blks = a.split_blks;
+  P.n_splits = a.n_splits;
+  P.capacity = a.capacity;
+  P.max_splits = kPrefillMaxSplits;
+  P.scale_log2 = a.scale_log2;
+  const int grid = a.n_splits * a.H + a.H;
+  if (a.D == 64) return launch_prefill_d<64>(P, grid, st);
+  if (a.D == 128) return launch_prefill_d<128>(P, grid, st);
+  return cudaErrorInvalidValue;
+}
+
 }  // namespace smem

@@ -107,6 +107,25 @@ class DeviceCache:
             return None, None
         return f64(self.k_null[layer]), f64(self.v_null[layer])
 
+    # -------------------------------------------------------------- prefill
+    def prefill_inputs(self, layer, tag=0):
+        shape = (B_TOK, self.H, self.D)
+        return [synth.tensor_np(self.seed, k, shape, layer, tag)
+                for k in (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+
+    def prefill(self, seq, layer, q_idx, tag=0):
+        qs, ks, vs, qc = self.prefill_inputs(layer, tag)
+        osa = torch.empty((B_TOK, self.H, self.D), dtype=torch.bfloat16, device="cuda")
+        oca = torch.empty_like(osa)
+        smem.smem_prefill_block(self.h, seq, layer, q_idx, to_dev(qs), to_dev(ks), to_dev(vs), to_dev(qc), osa, oca)
+        torch.cuda.synchronize()
+        return (qs, ks, vs, qc), osa, oca
+
+    def oracle_prefill(self, seq, layer, q_idx, qs, ks, vs, qc):
+        idx, mk, mv = self.oracle_memory(seq, layer)
+        kn0, vn0 = self.null(layer)
+        return oracle.reader_prefill(idx, mk, mv, q_idx, f64(qs), f64(ks), f64(vs), f64(qc), kn0, vn0)
+
     # -------------------------------------------------------------- decode
     def decode_inputs(self, nb, layer, step):
         H, D = self.H, self.D
