@@ -44,6 +44,9 @@ def parse_args():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-serve", action="store_true")
+    ap.add_argument("--only-serve", action="store_true",
+                    help="time only the one-block cached-serve cells (profiling)")
     ap.add_argument("--seqs", type=int, default=WORKLOAD["seqs"])
     ap.add_argument("--layers", type=int, default=WORKLOAD["L"],
                     help="fewer layers: same per-launch work, smaller pool (profiling captures)")
@@ -265,6 +268,110 @@ class DecodeWorkload:
         return launches
 
 
+# ----------------------------------------------------------------------------- prefill workload
+SERVE = dict(name="160M-shaped one-block cached-context prefill", L=12, H=12, D=64, contexts=(16, 64, 256), seed=1)
+
+
+class PrefillWorkload:
+    """A fully cached context of `nblk` memory blocks (160M reader shape,
+    shuffled slots) served by running the reader's attention on the final
+    block alone: 12 one-block prefill launches, one per layer."""
+
+    def __init__(self, nblk, device, L=None, H=None, D=None, seed=None):
+        import torch
+
+        import synth
+        from paper_2609_32395_gb300 import smem
+
+        self.L = L or SERVE["L"]
+        self.H = H or SERVE["H"]
+        self.D = D or SERVE["D"]
+        self.nblk = nblk
+        seed = SERVE["seed"] if seed is None else seed
+        cap = nblk + 2
+        self.cfg = smem.make_config(self.L, self.H, self.D, 1, nblk + 1, cap,
+                                    free_order=synth.slot_permutation(seed + nblk, cap))
+        self.cache = smem.SmemCache(self.cfg, device=device)
+        self.h = self.cache.h
+        for b0 in range(0, nblk, 16):
+            ids = list(range(b0, min(nblk, b0 + 16)))
+            K, V = synth.block_rows_torch(seed, 0, ids, self.L, self.H, R, self.D, device)
+            for i, j in enumerate(ids):
+                smem.smem_append_block(self.h, 0, j, K[i], V[i])
+        shape = (B_TOK, self.H, self.D)
+        self.inputs = [[synth.tensor_torch(seed, k, shape, layer, 0, device=device)
+                        for k in (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+                       for layer in range(self.L)]
+        self.outputs = [(torch.empty(shape, dtype=torch.bfloat16, device=device),
+                         torch.empty(shape, dtype=torch.bfloat16, device=device)) for _ in range(self.L)]
+        torch.cuda.synchronize()
+
+    def layer(self, layer):
+        from paper_2609_32395_gb300 import smem
+
+        qs, ks, vs, qc = self.inputs[layer]
+        osa, oca = self.outputs[layer]
+        smem.smem_prefill_block(self.h, 0, layer, self.nblk, qs, ks, vs, qc, osa, oca)
+
+    def serve(self):
+        for layer in range(self.L):
+            self.layer(layer)
+
+    def bytes_per_launch(self):
+        # K/V of every memory row read (4*H*d_h bytes per row) + Qs, Ks, Vs, Qc read and Osa, Oca written
+        return self.nblk * R * 4 * self.H * self.D + 6 * B_TOK * self.H * self.D * 2
+
+    def flops_per_launch(self):
+        # CA: QK^T and P.V over all memory rows; SA: the causal half of the 64 x 64 block
+        ca = 4 * B_TOK * self.nblk * R * self.H * self.D
+        sa = 4 * (B_TOK * (B_TOK + 1) // 2) * self.H * self.D
+        return ca + sa
+
+
+def measure_serve(nblk, device, iters=30, flush_bytes=512 << 20):
+    """Latency of one cached-context serve (12 layers) replayed from a CUDA
+    graph, and the mean duration of one prefill launch; L2 is flushed before
+    each timed iteration (the flush also keeps the stream busy while the
+    timed work is enqueued)."""
+    import torch
+
+    wl = PrefillWorkload(nblk, device)
+    flush = torch.empty(flush_bytes, dtype=torch.uint8, device=device)
+    st = torch.cuda.current_stream()
+    for _ in range(3):
+        wl.serve()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        wl.serve()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(iters)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(iters)]
+    k0 = [torch.cuda.Event(enable_timing=True) for _ in range(iters)]
+    k1 = [torch.cuda.Event(enable_timing=True) for _ in range(iters)]
+    for i in range(iters):
+        flush.zero_()
+        e0[i].record(st)
+        g.replay()
+        e1[i].record(st)
+    for i in range(iters):
+        flush.zero_()
+        k0[i].record(st)
+        wl.layer(i % wl.L)
+        k1[i].record(st)
+    torch.cuda.synchronize()
+    serve_ms = sorted(a.elapsed_time(b) for a, b in zip(e0, e1))
+    kern_ms = [a.elapsed_time(b) for a, b in zip(k0, k1)]
+    del g
+    out = {"context_blocks": nblk, "memory_rows": nblk * R, "latency_ms": serve_ms[len(serve_ms) // 2],
+           "latency_ms_min": serve_ms[0], "kernel_ms_mean": float(np.mean(kern_ms)),
+           "bytes_per_launch": wl.bytes_per_launch(), "flops_per_launch": wl.flops_per_launch()}
+    wl.cache.close()
+    return out
+
+
 # ----------------------------------------------------------------------------- oracle (cpu) timing
 class OracleDecodeSample:
     """A bounded sample of the default workload for the fp64 CPU oracle: the
@@ -449,6 +556,15 @@ def run_ours(args):
     if err != smem.OK:
         raise RuntimeError("device error recorded during the benchmark")
 
+    # --- one-block cached-context serve (prefill), the metric's second half
+    serve = None
+    if not args.no_serve:
+        wl.cache.close()
+        wl.cache.buf = None
+        del wl.new_K, wl.new_V
+        torch.cuda.empty_cache()
+        serve = [measure_serve(n, device) for n in SERVE["contexts"]]
+
     if rank != 0:
         if ws > 1:
             import torch.distributed as dist
@@ -479,6 +595,18 @@ def run_ours(args):
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
+    if serve:
+        bf16_peak = float(peaks.get("bf16_tflops", 1900.0))
+        for sv in serve:
+            gbs = sv["bytes_per_launch"] / (sv["kernel_ms_mean"] / 1e3) / 1e9
+            tfs = sv["flops_per_launch"] / (sv["kernel_ms_mean"] / 1e3) / 1e12
+            sv["roofline"] = {"bound": "hbm", "achieved_gbs": gbs, "hbm_frac": gbs / peak,
+                              "achieved_tflops": tfs, "tensor_frac": tfs / bf16_peak,
+                              "peak_tflops_bf16": bf16_peak}
+        line["serve"] = {"workload": SERVE["name"], "layers": SERVE["L"], "heads": SERVE["H"],
+                         "head_dim": SERVE["D"], "metric": "one-block cached-serve latency (12 layers)",
+                         "unit": "ms", "timing": "CUDA graph of the 12 per-layer launches, L2 flushed before each",
+                         "cells": serve}
     if e2e:
         line["e2e"] = e2e
     if cpu:
@@ -490,8 +618,22 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_serve_only(args):
+    import torch
+
+    from paper_2609_32395_gb300 import smem
+
+    torch.cuda.set_device(0)
+    smem.lib()
+    cells = [measure_serve(n, torch.device("cuda", 0)) for n in SERVE["contexts"]]
+    print(json.dumps({"serve_only": True, "workload": SERVE["name"], "cells": cells}), flush=True)
+
+
 def main():
     args = parse_args()
+    if args.only_serve:
+        run_serve_only(args)
+        return
     if args.impl == "reference":
         run_reference(args)
     else:

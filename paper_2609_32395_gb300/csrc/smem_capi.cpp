@@ -356,7 +356,7 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
   a.D = c->lay.D;
   a.layer = layer;
   a.nblk = nblk;
-  a.split_blks = nblk ? smem::prefill_split_blocks(nblk, c->lay.H) : 1;
+  a.split_blks = nblk ? smem::prefill_split_blocks(nblk, c->lay.H, c->lay.D) : 1;
   a.n_splits = nblk ? smem::ceil_div(nblk, a.split_blks) : 0;
   a.capacity = c->lay.capacity;
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->lay.D));

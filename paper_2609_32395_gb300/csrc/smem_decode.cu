@@ -608,12 +608,12 @@ int decode_warps_per_cta() { return Dec<64>::NW; }
 cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st) {
   if (D == 64) {
     using C = Dec<64>;
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e = ensure_smem_limit<64>(decode_kernel<64>, C::SMEM);
     if (e != cudaSuccess) return e;
     decode_kernel<64><<<grid, C::THREADS, C::SMEM, st>>>(p);
   } else if (D == 128) {
     using C = Dec<128>;
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e = ensure_smem_limit<128>(decode_kernel<128>, C::SMEM);
     if (e != cudaSuccess) return e;
     decode_kernel<128><<<grid, C::THREADS, C::SMEM, st>>>(p);
   } else {

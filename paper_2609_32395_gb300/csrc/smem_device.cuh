@@ -5,10 +5,28 @@
 // named barriers, and the device error word.
 #pragma once
 
-#include <cstdint>
 #include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
 
 namespace smem {
+
+// Raises a kernel's dynamic shared-memory limit once per device (a launch
+// that may run under stream capture then makes no attribute call). `Tag`
+// keeps one record per kernel.
+template <int Tag, typename Kernel>
+inline cudaError_t ensure_smem_limit(Kernel kernel, int bytes) {
+  static unsigned long long done = 0;  // bit d: device d configured
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (__atomic_load_n(&done, __ATOMIC_ACQUIRE) & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) __atomic_fetch_or(&done, bit, __ATOMIC_RELEASE);
+  return e;
+}
 
 // Codes a kernel stores in the device error word (first writer wins).
 enum DeviceError : int {

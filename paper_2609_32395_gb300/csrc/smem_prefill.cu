@@ -54,6 +54,7 @@ struct Pf {
   static constexpr int OFF_MISC = OFF_BAR + NBARS * 8;
   static constexpr int SMEM = OFF_MISC + 64 + 1024;
   static constexpr int THREADS = 192;             // 4 softmax warps, producer, MMA
+  static constexpr int MIN_CTAS = D == 64 ? 2 : 1; // resident CTAs per SM (smem and TMEM allow it)
   static constexpr uint32_t TMEM_COLS = 256;      // S0 | S1 | O
   static constexpr uint32_t COL_O = 128;
   static constexpr uint32_t ID_QK = tc::idesc_bf16(64, 64, 0, 0);
@@ -78,7 +79,7 @@ struct PrefillParams {
 };
 
 template <int D>
-__global__ void __launch_bounds__(Pf<D>::THREADS, 1) prefill_kernel(const __grid_constant__ PrefillParams p) {
+__global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kernel(const __grid_constant__ PrefillParams p) {
   using C = Pf<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -367,8 +368,18 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, 1) prefill_kernel(const __grid
         }
         const float* pb = p.part + ((size_t)h * p.max_splits * C::B + r) * (D + 4);
         const size_t ps = (size_t)C::B * (D + 4);
+        const int ns = p.n_splits;
+        // every split's (m, l) in one batch of independent loads
+        float ms[kPrefillMaxSplits], ls[kPrefillMaxSplits];
+#pragma unroll
+        for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) {
+          const float2 v = s2 < ns ? __ldcg(reinterpret_cast<const float2*>(pb + s2 * ps)) : make_float2(-INFINITY, 0.f);
+          ms[s2] = v.x;
+          ls[s2] = v.y;
+        }
         float M = nscore;
-        for (int s2 = 0; s2 < p.n_splits; ++s2) M = fmaxf(M, __ldcg(pb + s2 * ps));
+#pragma unroll
+        for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) M = fmaxf(M, ms[s2]);
         float Lsum = 0.f, A[D / 2];
 #pragma unroll
         for (int c = 0; c < D / 2; ++c) A[c] = 0.f;
@@ -379,17 +390,32 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, 1) prefill_kernel(const __grid
 #pragma unroll
           for (int c = 0; c < D / 2; ++c) A[c] = f * bf16lo(vn[c]);
         }
-        for (int s2 = 0; s2 < p.n_splits; ++s2) {
-          const float* ps2 = pb + s2 * ps;
-          const float f = exp2f(__ldcg(ps2) - M);
-          Lsum = fmaf(f, __ldcg(ps2 + 1), Lsum);
+        // O of GROUP splits loaded before any is used; summed in split order
+        constexpr int GROUP = D == 64 ? 4 : 2;
+        for (int s0 = 0; s0 < ns; s0 += GROUP) {
+          float4 buf[GROUP][D / 8];
 #pragma unroll
-          for (int c = 0; c < D / 2; c += 4) {
-            const float4 v = __ldcg(reinterpret_cast<const float4*>(ps2 + 4 + col0 + c));
-            A[c] = fmaf(f, v.x, A[c]);
-            A[c + 1] = fmaf(f, v.y, A[c + 1]);
-            A[c + 2] = fmaf(f, v.z, A[c + 2]);
-            A[c + 3] = fmaf(f, v.w, A[c + 3]);
+          for (int g2 = 0; g2 < GROUP; ++g2)
+#pragma unroll
+            for (int c = 0; c < D / 8; ++c)
+              buf[g2][c] = s0 + g2 < ns ? __ldcg(reinterpret_cast<const float4*>(pb + (s0 + g2) * ps + 4 + col0) + c)
+                                        : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int g2 = 0; g2 < GROUP; ++g2) {
+            if (s0 + g2 >= ns) break;
+            float f = 0.f, msg = 0.f, lsg = 0.f;
+#pragma unroll
+            for (int t2 = 0; t2 < kPrefillMaxSplits; ++t2)
+              if (t2 == s0 + g2) { msg = ms[t2]; lsg = ls[t2]; }
+            f = exp2f(msg - M);
+            Lsum = fmaf(f, lsg, Lsum);
+#pragma unroll
+            for (int c = 0; c < D / 8; ++c) {
+              A[4 * c] = fmaf(f, buf[g2][c].x, A[4 * c]);
+              A[4 * c + 1] = fmaf(f, buf[g2][c].y, A[4 * c + 1]);
+              A[4 * c + 2] = fmaf(f, buf[g2][c].z, A[4 * c + 2]);
+              A[4 * c + 3] = fmaf(f, buf[g2][c].w, A[4 * c + 3]);
+            }
           }
         }
         const float inv = 1.f / Lsum;
@@ -418,7 +444,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, 1) prefill_kernel(const __grid
 template <int D>
 static cudaError_t launch_prefill_d(const PrefillParams& p, int grid, cudaStream_t st) {
   using C = Pf<D>;
-  cudaError_t e = cudaFuncSetAttribute(prefill_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  cudaError_t e = ensure_smem_limit<1000 + D>(prefill_kernel<D>, C::SMEM);
   if (e != cudaSuccess) return e;
   prefill_kernel<D><<<grid, C::THREADS, C::SMEM, st>>>(p);
   return cudaGetLastError();
