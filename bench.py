@@ -45,6 +45,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-serve", action="store_true")
+    ap.add_argument("--workload", default="decode", choices=["decode", "long"],
+                    help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
     ap.add_argument("--only-serve", action="store_true",
                     help="time only the one-block cached-serve cells (profiling)")
     ap.add_argument("--seqs", type=int, default=WORKLOAD["seqs"])
@@ -372,6 +374,140 @@ def measure_serve(nblk, device, iters=30, flush_bytes=512 << 20):
     return out
 
 
+# ----------------------------------------------------------------------------- long-context workload
+LONG = dict(name="1.5B-shaped long cached context", L=24, H=16, D=128, contexts=(512, 1024, 4096), batches=(1, 16),
+            seed=2)
+
+
+def run_long(args):
+    """One-block prefill latency and decode tok/s per context length at the
+    1.5B reader shape. Each batch builds one cache at the longest context;
+    shorter contexts read its block prefix (block-causal mask). Layers that
+    do not fit in HBM are emulated: the 24 logical layers cycle over the
+    physical layers that fit (per-layer working set >> L2)."""
+    import torch
+
+    import synth
+    from paper_2609_32395_gb300 import smem
+
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    smem.lib()
+    W = LONG
+    H, D, L = W["H"], W["D"], W["L"]
+    nmax = max(W["contexts"])
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    bf16_peak = float(peaks.get("bf16_tflops", 1900.0))
+    block_bytes = 2 * H * R * D * 2  # K and V of one layer
+    cells = []
+    for batch in W["batches"]:
+        free, _ = torch.cuda.mem_get_info()
+        budget = free - (16 << 30)
+        l_phys = max(2, min(L, budget // (batch * (nmax + 8) * block_bytes)))
+        cap = batch * (nmax + 4)
+        cfg = smem.make_config(int(l_phys), H, D, batch, nmax + 4, cap,
+                               free_order=synth.slot_permutation(W["seed"] + batch, cap))
+        cache = smem.SmemCache(cfg, device=device)
+        for s in range(batch):
+            for b0 in range(0, nmax, 16):
+                ids = list(range(b0, min(nmax, b0 + 16)))
+                K, V = synth.block_rows_torch(W["seed"], s, ids, int(l_phys), H, R, D, device)
+                for i, j in enumerate(ids):
+                    smem.smem_append_block(cache.h, s, j, K[i], V[i])
+                del K, V
+        shape = (batch, H, D)
+        dins = [synth.tensor_torch(W["seed"], k, shape, 0, 0, device=device)
+                for k in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
+        osa = torch.empty(shape, dtype=torch.bfloat16, device=device)
+        oca = torch.empty_like(osa)
+        pshape = (B_TOK, H, D)
+        pins = [synth.tensor_torch(W["seed"], k, pshape, 0, 0, device=device)
+                for k in (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+        posa = torch.empty(pshape, dtype=torch.bfloat16, device=device)
+        poca = torch.empty_like(posa)
+        seqs = np.arange(batch, dtype=np.int32)
+        st = torch.cuda.current_stream()
+        for ctx in W["contexts"]:
+            qidx = np.full(batch, ctx, dtype=np.int32)
+            pos = np.zeros(batch, dtype=np.int32)
+
+            def step():
+                for layer in range(L):
+                    smem.smem_decode(cache.h, layer % int(l_phys), seqs, pos, qidx, *dins, osa, oca)
+
+            for _ in range(2):
+                step()
+            n_steps = 8
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * L * n_steps)]
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            t0.record(st)
+            for i in range(n_steps):
+                for layer in range(L):
+                    ev[2 * (i * L + layer)].record(st)
+                    smem.smem_decode(cache.h, layer % int(l_phys), seqs, pos, qidx, *dins, osa, oca)
+                    ev[2 * (i * L + layer) + 1].record(st)
+            t1.record(st)
+            torch.cuda.synchronize()
+            step_ms = t0.elapsed_time(t1) / n_steps
+            kms = float(np.mean([ev[2 * k].elapsed_time(ev[2 * k + 1]) for k in range(L * n_steps)]))
+            dec_bytes = batch * (ctx * R + 1) * 4 * H * D
+            cell = {"batch": batch, "context_blocks": ctx, "memory_rows": ctx * R,
+                    "layers_physical": int(l_phys), "layers_logical": L,
+                    "emulated": bool(l_phys < L),
+                    "decode_tok_s": batch / (step_ms / 1e3), "decode_ms_per_step": step_ms,
+                    "decode_kernel_ms": kms, "decode_gbs": dec_bytes / (kms / 1e3) / 1e9,
+                    "decode_hbm_frac": dec_bytes / (kms / 1e3) / 1e9 / peak}
+            if batch == 1:
+                # one-block cached serve: 24 prefill launches, graph-replayed, L2 flushed
+                def serve():
+                    for layer in range(L):
+                        smem.smem_prefill_block(cache.h, 0, layer % int(l_phys), ctx, *pins, posa, poca)
+
+                serve()
+                torch.cuda.synchronize()
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    serve()
+                flush = torch.empty(512 << 20, dtype=torch.uint8, device=device)
+                lat, kern = [], []
+                for i in range(6):
+                    flush.zero_()
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record(st)
+                    g.replay()
+                    b.record(st)
+                    torch.cuda.synchronize()
+                    lat.append(a.elapsed_time(b))
+                for i in range(6):
+                    flush.zero_()
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record(st)
+                    smem.smem_prefill_block(cache.h, 0, i % int(l_phys), ctx, *pins, posa, poca)
+                    b.record(st)
+                    torch.cuda.synchronize()
+                    kern.append(a.elapsed_time(b))
+                del g, flush
+                pf_bytes = ctx * R * 4 * H * D + 6 * B_TOK * H * D * 2
+                pf_flops = 4 * B_TOK * ctx * R * H * D + 4 * (B_TOK * (B_TOK + 1) // 2) * H * D
+                km = float(np.median(kern))
+                cell.update({"serve_latency_ms": float(np.median(lat)), "prefill_kernel_ms": km,
+                             "prefill_gbs": pf_bytes / (km / 1e3) / 1e9,
+                             "prefill_hbm_frac": pf_bytes / (km / 1e3) / 1e9 / peak,
+                             "prefill_tflops": pf_flops / (km / 1e3) / 1e12,
+                             "prefill_tensor_frac": pf_flops / (km / 1e3) / 1e12 / bf16_peak})
+            cells.append(cell)
+            print(json.dumps(cell), file=sys.stderr, flush=True)
+        if smem.smem_check_device_error(cache.h) != smem.OK:
+            raise RuntimeError("device error recorded")
+        cache.close()
+        cache.buf = None
+        torch.cuda.empty_cache()
+    print(json.dumps({"workload": W["name"], "heads": H, "head_dim": D, "layers": L, "peak_hbm_gbs": peak,
+                      "peak_source": peak_src, "cells": cells}), flush=True)
+
+
 # ----------------------------------------------------------------------------- oracle (cpu) timing
 class OracleDecodeSample:
     """A bounded sample of the default workload for the fp64 CPU oracle: the
@@ -633,6 +769,9 @@ def main():
     args = parse_args()
     if args.only_serve:
         run_serve_only(args)
+        return
+    if args.workload == "long":
+        run_long(args)
         return
     if args.impl == "reference":
         run_reference(args)

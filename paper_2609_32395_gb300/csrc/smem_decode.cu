@@ -314,8 +314,16 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
   }
   const float* pb = p.part + ((size_t)pd.pair_begin * p.H + pd.h) * (D + 4);
   const size_t ps = (size_t)p.H * (D + 4);
+  constexpr int G = 16;  // splits whose loads are in flight together
+  // pass 1: the maximum over the null row and every split
   float M = nscore;
-  for (int s2 = 0; s2 < pd.nsplit; ++s2) M = fmaxf(M, __ldcg(pb + s2 * ps));
+  for (int s0 = 0; s0 < pd.nsplit; s0 += G) {
+    float mv[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) mv[g] = s0 + g < pd.nsplit ? __ldcg(pb + (s0 + g) * ps) : -INFINITY;
+#pragma unroll
+    for (int g = 0; g < G; ++g) M = fmaxf(M, mv[g]);
+  }
   float Lsum = 0.f, A[CPT];
 #pragma unroll
   for (int e = 0; e < CPT; ++e) A[e] = 0.f;
@@ -326,12 +334,27 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
 #pragma unroll
     for (int e = 0; e < CPT; ++e) A[e] = f * bf16lo(vn[lane * CPT + e]);
   }
-  for (int s2 = 0; s2 < pd.nsplit; ++s2) {
-    const float* ps2 = pb + s2 * ps;
-    const float f = exp2f(__ldcg(ps2) - M);
-    Lsum = fmaf(f, __ldcg(ps2 + 1), Lsum);
+  // pass 2: weighted sums in split order, G splits' loads issued first
+  for (int s0 = 0; s0 < pd.nsplit; s0 += G) {
+    float ml[G][2], av[G][CPT];
 #pragma unroll
-    for (int e = 0; e < CPT; ++e) A[e] = fmaf(f, __ldcg(ps2 + 4 + lane * CPT + e), A[e]);
+    for (int g = 0; g < G; ++g) {
+      const bool in = s0 + g < pd.nsplit;
+      const float* ps2 = pb + (s0 + g) * ps;
+      const float2 v = in ? __ldcg(reinterpret_cast<const float2*>(ps2)) : make_float2(-INFINITY, 0.f);
+      ml[g][0] = v.x;
+      ml[g][1] = v.y;
+#pragma unroll
+      for (int e = 0; e < CPT; ++e) av[g][e] = in ? __ldcg(ps2 + 4 + lane * CPT + e) : 0.f;
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      if (s0 + g >= pd.nsplit) break;
+      const float f = exp2f(ml[g][0] - M);
+      Lsum = fmaf(f, ml[g][1], Lsum);
+#pragma unroll
+      for (int e = 0; e < CPT; ++e) A[e] = fmaf(f, av[g][e], A[e]);
+    }
   }
   const float inv = 1.f / Lsum;
   uint32_t* o32 = reinterpret_cast<uint32_t*>(p.oca + qoff) + lane * (CPT / 2);

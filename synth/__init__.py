@@ -97,10 +97,11 @@ def _round_f32_bits_to_bf16(bits):
     return ((bits + 0x7FFF + ((bits >> 16) & 1)) >> 16) & 0xFFFF
 
 
-def normal_bf16_np(keys: np.ndarray, n: int) -> np.ndarray:
-    """bf16 bit patterns (uint16), shape keys.shape + (n,)."""
+def normal_bf16_np(keys: np.ndarray, n: int, start: int = 0) -> np.ndarray:
+    """bf16 bit patterns (uint16), shape keys.shape + (n,), element counters
+    start .. start+n-1 of each stream."""
     keys = np.asarray(keys, dtype=np.int64)[..., None]
-    ctr = np.arange(n, dtype=np.int64)
+    ctr = np.arange(start, start + n, dtype=np.int64)
     s = _unif_sum(keys, ctr)
     z = (s - _MEAN).astype(np.float32) * _SCALE_F32
     bits = z.view(np.uint32).astype(np.int64)
@@ -136,6 +137,16 @@ def block_rows_np(seed, seq, block_idx, L, H, R, D):
     for kind in (KIND_K, KIND_V):
         keys = np.array(block_keys(seed, seq, block_idx, L, kind), dtype=np.int64)
         out.append(normal_bf16_np(keys, H * R * D).reshape(L, H, R, D))
+    return out[0], out[1]
+
+
+def block_head_rows_np(seed, seq, block_ids, layer, head, R, D):
+    """(K, V) uint16 arrays [n_blocks][R][D]: one head of one layer of many
+    blocks (the same values as the matching slice of :func:`block_rows_np`)."""
+    out = []
+    for kind in (KIND_K, KIND_V):
+        keys = np.array([stream_key(seed, 1, seq, b, layer, kind) for b in block_ids], dtype=np.int64)
+        out.append(normal_bf16_np(keys, R * D, start=head * R * D).reshape(len(block_ids), R, D))
     return out[0], out[1]
 
 
