@@ -24,6 +24,10 @@ inline cudaError_t ensure_smem_limit(Kernel kernel, int bytes) {
   const unsigned long long bit = 1ull << (dev & 63);
   if (__atomic_load_n(&done, __ATOMIC_ACQUIRE) & bit) return cudaSuccess;
   e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  // prefer the largest shared-memory carveout so that the intended number of
+  // CTAs per SM fits
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
   if (e == cudaSuccess) __atomic_fetch_or(&done, bit, __ATOMIC_RELEASE);
   return e;
 }

@@ -40,13 +40,14 @@ SMEM_HD inline int decode_split_blocks(int nblk) {
 SMEM_HD inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
 // Split plan of the one-block prefill cross-attention, a function of the
-// block count and the cache's fixed head count and head dimension alone:
-// about one wave of CTAs on a GB300 (two per SM at d_h = 64, one at 128),
-// at most kPrefillMaxSplits splits per head, at least two blocks per split.
+// block count and the cache's fixed head count and head dimension alone: the
+// cross-attention CTAs fit one wave on a GB300 (152 SMs; two CTAs per SM at
+// d_h = 64, one at 128), at most kPrefillMaxSplits splits per head, at least
+// two blocks per split.
 constexpr int kPrefillMaxSplits = 16;
 SMEM_HD inline int prefill_split_blocks(int nblk, int H, int D) {
   const int target = D == 64 ? 304 : 152;
-  int ns = (target + H - 1) / H;
+  int ns = target / H;
   if (ns > kPrefillMaxSplits) ns = kPrefillMaxSplits;
   if (ns > (nblk + 1) / 2) ns = (nblk + 1) / 2;
   if (ns < 1) ns = 1;

@@ -43,14 +43,14 @@ struct Pf {
   static constexpr int BOX = 64 * 128;            // one [64 rows][128 B] box
   static constexpr int TILE = BOXES * BOX;        // K or V of one block and head
   static constexpr int STAGE = 2 * TILE;
-  static constexpr int NS = D == 64 ? 4 : 3;
+  static constexpr int NS = D == 64 ? 5 : 4;      // ring stages (2 CTAs per SM fit at d_h = 64)
   static constexpr int PBYTES = 64 * 64 * 2;      // P tile [64 queries][64 keys] bf16
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_RING = TILE;
   static constexpr int OFF_P = OFF_RING + NS * STAGE;
   static constexpr int OFF_BAR = OFF_P + 2 * PBYTES;
-  // barriers: q_full | full[NS] | empty[NS] | s_full[2] | s_free[2] | p_full[2] | o_done[2] | drain
-  static constexpr int NBARS = 1 + 2 * NS + 9;
+  // barriers: q_full | full[NS] | empty[NS] | s_full[2] | s_free[2] | p_full[2] | o_done[2] | drain | merge
+  static constexpr int NBARS = 1 + 2 * NS + 10;
   static constexpr int OFF_MISC = OFF_BAR + NBARS * 8;
   static constexpr int SMEM = OFF_MISC + 64 + 1024;
   static constexpr int THREADS = 192;             // 4 softmax warps, producer, MMA
@@ -59,6 +59,8 @@ struct Pf {
   static constexpr uint32_t COL_O = 128;
   static constexpr uint32_t ID_QK = tc::idesc_bf16(64, 64, 0, 0);
   static constexpr uint32_t ID_PV = tc::idesc_bf16(64, D, 0, 1);
+  static constexpr int PART_BYTES = B * (D + 4) * 4;          // one split's partial rows
+  static constexpr int MERGE_SPR = NS * STAGE / PART_BYTES;   // split partials staged per round
 };
 
 constexpr float kRescaleLog2 = 8.0f;  // raise the running max when it grows by more than 2^8
@@ -95,16 +97,18 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   uint64_t* p_full = s_free + 2;
   uint64_t* o_done = p_full + 2;
   uint64_t* drain = o_done + 2;
+  uint64_t* mbar_merge = drain + 1;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(base + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::OFF_MISC + 4);
   volatile unsigned* ticket = reinterpret_cast<volatile unsigned*>(base + C::OFF_MISC + 8);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int n_ca = p.n_splits * p.H;
-  const bool sa = (int)blockIdx.x >= n_ca;
-  const int h = sa ? (int)blockIdx.x - n_ca : (int)blockIdx.x % p.H;
-  const int split = sa ? 0 : (int)blockIdx.x / p.H;
+  // the short self-attention CTAs come first and leave their SMs early
+  const bool sa = (int)blockIdx.x < p.H;
+  const int cb = (int)blockIdx.x - p.H;
+  const int h = sa ? (int)blockIdx.x : cb % p.H;
+  const int split = sa ? 0 : cb / p.H;
   const int b0 = split * p.split_blks;
   const int nt = sa ? 1 : min(p.split_blks, p.nblk - b0);
 
@@ -121,6 +125,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       mbar_init(&o_done[b], 1);
     }
     mbar_init(drain, 1);
+    mbar_init(mbar_merge, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -390,33 +395,40 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
 #pragma unroll
           for (int c = 0; c < D / 2; ++c) A[c] = f * bf16lo(vn[c]);
         }
-        // O of GROUP splits loaded before any is used; summed in split order
-        constexpr int GROUP = D == 64 ? 4 : 2;
-        for (int s0 = 0; s0 < ns; s0 += GROUP) {
-          float4 buf[GROUP][D / 8];
-#pragma unroll
-          for (int g2 = 0; g2 < GROUP; ++g2)
-#pragma unroll
-            for (int c = 0; c < D / 8; ++c)
-              buf[g2][c] = s0 + g2 < ns ? __ldcg(reinterpret_cast<const float4*>(pb + (s0 + g2) * ps + 4 + col0) + c)
-                                        : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-          for (int g2 = 0; g2 < GROUP; ++g2) {
-            if (s0 + g2 >= ns) break;
-            float f = 0.f, msg = 0.f, lsg = 0.f;
+        // O rows of the splits come through the (now idle) K/V ring by bulk
+        // copy, MERGE_SPR splits per round, and are summed in split order
+        const float* head_part = p.part + (size_t)h * p.max_splits * C::B * (D + 4);
+        for (int s0 = 0, round = 0; s0 < ns; s0 += C::MERGE_SPR, ++round) {
+          const int cnt = min(C::MERGE_SPR, ns - s0);
+          if (threadIdx.x == 0) {
+            mbar_arrive_expect_tx(mbar_merge, (uint32_t)(cnt * C::PART_BYTES));
+            for (int g2 = 0; g2 < cnt; ++g2)
+              bulk_g2s(ring + g2 * C::PART_BYTES, head_part + (size_t)(s0 + g2) * C::B * (D + 4), C::PART_BYTES,
+                       mbar_merge);
+          }
+          if (!bar_all(1, 128, mbar_wait_bounded(mbar_merge, round & 1, nullptr))) {
+            if (threadIdx.x == 0) record_error(p.err, kDevErrWaitFull);
+            break;  // uniform: every softmax thread saw the same outcome
+          }
+          for (int g2 = 0; g2 < cnt; ++g2) {
+            float msg = 0.f, lsg = 0.f;
 #pragma unroll
             for (int t2 = 0; t2 < kPrefillMaxSplits; ++t2)
               if (t2 == s0 + g2) { msg = ms[t2]; lsg = ls[t2]; }
-            f = exp2f(msg - M);
+            const float f = exp2f(msg - M);
             Lsum = fmaf(f, lsg, Lsum);
+            const float4* row = reinterpret_cast<const float4*>(ring + g2 * C::PART_BYTES + r * (D + 4) * 4 + 16) +
+                                col0 / 4;
 #pragma unroll
             for (int c = 0; c < D / 8; ++c) {
-              A[4 * c] = fmaf(f, buf[g2][c].x, A[4 * c]);
-              A[4 * c + 1] = fmaf(f, buf[g2][c].y, A[4 * c + 1]);
-              A[4 * c + 2] = fmaf(f, buf[g2][c].z, A[4 * c + 2]);
-              A[4 * c + 3] = fmaf(f, buf[g2][c].w, A[4 * c + 3]);
+              const float4 v = row[c];
+              A[4 * c] = fmaf(f, v.x, A[4 * c]);
+              A[4 * c + 1] = fmaf(f, v.y, A[4 * c + 1]);
+              A[4 * c + 2] = fmaf(f, v.z, A[4 * c + 2]);
+              A[4 * c + 3] = fmaf(f, v.w, A[4 * c + 3]);
             }
           }
+          named_bar_sync(1, 128);  // the staging area is refilled next round
         }
         const float inv = 1.f / Lsum;
         uint16_t* out = p.oca + qoff + col0;
