@@ -47,6 +47,10 @@ def parse_args():
     ap.add_argument("--no-serve", action="store_true")
     ap.add_argument("--workload", default="decode", choices=["decode", "long"],
                     help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
+    ap.add_argument("--long-batches", default="1,16", help="batches of the long-context cells")
+    ap.add_argument("--long-layers", type=int, default=None,
+                    help="physical layers of the long-context cache (profiling captures)")
+    ap.add_argument("--long-contexts", default="512,1024,4096")
     ap.add_argument("--only-serve", action="store_true",
                     help="time only the one-block cached-serve cells (profiling)")
     ap.add_argument("--seqs", type=int, default=WORKLOAD["seqs"])
@@ -133,24 +137,50 @@ def source_sha(path):
         return hashlib.sha256(f.read()).hexdigest()
 
 
-def profiled_traffic(profile_name, kernel_src, units_now):
+def profiled_traffic(profile_name, units_now, exact=False):
     """DRAM bytes per launch from a committed ncu summary, scaled to this
-    launch's units, or None if the kernel source changed since the capture."""
+    launch's units; None if any source the summary lists changed since the
+    capture (so a stale count is never reported)."""
     path = os.path.join(ROOT, "profiles", profile_name)
     if not os.path.exists(path):
         return None
-    kv = {}
+    kv, shas = {}, []
     for line in open(path):
-        if ":" in line and not line.startswith("#"):
-            k, v = line.split(":", 1)
-            kv[k.strip()] = v.strip()
+        if line.startswith("#") or ":" not in line:
+            continue
+        k, v = line.split(":", 1)
+        k, v = k.strip(), v.strip()
+        if k == "source_sha256":
+            name, digest = v.split()
+            shas.append((name, digest))
+        else:
+            kv[k] = v
     try:
-        if kv.get("kernel_source_sha256") != source_sha(kernel_src):
+        if not shas or any(source_sha(os.path.join(ROOT, n)) != d for n, d in shas):
             return None
+        if exact:  # traffic with a fixed part: only the captured size is known
+            return float(kv["dram_bytes_per_launch"]) if float(kv["units_per_launch"]) == units_now else None
         per_unit = float(kv["dram_bytes_per_launch"]) / float(kv["units_per_launch"])
         return per_unit * units_now
-    except (KeyError, ValueError):
+    except (KeyError, ValueError, OSError):
         return None
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    """Max of a per-rank float over the process group (identity without one)."""
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def rank_seed(seed: int, rank: int) -> int:
+    """Each rank serves its own sequences: the seed is offset by the rank."""
+    return seed + 1000 * rank
 
 
 # ----------------------------------------------------------------------------- decode workload
@@ -166,7 +196,7 @@ class DecodeWorkload:
         W = WORKLOAD
         self.L, self.H, self.D = (layers or W["L"]), W["H"], W["D"]
         self.S = seqs
-        self.seed = seed + 1000 * rank
+        self.seed = rank_seed(seed, rank)
         self.device = device
         self.nblk = synth.ragged_contexts(self.seed, seqs, W["ctx_lo"], W["ctx_hi"]).astype(np.int64)
         self.pos = synth.inblock_positions(self.seed, seqs, B_TOK).astype(np.int64)
@@ -395,16 +425,20 @@ def run_long(args):
     smem.lib()
     W = LONG
     H, D, L = W["H"], W["D"], W["L"]
-    nmax = max(W["contexts"])
+    contexts = [int(x) for x in args.long_contexts.split(",")]
+    batches = [int(x) for x in args.long_batches.split(",")]
+    nmax = max(contexts)
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     bf16_peak = float(peaks.get("bf16_tflops", 1900.0))
     block_bytes = 2 * H * R * D * 2  # K and V of one layer
     cells = []
-    for batch in W["batches"]:
+    for batch in batches:
         free, _ = torch.cuda.mem_get_info()
         budget = free - (16 << 30)
-        l_phys = max(2, min(L, budget // (batch * (nmax + 8) * block_bytes)))
+        l_phys = max(1, min(L, budget // (batch * (nmax + 8) * block_bytes)))
+        if args.long_layers:
+            l_phys = min(l_phys, args.long_layers)
         cap = batch * (nmax + 4)
         cfg = smem.make_config(int(l_phys), H, D, batch, nmax + 4, cap,
                                free_order=synth.slot_permutation(W["seed"] + batch, cap))
@@ -428,7 +462,7 @@ def run_long(args):
         poca = torch.empty_like(posa)
         seqs = np.arange(batch, dtype=np.int32)
         st = torch.cuda.current_stream()
-        for ctx in W["contexts"]:
+        for ctx in contexts:
             qidx = np.full(batch, ctx, dtype=np.int32)
             pos = np.zeros(batch, dtype=np.int32)
 
@@ -508,6 +542,63 @@ def run_long(args):
                       "peak_source": peak_src, "cells": cells}), flush=True)
 
 
+# ----------------------------------------------------------------------------- edit latency
+EDIT = dict(name="410M-shaped edit churn, 32 sequences", H=16, D=64, seqs=32, contexts=(512, 4096), seed=4)
+
+
+def measure_edit_latency(ctx, device, n_ops=400):
+    """Per-delete and per-append latency with every sequence holding `ctx`
+    blocks (block contents do not affect an edit, so every block is filled
+    from one zero block). Host time is the whole C ABI call (bookkeeping,
+    validation and the launch of the table-edit kernel); device time is the
+    table-edit kernel alone."""
+    import torch
+
+    from paper_2609_32395_gb300 import smem
+
+    W = EDIT
+    S, H, D = W["seqs"], W["H"], W["D"]
+    cap = S * ctx + 8
+    cfg = smem.make_config(1, H, D, S, ctx + 8, cap)
+    cache = smem.SmemCache(cfg, device=device)
+    z = torch.zeros((1, H, R, D), dtype=torch.bfloat16, device=device)
+    for s in range(S):
+        for j in range(ctx):
+            smem.smem_append_block(cache.h, s, j, z, z)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(W["seed"] + ctx)
+    st = torch.cuda.current_stream()
+    host_del, host_app, dev_del = [], [], []
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_ops)]
+    for i in range(n_ops):
+        s = int(rng.integers(0, S))
+        j = int(rng.integers(0, ctx))
+        ev[i][0].record(st)
+        t0 = time.perf_counter()
+        smem.smem_delete_block(cache.h, s, j)
+        t1 = time.perf_counter()
+        ev[i][1].record(st)
+        smem.smem_append_block(cache.h, s, j, z, z)
+        t2 = time.perf_counter()
+        host_del.append(t1 - t0)
+        host_app.append(t2 - t1)
+        if i % 50 == 49:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+    dev_del = [a.elapsed_time(b) * 1e3 for a, b in ev]
+    err = smem.smem_check_device_error(cache.h)
+    cache.close()
+    cache.buf = None
+    torch.cuda.empty_cache()
+    if err != smem.OK:
+        raise RuntimeError("device error recorded during the edit measurement")
+    us = lambda v, q: float(np.percentile(np.array(v) * 1e6, q))  # noqa: E731
+    return {"context_blocks": ctx, "sequences": S, "delete_host_us_p50": us(host_del, 50),
+            "delete_host_us_p99": us(host_del, 99), "append_host_us_p50": us(host_app, 50),
+            "delete_device_us_p50": float(np.percentile(dev_del, 50)),
+            "append_bytes": 2 * H * R * D * 2}
+
+
 # ----------------------------------------------------------------------------- oracle (cpu) timing
 class OracleDecodeSample:
     """A bounded sample of the default workload for the fp64 CPU oracle: the
@@ -520,7 +611,7 @@ class OracleDecodeSample:
 
         W = WORKLOAD
         self.L, self.H, self.D = W["L"], W["H"], W["D"]
-        s_seed = W["seed"] + 1000 * rank
+        s_seed = rank_seed(W["seed"], rank)
         nblk = synth.ragged_contexts(s_seed, seqs, W["ctx_lo"], W["ctx_hi"])
         pos = synth.inblock_positions(s_seed, seqs, B_TOK)
         self.mean_rows = float(nblk.mean()) * R + float(pos.mean()) + 1
@@ -652,12 +743,7 @@ def run_ours(args):
     achieved = sum(alg_bytes) / (sum(kern_ms) / 1e3) / 1e9
 
     tokens = args.steps * args.seqs
-    if ws > 1:
-        import torch.distributed as dist
-
-        t = torch.tensor([elapsed], device=device, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed = float(t.item())
+    elapsed = max_over_ranks(elapsed, device)
     value = tokens * ws / elapsed
 
     # --- end to end: host inputs / outputs / appended rows through the C ABI
@@ -679,12 +765,7 @@ def run_ours(args):
         n_app = sum(wl.new_used) - appends_before
         h2d = wl.L * 4 * args.seqs * wl.H * wl.D * 2 + n_app / e2e_steps * 2 * host_blk[0].numel() * 2
         d2h = wl.L * 2 * args.seqs * wl.H * wl.D * 2
-        if ws > 1:
-            import torch.distributed as dist
-
-            t = torch.tensor([e2e_el], device=device, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_el = float(t.item())
+        e2e_el = max_over_ranks(e2e_el, device)
         e2e = {"value": e2e_steps * args.seqs * ws / e2e_el, "unit": "tok/s",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
@@ -700,6 +781,7 @@ def run_ours(args):
         del wl.new_K, wl.new_V
         torch.cuda.empty_cache()
         serve = [measure_serve(n, device) for n in SERVE["contexts"]]
+    edit = None if args.no_serve else [measure_edit_latency(n, device) for n in EDIT["contexts"]]
 
     if rank != 0:
         if ws > 1:
@@ -711,8 +793,7 @@ def run_ours(args):
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     units_launch = float(np.mean(rows))
-    traffic = profiled_traffic("decode_410m.txt", os.path.join(ROOT, "paper_2609_32395_gb300", "csrc",
-                                                                   "smem_decode.cu"), units_launch)
+    traffic = profiled_traffic("decode_410m.txt", units_launch)
     cpu = None if args.no_cpu_baseline else oracle_baseline(args.seqs)
     line = {
         "metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": ws, "steps": args.steps,
@@ -736,13 +817,17 @@ def run_ours(args):
         for sv in serve:
             gbs = sv["bytes_per_launch"] / (sv["kernel_ms_mean"] / 1e3) / 1e9
             tfs = sv["flops_per_launch"] / (sv["kernel_ms_mean"] / 1e3) / 1e12
-            sv["roofline"] = {"bound": "hbm", "achieved_gbs": gbs, "hbm_frac": gbs / peak,
+            tr = profiled_traffic("prefill_160m.txt", sv["memory_rows"], exact=True)
+            sv["roofline"] = {"bound": "hbm", "achieved_gbs": gbs, "hbm_frac": gbs / peak, "traffic": tr,
                               "achieved_tflops": tfs, "tensor_frac": tfs / bf16_peak,
                               "peak_tflops_bf16": bf16_peak}
         line["serve"] = {"workload": SERVE["name"], "layers": SERVE["L"], "heads": SERVE["H"],
                          "head_dim": SERVE["D"], "metric": "one-block cached-serve latency (12 layers)",
                          "unit": "ms", "timing": "CUDA graph of the 12 per-layer launches, L2 flushed before each",
                          "cells": serve}
+    if edit:
+        line["edit"] = {"workload": EDIT["name"], "unit": "us",
+                        "note": "host = whole C ABI call; device = table-edit kernel; no row moves", "cells": edit}
     if e2e:
         line["e2e"] = e2e
     if cpu:

@@ -34,7 +34,7 @@ struct Layout {
 // split reads, a function of the sequence's block count alone (so the same
 // block set always reduces in the same order).
 SMEM_HD inline int decode_split_blocks(int nblk) {
-  int sb = (nblk + 127) / 128;
+  int sb = (nblk + 31) / 32;
   return sb < 4 ? 4 : (sb > 16 ? 16 : sb);
 }
 SMEM_HD inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
