@@ -13,6 +13,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <deque>
 #include <new>
@@ -37,6 +38,7 @@ struct smem_cache {
   std::vector<uint32_t> seen;              // decode: duplicate-sequence check
   uint32_t seen_epoch = 0;
   int fail_after = 0;                      // test hook: n-th next launch fails
+  int pf_cluster_max = 0;                  // prefill cluster limit on this device (0: no clusters)
 };
 
 namespace {
@@ -212,6 +214,8 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
       delete c;
       return SMEM_ERR_CUDA;
     }
+    const char* knob = std::getenv("SMEM_PREFILL_CLUSTERS");
+    c->pf_cluster_max = (knob && knob[0] == '0') ? 0 : smem::prefill_cluster_max(L.H, L.D);
   }
   *out = c;
   return SMEM_OK;
@@ -356,7 +360,11 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
   a.D = c->lay.D;
   a.layer = layer;
   a.nblk = nblk;
-  a.split_blks = nblk ? smem::prefill_split_blocks(nblk, c->lay.H, c->lay.D) : 1;
+  a.cluster = (c->pf_cluster_max >= 2 && nblk <= smem::kPrefillClusterMaxBlocks) ? 1 : 0;
+  if (a.cluster)
+    a.split_blks = nblk ? smem::prefill_cluster_split_blocks(nblk, c->pf_cluster_max) : 1;
+  else
+    a.split_blks = nblk ? smem::prefill_split_blocks(nblk, c->lay.H, c->lay.D) : 1;
   a.n_splits = nblk ? smem::ceil_div(nblk, a.split_blks) : 0;
   a.capacity = c->lay.capacity;
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->lay.D));

@@ -132,8 +132,22 @@ struct PrefillArgs {
   int* err;
   long long slot_elems;
   int L, H, D, layer, nblk, split_blks, n_splits, capacity;
+  int cluster;                // 1: cluster mode (one cluster of n_splits + 1 CTAs per head)
   float scale_log2;
 };
 cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);
+// Largest cluster size (<= 16) with one cluster per head resident at once on
+// the current device for the d_h = 64 prefill; 0 if cluster mode is unavailable.
+int prefill_cluster_max(int H, int D);
+// Cluster mode pays off while the launch is latency-bound (short contexts);
+// beyond this many blocks the cluster-free grid, spread over every SM, wins.
+constexpr int kPrefillClusterMaxBlocks = 128;
+// Split plan of the cluster mode: blocks per split for a cluster limit cs_max.
+SMEM_HD inline int prefill_cluster_split_blocks(int nblk, int cs_max) {
+  int ns = cs_max - 1;
+  if (ns > (nblk + 1) / 2) ns = (nblk + 1) / 2;
+  if (ns < 1) ns = 1;
+  return (nblk + ns - 1) / ns;
+}
 
 }  // namespace smem

@@ -80,7 +80,80 @@ struct PrefillParams {
   float scale_log2;
 };
 
+// Cluster mode (d_h = 64): one cluster of n_splits + 1 CTAs per head, rank 0
+// the in-block SA tile and rank k the split k-1. Each split CTA parks its
+// partial rows (m, l, O) in its own shared memory; after a cluster barrier
+// every CTA merges a slice of the 64 rows by reading the others' partials
+// over distributed shared memory, in split order (null row first).
 template <int D>
+__device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint32_t cs, uint32_t stage_saddr,
+                              int warp, int lane) {
+  constexpr int CPL = D / 32;  // columns per lane
+  const int ns = (int)cs - 1;
+  const int rp = (kBlockTok + (int)cs - 1) / (int)cs;
+  const int r0 = (int)rank * rp, r1 = min(kBlockTok, r0 + rp);
+  for (int row = r0 + warp; row < r1; row += 6) {
+    const size_t qoff = ((size_t)row * p.H + h) * D;
+    float nscore = -INFINITY;
+    if (p.null_kv) {
+      const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
+      float dot = 0.f;
+#pragma unroll
+      for (int e = 0; e < CPL; ++e)
+        dot = fmaf(bf16lo(p.qc_ptr[qoff + lane * CPL + e]), bf16lo(kn[lane * CPL + e]), dot);
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+      nscore = dot * p.scale_log2;
+    }
+    const uint32_t row_saddr = stage_saddr + (uint32_t)(row * (D + 4) * 4);
+    float ms[kPrefillMaxSplits], ls[kPrefillMaxSplits];
+#pragma unroll
+    for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) {
+      const float2 v = s2 < ns ? tc::ld_dsmem_f32x2(tc::dsmem_addr(row_saddr, (uint32_t)(s2 + 1)))
+                               : make_float2(-INFINITY, 0.f);
+      ms[s2] = v.x;
+      ls[s2] = v.y;
+    }
+    float M = nscore;
+#pragma unroll
+    for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) M = fmaxf(M, ms[s2]);
+    float Lsum = 0.f, A[CPL];
+#pragma unroll
+    for (int e = 0; e < CPL; ++e) A[e] = 0.f;
+    if (p.null_kv) {
+      const float f = exp2f(nscore - M);
+      Lsum = f;
+      const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D + D;
+#pragma unroll
+      for (int e = 0; e < CPL; ++e) A[e] = f * bf16lo(vn[lane * CPL + e]);
+    }
+    float2 ov[kPrefillMaxSplits][CPL / 2];
+#pragma unroll
+    for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2)
+#pragma unroll
+      for (int e = 0; e < CPL / 2; ++e)
+        ov[s2][e] = s2 < ns ? tc::ld_dsmem_f32x2(
+                                  tc::dsmem_addr(row_saddr + 16 + (lane * CPL + 2 * e) * 4, (uint32_t)(s2 + 1)))
+                            : make_float2(0.f, 0.f);
+#pragma unroll
+    for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) {
+      if (s2 >= ns) break;
+      const float f = exp2f(ms[s2] - M);
+      Lsum = fmaf(f, ls[s2], Lsum);
+#pragma unroll
+      for (int e = 0; e < CPL / 2; ++e) {
+        A[2 * e] = fmaf(f, ov[s2][e].x, A[2 * e]);
+        A[2 * e + 1] = fmaf(f, ov[s2][e].y, A[2 * e + 1]);
+      }
+    }
+    const float inv = 1.f / Lsum;
+    uint32_t* o32 = reinterpret_cast<uint32_t*>(p.oca + qoff) + lane * (CPL / 2);
+#pragma unroll
+    for (int e = 0; e < CPL / 2; ++e) o32[e] = pack_bf16x2(A[2 * e] * inv, A[2 * e + 1] * inv);
+  }
+}
+
+template <int D, bool CL>
 __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kernel(const __grid_constant__ PrefillParams p) {
   using C = Pf<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -104,11 +177,14 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // the short self-attention CTAs come first and leave their SMs early
-  const bool sa = (int)blockIdx.x < p.H;
+  // without clusters the short self-attention CTAs come first and leave
+  // their SMs early; in cluster mode a head is a cluster and rank 0 its SA
+  const uint32_t cs = (uint32_t)p.n_splits + 1;
+  const uint32_t crank = CL ? tc::cluster_ctarank() : 0u;
+  const bool sa = CL ? crank == 0 : (int)blockIdx.x < p.H;
   const int cb = (int)blockIdx.x - p.H;
-  const int h = sa ? (int)blockIdx.x : cb % p.H;
-  const int split = sa ? 0 : cb / p.H;
+  const int h = CL ? (int)(blockIdx.x / cs) : (sa ? (int)blockIdx.x : cb % p.H);
+  const int split = CL ? (int)crank - 1 : (sa ? 0 : cb / p.H);
   const int b0 = split * p.split_blks;
   const int nt = sa ? 1 : min(p.split_blks, p.nblk - b0);
 
@@ -320,7 +396,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
     }
     const float lrow = l + __shfl_xor_sync(0xffffffffu, l, 16);
     const int col0 = hf * (D / 2);  // this thread's columns of O
-    const bool direct = sa || (p.n_splits == 1 && !p.null_kv);
+    const bool direct = sa || (!CL && p.n_splits == 1 && !p.null_kv);
     if (ok && direct) {
       uint16_t* out = (sa ? p.osa : p.oca) + ((size_t)r * p.H + h) * D + col0;
       const float inv = 1.f / lrow;
@@ -342,7 +418,19 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       for (int c = 0; c < D / 2; c += 8)
         *reinterpret_cast<uint4*>(out + c) = vn ? *reinterpret_cast<const uint4*>(vn + c) : make_uint4(0, 0, 0, 0);
     }
-    if (ok && !direct) {
+    if (CL && !sa) {
+      // park this split's partial rows in shared memory for the cluster merge
+      float* pp = reinterpret_cast<float*>(ring) + (size_t)r * (D + 4);
+#pragma unroll
+      for (int c = 0; c < D / 2; c += 4)
+        *reinterpret_cast<float4*>(pp + 4 + col0 + c) =
+            ok ? make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]) : make_float4(0.f, 0.f, 0.f, 0.f);
+      if (hf == 0) {
+        pp[0] = ok ? m_used : -INFINITY;
+        pp[1] = ok ? lrow : 0.f;
+      }
+    }
+    if (!CL && ok && !direct) {
       float* pp = p.part + (((size_t)h * p.max_splits + split) * C::B + r) * (D + 4);
 #pragma unroll
       for (int c = 0; c < D / 2; c += 4)
@@ -355,7 +443,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
     }
     // the four softmax warps agree on the outcome before the ticket
     const bool all_ok = bar_all(1, 128, ok);
-    if (all_ok && !direct) {
+    if (!CL && all_ok && !direct) {
       if (threadIdx.x == 0) *ticket = atomicAdd(&p.counters[h], 1u);
       named_bar_sync(1, 128);
       if (*ticket == (unsigned)(p.n_splits - 1)) {
@@ -447,6 +535,11 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   }
   tc::fence_before();
   __syncthreads();
+  if (CL && p.n_splits > 0) {
+    tc::cluster_sync();  // every split's partial rows are parked
+    cluster_merge<D>(p, h, crank, cs, smem_u32(ring), warp, lane);
+    tc::cluster_sync();  // no CTA leaves while others read its shared memory
+  }
   if (warp == 4) {
     tc::fence_after();
     tc::dealloc(tmem, C::TMEM_COLS);
@@ -456,10 +549,64 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
 template <int D>
 static cudaError_t launch_prefill_d(const PrefillParams& p, int grid, cudaStream_t st) {
   using C = Pf<D>;
-  cudaError_t e = ensure_smem_limit<1000 + D>(prefill_kernel<D>, C::SMEM);
+  cudaError_t e = ensure_smem_limit<1000 + D>(prefill_kernel<D, false>, C::SMEM);
   if (e != cudaSuccess) return e;
-  prefill_kernel<D><<<grid, C::THREADS, C::SMEM, st>>>(p);
+  prefill_kernel<D, false><<<grid, C::THREADS, C::SMEM, st>>>(p);
   return cudaGetLastError();
+}
+
+static cudaError_t cluster_kernel_setup() {
+  cudaError_t e = ensure_smem_limit<2064>(prefill_kernel<64, true>, Pf<64>::SMEM);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(prefill_kernel<64, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  return e;
+}
+
+static cudaError_t launch_prefill_cluster(const PrefillParams& p, cudaStream_t st) {
+  cudaError_t e = cluster_kernel_setup();
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  const unsigned cs = (unsigned)p.n_splits + 1;
+  cfg.gridDim = dim3((unsigned)p.H * cs);
+  cfg.blockDim = dim3(Pf<64>::THREADS);
+  cfg.dynamicSmemBytes = Pf<64>::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, prefill_kernel<64, true>, p);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+int prefill_cluster_max(int H, int D) {
+  // the largest cluster (at most 16 CTAs) of which one per head can be
+  // resident at once on the current device; 0: cluster mode unavailable
+  if (D != 64) return 0;
+  if (cluster_kernel_setup() != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  for (int cs : {16, 12, 8, 4}) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(H * cs));
+    cfg.blockDim = dim3(Pf<64>::THREADS);
+    cfg.dynamicSmemBytes = Pf<64>::SMEM;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, prefill_kernel<64, true>, &cfg) == cudaSuccess && n >= H) return cs;
+    cudaGetLastError();
+  }
+  return 0;
 }
 
 static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D) {
@@ -506,6 +653,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   P.max_splits = kPrefillMaxSplits;
   P.scale_log2 = a.scale_log2;
   const int grid = a.n_splits * a.H + a.H;
+  if (a.D == 64 && a.cluster) return launch_prefill_cluster(P, st);
   if (a.D == 64) return launch_prefill_d<64>(P, grid, st);
   if (a.D == 128) return launch_prefill_d<128>(P, grid, st);
   return cudaErrorInvalidValue;

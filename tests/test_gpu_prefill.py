@@ -12,6 +12,16 @@ from tests.gpu_helpers import DeviceCache, assert_close, out_f64
 pytestmark = pytest.mark.gpu
 
 
+@pytest.fixture(params=["clusters", "no_clusters"])
+def cluster_mode(request, monkeypatch):
+    """d_h = 64 prefill with one cluster per head, or the cluster-free kernel."""
+    if request.param == "no_clusters":
+        monkeypatch.setenv("SMEM_PREFILL_CLUSTERS", "0")
+    else:
+        monkeypatch.delenv("SMEM_PREFILL_CLUSTERS", raising=False)
+    return request.param
+
+
 def _check_prefill(dc, seq, layer, q_idx, tag=0):
     ins, osa, oca = dc.prefill(seq, layer, q_idx, tag)
     ref_sa, ref_ca = dc.oracle_prefill(seq, layer, q_idx, *ins)
@@ -20,7 +30,7 @@ def _check_prefill(dc, seq, layer, q_idx, tag=0):
     return osa, oca
 
 
-def test_tiny_config_prefill_and_delete_reappend():
+def test_tiny_config_prefill_and_delete_reappend(cluster_mode):
     """Tiny reader: H=4, d_h=64, 8 memory blocks (512 rows), one 64-token
     query block; delete block 3, re-append it to another slot: bitwise equal."""
     dc = DeviceCache(L=1, H=4, D=64, max_seqs=1, max_blocks=16, capacity=16)
@@ -39,7 +49,7 @@ def test_tiny_config_prefill_and_delete_reappend():
 
 @pytest.mark.parametrize("D", [64, 128])
 @pytest.mark.parametrize("has_null", [False, True])
-def test_ragged_contexts(D, has_null):
+def test_ragged_contexts(D, has_null, cluster_mode):
     """Contexts from empty to many splits with a ragged last split, and a
     query block in the middle of the table."""
     nblks = [0, 1, 2, 5, 33, 64, 130]
@@ -59,7 +69,7 @@ def test_ragged_contexts(D, has_null):
 
 
 @pytest.mark.parametrize("nblk", [16, 64, 256])
-def test_160m_shape_one_layer(nblk):
+def test_160m_shape_one_layer(nblk, cluster_mode):
     """160M reader shape (H=12, d_h=64) at 16 / 64 / 256 cached blocks."""
     dc = DeviceCache(L=1, H=12, D=64, max_seqs=1, max_blocks=nblk + 1, capacity=nblk + 8, seed=5,
                      free_order=synth.slot_permutation(5, nblk + 8))
@@ -69,11 +79,12 @@ def test_160m_shape_one_layer(nblk):
     assert smem.smem_check_device_error(dc.h) == smem.OK
 
 
-def test_path_independence_bitwise():
+@pytest.mark.parametrize("D", [64, 128])
+def test_path_independence_bitwise(D):
     outs = []
     target = list(range(0, 40, 2)) + [41, 45]
     for trial in range(3):
-        dc = DeviceCache(L=1, H=2, D=128, max_seqs=1, max_blocks=64, capacity=100, seed=13,
+        dc = DeviceCache(L=1, H=2, D=D, max_seqs=1, max_blocks=64, capacity=100, seed=13,
                          free_order=synth.slot_permutation(50 + trial, 100))
         rng = np.random.default_rng(100 + trial)
         live = set()
