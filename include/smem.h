@@ -38,9 +38,10 @@
  *     owns it; it must outlive the cache.
  *   - Supported shapes: block_tokens == rows_per_block == 64,
  *     head_dim 64 or 128 (SMEM_ERR_UNSUPPORTED otherwise).
- *   - At head_dim 64 and up to 128 readable blocks the one-block prefill
- *     runs one thread-block cluster per head when the device can hold all of
- *     them at once (checked at cache creation); the environment variable
+ *   - At head_dim 64 the one-block prefill runs one thread-block cluster per
+ *     head when the device can hold all of them at once (checked at cache
+ *     creation; with clusters smaller than 16 CTAs only up to 128 readable
+ *     blocks); the environment variable
  *     SMEM_PREFILL_CLUSTERS=0, read at creation, selects the cluster-free
  *     kernel instead. Both are deterministic; their split plans (hence
  *     rounding) differ.

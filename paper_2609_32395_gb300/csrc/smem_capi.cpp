@@ -360,7 +360,7 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
   a.D = c->lay.D;
   a.layer = layer;
   a.nblk = nblk;
-  a.cluster = (c->pf_cluster_max >= 2 && nblk <= smem::kPrefillClusterMaxBlocks) ? 1 : 0;
+  a.cluster = smem::prefill_use_clusters(nblk, c->pf_cluster_max) ? 1 : 0;
   if (a.cluster)
     a.split_blks = nblk ? smem::prefill_cluster_split_blocks(nblk, c->pf_cluster_max) : 1;
   else

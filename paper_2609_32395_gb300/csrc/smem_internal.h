@@ -139,9 +139,13 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);
 // Largest cluster size (<= 16) with one cluster per head resident at once on
 // the current device for the d_h = 64 prefill; 0 if cluster mode is unavailable.
 int prefill_cluster_max(int H, int D);
-// Cluster mode pays off while the launch is latency-bound (short contexts);
-// beyond this many blocks the cluster-free grid, spread over every SM, wins.
+// Cluster mode removes the global split merge. With clusters of 16 it wins at
+// every context length; with smaller clusters (fewer splits than the
+// cluster-free plan) only while the launch is latency-bound.
 constexpr int kPrefillClusterMaxBlocks = 128;
+SMEM_HD inline bool prefill_use_clusters(int nblk, int cs_max) {
+  return cs_max >= 2 && (cs_max >= 16 || nblk <= kPrefillClusterMaxBlocks);
+}
 // Split plan of the cluster mode: blocks per split for a cluster limit cs_max.
 SMEM_HD inline int prefill_cluster_split_blocks(int nblk, int cs_max) {
   int ns = cs_max - 1;

@@ -582,11 +582,25 @@ static cudaError_t launch_prefill_cluster(const PrefillParams& p, cudaStream_t s
   return cudaGetLastError();
 }
 
+// A kernel with the cluster prefill's launch footprint (threads and dynamic
+// shared memory) but no tensor-memory allocation: the occupancy query counts
+// one CTA per SM for kernels that allocate tensor memory at run time, while
+// the hardware holds two of these (256 of 512 TMEM columns each; registers
+// and shared memory both allow two).
+__global__ void __launch_bounds__(192, 2) prefill_footprint_kernel(int* p) {
+  extern __shared__ uint8_t sm[];
+  if (p) p[threadIdx.x] = sm[threadIdx.x];
+}
+
 int prefill_cluster_max(int H, int D) {
   // the largest cluster (at most 16 CTAs) of which one per head can be
   // resident at once on the current device; 0: cluster mode unavailable
   if (D != 64) return 0;
-  if (cluster_kernel_setup() != cudaSuccess) {
+  if (cluster_kernel_setup() != cudaSuccess ||
+      cudaFuncSetAttribute(prefill_footprint_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, Pf<64>::SMEM) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(prefill_footprint_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+          cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -603,7 +617,7 @@ int prefill_cluster_max(int H, int D) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, prefill_kernel<64, true>, &cfg) == cudaSuccess && n >= H) return cs;
+    if (cudaOccupancyMaxActiveClusters(&n, prefill_footprint_kernel, &cfg) == cudaSuccess && n >= H) return cs;
     cudaGetLastError();
   }
   return 0;
