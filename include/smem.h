@@ -35,7 +35,10 @@
  *     as it was. No C++ exception crosses this interface.
  *   - The library allocates no device memory: the caller passes one device
  *     buffer of smem_cache_required_bytes() bytes to smem_cache_create and
- *     owns it; it must outlive the cache.
+ *     owns it; it must outlive the cache. The one exception is the
+ *     reader-layer group at the end: its first call on a cache creates a
+ *     cuBLAS handle (cuBLAS's own small device state, freed by
+ *     smem_cache_destroy); the GEMM workspace there is the caller's too.
  *   - Supported shapes: block_tokens == rows_per_block == 64,
  *     head_dim 64 or 128 (SMEM_ERR_UNSUPPORTED otherwise).
  *   - At head_dim 64 the one-block prefill runs one thread-block cluster per
@@ -56,7 +59,7 @@
 extern "C" {
 #endif
 
-#define SMEM_ABI_VERSION 1
+#define SMEM_ABI_VERSION 2
 
 enum {
     SMEM_OK = 0,
@@ -201,6 +204,78 @@ int smem_decode_static_scratch(smem_cache *c, int32_t layer, int32_t nb, const i
                                const int32_t *pos, const int32_t *q_block_idx, const void *qs,
                                const void *k_new, const void *v_new, const void *qc, void *osa,
                                void *oca, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Full reader layer (arXiv 2609.32395, Sec. 2 "Model", App. A "Reader").
+ * With d = H * d_h, one reader layer maps the residual stream x (fp32) by
+ * three pre-LN residual branches:
+ *   x1 = x  + SA(LN1(x) W_qkv) W_os        block-local causal self-attention
+ *   x2 = x1 + CA(LN2(x1) W_qc) W_oc        cross-attention into memory rows
+ *   x3 = x2 + GELU(LN3(x2) W_1) W_2        FFN of width 4d, GELU = x Phi(x)
+ * LN(x) = (x - mean) / sqrt(biased variance + 1e-5) * g + b per token.
+ * A memory row mu (d wide, the block-local encoder's output, shared by all
+ * layers) has per-layer keys mu W_kc and values mu W_vc; the null row is one
+ * d-vector nu projected the same way. The attentions are those of
+ * smem_prefill_block / smem_decode on the same cache; projections are bf16
+ * GEMMs with fp32 accumulation (cuBLAS); intermediates LN outputs, q/k/v,
+ * attention outputs and GELU outputs are rounded to bf16, the residual
+ * stream stays fp32.
+ *
+ * Workspace: every call below takes a device buffer `ws` of at least
+ * smem_layer_workspace_bytes(c, n_rows) bytes (256-byte aligned, the
+ * caller's), n_rows = b for a prefill, nb for a decode, 0 for the memory
+ * projections. Calls that share a workspace must be ordered. */
+typedef struct smem_layer_weights {
+    const float *ln1_g, *ln1_b; /* [d] fp32                                     */
+    const void *w_qkv;          /* bf16 [d][3d], columns Q | K | V, each [H][d_h] */
+    const void *w_os;           /* bf16 [d][d]                                  */
+    const float *ln2_g, *ln2_b; /* [d]                                          */
+    const void *w_qc;           /* bf16 [d][d], cross-attention query map       */
+    const void *w_oc;           /* bf16 [d][d]                                  */
+    const void *w_kc, *w_vc;    /* bf16 [d][d], memory-row key / value maps     */
+    const float *ln3_g, *ln3_b; /* [d]                                          */
+    const void *w_1;            /* bf16 [d][4d]                                 */
+    const void *w_2;            /* bf16 [4d][d]                                 */
+} smem_layer_weights;
+
+/* Workspace bytes of a layer call over n_rows tokens (0 <= n_rows <=
+ * max(b, max_decode_batch)); 0 for a bad argument. */
+size_t smem_layer_workspace_bytes(const smem_cache *c, int32_t n_rows);
+
+/* Appends memory block `block_idx` of `seq` given its memory rows: mu is
+ * device bf16 [R][d]; w points to L HOST structs (layer 0..L-1) of which
+ * w_kc and w_vc are read. The slot receives, for every layer l and head h,
+ * K = mu W_kc^l[:, h d_h : (h+1) d_h] and V likewise (bf16), then the table
+ * insert follows as in smem_append_block (same validation, errors and
+ * FIFO order). */
+int smem_append_block_rows(smem_cache *c, int32_t seq, int32_t block_idx, const void *mu,
+                           const smem_layer_weights *w, void *ws, size_t ws_bytes, void *stream,
+                           int32_t *slot_out);
+
+/* Sets the null row from the d-vector nu (device bf16 [d]): per layer,
+ * k_null = nu W_kc^l, v_null = nu W_vc^l. w: L host structs. Requires
+ * has_null_row. */
+int smem_set_null_vector(smem_cache *c, const void *nu, const smem_layer_weights *w, void *ws,
+                         size_t ws_bytes, void *stream);
+
+/* One reader layer on the b tokens of block `q_block_idx` of `seq`
+ * (block-skip serving, Sec. 3.1): x is device fp32 [b][d], read and
+ * overwritten with the layer's output; w is one host struct (this layer's
+ * weights). The block's self-attention keys/values (LN1(x) W_qkv, K and V
+ * parts) are also stored as in-block rows 0..b-1 of (seq, layer), as
+ * smem_write_inblock would, for later decode steps. Cross-attention reads
+ * the null row and the table blocks with index < q_block_idx. */
+int smem_reader_layer_prefill(smem_cache *c, int32_t seq, int32_t layer, int32_t q_block_idx,
+                              const smem_layer_weights *w, float *x, void *ws, size_t ws_bytes,
+                              void *stream);
+
+/* One reader layer for one decode step of nb sequences (arguments as in
+ * smem_decode): x is device fp32 [nb][d], read and overwritten; the new
+ * tokens' self-attention k, v become in-block rows pos[i]. */
+int smem_reader_layer_decode(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids,
+                             const int32_t *pos, const int32_t *q_block_idx,
+                             const smem_layer_weights *w, float *x, void *ws, size_t ws_bytes,
+                             void *stream);
 
 /* Introspection for bit-exact bookkeeping checks (host state, no CUDA).
  * smem_get_table: the table of `seq` in ascending block index; up to `cap`

@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OBJ = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsmem.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["smem_capi.cpp", "smem_copy.cu", "smem_decode.cu", "smem_prefill.cu"]
+SOURCES = ["smem_capi.cpp", "smem_copy.cu", "smem_decode.cu", "smem_layer.cu", "smem_prefill.cu"]
 HEADERS = ["smem_device.cuh", "smem_internal.h", "smem_tc.cuh"]
 
 
@@ -76,7 +76,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
                 print(log)
     tmp = LIB + f".tmp{os.getpid()}"
     cmd = [nvcc, "-shared", "-o", tmp] + [o for o, _ in results] + ARCH + [
-        "-cudart", "shared", "-Xlinker", f"-rpath,{_cuda_lib_dir(nvcc)}"]
+        "-cudart", "shared", "-lcublas", "-Xlinker", f"-rpath,{_cuda_lib_dir(nvcc)}"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -39,6 +39,8 @@ struct smem_cache {
   uint32_t seen_epoch = 0;
   int fail_after = 0;                      // test hook: n-th next launch fails
   int pf_cluster_max = 0;                  // prefill cluster limit on this device (0: no clusters)
+  void* blas = nullptr;                    // cuBLAS handle of the reader-layer calls (created on first use)
+  ~smem_cache() { smem::blas_destroy(blas); }
 };
 
 namespace {
@@ -150,6 +152,201 @@ inline uint16_t* inblock_layer(smem_cache* c, int seq, int layer) {
 }
 inline const uint16_t* null_kv(smem_cache* c) {
   return c->lay.has_null ? reinterpret_cast<const uint16_t*>(c->dev + c->lay.off_null) : nullptr;
+}
+
+// Workspace of a reader-layer call over n rows (offsets from the caller's
+// 256-byte aligned buffer): cuBLAS workspace, then bf16 h [n][d], qkv
+// [n][3d], att [n][d], qc [n][d], fp32 f [n][4d], bf16 g [n][4d].
+struct LayerWs {
+  size_t blas, h, qkv, att, qc, f, g, total;
+};
+
+LayerWs layer_ws(const Layout& L, int n) {
+  const size_t d = (size_t)L.H * L.D;
+  LayerWs w{};
+  size_t off = 0;
+  w.blas = off;
+  off += smem::kBlasWorkspaceBytes;
+  w.h = off;
+  off = align_up(off + (size_t)n * d * 2, 256);
+  w.qkv = off;
+  off = align_up(off + (size_t)n * 3 * d * 2, 256);
+  w.att = off;
+  off = align_up(off + (size_t)n * d * 2, 256);
+  w.qc = off;
+  off = align_up(off + (size_t)n * d * 2, 256);
+  w.f = off;
+  off = align_up(off + (size_t)n * 4 * d * 4, 256);
+  w.g = off;
+  off = align_up(off + (size_t)n * 4 * d * 2, 256);
+  w.total = off;
+  return w;
+}
+
+int layer_rows_max(const Layout& L) { return std::max(smem::kBlockTok, L.max_batch); }
+
+// Checks the workspace and binds cuBLAS to it and the stream (creating the
+// handle on first use).
+int layer_begin(smem_cache* c, void* ws, size_t ws_bytes, int n_rows, cudaStream_t st) {
+  if (!ws) return SMEM_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(ws) & 255u) return SMEM_ERR_ALIGN;
+  if (ws_bytes < layer_ws(c->lay, n_rows).total) return SMEM_ERR_INVALID_ARG;
+  if (!c->blas && smem::blas_create(&c->blas, g_detail, sizeof(g_detail))) return SMEM_ERR_CUDA;
+  if (smem::blas_bind(c->blas, st, ws, smem::kBlasWorkspaceBytes, g_detail, sizeof(g_detail))) return SMEM_ERR_CUDA;
+  return SMEM_OK;
+}
+
+bool ok16(const void* p) { return p && aligned16(p); }
+
+// The fields of one layer's weights a call reads: all (full layer) or only
+// the memory key/value maps.
+int check_weights(const smem_layer_weights* w, bool full) {
+  if (!w) return SMEM_ERR_INVALID_ARG;
+  const void* kv[2] = {w->w_kc, w->w_vc};
+  for (const void* p : kv)
+    if (!p) return SMEM_ERR_INVALID_ARG;
+  for (const void* p : kv)
+    if (!aligned16(p)) return SMEM_ERR_ALIGN;
+  if (!full) return SMEM_OK;
+  const void* all[14] = {w->ln1_g, w->ln1_b, w->w_qkv, w->w_os, w->ln2_g, w->ln2_b, w->w_qc,
+                         w->w_oc, w->ln3_g, w->ln3_b, w->w_1,  w->w_2,  w->w_kc, w->w_vc};
+  for (const void* p : all)
+    if (!p) return SMEM_ERR_INVALID_ARG;
+  for (const void* p : all)
+    if (!aligned16(p)) return SMEM_ERR_ALIGN;
+  return SMEM_OK;
+}
+
+int cuda_rc(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return SMEM_OK;
+  set_detail(what, e);
+  return SMEM_ERR_CUDA;
+}
+
+inline int blas_rc(int r) { return r ? SMEM_ERR_CUDA : SMEM_OK; }
+
+// One-block attention of one layer (arguments validated by the caller).
+// mode bit 0: self-attention, bit 1: cross-attention; tok_s, tok_c: token
+// strides (elements) of Qs/Ks/Vs and of Qc, 0 for H*D.
+int prefill_impl(smem_cache* c, int seq, int layer, int q_block_idx, const void* Qs, const void* Ks, const void* Vs,
+                 const void* Qc, void* Osa, void* Oca, int mode, int tok_s, int tok_c, cudaStream_t st) {
+  const std::vector<int32_t>& ix = c->idx[seq];
+  const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx) - ix.begin());
+  smem::PrefillArgs a{};
+  a.pool_map = &c->pool_map_pf;
+  a.pool = reinterpret_cast<const uint16_t*>(c->dev + c->lay.off_pool);
+  a.table_row = table_row(c, seq);
+  a.null_kv = null_kv(c);
+  a.qs = static_cast<const uint16_t*>(Qs);
+  a.ks = static_cast<const uint16_t*>(Ks);
+  a.vs = static_cast<const uint16_t*>(Vs);
+  a.qc = static_cast<const uint16_t*>(Qc);
+  a.osa = static_cast<uint16_t*>(Osa);
+  a.oca = static_cast<uint16_t*>(Oca);
+  a.part = reinterpret_cast<float*>(c->dev + c->lay.off_pf_part);
+  a.counters = reinterpret_cast<unsigned*>(c->dev + c->lay.off_pf_cnt);
+  a.err = reinterpret_cast<int*>(c->dev + c->lay.off_err);
+  a.slot_elems = (long long)c->lay.slot_elems;
+  a.L = c->lay.L;
+  a.H = c->lay.H;
+  a.D = c->lay.D;
+  a.layer = layer;
+  a.nblk = nblk;
+  a.cluster = smem::prefill_use_clusters(nblk, c->pf_cluster_max) ? 1 : 0;
+  if (a.cluster)
+    a.split_blks = nblk ? smem::prefill_cluster_split_blocks(nblk, c->pf_cluster_max) : 1;
+  else
+    a.split_blks = nblk ? smem::prefill_split_blocks(nblk, c->lay.H, c->lay.D) : 1;
+  a.n_splits = nblk ? smem::ceil_div(nblk, a.split_blks) : 0;
+  a.capacity = c->lay.capacity;
+  a.mode = mode;
+  a.tok_s = tok_s;
+  a.tok_c = tok_c;
+  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->lay.D));
+  if (injected_failure(c)) return SMEM_ERR_CUDA;
+  return check_launch(c, smem::launch_prefill(a, st), "prefill");
+}
+
+// Host-side checks of a decode step (shared by every decode entry point).
+int check_decode_args(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const int32_t* pos,
+                      const int32_t* q_block_idx) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  const Layout& L = c->lay;
+  if (layer < 0 || layer >= L.L || nb < 1 || nb > L.max_batch) return SMEM_ERR_INVALID_ARG;
+  if (!seq_ids || !pos || !q_block_idx) return SMEM_ERR_INVALID_ARG;
+  if (++c->seen_epoch == 0) {
+    std::fill(c->seen.begin(), c->seen.end(), 0u);
+    c->seen_epoch = 1;
+  }
+  for (int i = 0; i < nb; ++i) {
+    const int s = seq_ids[i];
+    if (s < 0 || s >= L.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
+    if (c->seen[s] == c->seen_epoch) return SMEM_ERR_INVALID_ARG;  // one token per sequence per step
+    c->seen[s] = c->seen_epoch;
+    if (pos[i] < 0 || pos[i] >= smem::kBlockTok || q_block_idx[i] < 0) return SMEM_ERR_INVALID_ARG;
+  }
+  return SMEM_OK;
+}
+
+// One decode step of one layer (arguments validated by the caller). mode as
+// in prefill_impl; s_stride, c_stride: elements between items of
+// qs/k_new/v_new and of qc. Outputs are [nb][H][D].
+int decode_impl(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const int32_t* pos,
+                const int32_t* q_block_idx, const void* qs, const void* k_new, const void* v_new, const void* qc,
+                void* osa, void* oca, int mode, int s_stride, int c_stride, cudaStream_t st) {
+  const Layout& L = c->lay;
+  const size_t tok = (size_t)L.H * L.D;  // output elements per item
+  static thread_local smem::DecodeParams P;
+  for (int i0 = 0; i0 < nb; i0 += smem::kMaxDecodeItems) {
+    const int n = std::min(nb - i0, smem::kMaxDecodeItems);
+    P.tmap = c->pool_map;
+    P.pool = reinterpret_cast<const uint16_t*>(c->dev + L.off_pool);
+    P.inblock = reinterpret_cast<uint16_t*>(c->dev + L.off_inblock);
+    P.table = reinterpret_cast<const int*>(c->dev + L.off_table);
+    P.null_kv = null_kv(c);
+    P.part = reinterpret_cast<float*>(c->dev + L.off_dec_part);
+    P.counters = reinterpret_cast<unsigned*>(c->dev + L.off_dec_cnt);
+    P.sched = reinterpret_cast<unsigned long long*>(c->dev + L.off_dec_cnt +
+                                                    ((size_t)L.max_batch * L.H * 4 + 15) / 16 * 16);
+    P.err = reinterpret_cast<int*>(c->dev + L.off_err);
+    P.qs = static_cast<const uint16_t*>(qs) + (size_t)i0 * s_stride;
+    P.k_new = static_cast<const uint16_t*>(k_new) + (size_t)i0 * s_stride;
+    P.v_new = static_cast<const uint16_t*>(v_new) + (size_t)i0 * s_stride;
+    P.qc = static_cast<const uint16_t*>(qc) + (size_t)i0 * c_stride;
+    P.osa = static_cast<uint16_t*>(osa) + i0 * tok;
+    P.oca = static_cast<uint16_t*>(oca) + i0 * tok;
+    P.slot_elems = (long long)L.slot_elems;
+    P.L = L.L;
+    P.H = L.H;
+    P.layer = layer;
+    P.max_blocks = L.max_blocks;
+    P.capacity = L.capacity;
+    P.n_items = n;
+    P.mode = mode;
+    P.s_stride = s_stride;
+    P.c_stride = c_stride;
+    P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
+    int pairs = 0;
+    for (int i = 0; i < n; ++i) {
+      const int s = seq_ids[i0 + i];
+      const std::vector<int32_t>& ix = c->idx[s];
+      const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx[i0 + i]) - ix.begin());
+      P.items[i].seq = s;
+      P.items[i].nblk = nblk;
+      P.items[i].pos = pos[i0 + i];
+      P.items[i].pair_begin = pairs;
+      if (nblk && (mode & 2)) pairs += smem::ceil_div(nblk, smem::decode_split_blocks(nblk));
+    }
+    P.n_pairs = pairs;
+    const long long units = (long long)(pairs + n) * L.H;
+    const long long wpc = smem::decode_warps_per_cta();
+    const int grid = (int)std::min<long long>((units + wpc - 1) / wpc, smem::decode_max_grid(L.D, c->num_sms));
+    if (injected_failure(c)) return SMEM_ERR_CUDA;
+    const int rc = check_launch(c, smem::launch_decode(P, L.D, grid, st), "decode");
+    if (rc) return rc;
+  }
+  return SMEM_OK;
 }
 
 }  // namespace
@@ -338,114 +535,24 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
     if (!p) return SMEM_ERR_INVALID_ARG;
     if (!aligned16(p)) return SMEM_ERR_ALIGN;
   }
-  const std::vector<int32_t>& ix = c->idx[seq];
-  const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx) - ix.begin());
-  smem::PrefillArgs a{};
-  a.pool_map = &c->pool_map_pf;
-  a.pool = reinterpret_cast<const uint16_t*>(c->dev + c->lay.off_pool);
-  a.table_row = table_row(c, seq);
-  a.null_kv = null_kv(c);
-  a.qs = static_cast<const uint16_t*>(Qs);
-  a.ks = static_cast<const uint16_t*>(Ks);
-  a.vs = static_cast<const uint16_t*>(Vs);
-  a.qc = static_cast<const uint16_t*>(Qc);
-  a.osa = static_cast<uint16_t*>(Osa);
-  a.oca = static_cast<uint16_t*>(Oca);
-  a.part = reinterpret_cast<float*>(c->dev + c->lay.off_pf_part);
-  a.counters = reinterpret_cast<unsigned*>(c->dev + c->lay.off_pf_cnt);
-  a.err = reinterpret_cast<int*>(c->dev + c->lay.off_err);
-  a.slot_elems = (long long)c->lay.slot_elems;
-  a.L = c->lay.L;
-  a.H = c->lay.H;
-  a.D = c->lay.D;
-  a.layer = layer;
-  a.nblk = nblk;
-  a.cluster = smem::prefill_use_clusters(nblk, c->pf_cluster_max) ? 1 : 0;
-  if (a.cluster)
-    a.split_blks = nblk ? smem::prefill_cluster_split_blocks(nblk, c->pf_cluster_max) : 1;
-  else
-    a.split_blks = nblk ? smem::prefill_split_blocks(nblk, c->lay.H, c->lay.D) : 1;
-  a.n_splits = nblk ? smem::ceil_div(nblk, a.split_blks) : 0;
-  a.capacity = c->lay.capacity;
-  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->lay.D));
   DeviceGuard g(c->device);
-  if (injected_failure(c)) return SMEM_ERR_CUDA;
-  return check_launch(c, smem::launch_prefill(a, as_stream(stream)), "prefill");
+  return prefill_impl(c, seq, layer, q_block_idx, Qs, Ks, Vs, Qc, Osa, Oca, 3, 0, 0, as_stream(stream));
 }
 
 int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,
                 const int32_t* q_block_idx, const void* qs, const void* k_new, const void* v_new, const void* qc,
                 void* osa, void* oca, void* stream) {
-  if (!c) return SMEM_ERR_INVALID_ARG;
-  if (!c->dev) return SMEM_ERR_NO_DEVICE;
-  const Layout& L = c->lay;
-  if (layer < 0 || layer >= L.L || nb < 1 || nb > L.max_batch) return SMEM_ERR_INVALID_ARG;
-  if (!seq_ids || !pos || !q_block_idx) return SMEM_ERR_INVALID_ARG;
+  const int rc = check_decode_args(c, layer, nb, seq_ids, pos, q_block_idx);
+  if (rc) return rc;
   const void* ptrs[6] = {qs, k_new, v_new, qc, osa, oca};
   for (const void* p : ptrs) {
     if (!p) return SMEM_ERR_INVALID_ARG;
     if (!aligned16(p)) return SMEM_ERR_ALIGN;
   }
-  if (++c->seen_epoch == 0) {
-    std::fill(c->seen.begin(), c->seen.end(), 0u);
-    c->seen_epoch = 1;
-  }
-  for (int i = 0; i < nb; ++i) {
-    const int s = seq_ids[i];
-    if (s < 0 || s >= L.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
-    if (c->seen[s] == c->seen_epoch) return SMEM_ERR_INVALID_ARG;  // one token per sequence per step
-    c->seen[s] = c->seen_epoch;
-    if (pos[i] < 0 || pos[i] >= smem::kBlockTok || q_block_idx[i] < 0) return SMEM_ERR_INVALID_ARG;
-  }
   DeviceGuard g(c->device);
-  const size_t tok = (size_t)L.H * L.D;  // elements per item
-  static thread_local smem::DecodeParams P;
-  for (int i0 = 0; i0 < nb; i0 += smem::kMaxDecodeItems) {
-    const int n = std::min(nb - i0, smem::kMaxDecodeItems);
-    P.tmap = c->pool_map;
-    P.pool = reinterpret_cast<const uint16_t*>(c->dev + L.off_pool);
-    P.inblock = reinterpret_cast<uint16_t*>(c->dev + L.off_inblock);
-    P.table = reinterpret_cast<const int*>(c->dev + L.off_table);
-    P.null_kv = null_kv(c);
-    P.part = reinterpret_cast<float*>(c->dev + L.off_dec_part);
-    P.counters = reinterpret_cast<unsigned*>(c->dev + L.off_dec_cnt);
-    P.sched = reinterpret_cast<unsigned long long*>(c->dev + L.off_dec_cnt +
-                                                    ((size_t)L.max_batch * L.H * 4 + 15) / 16 * 16);
-    P.err = reinterpret_cast<int*>(c->dev + L.off_err);
-    P.qs = static_cast<const uint16_t*>(qs) + i0 * tok;
-    P.k_new = static_cast<const uint16_t*>(k_new) + i0 * tok;
-    P.v_new = static_cast<const uint16_t*>(v_new) + i0 * tok;
-    P.qc = static_cast<const uint16_t*>(qc) + i0 * tok;
-    P.osa = static_cast<uint16_t*>(osa) + i0 * tok;
-    P.oca = static_cast<uint16_t*>(oca) + i0 * tok;
-    P.slot_elems = (long long)L.slot_elems;
-    P.L = L.L;
-    P.H = L.H;
-    P.layer = layer;
-    P.max_blocks = L.max_blocks;
-    P.capacity = L.capacity;
-    P.n_items = n;
-    P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
-    int pairs = 0;
-    for (int i = 0; i < n; ++i) {
-      const int s = seq_ids[i0 + i];
-      const std::vector<int32_t>& ix = c->idx[s];
-      const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx[i0 + i]) - ix.begin());
-      P.items[i].seq = s;
-      P.items[i].nblk = nblk;
-      P.items[i].pos = pos[i0 + i];
-      P.items[i].pair_begin = pairs;
-      if (nblk) pairs += smem::ceil_div(nblk, smem::decode_split_blocks(nblk));
-    }
-    P.n_pairs = pairs;
-    const long long units = (long long)(pairs + n) * L.H;
-    const long long wpc = smem::decode_warps_per_cta();
-    const int grid = (int)std::min<long long>((units + wpc - 1) / wpc, smem::decode_max_grid(L.D, c->num_sms));
-    if (injected_failure(c)) return SMEM_ERR_CUDA;
-    const int rc = check_launch(c, smem::launch_decode(P, L.D, grid, as_stream(stream)), "decode");
-    if (rc) return rc;
-  }
-  return SMEM_OK;
+  const int tok = c->lay.H * c->lay.D;
+  return decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, qs, k_new, v_new, qc, osa, oca, 3, tok, tok,
+                     as_stream(stream));
 }
 
 int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,
@@ -523,6 +630,8 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     P.max_blocks = L.max_blocks;
     P.capacity = L.capacity;
     P.n_items = n;
+    P.mode = 3;
+    P.s_stride = P.c_stride = L.H * L.D;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
     int pairs = 0;
     for (int i = 0; i < n; ++i) {
@@ -545,6 +654,193 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     if (rc) return rc;
   }
   return SMEM_OK;
+}
+
+// ---------------------------------------------------------------------------
+// reader layer
+// ---------------------------------------------------------------------------
+size_t smem_layer_workspace_bytes(const smem_cache* c, int32_t n_rows) {
+  if (!c || n_rows < 0 || n_rows > layer_rows_max(c->lay)) return 0;
+  return layer_ws(c->lay, n_rows).total;
+}
+
+int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const void* mu,
+                           const smem_layer_weights* w, void* ws, size_t ws_bytes, void* stream, int32_t* slot_out) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
+  if (block_idx < 0 || !mu || !w) return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(mu)) return SMEM_ERR_ALIGN;
+  const Layout& L = c->lay;
+  for (int l = 0; l < L.L; ++l) {
+    const int rc = check_weights(&w[l], false);
+    if (rc) return rc;
+  }
+  std::vector<int32_t>& ix = c->idx[seq];
+  const auto it = std::lower_bound(ix.begin(), ix.end(), block_idx);
+  const int pos = (int)(it - ix.begin());
+  if (it != ix.end() && *it == block_idx) return SMEM_ERR_DUPLICATE_BLOCK;
+  if ((int)ix.size() >= L.max_blocks) return SMEM_ERR_TABLE_FULL;
+  if (c->fifo.empty()) return SMEM_ERR_POOL_FULL;
+  DeviceGuard g(c->device);
+  const cudaStream_t st = as_stream(stream);
+  int rc = layer_begin(c, ws, ws_bytes, 0, st);
+  if (rc) return rc;
+  if (injected_failure(c)) return SMEM_ERR_CUDA;
+  const int32_t s = c->fifo.front();
+  // the slot is still free: a failure below leaves only a free slot's rows written
+  uint16_t* slot = pool_slot(c, s);
+  const int d = L.H * L.D;
+  const size_t head_stride = (size_t)2 * smem::kRows * L.D;
+  for (int l = 0; l < L.L && !rc; ++l)
+    for (int kv = 0; kv < 2 && !rc; ++kv)
+      rc = blas_rc(smem::blas_project_heads(c->blas, smem::kRows, d, L.H, L.D, static_cast<const uint16_t*>(mu),
+                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc),
+                                            slot + ((size_t)l * L.H * 2 + kv) * smem::kRows * L.D,
+                                            (long long)head_stride, g_detail, sizeof(g_detail)));
+  if (!rc) rc = cuda_rc(smem::launch_table_insert(table_row(c, seq), pos, (int)ix.size(), s, st), "append rows");
+  if (rc) return rc;
+  c->fifo.pop_front();
+  ix.insert(ix.begin() + pos, block_idx);
+  c->slot[seq].insert(c->slot[seq].begin() + pos, s);
+  if (slot_out) *slot_out = s;
+  return SMEM_OK;
+}
+
+int smem_set_null_vector(smem_cache* c, const void* nu, const smem_layer_weights* w, void* ws, size_t ws_bytes,
+                         void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  const Layout& L = c->lay;
+  if (!L.has_null || !nu || !w) return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(nu)) return SMEM_ERR_ALIGN;
+  for (int l = 0; l < L.L; ++l) {
+    const int rc = check_weights(&w[l], false);
+    if (rc) return rc;
+  }
+  DeviceGuard g(c->device);
+  int rc = layer_begin(c, ws, ws_bytes, 0, as_stream(stream));
+  if (rc) return rc;
+  if (injected_failure(c)) return SMEM_ERR_CUDA;
+  uint16_t* nk = reinterpret_cast<uint16_t*>(c->dev + L.off_null);
+  const int d = L.H * L.D;
+  for (int l = 0; l < L.L && !rc; ++l)
+    for (int kv = 0; kv < 2 && !rc; ++kv)
+      rc = blas_rc(smem::blas_project_heads(c->blas, 1, d, L.H, L.D, static_cast<const uint16_t*>(nu),
+                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc),
+                                            nk + ((size_t)l * L.H * 2 + kv) * L.D, (long long)2 * L.D, g_detail,
+                                            sizeof(g_detail)));
+  return rc;
+}
+
+namespace {
+
+// The dense tail shared by prefill and decode layers: after the attention
+// outputs are in place, x += att W_o etc. Steps are issued in the layer's
+// order on one stream.
+struct LayerRun {
+  smem_cache* c;
+  const smem_layer_weights* w;
+  float* x;
+  uint8_t* ws;
+  LayerWs o;
+  int n, d;
+  cudaStream_t st;
+  uint16_t* h() const { return reinterpret_cast<uint16_t*>(ws + o.h); }
+  uint16_t* qkv() const { return reinterpret_cast<uint16_t*>(ws + o.qkv); }
+  uint16_t* att() const { return reinterpret_cast<uint16_t*>(ws + o.att); }
+  uint16_t* qc() const { return reinterpret_cast<uint16_t*>(ws + o.qc); }
+  float* f() const { return reinterpret_cast<float*>(ws + o.f); }
+  uint16_t* g() const { return reinterpret_cast<uint16_t*>(ws + o.g); }
+  int ln(const float* gain, const float* bias) {
+    return cuda_rc(smem::launch_layernorm(x, n, d, gain, bias, smem::kLayerNormEps, h(), st), "layernorm");
+  }
+  int gemm(int cols, int k, const uint16_t* A, const void* W, void* C, bool f32, bool acc) {
+    return blas_rc(smem::blas_gemm(c->blas, n, cols, k, A, static_cast<const uint16_t*>(W), C, f32, acc, g_detail,
+                                   sizeof(g_detail)));
+  }
+  // h1 = LN1(x); qkv = h1 W_qkv
+  int qkv_proj() {
+    int rc = ln(w->ln1_g, w->ln1_b);
+    return rc ? rc : gemm(3 * d, d, h(), w->w_qkv, qkv(), false, false);
+  }
+  // x += att W_os; h2 = LN2(x); qc = h2 W_qc
+  int after_sa() {
+    int rc = gemm(d, d, att(), w->w_os, x, true, true);
+    if (!rc) rc = ln(w->ln2_g, w->ln2_b);
+    return rc ? rc : gemm(d, d, h(), w->w_qc, qc(), false, false);
+  }
+  // x += att W_oc; x += GELU(LN3(x) W_1) W_2
+  int after_ca() {
+    int rc = gemm(d, d, att(), w->w_oc, x, true, true);
+    if (!rc) rc = ln(w->ln3_g, w->ln3_b);
+    if (!rc) rc = gemm(4 * d, d, h(), w->w_1, f(), true, false);
+    if (!rc) rc = cuda_rc(smem::launch_gelu(f(), g(), (long long)n * 4 * d, st), "gelu");
+    return rc ? rc : gemm(d, 4 * d, g(), w->w_2, x, true, true);
+  }
+};
+
+}  // namespace
+
+int smem_reader_layer_prefill(smem_cache* c, int32_t seq, int32_t layer, int32_t q_block_idx,
+                              const smem_layer_weights* w, float* x, void* ws, size_t ws_bytes, void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
+  if (layer < 0 || layer >= c->lay.L || q_block_idx < 0 || !x) return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(x)) return SMEM_ERR_ALIGN;
+  int rc = check_weights(w, true);
+  if (rc) return rc;
+  DeviceGuard g(c->device);
+  const cudaStream_t st = as_stream(stream);
+  const int n = smem::kBlockTok;
+  rc = layer_begin(c, ws, ws_bytes, n, st);
+  if (rc) return rc;
+  const Layout& L = c->lay;
+  LayerRun r{c, w, x, static_cast<uint8_t*>(ws), layer_ws(L, n), n, L.H * L.D, st};
+  const int d = r.d;
+  rc = r.qkv_proj();
+  // the block's self-attention keys/values become its in-block rows
+  if (!rc)
+    rc = cuda_rc(smem::launch_inblock_write(inblock_layer(c, seq, layer), r.qkv() + d, r.qkv() + 2 * d, n, L.H, L.D,
+                                            st, 3 * d),
+                 "in-block write");
+  if (!rc)
+    rc = prefill_impl(c, seq, layer, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + 2 * d, r.qkv(), r.att(), r.att(), 1,
+                      3 * d, 3 * d, st);
+  if (!rc) rc = r.after_sa();
+  if (!rc)
+    rc = prefill_impl(c, seq, layer, q_block_idx, r.qc(), r.qc(), r.qc(), r.qc(), r.att(), r.att(), 2, d, d, st);
+  if (!rc) rc = r.after_ca();
+  return rc;
+}
+
+int smem_reader_layer_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,
+                             const int32_t* q_block_idx, const smem_layer_weights* w, float* x, void* ws,
+                             size_t ws_bytes, void* stream) {
+  int rc = check_decode_args(c, layer, nb, seq_ids, pos, q_block_idx);
+  if (rc) return rc;
+  if (!x) return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(x)) return SMEM_ERR_ALIGN;
+  rc = check_weights(w, true);
+  if (rc) return rc;
+  DeviceGuard g(c->device);
+  const cudaStream_t st = as_stream(stream);
+  rc = layer_begin(c, ws, ws_bytes, nb, st);
+  if (rc) return rc;
+  const Layout& L = c->lay;
+  LayerRun r{c, w, x, static_cast<uint8_t*>(ws), layer_ws(L, nb), nb, L.H * L.D, st};
+  const int d = r.d;
+  rc = r.qkv_proj();
+  if (!rc)
+    rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + 2 * d, r.qkv(), r.att(),
+                     r.att(), 1, 3 * d, 3 * d, st);
+  if (!rc) rc = r.after_sa();
+  if (!rc)
+    rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qc(), r.qc(), r.qc(), r.qc(), r.att(), r.att(), 2, d,
+                     d, st);
+  if (!rc) rc = r.after_ca();
+  return rc;
 }
 
 int smem_get_table(const smem_cache* c, int32_t seq, int32_t* idx_out, int32_t* slot_out, int32_t cap,

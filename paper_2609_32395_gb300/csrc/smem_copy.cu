@@ -69,8 +69,9 @@ __global__ void __launch_bounds__(kCopyThreads) table_remove_kernel(int* row, in
   table_remove_cta(row, pos, n);
 }
 
-// rows [n][H][D] (K and V) -> in-block layout [H][2][b][D] of one layer
-__global__ void inblock_write_kernel(uint4* ib, const uint4* K, const uint4* V, int n, int H, int cpr) {
+// rows [n][H][D] (K and V, token stride `tok16` chunks of 16 bytes) ->
+// in-block layout [H][2][b][D] of one layer
+__global__ void inblock_write_kernel(uint4* ib, const uint4* K, const uint4* V, int n, int H, int cpr, int tok16) {
   const int total = 2 * n * H * cpr;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
     const int kv = i >= n * H * cpr;
@@ -78,7 +79,8 @@ __global__ void inblock_write_kernel(uint4* ib, const uint4* K, const uint4* V, 
     const int t = j / (H * cpr);
     const int h = (j / cpr) % H;
     const int c = j % cpr;
-    ib[((h * 2 + kv) * kBlockTok + t) * cpr + c] = kv ? V[j] : K[j];
+    const size_t src = (size_t)t * tok16 + (size_t)h * cpr + c;
+    ib[((h * 2 + kv) * kBlockTok + t) * cpr + c] = kv ? V[src] : K[src];
   }
 }
 
@@ -111,20 +113,26 @@ cudaError_t launch_append(uint16_t* slot_base, const uint16_t* K, const uint16_t
   return cudaGetLastError();
 }
 
+cudaError_t launch_table_insert(int* table_row, int pos, int n_old, int slot, cudaStream_t st) {
+  append_kernel<<<1, kCopyThreads, 0, st>>>(nullptr, nullptr, nullptr, 0, 0, table_row, pos, n_old, slot, 0);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_table_remove(int* table_row, int pos, int n_old, cudaStream_t st) {
   table_remove_kernel<<<1, kCopyThreads, 0, st>>>(table_row, pos, n_old);
   return cudaGetLastError();
 }
 
 cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
-                                 int D, cudaStream_t st) {
+                                 int D, cudaStream_t st, int tok) {
   if (n == 0) return cudaSuccess;
   const int cpr = D * 2 / 16;
+  const int tok16 = (tok ? tok : H * D) * 2 / 16;
   const int total = 2 * n * H * cpr;
   const int blocks = (total + 255) / 256;
   inblock_write_kernel<<<blocks, 256, 0, st>>>(reinterpret_cast<uint4*>(ib_layer_base),
                                                reinterpret_cast<const uint4*>(K),
-                                               reinterpret_cast<const uint4*>(V), n, H, cpr);
+                                               reinterpret_cast<const uint4*>(V), n, H, cpr, tok16);
   return cudaGetLastError();
 }
 

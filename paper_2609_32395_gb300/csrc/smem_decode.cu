@@ -184,7 +184,7 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
       tma_load_3d(stage + bx * C::BOX_BYTES, &p.tmap, bx * 64, y, slot, bar);
       tma_load_3d(stage + C::HALF + bx * C::BOX_BYTES, &p.tmap, bx * 64, y + C::R, slot, bar);
     }
-    if (qbytes) bulk_g2s(qslot, p.qc + ((size_t)is.item * p.H + is.h) * D, qbytes, bar);
+    if (qbytes) bulk_g2s(qslot, p.qc + (size_t)is.item * p.c_stride + (size_t)is.h * D, qbytes, bar);
   }
   if (++is.c == is.nc) issue_begin_unit<D>(p, is, is.next_u, uq);
   return true;
@@ -199,85 +199,88 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
   constexpr int RPP = 32 / LPR;  // rows per pass
   const DecodeItem& it = p.items[U.item];
   const int n = it.pos + 1;
-  const size_t qoff = ((size_t)U.item * p.H + U.h) * D;
+  const size_t qoff = ((size_t)U.item * p.H + U.h) * D;           // outputs
+  const size_t soff = (size_t)U.item * p.s_stride + (size_t)U.h * D;  // qs, k_new, v_new
   const uint16_t* ib = p.inblock + (((size_t)it.seq * p.L + p.layer) * p.H + U.h) * (size_t)2 * kBlockTok * D;
   const int hh = lane % LPR;  // which 64 columns of the row
-  float q[64];
+  if (p.mode & 1) {
+    float q[64];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    float t[8];
-    unpack8(ld_nc16(p.qs + qoff + hh * 64 + j * 8), t);
+    for (int j = 0; j < 8; ++j) {
+      float t[8];
+      unpack8(ld_nc16(p.qs + soff + hh * 64 + j * 8), t);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
-  }
-  // scores of rows lane/LPR + k*RPP
-  float s[kBlockTok / RPP];
-  float mx = -INFINITY;
+      for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
+    }
+    // scores of rows lane/LPR + k*RPP
+    float s[kBlockTok / RPP];
+    float mx = -INFINITY;
 #pragma unroll
-  for (int k = 0; k < kBlockTok / RPP; ++k) {
-    const int r = k * RPP + lane / LPR;
-    float dot = 0.f;
-    if (r < n) {
-      const uint16_t* row = r == it.pos ? p.k_new + qoff : ib + (size_t)r * D;
+    for (int k = 0; k < kBlockTok / RPP; ++k) {
+      const int r = k * RPP + lane / LPR;
+      float dot = 0.f;
+      if (r < n) {
+        const uint16_t* row = r == it.pos ? p.k_new + soff : ib + (size_t)r * D;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        float t[8];
-        unpack8(ld_nc16(row + hh * 64 + j * 8), t);
+        for (int j = 0; j < 8; ++j) {
+          float t[8];
+          unpack8(ld_nc16(row + hh * 64 + j * 8), t);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
+          for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
+        }
+      }
+      if (LPR == 2) dot += __shfl_xor_sync(0xffffffffu, dot, 1);
+      s[k] = r < n ? dot : -INFINITY;
+      mx = fmaxf(mx, s[k]);
+    }
+#pragma unroll
+    for (int o = LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float l = 0.f;
+#pragma unroll
+    for (int k = 0; k < kBlockTok / RPP; ++k) {
+      const int r = k * RPP + lane / LPR;
+      const float pr = r < n ? exp2f(s[k] - mx) : 0.f;
+      if (hh == 0) {
+        l += pr;
+        pbuf[r] = pr;
       }
     }
-    if (LPR == 2) dot += __shfl_xor_sync(0xffffffffu, dot, 1);
-    s[k] = r < n ? dot : -INFINITY;
-    mx = fmaxf(mx, s[k]);
-  }
+    __syncwarp();
 #pragma unroll
-  for (int o = LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  float l = 0.f;
+    for (int o = 1; o < 32; o <<= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    // P.V: lane (g, c) owns column chunk c of rows g*RG .. g*RG+RG-1
+    constexpr int CPL = D / 8;        // column chunks
+    constexpr int G = 32 / CPL;       // row groups
+    constexpr int RG = kBlockTok / G; // rows per group
+    const int g = lane / CPL, c = lane % CPL;
+    float acc[8];
 #pragma unroll
-  for (int k = 0; k < kBlockTok / RPP; ++k) {
-    const int r = k * RPP + lane / LPR;
-    const float pr = r < n ? exp2f(s[k] - mx) : 0.f;
-    if (hh == 0) {
-      l += pr;
-      pbuf[r] = pr;
+    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+    for (int i = 0; i < RG; ++i) {
+      const int r = g * RG + i;
+      if (r < n) {
+        const float pr = pbuf[r];
+        const uint16_t* row = r == it.pos ? p.v_new + soff : ib + (size_t)kBlockTok * D + (size_t)r * D;
+        float t[8];
+        unpack8(ld_nc16(row + c * 8), t);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] = fmaf(pr, t[e], acc[e]);
+      }
     }
-  }
-  __syncwarp();
 #pragma unroll
-  for (int o = 1; o < 32; o <<= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-  // P.V: lane (g, c) owns column chunk c of rows g*RG .. g*RG+RG-1
-  constexpr int CPL = D / 8;        // column chunks
-  constexpr int G = 32 / CPL;       // row groups
-  constexpr int RG = kBlockTok / G; // rows per group
-  const int g = lane / CPL, c = lane % CPL;
-  float acc[8];
+    for (int o = CPL; o < 32; o <<= 1)
 #pragma unroll
-  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-  for (int i = 0; i < RG; ++i) {
-    const int r = g * RG + i;
-    if (r < n) {
-      const float pr = pbuf[r];
-      const uint16_t* row = r == it.pos ? p.v_new + qoff : ib + (size_t)kBlockTok * D + (size_t)r * D;
-      float t[8];
-      unpack8(ld_nc16(row + c * 8), t);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] = fmaf(pr, t[e], acc[e]);
+      for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
+    if (g == 0) store_bf16x8(p.osa + qoff + c * 8, acc, 1.f / l);
+    // the new token's k and v become in-block row p for later steps
+    if (lane < 2 * CPL) {
+      const int kv = lane / CPL, cc = lane % CPL;
+      uint16_t* dst = (uint16_t*)ib + (size_t)kv * kBlockTok * D + (size_t)it.pos * D + cc * 8;
+      *reinterpret_cast<uint4*>(dst) = ld_nc16((kv ? p.v_new : p.k_new) + soff + cc * 8);
     }
-  }
-#pragma unroll
-  for (int o = CPL; o < 32; o <<= 1)
-#pragma unroll
-    for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
-  if (g == 0) store_bf16x8(p.osa + qoff + c * 8, acc, 1.f / l);
-  // the new token's k and v become in-block row p for later steps
-  if (lane < 2 * CPL) {
-    const int kv = lane / CPL, cc = lane % CPL;
-    uint16_t* dst = (uint16_t*)ib + (size_t)kv * kBlockTok * D + (size_t)it.pos * D + cc * 8;
-    *reinterpret_cast<uint4*>(dst) = ld_nc16((kv ? p.v_new : p.k_new) + qoff + cc * 8);
-  }
+  }  // self-attention half
   // no readable memory block: oca is the null row's value or zero
-  if (it.nblk == 0 && lane < CPL) {
+  if ((p.mode & 2) && it.nblk == 0 && lane < D / 8) {
     float v[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) v[e] = 0.f;
@@ -300,6 +303,7 @@ template <int D>
 __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane) {
   constexpr int CPT = D / 32;  // columns per lane
   const size_t qoff = ((size_t)pd.item * p.H + pd.h) * D;
+  const size_t qcoff = (size_t)pd.item * p.c_stride + (size_t)pd.h * D;
   float nscore = -INFINITY;
   if (p.null_kv) {
     // null-row score with the same scaled-query dot product as the rows
@@ -307,7 +311,7 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
     float dot = 0.f;
 #pragma unroll
     for (int e = 0; e < CPT; ++e)
-      dot = fmaf(bf16lo(p.qc[qoff + lane * CPT + e]) * p.scale_log2, bf16lo(kn[lane * CPT + e]), dot);
+      dot = fmaf(bf16lo(p.qc[qcoff + lane * CPT + e]) * p.scale_log2, bf16lo(kn[lane * CPT + e]), dot);
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
     nscore = dot;

@@ -85,6 +85,8 @@ struct DecodeParams {
   long long slot_elems;      // elements per pool slot
   int L, H, layer, max_blocks, capacity;
   int n_items, n_pairs;      // items and CA (item, split) pairs in this launch
+  int mode;                  // bit 0: in-block self-attention, bit 1: cross-attention
+  int s_stride, c_stride;    // elements between items of qs/k_new/v_new and of qc
   float scale_log2;          // log2(e) / sqrt(D)
   DecodeItem items[kMaxDecodeItems];
 };
@@ -109,13 +111,36 @@ cudaError_t launch_append(uint16_t* slot_base, const uint16_t* K, const uint16_t
                           int* table_row, int pos, int n_old, int slot, cudaStream_t st);
 // Removes table position `pos` of a row holding n_old entries.
 cudaError_t launch_table_remove(int* table_row, int pos, int n_old, cudaStream_t st);
-// In-block write: rows [n][H][D] -> inblock[seq][layer][h][2][b][D].
+// In-block write: rows [n][H][D] (token stride `tok` elements, 0: H*D) ->
+// inblock[seq][layer][h][2][b][D].
 cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
-                                 int D, cudaStream_t st);
+                                 int D, cudaStream_t st, int tok = 0);
 // Null row: k,v [L][H][D] -> null_kv [L][H][2][D].
 cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
                               cudaStream_t st);
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st);
+
+// Table insert alone (the slot's rows written by other kernels before it).
+cudaError_t launch_table_insert(int* table_row, int pos, int n_old, int slot, cudaStream_t st);
+
+// ---------------------------------------------------------------------------
+// dense parts of the reader layer (LayerNorm, GELU, cuBLAS projections)
+// ---------------------------------------------------------------------------
+constexpr float kLayerNormEps = 1e-5f;
+constexpr size_t kBlasWorkspaceBytes = (size_t)32 << 20;
+// h [n][d] bf16 = LayerNorm(x [n][d] fp32) * g + b.
+cudaError_t launch_layernorm(const float* x, int n, int d, const float* g, const float* b, float eps, uint16_t* h,
+                             cudaStream_t st);
+// out [n] bf16 = GELU(f [n] fp32), n a multiple of 4.
+cudaError_t launch_gelu(const float* f, uint16_t* out, long long n, cudaStream_t st);
+// An opaque cuBLAS handle; nonzero return = failure, message in `detail`.
+int blas_create(void** out, char* detail, size_t detail_len);
+void blas_destroy(void* blas);
+int blas_bind(void* blas, cudaStream_t st, void* ws, size_t ws_bytes, char* detail, size_t detail_len);
+int blas_gemm(void* blas, int m, int n, int k, const uint16_t* A, const uint16_t* W, void* C, bool c_f32,
+              bool accumulate, char* detail, size_t detail_len);
+int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t* X, const uint16_t* W,
+                       uint16_t* out, long long head_stride, char* detail, size_t detail_len);
 
 // ---------------------------------------------------------------------------
 // prefill
@@ -133,6 +158,8 @@ struct PrefillArgs {
   long long slot_elems;
   int L, H, D, layer, nblk, split_blks, n_splits, capacity;
   int cluster;                // 1: cluster mode (one cluster of n_splits + 1 CTAs per head)
+  int mode;                   // bit 0: self-attention, bit 1: cross-attention (0: both)
+  int tok_s, tok_c;           // elements between tokens of Qs/Ks/Vs and of Qc (0: H*D)
   float scale_log2;
 };
 cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);

@@ -77,6 +77,9 @@ struct PrefillParams {
   unsigned* counters;
   int* err;
   int L, H, layer, nblk, split_blks, n_splits, capacity, max_splits;
+  int mode;            // bit 0: in-block self-attention, bit 1: cross-attention
+  int n_sa;            // self-attention CTAs of the cluster-free grid (0 or H)
+  int tok_c;           // elements between consecutive tokens of Qc
   float scale_log2;
 };
 
@@ -94,13 +97,14 @@ __device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint
   const int r0 = (int)rank * rp, r1 = min(kBlockTok, r0 + rp);
   for (int row = r0 + warp; row < r1; row += 6) {
     const size_t qoff = ((size_t)row * p.H + h) * D;
+    const size_t qcoff = (size_t)row * p.tok_c + (size_t)h * D;
     float nscore = -INFINITY;
     if (p.null_kv) {
       const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
       float dot = 0.f;
 #pragma unroll
       for (int e = 0; e < CPL; ++e)
-        dot = fmaf(bf16lo(p.qc_ptr[qoff + lane * CPL + e]), bf16lo(kn[lane * CPL + e]), dot);
+        dot = fmaf(bf16lo(p.qc_ptr[qcoff + lane * CPL + e]), bf16lo(kn[lane * CPL + e]), dot);
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
       nscore = dot * p.scale_log2;
@@ -181,12 +185,15 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   // their SMs early; in cluster mode a head is a cluster and rank 0 its SA
   const uint32_t cs = (uint32_t)p.n_splits + 1;
   const uint32_t crank = CL ? tc::cluster_ctarank() : 0u;
-  const bool sa = CL ? crank == 0 : (int)blockIdx.x < p.H;
-  const int cb = (int)blockIdx.x - p.H;
+  const bool sa = CL ? crank == 0 : (int)blockIdx.x < p.n_sa;
+  const int cb = (int)blockIdx.x - p.n_sa;
   const int h = CL ? (int)(blockIdx.x / cs) : (sa ? (int)blockIdx.x : cb % p.H);
   const int split = CL ? (int)crank - 1 : (sa ? 0 : cb / p.H);
   const int b0 = split * p.split_blks;
-  const int nt = sa ? 1 : min(p.split_blks, p.nblk - b0);
+  // an SA CTA without the SA half to do only joins the merge (cluster mode)
+  // or writes the empty-memory cross-attention output
+  const int nt = sa ? ((p.mode & 1) ? 1 : 0) : min(p.split_blks, p.nblk - b0);
+  const bool work = nt > 0;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
@@ -213,7 +220,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
 
   if (warp == 4) {
     // ------------------------------------------------------------ TMA producer
-    if (lane == 0) {
+    if (lane == 0 && work) {
       const CUtensorMap* qmap = sa ? &p.qs : &p.qc;
       mbar_arrive_expect_tx(q_full, C::TILE);
 #pragma unroll
@@ -259,7 +266,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------- MMA issuer
-    if (lane == 0) {
+    if (lane == 0 && work) {
       bool ok = mbar_wait_bounded(q_full, 0, abort_flag);
       tc::fence_after();
       const uint32_t qa = smem_u32(qt);
@@ -381,9 +388,10 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       *abort_flag = 1;
     }
     // ---------------------------------------------------------- epilogue
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait_bounded(&o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, abort_flag));
+    if (ok && work)
+      ok = __all_sync(0xffffffffu, mbar_wait_bounded(&o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, abort_flag));
     float o[D / 2];
-    if (ok) {
+    if (ok && work) {
       tc::fence_after();
 #pragma unroll
       for (int cb = 0; cb < D / 64; ++cb) {
@@ -397,7 +405,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
     const float lrow = l + __shfl_xor_sync(0xffffffffu, l, 16);
     const int col0 = hf * (D / 2);  // this thread's columns of O
     const bool direct = sa || (!CL && p.n_splits == 1 && !p.null_kv);
-    if (ok && direct) {
+    if (ok && direct && work) {
       uint16_t* out = (sa ? p.osa : p.oca) + ((size_t)r * p.H + h) * D + col0;
       const float inv = 1.f / lrow;
 #pragma unroll
@@ -410,7 +418,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         *reinterpret_cast<uint4*>(out + c) = w;
       }
     }
-    if (ok && sa && p.nblk == 0) {
+    if (ok && sa && p.nblk == 0 && (p.mode & 2)) {
       // no readable memory block: oca is the null row's value or zero
       uint16_t* out = p.oca + ((size_t)r * p.H + h) * D + col0;
       const uint16_t* vn = p.null_kv ? p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D + D + col0 : nullptr;
@@ -450,12 +458,13 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         __threadfence();
         // merge all splits of this head for row r, columns col0.., in split order
         const size_t qoff = ((size_t)r * p.H + h) * D;
+        const size_t qcoff = (size_t)r * p.tok_c + (size_t)h * D;
         float nscore = -INFINITY;
         if (p.null_kv) {
           const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
           float dot = 0.f;
           for (int c = 0; c < D / 2; ++c)
-            dot = fmaf(bf16lo(p.qc_ptr[qoff + col0 + c]), bf16lo(kn[col0 + c]), dot);
+            dot = fmaf(bf16lo(p.qc_ptr[qcoff + col0 + c]), bf16lo(kn[col0 + c]), dot);
           dot += __shfl_xor_sync(0xffffffffu, dot, 16);
           nscore = dot * p.scale_log2;
         }
@@ -623,7 +632,7 @@ int prefill_cluster_max(int H, int D) {
   return 0;
 }
 
-static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D) {
+static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D, int tok_stride) {
   static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
   if (!encode) {
     void* fn = nullptr;
@@ -634,7 +643,7 @@ static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D) {
     encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   }
   const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)kBlockTok};
-  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)tok_stride * 2};
   const cuuint32_t box[3] = {64, 1, (cuuint32_t)kBlockTok};
   const cuuint32_t estr[3] = {1, 1, 1};
   const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
@@ -646,9 +655,20 @@ static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D) {
 cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   static thread_local PrefillParams P;
   P.pool = *a.pool_map;
-  if (encode_bhd(&P.qs, a.qs, a.H, a.D) || encode_bhd(&P.ks, a.ks, a.H, a.D) || encode_bhd(&P.vs, a.vs, a.H, a.D) ||
-      encode_bhd(&P.qc, a.qc, a.H, a.D))
+  const int tok_s = a.tok_s ? a.tok_s : a.H * a.D;
+  const int tok_c = a.tok_c ? a.tok_c : a.H * a.D;
+  const int mode = a.mode ? a.mode : 3;
+  // a half that is not requested keeps a harmless map (its pointer is valid)
+  const void* qs = (mode & 1) ? a.qs : a.qc;
+  const void* ks = (mode & 1) ? a.ks : a.qc;
+  const void* vs = (mode & 1) ? a.vs : a.qc;
+  const void* qc = (mode & 2) ? a.qc : a.qs;
+  const int ts = (mode & 1) ? tok_s : tok_c, tc2 = (mode & 2) ? tok_c : tok_s;
+  if (encode_bhd(&P.qs, qs, a.H, a.D, ts) || encode_bhd(&P.ks, ks, a.H, a.D, ts) ||
+      encode_bhd(&P.vs, vs, a.H, a.D, ts) || encode_bhd(&P.qc, qc, a.H, a.D, tc2))
     return cudaErrorInvalidValue;
+  P.mode = mode;
+  P.tok_c = tok_c;
   P.table_row = a.table_row;
   P.null_kv = a.null_kv;
   P.qc_ptr = a.qc;
@@ -662,12 +682,13 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   P.layer = a.layer;
   P.nblk = a.nblk;
   P.split_blks = a.split_blks;
-  P.n_splits = a.n_splits;
+  P.n_splits = (mode & 2) ? a.n_splits : 0;
   P.capacity = a.capacity;
   P.max_splits = kPrefillMaxSplits;
   P.scale_log2 = a.scale_log2;
-  const int grid = a.n_splits * a.H + a.H;
-  if (a.D == 64 && a.cluster) return launch_prefill_cluster(P, st);
+  P.n_sa = ((mode & 1) || ((mode & 2) && a.nblk == 0)) ? a.H : 0;
+  const int grid = P.n_splits * a.H + P.n_sa;
+  if (a.D == 64 && a.cluster && P.n_splits > 0) return launch_prefill_cluster(P, st);
   if (a.D == 64) return launch_prefill_d<64>(P, grid, st);
   if (a.D == 128) return launch_prefill_d<128>(P, grid, st);
   return cudaErrorInvalidValue;

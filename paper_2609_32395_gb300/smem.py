@@ -36,6 +36,8 @@ EXPORTED = [
     "smem_append_block", "smem_delete_block", "smem_release_seq", "smem_write_inblock", "smem_prefill_block",
     "smem_decode", "smem_decode_static_scratch", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table", "smem_check_device_error",
     "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
+    "smem_layer_workspace_bytes", "smem_append_block_rows", "smem_set_null_vector", "smem_reader_layer_prefill",
+    "smem_reader_layer_decode",
 ]
 
 
@@ -58,10 +60,21 @@ class SmemConfig(ctypes.Structure):
     ]
 
 
+class SmemLayerWeights(ctypes.Structure):
+    """struct smem_layer_weights: device pointers of one reader layer."""
+    _fields_ = [(n, ctypes.c_void_p) for n in (
+        "ln1_g", "ln1_b", "w_qkv", "w_os", "ln2_g", "ln2_b", "w_qc", "w_oc", "w_kc", "w_vc", "ln3_g", "ln3_b",
+        "w_1", "w_2")]
+
+
+LAYER_FIELDS = [f for f, _ in SmemLayerWeights._fields_]
+
+
 _lib = None
 _vp = ctypes.c_void_p
 _i32 = ctypes.c_int32
 _i32p = ctypes.POINTER(ctypes.c_int32)
+_wp = ctypes.POINTER(SmemLayerWeights)
 
 
 def lib():
@@ -95,6 +108,13 @@ def lib():
             "smem_debug_fail_after": (ctypes.c_int, [_vp, _i32]),
             "smem_strerror": (ctypes.c_char_p, [ctypes.c_int]),
             "smem_abi_version": (ctypes.c_int, []),
+            "smem_layer_workspace_bytes": (ctypes.c_size_t, [_vp, _i32]),
+            "smem_append_block_rows": (ctypes.c_int, [_vp, _i32, _i32, _vp, _wp, _vp, ctypes.c_size_t, _vp, _i32p]),
+            "smem_set_null_vector": (ctypes.c_int, [_vp, _vp, _wp, _vp, ctypes.c_size_t, _vp]),
+            "smem_reader_layer_prefill": (ctypes.c_int, [_vp, _i32, _i32, _i32, _wp, _vp, _vp, ctypes.c_size_t,
+                                                         _vp]),
+            "smem_reader_layer_decode": (ctypes.c_int, [_vp, _i32, _i32, _i32p, _i32p, _i32p, _wp, _vp, _vp,
+                                                        ctypes.c_size_t, _vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -256,6 +276,63 @@ def smem_debug_fail_after(h, n: int):
 
 def smem_abi_version() -> int:
     return int(lib().smem_abi_version())
+
+
+def layer_weights(tensors: dict) -> SmemLayerWeights:
+    """A SmemLayerWeights from a dict of device tensors keyed by field name
+    (LayerNorm gains/biases fp32 [d], matrices bf16 row-major). The caller
+    keeps the tensors alive."""
+    return SmemLayerWeights(*[tensors[f].data_ptr() if tensors.get(f) is not None else None for f in LAYER_FIELDS])
+
+
+def _warr(weights):
+    if isinstance(weights, SmemLayerWeights):
+        weights = [weights]
+    arr = (SmemLayerWeights * len(weights))(*weights)
+    return arr
+
+
+def _ws(ws):
+    return _ptr(ws), (0 if ws is None else ws.numel() * ws.element_size())
+
+
+def smem_layer_workspace_bytes(h, n_rows) -> int:
+    return int(lib().smem_layer_workspace_bytes(h, n_rows))
+
+
+def smem_append_block_rows(h, seq, block_idx, mu, weights, ws, stream=None) -> int:
+    """weights: a list of SmemLayerWeights, one per layer."""
+    slot = ctypes.c_int32(-1)
+    arr = _warr(weights)
+    wp, wn = _ws(ws)
+    _check(lib().smem_append_block_rows(h, seq, block_idx, _ptr(mu), arr, wp, wn, _stream(stream),
+                                        ctypes.byref(slot)), "smem_append_block_rows")
+    return slot.value
+
+
+def smem_set_null_vector(h, nu, weights, ws, stream=None):
+    arr = _warr(weights)
+    wp, wn = _ws(ws)
+    return _check(lib().smem_set_null_vector(h, _ptr(nu), arr, wp, wn, _stream(stream)), "smem_set_null_vector")
+
+
+def smem_reader_layer_prefill(h, seq, layer, q_block_idx, weights, x, ws, stream=None):
+    """weights: this layer's SmemLayerWeights; x: fp32 [b][d], updated in place."""
+    arr = _warr(weights)
+    wp, wn = _ws(ws)
+    return _check(lib().smem_reader_layer_prefill(h, seq, layer, q_block_idx, arr, _ptr(x), wp, wn, _stream(stream)),
+                  "smem_reader_layer_prefill")
+
+
+def smem_reader_layer_decode(h, layer, seq_ids, pos, q_block_idx, weights, x, ws, stream=None):
+    """x: fp32 [nb][d], updated in place."""
+    s, sp = _i32arr(seq_ids)
+    p, pp = _i32arr(pos)
+    q, qp = _i32arr(q_block_idx)
+    arr = _warr(weights)
+    wp, wn = _ws(ws)
+    return _check(lib().smem_reader_layer_decode(h, layer, len(s), sp, pp, qp, arr, _ptr(x), wp, wn,
+                                                 _stream(stream)), "smem_reader_layer_decode")
 
 
 class SmemCache:

@@ -40,6 +40,8 @@ KIND_QS, KIND_QC, KIND_KS, KIND_VS = 2, 3, 4, 5
 KIND_KNULL, KIND_VNULL = 6, 7
 KIND_KIN, KIND_VIN = 8, 9
 KIND_QDEC_S, KIND_QDEC_C, KIND_KNEW, KIND_VNEW = 10, 11, 12, 13
+KIND_MU, KIND_NU, KIND_X = 14, 15, 16
+KIND_WEIGHT, KIND_LN = 17, 18
 
 
 # ---------------------------------------------------------------------------
@@ -212,3 +214,56 @@ def inblock_positions(seed: int, n_seqs: int, b: int) -> np.ndarray:
     """Per-sequence in-block decode offsets uniform in [0, b-1]."""
     rng = np.random.Generator(np.random.PCG64(seed ^ 0xB10C))
     return rng.integers(0, b, size=n_seqs).astype(np.int32)
+
+
+# ---------------------------------------------------------------------------
+# random-init reader-layer weights (the recipe: matrices N(0, 1/fan_in) as
+# bf16, LayerNorm gains 1 + 0.1 N(0,1) and biases 0.1 N(0,1) as float32;
+# every scaling is one float32 multiply, then round-to-nearest-even)
+# ---------------------------------------------------------------------------
+# (name, fan_in / d, fan_out / d), stored [fan_in][fan_out] row-major
+LAYER_MATRICES = (("w_qkv", 1, 3), ("w_os", 1, 1), ("w_qc", 1, 1), ("w_oc", 1, 1), ("w_kc", 1, 1),
+                  ("w_vc", 1, 1), ("w_1", 1, 4), ("w_2", 4, 1))
+LAYER_NORMS = ("ln1", "ln2", "ln3")
+
+
+def _matrix_scale(fan_in: int) -> np.float32:
+    return np.float32(1.0 / np.sqrt(fan_in))
+
+
+def reader_layer_weights_np(seed: int, layer: int, d: int) -> dict:
+    """One layer's weights: matrices as bf16 bits (uint16 [fan_in][fan_out]),
+    LayerNorm parameters as float32 [d]."""
+    out = {}
+    for i, (name, fi, fo) in enumerate(LAYER_MATRICES):
+        z = tensor_np(seed, KIND_WEIGHT, (fi * d, fo * d), layer, i)
+        f = (z.astype(np.uint32) << 16).view(np.float32) * _matrix_scale(fi * d)
+        out[name] = _round_f32_bits_to_bf16(f.view(np.uint32).astype(np.int64)).astype(np.uint16)
+    for i, name in enumerate(LAYER_NORMS):
+        z = tensor_np(seed, KIND_LN, (2, d), layer, i)
+        zf = (z.astype(np.uint32) << 16).view(np.float32)
+        out[name + "_g"] = np.float32(1.0) + np.float32(0.1) * zf[0]
+        out[name + "_b"] = np.float32(0.1) * zf[1]
+    return out
+
+
+def reader_layer_weights_torch(seed: int, layer: int, d: int, device=None) -> dict:
+    """Same values as :func:`reader_layer_weights_np`, as torch tensors
+    (bfloat16 matrices, float32 LayerNorm parameters) on `device`."""
+    import torch
+
+    out = {}
+    for i, (name, fi, fo) in enumerate(LAYER_MATRICES):
+        z = tensor_torch(seed, KIND_WEIGHT, (fi * d, fo * d), layer, i, device=device)
+        f = z.to(torch.float32) * torch.tensor(float(_matrix_scale(fi * d)), dtype=torch.float32, device=z.device)
+        bits = f.view(torch.int32).to(torch.int64) & M32
+        r = _round_f32_bits_to_bf16(bits)
+        r = r - ((r >> 15) << 16)
+        out[name] = r.to(torch.int16).view(torch.bfloat16)
+    for i, name in enumerate(LAYER_NORMS):
+        zf = tensor_torch(seed, KIND_LN, (2, d), layer, i, device=device).to(torch.float32)
+        one = torch.tensor(1.0, dtype=torch.float32, device=zf.device)
+        tenth = torch.tensor(float(np.float32(0.1)), dtype=torch.float32, device=zf.device)
+        out[name + "_g"] = (one + tenth * zf[0]).contiguous()
+        out[name + "_b"] = (tenth * zf[1]).contiguous()
+    return out

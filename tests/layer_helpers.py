@@ -1,0 +1,87 @@
+"""Shared pieces of the reader-layer tests: seeded weights and inputs (from
+``synth``), their fp64 view for the layer oracle and device copies for the C
+ABI, and the layer tolerance.
+
+Tolerance of a layer output x_out (fp32) against the fp64 oracle on the same
+bf16 weights and inputs. The device path rounds to bf16 (unit roundoff
+2^-8) at nine places per layer -- LN1/LN2/LN3 outputs, q/k/v, the
+cross-attention query, the memory keys/values in the pool, both attention
+outputs and the GELU output -- and accumulates in fp32. With inputs and
+branch outputs of unit scale, each rounding perturbs a branch by about
+2^-8 / sqrt(3) relative (rms), and the errors of independent roundings add
+in quadrature: about 3e-3 rms relative to the layer's update x_out - x_in.
+A CPU emulation of exactly those roundings (fp32 elsewhere) at H = 4..16,
+d_h = 64/128 and 8..256 memory blocks gave max-abs 0.012-0.015, mean-abs
+0.0018 and relative L2 error of the update 0.003. The bounds below leave a
+factor of about three for accumulation-order differences.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import synth
+from oracle.reader_layer import LayerWeights
+from paper_2609_32395_gb300 import smem
+
+R = 64
+B_TOK = 64
+LAYER_MAX_ABS = 5e-2
+LAYER_MEAN_ABS = 5e-3
+LAYER_REL_UPDATE = 1e-2
+
+
+def bits_f64(bits: np.ndarray) -> np.ndarray:
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def bits_dev(bits: np.ndarray, device="cuda"):
+    return synth.bits_to_torch_bf16(bits).to(device)
+
+
+class LayerModel:
+    """L reader layers of width d: host fp64 weights for the oracle, device
+    tensors and their SmemLayerWeights for the library."""
+
+    def __init__(self, L: int, d: int, seed: int, device="cuda"):
+        self.L, self.d, self.seed = L, d, seed
+        self.host = [synth.reader_layer_weights_np(seed, l, d) for l in range(L)]
+        self.oracle = []
+        self.dev = []
+        self.sw = []
+        for hw in self.host:
+            kw = {}
+            dw = {}
+            for name, _, _ in synth.LAYER_MATRICES:
+                kw[name] = bits_f64(hw[name])
+                dw[name] = bits_dev(hw[name], device)
+            for name in synth.LAYER_NORMS:
+                for s in ("_g", "_b"):
+                    kw[name + s] = hw[name + s].astype(np.float64)
+                    dw[name + s] = torch.from_numpy(hw[name + s]).to(device)
+            self.oracle.append(LayerWeights(**kw))
+            self.dev.append(dw)
+            self.sw.append(smem.layer_weights(dw))
+
+
+def mu_bits(seed, seq, idx, d):
+    """Memory rows of block idx of seq: bf16 bits [R][d]."""
+    return synth.tensor_np(seed, synth.KIND_MU, (R, d), seq, idx)
+
+
+def nu_bits(seed, d):
+    return synth.tensor_np(seed, synth.KIND_NU, (d,))
+
+
+def x_rows(seed, seq, q_idx, d, n=B_TOK) -> np.ndarray:
+    """Residual-stream input of a block's tokens: fp32 [n][d] (bf16 values)."""
+    return bits_f64(synth.tensor_np(seed, synth.KIND_X, (n, d), seq, q_idx)).astype(np.float32)
+
+
+def assert_layer_close(got: np.ndarray, ref: np.ndarray, x_in: np.ndarray, what: str):
+    err = np.abs(got - ref)
+    mx, mean = float(err.max()), float(err.mean())
+    rel = float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref - x_in), 1e-30))
+    assert mx <= LAYER_MAX_ABS and mean <= LAYER_MEAN_ABS and rel <= LAYER_REL_UPDATE, \
+        f"{what}: max_abs {mx:.3e} mean_abs {mean:.3e} rel_l2(update) {rel:.3e}"
+    return mx, mean, rel

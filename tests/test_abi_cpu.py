@@ -28,7 +28,7 @@ def test_exports_every_declared_symbol():
     for n in names:
         assert hasattr(L, n), n
     assert set(names) == set(smem.EXPORTED)
-    assert smem.smem_abi_version() == 1
+    assert smem.smem_abi_version() == 2
 
 
 def test_required_bytes_validation():
@@ -120,3 +120,30 @@ def test_error_codes_agree_with_mirror_constants():
             smem.ERR_POOL_FULL, smem.ERR_TABLE_FULL) == (bk.ERR_INVALID_ARG, bk.ERR_NO_SUCH_SEQ,
                                                          bk.ERR_DUPLICATE_BLOCK, bk.ERR_NO_SUCH_BLOCK,
                                                          bk.ERR_POOL_FULL, bk.ERR_TABLE_FULL)
+
+
+def test_layer_entry_points_on_a_bookkeeping_cache():
+    """Workspace sizing is host arithmetic; the layer calls need a device."""
+    cfg = smem.make_config(2, 4, 64, 3, 16, 32, has_null_row=True)
+    h = smem.smem_cache_create(cfg, None)
+    try:
+        d = 4 * 64
+        w0 = smem.smem_layer_workspace_bytes(h, 0)
+        w64 = smem.smem_layer_workspace_bytes(h, 64)
+        assert w0 >= 32 << 20
+        # h, qkv, att, qc (bf16: 6d) + f (fp32: 4d) + g (bf16: 4d) per row
+        assert w64 - w0 == 64 * (6 * d * 2 + 4 * d * 4 + 4 * d * 2)
+        assert smem.smem_layer_workspace_bytes(h, 65) == 0      # above max(b, max_decode_batch)
+        assert smem.smem_layer_workspace_bytes(h, -1) == 0
+        w = [smem.SmemLayerWeights()] * 2
+        L = smem.lib()
+        import ctypes
+        arr = (smem.SmemLayerWeights * 2)(*w)
+        assert L.smem_reader_layer_prefill(h, 0, 0, 0, arr, None, None, 0, None) == smem.ERR_NO_DEVICE
+        assert L.smem_append_block_rows(h, 0, 0, None, arr, None, 0, None, None) == smem.ERR_NO_DEVICE
+        assert L.smem_set_null_vector(h, None, arr, None, 0, None) == smem.ERR_NO_DEVICE
+        seq = (ctypes.c_int32 * 1)(0)
+        assert L.smem_reader_layer_decode(h, 0, 1, seq, seq, seq, arr, None, None, 0, None) == smem.ERR_NO_DEVICE
+        assert smem.smem_get_table(h, 0) == ([], [])
+    finally:
+        smem.smem_cache_destroy(h)

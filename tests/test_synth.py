@@ -27,3 +27,16 @@ def test_distribution_is_standard_normal_like():
     x = synth.bits_to_torch_bf16(synth.tensor_np(0, 2, (64, 4096), 1)).float().numpy()
     assert abs(x.mean()) < 0.01 and abs(x.std() - 1.0) < 0.01
     assert 3.5 < np.abs(x).max() < 4.3
+
+
+def test_layer_weights_numpy_and_torch_agree():
+    d = 64
+    a = synth.reader_layer_weights_np(11, 2, d)
+    b = synth.reader_layer_weights_torch(11, 2, d)
+    for name, fi, fo in synth.LAYER_MATRICES:
+        assert a[name].shape == (fi * d, fo * d)
+        np.testing.assert_array_equal(a[name], synth.torch_bf16_to_bits(b[name]))
+    for name in synth.LAYER_NORMS:
+        for s in ("_g", "_b"):
+            assert a[name + s].dtype == np.float32
+            np.testing.assert_array_equal(a[name + s], b[name + s].numpy())
