@@ -45,6 +45,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-serve", action="store_true")
+    ap.add_argument("--no-layer", action="store_true", help="skip the full-reader-layer cells")
     ap.add_argument("--workload", default="decode", choices=["decode", "long"],
                     help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
     ap.add_argument("--long-batches", default="1,16", help="batches of the long-context cells")
@@ -300,6 +301,97 @@ class DecodeWorkload:
         return launches
 
 
+class LayerStack:
+    """Random-init weights of L reader layers of width d on the device (the
+    seeded recipe of ``synth.reader_layer_weights_torch``)."""
+
+    def __init__(self, L, d, seed, device):
+        import synth
+        from paper_2609_32395_gb300 import smem
+
+        self.L, self.d = L, d
+        self.tensors = [synth.reader_layer_weights_torch(seed, l, d, device=device) for l in range(L)]
+        self.sw = [smem.layer_weights(t) for t in self.tensors]
+
+    def bytes_per_layer(self):
+        # every weight matrix read once (bf16) + LayerNorm parameters (fp32)
+        return 14 * self.d * self.d * 2 + 6 * self.d * 4
+
+    def flops_per_layer(self, rows):
+        # the six token projections (memory-row projections happen at append)
+        return 2 * rows * (3 + 1 + 1 + 1 + 4 + 4) * self.d * self.d
+
+
+def layer_decode_step(wl, stack, x, ws, mu, events=None):
+    """One decode token for every sequence through all layers of the full
+    reader layer (LayerNorm, projections, attention, FFN); a finished block
+    is appended from synthetic memory rows through the layer's key/value
+    maps. Returns (our kernel launches, cuBLAS calls)."""
+    import torch
+
+    from paper_2609_32395_gb300 import smem
+
+    st = torch.cuda.current_stream()
+    if events is not None:
+        events[0].record(st)
+    for layer in range(wl.L):
+        smem.smem_reader_layer_decode(wl.h, layer, wl.seq_ids, wl.pos.astype(np.int32), wl.nblk.astype(np.int32),
+                                      stack.sw[layer], x, ws)
+    if events is not None:
+        events[1].record(st)
+    ours, blas = 6 * wl.L, 6 * wl.L  # 3 LayerNorm, GELU, 2 attention; 6 GEMMs per layer
+    wl.pos += 1
+    for s in np.nonzero(wl.pos == B_TOK)[0]:
+        smem.smem_append_block_rows(wl.h, int(s), int(wl.nblk[s]), mu, stack.sw, ws)
+        ours += 1
+        blas += 2 * wl.L
+        wl.new_used[s] += 1
+        wl.nblk[s] += 1
+        wl.pos[s] = 0
+    wl.step_no += 1
+    return ours, blas
+
+
+def measure_layer_decode(wl, steps, warmup, device):
+    """Full-reader-layer decode on the decode workload's cache (its memory
+    rows stand in for projected ones): tok/s, and the HBM roofline of a step
+    (weights of every layer + the K/V rows the attention reads)."""
+    import torch
+
+    import synth
+    from paper_2609_32395_gb300 import smem
+
+    d = wl.H * wl.D
+    stack = LayerStack(wl.L, d, 5, device)
+    ws = torch.empty(smem.smem_layer_workspace_bytes(wl.h, wl.S), dtype=torch.uint8, device=device)
+    x0 = synth.tensor_torch(wl.seed, synth.KIND_X, (wl.S, d), 0, device=device).float()
+    x = x0.clone()
+    mu = synth.tensor_torch(wl.seed, synth.KIND_MU, (R, d), 0, device=device)
+    for _ in range(warmup):
+        layer_decode_step(wl, stack, x, ws, mu)
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+    rows, ours, blas = [], 0, 0
+    for i in range(steps):
+        x.copy_(x0)
+        rows.append(wl.rows_read())
+        o, b = layer_decode_step(wl, stack, x, ws, mu, events=ev[i])
+        ours, blas = ours + o, blas + b
+    torch.cuda.synchronize()
+    if smem.smem_check_device_error(wl.h) != smem.OK:
+        raise RuntimeError("device error recorded during the full-layer decode")
+    ms = [a.elapsed_time(b) for a, b in ev]
+    step_ms = float(np.mean(ms))
+    kv = float(np.mean(rows)) * 4 * d * wl.L  # K + V bf16 per row per layer
+    w = stack.bytes_per_layer() * wl.L
+    act = wl.L * wl.S * d * 4 * 2 * 3  # residual stream read + written per branch (fp32)
+    alg = kv + w + act
+    return {"tok_per_s": wl.S / (step_ms / 1e3), "step_ms": step_ms, "step_ms_p50": float(np.median(ms)),
+            "alg_bytes_per_step": alg, "weight_bytes_per_step": w, "kv_bytes_per_step": kv,
+            "achieved_gbs": alg / (step_ms / 1e3) / 1e9, "our_launches": ours, "cublas_calls": blas,
+            "timing": "CUDA events around the layer calls of each step (appends excluded), inputs resident"}
+
+
 # ----------------------------------------------------------------------------- prefill workload
 SERVE = dict(name="160M-shaped one-block cached-context prefill", L=12, H=12, D=64, contexts=(16, 64, 256), seed=1)
 
@@ -400,6 +492,63 @@ def measure_serve(nblk, device, iters=30, flush_bytes=512 << 20):
     out = {"context_blocks": nblk, "memory_rows": nblk * R, "latency_ms": serve_ms[len(serve_ms) // 2],
            "latency_ms_min": serve_ms[0], "kernel_ms_mean": float(np.mean(kern_ms)),
            "bytes_per_launch": wl.bytes_per_launch(), "flops_per_launch": wl.flops_per_launch()}
+    wl.cache.close()
+    return out
+
+
+def measure_layer_serve(nblk, device, iters=30, flush_bytes=512 << 20):
+    """Latency of one cached-context serve through the full reader layer
+    (12 layers of LayerNorm, projections, attention and FFN over the final
+    block's 64 tokens), replayed from a CUDA graph with L2 flushed before
+    each replay."""
+    import torch
+
+    import synth
+    from paper_2609_32395_gb300 import smem
+
+    wl = PrefillWorkload(nblk, device)
+    d = wl.H * wl.D
+    stack = LayerStack(wl.L, d, 6, device)
+    ws = torch.empty(smem.smem_layer_workspace_bytes(wl.h, B_TOK), dtype=torch.uint8, device=device)
+    x0 = synth.tensor_torch(SERVE["seed"], synth.KIND_X, (B_TOK, d), 0, nblk, device=device).float()
+    x = x0.clone()
+    flush = torch.empty(flush_bytes, dtype=torch.uint8, device=device)
+    st = torch.cuda.current_stream()
+
+    def serve():
+        x.copy_(x0)
+        for layer in range(wl.L):
+            smem.smem_reader_layer_prefill(wl.h, 0, layer, nblk, stack.sw[layer], x, ws)
+
+    for _ in range(3):
+        serve()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        serve()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    e0 = [torch.cuda.Event(enable_timing=True) for _ in range(iters)]
+    e1 = [torch.cuda.Event(enable_timing=True) for _ in range(iters)]
+    for i in range(iters):
+        flush.zero_()
+        e0[i].record(st)
+        g.replay()
+        e1[i].record(st)
+    torch.cuda.synchronize()
+    if smem.smem_check_device_error(wl.h) != smem.OK:
+        raise RuntimeError("device error recorded during the full-layer serve")
+    lat = sorted(a.elapsed_time(b) for a, b in zip(e0, e1))
+    del g
+    kv = nblk * R * 4 * d * wl.L
+    w = stack.bytes_per_layer() * wl.L
+    alg = kv + w
+    med = lat[len(lat) // 2]
+    out = {"context_blocks": nblk, "latency_ms": med, "latency_ms_min": lat[0], "alg_bytes": alg,
+           "weight_bytes": w, "kv_bytes": kv, "achieved_gbs": alg / (med / 1e3) / 1e9,
+           "flops": stack.flops_per_layer(B_TOK) * wl.L + wl.flops_per_launch() * wl.L,
+           "launches_per_serve": {"ours": 7 * wl.L, "cublas": 6 * wl.L}}
     wl.cache.close()
     return out
 
@@ -703,8 +852,9 @@ def run_ours(args):
     smem.lib()  # fails loudly without the CUDA library
 
     e2e_steps = 0 if args.no_e2e else min(args.steps, 64)
-    wl = DecodeWorkload(args.seqs, args.warmup + args.steps + e2e_steps + 2, WORKLOAD["seed"], device, rank,
-                        layers=args.layers)
+    layer_steps = 0 if args.no_layer else min(args.steps, 64)
+    wl = DecodeWorkload(args.seqs, args.warmup + args.steps + e2e_steps + 2 + (layer_steps + args.warmup),
+                        WORKLOAD["seed"], device, rank, layers=args.layers)
 
     def barrier():
         if ws > 1:
@@ -773,14 +923,18 @@ def run_ours(args):
     if err != smem.OK:
         raise RuntimeError("device error recorded during the benchmark")
 
+    # --- the full reader layer around the attention (projections, LayerNorm, FFN)
+    layer_dec = measure_layer_decode(wl, layer_steps, args.warmup, device) if layer_steps else None
+
     # --- one-block cached-context serve (prefill), the metric's second half
-    serve = None
+    serve = layer_serve = None
     if not args.no_serve:
         wl.cache.close()
         wl.cache.buf = None
         del wl.new_K, wl.new_V
         torch.cuda.empty_cache()
         serve = [measure_serve(n, device) for n in SERVE["contexts"]]
+        layer_serve = None if args.no_layer else [measure_layer_serve(n, device) for n in SERVE["contexts"]]
     edit = None if args.no_serve else [measure_edit_latency(n, device) for n in EDIT["contexts"]]
 
     if rank != 0:
@@ -825,6 +979,18 @@ def run_ours(args):
                          "head_dim": SERVE["D"], "metric": "one-block cached-serve latency (12 layers)",
                          "unit": "ms", "timing": "CUDA graph of the 12 per-layer launches, L2 flushed before each",
                          "cells": serve}
+    if layer_dec or layer_serve:
+        layer = {"what": "full reader layer: pre-LN self-attention, cross-attention and 4d GELU FFN "
+                         "branches with random-init bf16 weights (projections on cuBLAS)"}
+        if layer_dec:
+            layer_dec["hbm_frac"] = layer_dec["achieved_gbs"] / peak
+            layer["decode"] = dict(workload=WORKLOAD["name"], unit="tok/s", steps=layer_steps, **layer_dec)
+        if layer_serve:
+            for c in layer_serve:
+                c["hbm_frac"] = c["achieved_gbs"] / peak
+            layer["serve"] = {"workload": SERVE["name"], "unit": "ms", "cells": layer_serve,
+                              "timing": "CUDA graph of the 12 layer calls, L2 flushed before each"}
+        line["layer"] = layer
     if edit:
         line["edit"] = {"workload": EDIT["name"], "unit": "us",
                         "note": "host = whole C ABI call; device = table-edit kernel; no row moves", "cells": edit}
