@@ -59,7 +59,7 @@
 extern "C" {
 #endif
 
-#define SMEM_ABI_VERSION 2
+#define SMEM_ABI_VERSION 3
 
 enum {
     SMEM_OK = 0,
@@ -94,6 +94,14 @@ typedef struct smem_config {
     const int32_t *free_order;  /* host, C entries: initial FIFO order, a
                                    permutation of 0..C-1; NULL = ascending.
                                    Copied at create time.                      */
+    int32_t recompute_kv;       /* 0: a slot holds the block's projected K/V
+                                   for every layer (materialized, Sec. 3.1).
+                                   1: a slot holds only the block's memory
+                                   rows mu [R][d] (d = H*d_h, shared by all
+                                   layers); the reader-layer calls re-derive
+                                   each layer's keys and values from them
+                                   (the recompute regime, App. "Serving").
+                                   The pool is then 2L times smaller.          */
 } smem_config;
 
 typedef struct smem_cache smem_cache;
@@ -247,14 +255,15 @@ size_t smem_layer_workspace_bytes(const smem_cache *c, int32_t n_rows);
  * w_kc and w_vc are read. The slot receives, for every layer l and head h,
  * K = mu W_kc^l[:, h d_h : (h+1) d_h] and V likewise (bf16), then the table
  * insert follows as in smem_append_block (same validation, errors and
- * FIFO order). */
+ * FIFO order). On a recompute_kv cache the slot receives mu itself and w
+ * is not read (may be NULL). */
 int smem_append_block_rows(smem_cache *c, int32_t seq, int32_t block_idx, const void *mu,
                            const smem_layer_weights *w, void *ws, size_t ws_bytes, void *stream,
                            int32_t *slot_out);
 
 /* Sets the null row from the d-vector nu (device bf16 [d]): per layer,
  * k_null = nu W_kc^l, v_null = nu W_vc^l. w: L host structs. Requires
- * has_null_row. */
+ * has_null_row. On a recompute_kv cache nu itself is kept (w may be NULL). */
 int smem_set_null_vector(smem_cache *c, const void *nu, const smem_layer_weights *w, void *ws,
                          size_t ws_bytes, void *stream);
 
@@ -271,7 +280,16 @@ int smem_reader_layer_prefill(smem_cache *c, int32_t seq, int32_t layer, int32_t
 
 /* One reader layer for one decode step of nb sequences (arguments as in
  * smem_decode): x is device fp32 [nb][d], read and overwritten; the new
- * tokens' self-attention k, v become in-block rows pos[i]. */
+ * tokens' self-attention k, v become in-block rows pos[i].
+ *
+ * On a recompute_kv cache both layer calls compute the cross-attention from
+ * the memory rows: with q'_h = W_kc[:, h] q_h (times the softmax scale),
+ * scores q'_h . mu_r and output (sum_r p_r mu_r) W_vc[:, h] -- the same
+ * keys mu W_kc and values mu W_vc, re-associated so that each row is read
+ * once per layer for all heads. q' and sum_r p_r mu_r are rounded to bf16.
+ * smem_append_block, smem_set_null_row, smem_prefill_block, smem_decode and
+ * smem_decode_static_scratch return SMEM_ERR_UNSUPPORTED there (they take
+ * projected keys and values). */
 int smem_reader_layer_decode(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids,
                              const int32_t *pos, const int32_t *q_block_idx,
                              const smem_layer_weights *w, float *x, void *ws, size_t ws_bytes,

@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OBJ = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsmem.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["smem_capi.cpp", "smem_copy.cu", "smem_decode.cu", "smem_layer.cu", "smem_prefill.cu"]
+SOURCES = ["smem_capi.cpp", "smem_copy.cu", "smem_decode.cu", "smem_layer.cu", "smem_prefill.cu", "smem_recompute.cu"]
 HEADERS = ["smem_device.cuh", "smem_internal.h", "smem_tc.cuh"]
 
 

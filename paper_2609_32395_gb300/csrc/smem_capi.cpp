@@ -27,6 +27,7 @@ using smem::Layout;
 struct smem_cache {
   CUtensorMap pool_map{};     // decode kernel's view of the pool (device caches)
   CUtensorMap pool_map_pf{};  // prefill kernel's view (whole 64-row tiles)
+  CUtensorMap pool_map_mu{};  // memory-row view [C][R][d] (recompute caches)
   smem_config cfg{};
   Layout lay{};
   uint8_t* dev = nullptr;  // nullptr: bookkeeping-only
@@ -67,6 +68,11 @@ int make_layout(const smem_config* c, Layout* L) {
   if (c->head_dim != 64 && c->head_dim != 128) return SMEM_ERR_UNSUPPORTED;
   if (c->block_tokens != smem::kBlockTok || c->rows_per_block != smem::kRows) return SMEM_ERR_UNSUPPORTED;
   if (c->has_null_row != 0 && c->has_null_row != 1) return SMEM_ERR_INVALID_ARG;
+  if (c->recompute_kv != 0 && c->recompute_kv != 1) return SMEM_ERR_INVALID_ARG;
+  // recompute caches: rows of d = H*d_h in 128-column pairs, at most 64 heads per query tile
+  if (c->recompute_kv && ((c->n_heads * c->head_dim) % 128 != 0 || c->n_heads > 64 ||
+                          smem::mu_query_tile(c->n_heads, c->n_heads * c->head_dim) == 0))
+    return SMEM_ERR_UNSUPPORTED;
   L->L = c->n_layers;
   L->H = c->n_heads;
   L->D = c->head_dim;
@@ -75,13 +81,14 @@ int make_layout(const smem_config* c, Layout* L) {
   L->capacity = c->capacity_slots;
   L->has_null = c->has_null_row;
   L->max_batch = c->max_decode_batch;
+  L->recompute = c->recompute_kv;
   int ms = 1;
   for (int n = 1; n <= c->max_blocks_per_seq; ++n)
     ms = std::max(ms, smem::ceil_div(n, smem::decode_split_blocks(n)));
   L->dec_max_splits = ms;
   L->pf_max_splits = smem::kPrefillMaxSplits;
   const size_t D = (size_t)L->D;
-  L->slot_elems = (size_t)L->L * L->H * 2 * smem::kRows * D;
+  L->slot_elems = L->recompute ? (size_t)smem::kRows * L->H * D : (size_t)L->L * L->H * 2 * smem::kRows * D;
   size_t off = 0;
   const size_t A = 1024;
   L->off_pool = off;
@@ -89,7 +96,7 @@ int make_layout(const smem_config* c, Layout* L) {
   L->off_inblock = off;
   off = align_up(off + (size_t)L->max_seqs * L->L * L->H * 2 * smem::kBlockTok * D * 2, A);
   L->off_null = off;
-  off = align_up(off + (L->has_null ? (size_t)L->L * L->H * 2 * D * 2 : 0), A);
+  off = align_up(off + (!L->has_null ? 0 : L->recompute ? (size_t)L->H * D * 2 : (size_t)L->L * L->H * 2 * D * 2), A);
   L->off_table = off;
   off = align_up(off + (size_t)L->max_seqs * L->max_blocks * 4, A);
   L->off_dec_part = off;
@@ -100,6 +107,8 @@ int make_layout(const smem_config* c, Layout* L) {
   off = align_up(off + (size_t)L->H * L->pf_max_splits * smem::kBlockTok * (D + 4) * 4, A);
   L->off_pf_cnt = off;
   off = align_up(off + (size_t)L->H * 4, A);
+  L->off_mu_cnt = off;
+  off = align_up(off + (size_t)smem::kMaxMuGroups * 4, A);
   L->off_err = off;
   off = align_up(off + 256, A);
   L->total = off;
@@ -156,9 +165,11 @@ inline const uint16_t* null_kv(smem_cache* c) {
 
 // Workspace of a reader-layer call over n rows (offsets from the caller's
 // 256-byte aligned buffer): cuBLAS workspace, then bf16 h [n][d], qkv
-// [n][3d], att [n][d], qc [n][d], fp32 f [n][4d], bf16 g [n][4d].
+// [n][3d], att [n][d], qc [n][d], fp32 f [n][4d], bf16 g [n][4d]; on a
+// recompute cache also bf16 q' and O' [n][H][d] and the split partials of
+// the memory-row attention.
 struct LayerWs {
-  size_t blas, h, qkv, att, qc, f, g, total;
+  size_t blas, h, qkv, att, qc, f, g, qp, op, part, total;
 };
 
 LayerWs layer_ws(const Layout& L, int n) {
@@ -179,6 +190,18 @@ LayerWs layer_ws(const Layout& L, int n) {
   off = align_up(off + (size_t)n * 4 * d * 4, 256);
   w.g = off;
   off = align_up(off + (size_t)n * 4 * d * 2, 256);
+  w.qp = w.op = w.part = off;
+  if (L.recompute) {
+    const int nqd = smem::mu_query_tile(L.H, (int)d);
+    w.qp = off;
+    off = align_up(off + (size_t)n * L.H * d * 2, 256);
+    w.op = off;
+    off = align_up(off + (size_t)n * L.H * d * 2, 256);
+    w.part = off;
+    const size_t rows = std::max((size_t)std::min(n, smem::kMaxMuGroups) * nqd,
+                                 n >= smem::kBlockTok ? (size_t)smem::kBlockTok * L.H : (size_t)0);
+    off = align_up(off + rows * smem::kMuMaxSplits * (d + 4) * 4, 256);
+  }
   w.total = off;
   return w;
 }
@@ -402,10 +425,15 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
       delete c;
       return SMEM_ERR_CUDA;
     }
-    int er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity,
-                                   smem::decode_stage_rows(L.D));
-    if (er == 0)
-      er = smem::encode_pool_map(&c->pool_map_pf, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity, smem::kRows);
+    int er = 0;
+    if (L.recompute) {
+      er = smem::encode_mu_pool_map(&c->pool_map_mu, c->dev + L.off_pool, L.H * L.D, L.capacity);
+    } else {
+      er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity,
+                                 smem::decode_stage_rows(L.D));
+      if (er == 0)
+        er = smem::encode_pool_map(&c->pool_map_pf, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity, smem::kRows);
+    }
     if (er != 0) {
       std::snprintf(g_detail, sizeof(g_detail), "tensor map encode failed (%d)", er);
       delete c;
@@ -427,6 +455,7 @@ int smem_cache_destroy(smem_cache* c) {
 int smem_set_null_row(smem_cache* c, const void* k_null, const void* v_null, void* stream) {
   if (!c) return SMEM_ERR_INVALID_ARG;
   if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
   if (!c->lay.has_null || !k_null || !v_null) return SMEM_ERR_INVALID_ARG;
   if (!aligned16(k_null) || !aligned16(v_null)) return SMEM_ERR_ALIGN;
   DeviceGuard g(c->device);
@@ -445,6 +474,7 @@ int smem_append_block(smem_cache* c, int32_t seq, int32_t block_idx, const void*
   if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
   if (block_idx < 0) return SMEM_ERR_INVALID_ARG;
   if (c->dev) {
+    if (c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
     if (!K || !V) return SMEM_ERR_INVALID_ARG;
     if (!aligned16(K) || !aligned16(V)) return SMEM_ERR_ALIGN;
   } else if (K || V) {
@@ -530,6 +560,7 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
   if (!c->dev) return SMEM_ERR_NO_DEVICE;
   if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
   if (layer < 0 || layer >= c->lay.L || q_block_idx < 0) return SMEM_ERR_INVALID_ARG;
+  if (c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
   const void* ptrs[6] = {Qs, Ks, Vs, Qc, Osa, Oca};
   for (const void* p : ptrs) {
     if (!p) return SMEM_ERR_INVALID_ARG;
@@ -544,6 +575,7 @@ int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids
                 void* osa, void* oca, void* stream) {
   const int rc = check_decode_args(c, layer, nb, seq_ids, pos, q_block_idx);
   if (rc) return rc;
+  if (c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
   const void* ptrs[6] = {qs, k_new, v_new, qc, osa, oca};
   for (const void* p : ptrs) {
     if (!p) return SMEM_ERR_INVALID_ARG;
@@ -563,6 +595,7 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
   if (!c) return SMEM_ERR_INVALID_ARG;
   if (!c->dev) return SMEM_ERR_NO_DEVICE;
   const Layout& L = c->lay;
+  if (L.recompute) return SMEM_ERR_UNSUPPORTED;
   if (layer < 0 || layer >= L.L || nb < 1 || nb > L.max_batch) return SMEM_ERR_INVALID_ARG;
   if (!seq_ids || !pos || !q_block_idx) return SMEM_ERR_INVALID_ARG;
   const void* ptrs[6] = {qs, k_new, v_new, qc, osa, oca};
@@ -669,10 +702,10 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
   if (!c) return SMEM_ERR_INVALID_ARG;
   if (!c->dev) return SMEM_ERR_NO_DEVICE;
   if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
-  if (block_idx < 0 || !mu || !w) return SMEM_ERR_INVALID_ARG;
+  if (block_idx < 0 || !mu || (!w && !c->lay.recompute)) return SMEM_ERR_INVALID_ARG;
   if (!aligned16(mu)) return SMEM_ERR_ALIGN;
   const Layout& L = c->lay;
-  for (int l = 0; l < L.L; ++l) {
+  for (int l = 0; l < L.L && !L.recompute; ++l) {
     const int rc = check_weights(&w[l], false);
     if (rc) return rc;
   }
@@ -692,7 +725,9 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
   uint16_t* slot = pool_slot(c, s);
   const int d = L.H * L.D;
   const size_t head_stride = (size_t)2 * smem::kRows * L.D;
-  for (int l = 0; l < L.L && !rc; ++l)
+  if (L.recompute)  // the slot keeps the memory rows themselves
+    rc = cuda_rc(cudaMemcpyAsync(slot, mu, (size_t)smem::kRows * d * 2, cudaMemcpyDeviceToDevice, st), "append rows");
+  for (int l = 0; l < L.L && !rc && !L.recompute; ++l)
     for (int kv = 0; kv < 2 && !rc; ++kv)
       rc = blas_rc(smem::blas_project_heads(c->blas, smem::kRows, d, L.H, L.D, static_cast<const uint16_t*>(mu),
                                             static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc),
@@ -712,9 +747,9 @@ int smem_set_null_vector(smem_cache* c, const void* nu, const smem_layer_weights
   if (!c) return SMEM_ERR_INVALID_ARG;
   if (!c->dev) return SMEM_ERR_NO_DEVICE;
   const Layout& L = c->lay;
-  if (!L.has_null || !nu || !w) return SMEM_ERR_INVALID_ARG;
+  if (!L.has_null || !nu || (!w && !L.recompute)) return SMEM_ERR_INVALID_ARG;
   if (!aligned16(nu)) return SMEM_ERR_ALIGN;
-  for (int l = 0; l < L.L; ++l) {
+  for (int l = 0; l < L.L && !L.recompute; ++l) {
     const int rc = check_weights(&w[l], false);
     if (rc) return rc;
   }
@@ -724,6 +759,8 @@ int smem_set_null_vector(smem_cache* c, const void* nu, const smem_layer_weights
   if (injected_failure(c)) return SMEM_ERR_CUDA;
   uint16_t* nk = reinterpret_cast<uint16_t*>(c->dev + L.off_null);
   const int d = L.H * L.D;
+  if (L.recompute)
+    return cuda_rc(cudaMemcpyAsync(nk, nu, (size_t)d * 2, cudaMemcpyDeviceToDevice, as_stream(stream)), "null vector");
   for (int l = 0; l < L.L && !rc; ++l)
     for (int kv = 0; kv < 2 && !rc; ++kv)
       rc = blas_rc(smem::blas_project_heads(c->blas, 1, d, L.H, L.D, static_cast<const uint16_t*>(nu),
@@ -780,6 +817,89 @@ struct LayerRun {
   }
 };
 
+// Cross-attention of a layer call on a recompute cache (the memory rows mu
+// in the pool): q'_h = scale W_kc,h q_h, O'_h = attention of q'_h over the
+// rows, att_h = O'_h W_vc,h. Prefill: one row set, groups (head, query
+// tile); decode: one group per sequence holding all its heads.
+int mu_cross_attention(LayerRun& r, int layer, int nb, const int32_t* seq_ids, const int32_t* q_block_idx,
+                       bool prefill, int seq, int q_idx) {
+  smem_cache* c = r.c;
+  const Layout& L = c->lay;
+  const int d = r.d, H = L.H, D = L.D;
+  const float scale = (float)(1.4426950408889634 / std::sqrt((double)D));
+  const uint16_t* wkc = static_cast<const uint16_t*>(r.w->w_kc);
+  const uint16_t* wvc = static_cast<const uint16_t*>(r.w->w_vc);
+  uint16_t* qp = reinterpret_cast<uint16_t*>(r.ws + r.o.qp);
+  uint16_t* op = reinterpret_cast<uint16_t*>(r.ws + r.o.op);
+  const int nq = prefill ? smem::kBlockTok : nb;  // queries per head
+  // q'[.][h][i] = scale sum_j qc[.][h][j] W_kc[i][h D + j]; prefill stores [h][q][d], decode [s][h][d]
+  int rc = blas_rc(smem::blas_gemm_sb(c->blas, true, false, d, nq, D, scale, wkc, d, D, r.qc(), d, D, qp,
+                                      prefill ? d : H * d, prefill ? (long long)smem::kBlockTok * d : d, H, g_detail,
+                                      sizeof(g_detail)));
+  if (rc) return rc;
+  static thread_local smem::MuParams P;
+  P.pool = c->pool_map_mu;
+  P.table = reinterpret_cast<const int*>(c->dev + L.off_table);
+  P.nu = L.has_null ? reinterpret_cast<const uint16_t*>(c->dev + L.off_null) : nullptr;
+  P.part = reinterpret_cast<float*>(r.ws + r.o.part);
+  P.counters = reinterpret_cast<unsigned*>(c->dev + L.off_mu_cnt);
+  P.err = reinterpret_cast<int*>(c->dev + L.off_err);
+  P.d = d;
+  P.max_blocks = L.max_blocks;
+  P.capacity = L.capacity;
+  if (prefill) {
+    const int nqt = smem::mu_query_tile(smem::kBlockTok, d);
+    const std::vector<int32_t>& ix = c->idx[seq];
+    const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_idx) - ix.begin());
+    const int tiles = smem::kBlockTok / nqt;
+    const int groups = H * tiles;
+    const int sb = nblk ? smem::mu_prefill_split_blocks(nblk, groups) : 1;
+    const int nsplit = nblk ? smem::ceil_div(nblk, sb) : 1;
+    P.qptr = qp;
+    P.out = op;
+    P.nrows = smem::kBlockTok;
+    P.n_qg = H;
+    P.n_groups = groups;
+    int u = 0;
+    for (int h = 0; h < H; ++h)
+      for (int t = 0; t < tiles; ++t) {
+        smem::MuGroup& G = P.groups[h * tiles + t];
+        G = {seq, h, t * nqt, nblk, sb, nsplit, u, 0};
+        u += nsplit;
+      }
+    P.n_units = u;
+    if (injected_failure(c)) return SMEM_ERR_CUDA;
+    rc = cuda_rc(smem::launch_mu_attention(P, nqt, r.st), "memory-row attention");
+  } else {
+    const int nqt = smem::mu_query_tile(H, d);
+    for (int i0 = 0; i0 < nb && !rc; i0 += smem::kMaxMuGroups) {
+      const int n = std::min(nb - i0, smem::kMaxMuGroups);
+      P.qptr = qp + (size_t)i0 * H * d;
+      P.out = op + (size_t)i0 * H * d;
+      P.nrows = H;
+      P.n_qg = n;
+      P.n_groups = n;
+      int u = 0;
+      for (int i = 0; i < n; ++i) {
+        const std::vector<int32_t>& ix = c->idx[seq_ids[i0 + i]];
+        const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx[i0 + i]) - ix.begin());
+        const int sb = nblk ? smem::mu_decode_split_blocks(nblk) : 1;
+        const int nsplit = nblk ? smem::ceil_div(nblk, sb) : 1;
+        P.groups[i] = {seq_ids[i0 + i], i, 0, nblk, sb, nsplit, u, 0};
+        u += nsplit;
+      }
+      P.n_units = u;
+      if (injected_failure(c)) return SMEM_ERR_CUDA;
+      rc = cuda_rc(smem::launch_mu_attention(P, nqt, r.st), "memory-row attention");
+    }
+  }
+  if (rc) return rc;
+  // att[.][h][e] = sum_i O'[h-row][i] W_vc[i][h D + e]
+  return blas_rc(smem::blas_gemm_sb(c->blas, false, false, D, nq, d, 1.f, wvc, d, D, op,
+                                    prefill ? d : H * d, prefill ? (long long)smem::kBlockTok * d : d, r.att(), d, D,
+                                    H, g_detail, sizeof(g_detail)));
+}
+
 }  // namespace
 
 int smem_reader_layer_prefill(smem_cache* c, int32_t seq, int32_t layer, int32_t q_block_idx,
@@ -809,8 +929,12 @@ int smem_reader_layer_prefill(smem_cache* c, int32_t seq, int32_t layer, int32_t
     rc = prefill_impl(c, seq, layer, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + 2 * d, r.qkv(), r.att(), r.att(), 1,
                       3 * d, 3 * d, st);
   if (!rc) rc = r.after_sa();
-  if (!rc)
-    rc = prefill_impl(c, seq, layer, q_block_idx, r.qc(), r.qc(), r.qc(), r.qc(), r.att(), r.att(), 2, d, d, st);
+  if (!rc) {
+    if (L.recompute)
+      rc = mu_cross_attention(r, layer, 0, nullptr, nullptr, true, seq, q_block_idx);
+    else
+      rc = prefill_impl(c, seq, layer, q_block_idx, r.qc(), r.qc(), r.qc(), r.qc(), r.att(), r.att(), 2, d, d, st);
+  }
   if (!rc) rc = r.after_ca();
   return rc;
 }
@@ -836,9 +960,13 @@ int smem_reader_layer_decode(smem_cache* c, int32_t layer, int32_t nb, const int
     rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + 2 * d, r.qkv(), r.att(),
                      r.att(), 1, 3 * d, 3 * d, st);
   if (!rc) rc = r.after_sa();
-  if (!rc)
-    rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qc(), r.qc(), r.qc(), r.qc(), r.att(), r.att(), 2, d,
-                     d, st);
+  if (!rc) {
+    if (L.recompute)
+      rc = mu_cross_attention(r, layer, nb, seq_ids, q_block_idx, false, 0, 0);
+    else
+      rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qc(), r.qc(), r.qc(), r.qc(), r.att(), r.att(), 2,
+                       d, d, st);
+  }
   if (!rc) rc = r.after_ca();
   return rc;
 }

@@ -23,11 +23,12 @@ constexpr int kBlockTok = 64; // b: query tokens per block
 // ---------------------------------------------------------------------------
 struct Layout {
   int L, H, D, max_seqs, max_blocks, capacity, has_null, max_batch;
+  int recompute;       // 1: slots hold memory rows mu [R][d] instead of per-layer K/V
   int dec_max_splits;  // split-K partial slots per (decode item, head)
   int pf_max_splits;   // split-K partial slots per prefill head
-  size_t slot_elems;   // bf16 elements per pool slot = L*H*2*R*D
+  size_t slot_elems;   // bf16 elements per pool slot: L*H*2*R*D, or R*d (recompute)
   size_t off_pool, off_inblock, off_null, off_table, off_dec_part, off_dec_cnt, off_pf_part, off_pf_cnt,
-      off_err, total;
+      off_mu_cnt, off_err, total;
 };
 
 // Split-K plan of the decode cross-attention: the number of memory blocks a
@@ -141,6 +142,53 @@ int blas_gemm(void* blas, int m, int n, int k, const uint16_t* A, const uint16_t
               bool accumulate, char* detail, size_t detail_len);
 int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t* X, const uint16_t* W,
                        uint16_t* out, long long head_stride, char* detail, size_t detail_len);
+int blas_gemm_sb(void* blas, bool ta, bool tb, int m, int n, int k, float alpha, const uint16_t* A, int lda,
+                 long long sA, const uint16_t* B, int ldb, long long sB, uint16_t* C, int ldc, long long sC, int batch,
+                 char* detail, size_t detail_len);
+
+// ---------------------------------------------------------------------------
+// cross-attention over memory rows (recompute-K/V caches)
+// ---------------------------------------------------------------------------
+constexpr int kMaxMuGroups = 512;   // groups (row set x query tile) per launch
+constexpr int kMuMaxSplits = 16;    // splits of one group's blocks
+constexpr int kMuSmemBudget = 200 * 1024;
+// One group: NQ queries (rows n0.. of query set qg) that read the same row
+// set (the first nblk table blocks of `seq`), cut into nsplit units of
+// split_blks blocks; units of a group are consecutive from unit_begin.
+struct MuGroup {
+  int seq, qg, n0, nblk, split_blks, nsplit, unit_begin, pad;
+};
+struct MuParams {
+  CUtensorMap pool;           // memory rows [C][R][d], box 64 x 64 x 1
+  CUtensorMap q;              // Q' [n_qg][nrows][d], box 64 x NQ x 1 (set by the launcher)
+  const int* table;           // [max_seqs][max_blocks]
+  const uint16_t* qptr;       // Q' (bf16, softmax scale log2(e)/sqrt(d_h) folded in)
+  const uint16_t* nu;         // null row [d] or nullptr
+  uint16_t* out;              // O' [n_qg][nrows][d] bf16, normalized
+  float* part;                // [unit][NQ][d + 4]: m, l, pad, pad, O'[d]
+  unsigned* counters;         // [kMaxMuGroups], zero between launches
+  int* err;
+  int d, nrows, n_qg, max_blocks, capacity, n_groups, n_units;
+  int ns, off_ring, off_p, off_bar, off_misc;  // shared-memory plan (set by the launcher)
+  MuGroup groups[kMaxMuGroups];
+};
+// Widest query tile (16, 32 or 64) for nq_total queries per row set at width
+// d whose accumulators fit tensor memory; 0 if none does.
+int mu_query_tile(int nq_total, int d);
+int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity);
+cudaError_t launch_mu_attention(MuParams& P, int nq, cudaStream_t st);
+// Split plans (functions of the block count and the cache geometry only).
+SMEM_HD inline int mu_decode_split_blocks(int nblk) {
+  const int s = (nblk + kMuMaxSplits - 1) / kMuMaxSplits;
+  return s > 8 ? s : 8;
+}
+SMEM_HD inline int mu_prefill_split_blocks(int nblk, int groups) {
+  int ns = (304 + groups - 1) / groups;
+  if (ns > kMuMaxSplits) ns = kMuMaxSplits;
+  if (ns > nblk) ns = nblk;
+  if (ns < 1) ns = 1;
+  return (nblk + ns - 1) / ns;
+}
 
 // ---------------------------------------------------------------------------
 // prefill

@@ -145,4 +145,18 @@ int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t
                      "head projection", detail, detail_len);
 }
 
+// Column-major strided-batched GEMM (cuBLAS conventions), bf16 in and out,
+// fp32 accumulation: C_i = alpha op(A_i) op(B_i), i < batch.
+int blas_gemm_sb(void* blas, bool ta, bool tb, int m, int n, int k, float alpha, const uint16_t* A, int lda,
+                 long long sA, const uint16_t* B, int ldb, long long sB, uint16_t* C, int ldc, long long sC, int batch,
+                 char* detail, size_t detail_len) {
+  if (m == 0 || n == 0) return 0;
+  const float zero = 0.f;
+  return blas_status(cublasGemmStridedBatchedEx(handle(blas), ta ? CUBLAS_OP_T : CUBLAS_OP_N,
+                                                tb ? CUBLAS_OP_T : CUBLAS_OP_N, m, n, k, &alpha, A, CUDA_R_16BF, lda,
+                                                sA, B, CUDA_R_16BF, ldb, sB, &zero, C, CUDA_R_16BF, ldc, sC, batch,
+                                                CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT),
+                     "batched gemm", detail, detail_len);
+}
+
 }  // namespace smem

@@ -1,0 +1,521 @@
+// smem_recompute.cu -- cross-attention that reads the memory rows themselves
+// instead of materialized per-layer keys and values (the "recompute K/V"
+// regime of arXiv 2609.32395, Sec. 3.1 and App. "Serving": the cache keeps
+// only the memory rows mu, d values per row shared by every reader layer,
+// and each layer's keys mu W_kc and values mu W_vc are re-derived per step).
+//
+// The keys and values are linear in mu, so per head h (Sec. 2 "Model")
+//   q_h . (mu_r W_kc,h) = (W_kc,h q_h) . mu_r = q'_h . mu_r
+//   sum_r p_r (mu_r W_vc,h) = (sum_r p_r mu_r) W_vc,h
+// and the layer's cross-attention is an attention of d-wide queries q'_h
+// over the d-wide rows mu_r whose output O'_h = sum_r p_r mu_r is mapped by
+// W_vc,h afterwards. The two small per-head maps run as cuBLAS GEMMs before
+// and after this kernel; this kernel streams every row once per layer (2d
+// bytes per row, half the materialized 4 H d_h) and keeps all queries that
+// share a row set in one CTA:
+//   S^T [64 rows][NQ queries] = mu_tile Q'^T   (M = 64, K = d)
+//   O'^T [d][NQ]             += mu_tile^T P^T  (M = 128 per column pair, K = 64)
+// both on the tensor cores (tcgen05, fp32 accumulators in TMEM). A decode
+// step puts the H heads of one sequence in one CTA (NQ = H rounded up to 16);
+// a one-block prefill puts NQ of the block's 64 queries of one head in a
+// CTA. The row tile is streamed twice from the TMA ring -- once for S, once
+// for P.V (the second pass normally hits L2) -- so any d fits in shared
+// memory. Softmax runs column-wise (one query per column) with the same
+// conditional rescale as the prefill kernel (raise the running maximum only
+// when it grows by more than 2^8). Splits of a row set write (m, l, O') and
+// the CTA holding the last ticket merges them in split order, null row first
+// (the null row nu is just one more d-wide row). Reduction orders depend only
+// on the block count, so outputs are bitwise independent of the edit path.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include "smem_device.cuh"
+#include "smem_internal.h"
+#include "smem_tc.cuh"
+
+namespace smem {
+
+namespace {
+
+constexpr int kMuBox = 64 * 128;        // one [64 rows][64 columns] bf16 box
+constexpr int kMuThreads = 192;         // 4 softmax warps, producer, MMA
+constexpr float kMuRescaleLog2 = 8.0f;  // raise the running max when it grows by more than 2^8
+
+template <int NQ>
+struct MuCfg {
+  static constexpr int C2 = NQ / 2;                 // S columns per thread
+  static constexpr int PBYTES = NQ * 128;           // P tile [NQ][64 rows] bf16
+  static constexpr uint32_t ID_S = tc::idesc_bf16(64, NQ, 0, 0);
+  static constexpr uint32_t ID_PV = tc::idesc_bf16(128, NQ, 1, 0);
+};
+
+template <int NQ>
+__device__ __forceinline__ void ld_s(uint32_t taddr, uint32_t (&r)[NQ / 2]) {
+  if constexpr (NQ == 64) tc::ld_16x32bx2_x32<32>(taddr, r);
+  else if constexpr (NQ == 32) tc::ld_16x32bx2_x16<16>(taddr, r);
+  else tc::ld_16x32bx2_x8<8>(taddr, r);
+}
+
+__device__ __forceinline__ void store_bf16(uint16_t* p, float v) {
+  __nv_bfloat16 h = __float2bfloat16_rn(v);
+  *reinterpret_cast<__nv_bfloat16*>(p) = h;
+}
+
+}  // namespace
+
+template <int NQ>
+__global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __grid_constant__ MuParams p) {
+  using C = MuCfg<NQ>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const int d = p.d;
+  const int NC = d / 64;  // 64-column chunks of a row (even)
+  const int ns = p.ns;
+  uint8_t* qt = base;
+  uint8_t* ring = base + p.off_ring;
+  uint8_t* pt = base + p.off_p;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + p.off_bar);
+  uint64_t* q_full = bars;
+  uint64_t* full = bars + 1;
+  uint64_t* empty = full + ns;
+  uint64_t* s_full = empty + ns;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* o_done = p_full + 2;
+  uint64_t* drain = o_done + 2;
+  uint8_t* misc = base + p.off_misc;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+  volatile unsigned* ticket = reinterpret_cast<volatile unsigned*>(misc + 8);
+  float* red = reinterpret_cast<float*>(misc + 16);  // [2][4][NQ] column maxima per warp
+  float* alpha = red + 2 * 4 * NQ;                   // [2][NQ] rescale factors
+  float* lsum = alpha + 2 * NQ;                      // [4][NQ] column sums per warp
+  float* mfin = lsum + 4 * NQ;                       // [NQ]
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  // this CTA's unit: split `split` of group g
+  int lo = 0, hi = p.n_groups - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.groups[mid].unit_begin <= (int)blockIdx.x) lo = mid;
+    else hi = mid - 1;
+  }
+  const int g = lo;
+  const MuGroup& G = p.groups[g];
+  const int split = (int)blockIdx.x - G.unit_begin;
+  const int b0 = split * G.split_blks;
+  const int nt = G.nblk > 0 ? min(G.split_blks, G.nblk - b0) : 0;
+  const int* trow = p.table + (size_t)G.seq * p.max_blocks;
+  uint32_t ncols = 32;
+  while (ncols < (uint32_t)(NQ * (2 + NC / 2))) ncols <<= 1;
+  const uint32_t colO = 2 * NQ;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < ns; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_free[b], 4);
+      mbar_init(&p_full[b], 4);
+      mbar_init(&o_done[b], 1);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 4 && nt > 0) tc::alloc(tslot, ncols);
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = nt > 0 ? *tslot : 0u;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0 && nt > 0) {
+      mbar_arrive_expect_tx(q_full, (uint32_t)(NC * C::PBYTES));
+      for (int c = 0; c < NC; ++c) tc::tma_load_3d(qt + c * C::PBYTES, &p.q, c * 64, G.n0, G.qg, q_full);
+      int k = 0;
+      bool ok = true;
+      // one pass = the NC chunks of tile t; order S(0), S(1), PV(0), S(2), PV(1), ...
+      auto pass = [&](int t) {
+        const int slot = trow[b0 + t];
+        const bool good = slot >= 0 && slot < p.capacity;
+        if (!good) record_error(p.err, kDevErrBounds);
+        for (int c = 0; c < NC && ok; ++c, ++k) {
+          const int st = k % ns;
+          if (k >= ns && !mbar_wait_bounded(&empty[st], ((k / ns) - 1) & 1, abort_flag)) {
+            if (!*abort_flag) record_error(p.err, kDevErrWaitEmpty);
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+          if (good) {
+            mbar_arrive_expect_tx(&full[st], kMuBox);
+            tc::tma_load_3d(ring + st * kMuBox, &p.pool, c * 64, 0, slot, &full[st]);
+          } else {
+            mbar_arrive(&full[st]);
+          }
+        }
+      };
+      pass(0);
+      for (int t = 0; t < nt && ok; ++t) {
+        if (t + 1 < nt) pass(t + 1);
+        if (ok) pass(t);
+      }
+      if (!ok) {
+        // let every copy already issued land before the CTA can exit
+        mbar_wait_bounded(q_full, 0, nullptr);
+        for (int j = 0; j < k; ++j) mbar_wait_bounded(&full[j % ns], (j / ns) & 1, nullptr);
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------- MMA issuer
+    if (lane == 0 && nt > 0) {
+      bool ok = mbar_wait_bounded(q_full, 0, abort_flag);
+      tc::fence_after();
+      const uint32_t qa = smem_u32(qt);
+      const uint32_t ra = smem_u32(ring);
+      int k = 0;
+      auto issue_s = [&](int t) {
+        const int sb = t & 1;
+        if (ok && t >= 2) ok = mbar_wait_bounded(&s_free[sb], ((t >> 1) - 1) & 1, abort_flag);
+        for (int c = 0; c < NC && ok; ++c, ++k) {
+          const int st = k % ns;
+          ok = mbar_wait_bounded(&full[st], (k / ns) & 1, abort_flag);
+          if (!ok) break;
+          tc::fence_after();
+          const uint32_t a = ra + st * kMuBox, b = qa + c * C::PBYTES;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + sb * NQ, tc::sdesc_sw128(a + kk * 32, 16, 1024), tc::sdesc_sw128(b + kk * 32, 16, 1024),
+                         C::ID_S, (c | kk) > 0);
+          tc::commit(&empty[st]);
+        }
+        if (ok) tc::commit(&s_full[sb]);
+      };
+      auto issue_pv = [&](int t) {
+        const int pb = t & 1;
+        if (ok) ok = mbar_wait_bounded(&p_full[pb], (t >> 1) & 1, abort_flag);
+        if (!ok) return;
+        tc::fence_after();
+        const uint32_t b = smem_u32(pt + pb * C::PBYTES);
+        for (int cp = 0; cp < NC / 2 && ok; ++cp, k += 2) {
+          const int st = k % ns;  // even: the pair sits in slots st, st + 1
+          ok = mbar_wait_bounded(&full[st], (k / ns) & 1, abort_flag) &&
+               mbar_wait_bounded(&full[st + 1], ((k + 1) / ns) & 1, abort_flag);
+          if (!ok) break;
+          tc::fence_after();
+          const uint32_t a = ra + st * kMuBox;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + colO + cp * NQ, tc::sdesc_sw128(a + kk * 2048, kMuBox, 1024),
+                         tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_PV, (t > 0 || kk > 0));
+          tc::commit(&empty[st]);
+          tc::commit(&empty[st + 1]);
+        }
+        if (ok) tc::commit(&o_done[pb]);
+      };
+      issue_s(0);
+      for (int t = 0; t < nt && ok; ++t) {
+        if (t + 1 < nt) issue_s(t + 1);
+        issue_pv(t);
+      }
+      if (!ok) {
+        if (!*abort_flag) record_error(p.err, kDevErrWaitMma);
+        *abort_flag = 1;
+      }
+      tc::commit(drain);
+      mbar_wait_bounded(drain, 0, nullptr);
+    }
+  } else {
+    // ---------------------------------------------------------- softmax warps
+    const int tid = threadIdx.x;            // 0..127: TMEM lane of O'
+    const int r = 16 * warp + (lane & 15);  // row of the tile
+    const int hf = lane >> 4;               // column half of S
+    const int col0 = hf * C::C2;
+    const uint32_t tlane = tmem + ((uint32_t)(32 * warp) << 16);
+    float m_used[C::C2], lp[C::C2];
+#pragma unroll
+    for (int c = 0; c < C::C2; ++c) {
+      m_used[c] = -INFINITY;
+      lp[c] = 0.f;
+    }
+    // Every exit from this loop is decided through bar_all over the four
+    // warps, so they take the same named barriers in the same order.
+    bool ok = true;
+    for (int t = 0; t < nt; ++t) {
+      const int sb = t & 1;
+      ok = bar_all(3, 128, mbar_wait_bounded(&s_full[sb], (t >> 1) & 1, abort_flag));
+      if (!ok) break;
+      tc::fence_after();
+      uint32_t sr[C::C2];
+      ld_s<NQ>(tlane + sb * NQ, sr);
+      tc::wait_ld();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);
+      float x[C::C2];
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        x[c] = __uint_as_float(sr[c]);
+        float v = x[c];
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+        if ((lane & 15) == 0) red[(sb * 4 + warp) * NQ + col0 + c] = v;
+      }
+      named_bar_sync(1, 128);
+      bool need_mine = false;
+      float a_c[C::C2];
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        const int col = col0 + c;
+        float tmax = red[(sb * 4) * NQ + col];
+#pragma unroll
+        for (int w2 = 1; w2 < 4; ++w2) tmax = fmaxf(tmax, red[(sb * 4 + w2) * NQ + col]);
+        const bool need = tmax > m_used[c] + kMuRescaleLog2;
+        a_c[c] = 1.f;
+        if (need) {
+          a_c[c] = exp2f(m_used[c] - tmax);
+          lp[c] *= a_c[c];
+          m_used[c] = tmax;
+          need_mine = true;
+        }
+        if (warp == 0 && (lane & 15) == 0) alpha[sb * NQ + col] = a_c[c];
+      }
+      // any column of the tile raised its maximum (t > 0: O' holds earlier tiles)
+      const bool any = !bar_all(2, 128, !need_mine);
+      if (t > 0 && any) {
+        ok = bar_all(3, 128, mbar_wait_bounded(&o_done[(t - 1) & 1], ((t - 1) >> 1) & 1, abort_flag));
+        if (!ok) break;
+        tc::fence_after();
+        for (int cp = 0; cp < NC / 2; ++cp) {
+#pragma unroll
+          for (int cb = 0; cb < NQ / 16; ++cb) {
+            uint32_t o[16];
+            const uint32_t ta = tlane + colO + cp * NQ + cb * 16;
+            tc::ld_32x32b_x16(ta, o);
+            tc::wait_ld();
+#pragma unroll
+            for (int j = 0; j < 16; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha[sb * NQ + cb * 16 + j]);
+            tc::st_32x32b_x16(ta, o);
+          }
+        }
+        tc::wait_st();
+      }
+      // P buffer sb was last read by P.V of tile t-2
+      if (t >= 2) {
+        ok = bar_all(3, 128, mbar_wait_bounded(&o_done[sb], ((t - 2) >> 1) & 1, abort_flag));
+        if (!ok) break;
+      }
+      uint8_t* pb = pt + sb * C::PBYTES;
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        const int col = col0 + c;
+        const float pr = exp2f(x[c] - m_used[c]);
+        lp[c] += pr;
+        store_bf16(reinterpret_cast<uint16_t*>(pb + col * 128 + ((((r >> 3) ^ (col & 7)) & 7) << 4) + (r & 7) * 2),
+                   pr);
+      }
+      fence_proxy_async_smem();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[sb]);
+    }
+    if (!ok) {
+      if (lane == 0 && !*abort_flag) record_error(p.err, kDevErrWaitFull);
+      *abort_flag = 1;
+    }
+    // ---------------------------------------------------------- epilogue
+    const size_t part_stride = (size_t)d + 4;
+    float* part_u = p.part + (size_t)blockIdx.x * NQ * part_stride;
+    if (nt > 0) {
+      if (ok) ok = bar_all(3, 128, mbar_wait_bounded(&o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, abort_flag));
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        float v = lp[c];
+        v += __shfl_xor_sync(0xffffffffu, v, 1);
+        v += __shfl_xor_sync(0xffffffffu, v, 2);
+        v += __shfl_xor_sync(0xffffffffu, v, 4);
+        v += __shfl_xor_sync(0xffffffffu, v, 8);
+        if ((lane & 15) == 0) {
+          lsum[warp * NQ + col0 + c] = v;
+          if (warp == 0) mfin[col0 + c] = m_used[c];
+        }
+      }
+      const bool all_ok = bar_all(1, 128, ok);
+      if (all_ok) {
+        tc::fence_after();
+        for (int cp = 0; cp < NC / 2; ++cp) {
+#pragma unroll
+          for (int cb = 0; cb < NQ / 16; ++cb) {
+            uint32_t o[16];
+            tc::ld_32x32b_x16(tlane + colO + cp * NQ + cb * 16, o);
+            tc::wait_ld();
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+              __stcg(part_u + (size_t)(cb * 16 + j) * part_stride + 4 + cp * 128 + tid, __uint_as_float(o[j]));
+          }
+        }
+        if (tid < NQ) {
+          part_u[(size_t)tid * part_stride] = mfin[tid];
+          part_u[(size_t)tid * part_stride + 1] = lsum[tid] + lsum[NQ + tid] + lsum[2 * NQ + tid] + lsum[3 * NQ + tid];
+        }
+        __threadfence();
+      }
+      ok = all_ok;
+    }
+    // ---------------------------------------------------------- merge
+    const int nq_out = min(NQ, p.nrows - G.n0);  // queries of this group that exist
+    uint16_t* out_g = p.out + ((size_t)G.qg * p.nrows + G.n0) * d;
+    if (nt == 0) {
+      // no readable memory block: the null row's value (nu) or zero
+      for (int i = tid; i < nq_out * d; i += 128) {
+        const int dc = i % d;
+        out_g[i] = p.nu ? p.nu[dc] : (uint16_t)0;
+      }
+    } else if (ok) {
+      if (tid == 0) *ticket = atomicAdd(&p.counters[g], 1u);
+      named_bar_sync(1, 128);
+      if (*ticket == (unsigned)(G.nsplit - 1)) {
+        __threadfence();
+        const int nsp = G.nsplit;
+        const float* part_g = p.part + (size_t)G.unit_begin * NQ * part_stride;
+        float* wsc = reinterpret_cast<float*>(ring);  // [nsp][NQ] split weights, then [NQ] null weights
+        float* wnull = wsc + kMuMaxSplits * NQ;
+        float* snull = wnull + NQ;  // [4][NQ] partial null scores
+        // null scores q'_n . nu (q' carries the softmax scale)
+        if (p.nu) {
+          for (int n = 0; n < NQ; ++n) {
+            float dot = 0.f;
+            if (n < nq_out) {
+              const uint16_t* qrow = p.qptr + ((size_t)G.qg * p.nrows + G.n0 + n) * d;
+              for (int dc = tid; dc < d; dc += 128) dot = fmaf(bf16lo(qrow[dc]), bf16lo(p.nu[dc]), dot);
+            }
+#pragma unroll
+            for (int o = 16; o; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+            if (lane == 0) snull[warp * NQ + n] = dot;
+          }
+        }
+        named_bar_sync(1, 128);
+        if (tid < NQ) {
+          const int n = tid;
+          const float sn = p.nu ? snull[n] + snull[NQ + n] + snull[2 * NQ + n] + snull[3 * NQ + n] : -INFINITY;
+          float M = sn;
+          for (int s2 = 0; s2 < nsp; ++s2) M = fmaxf(M, __ldcg(part_g + ((size_t)s2 * NQ + n) * part_stride));
+          float L = p.nu ? exp2f(sn - M) : 0.f;
+          for (int s2 = 0; s2 < nsp; ++s2) {
+            const float* pr = part_g + ((size_t)s2 * NQ + n) * part_stride;
+            const float f = exp2f(__ldcg(pr) - M);
+            wsc[s2 * NQ + n] = f;
+            L = fmaf(f, __ldcg(pr + 1), L);
+          }
+          const float inv = 1.f / L;
+          for (int s2 = 0; s2 < nsp; ++s2) wsc[s2 * NQ + n] *= inv;
+          wnull[n] = p.nu ? exp2f(sn - M) * inv : 0.f;
+        }
+        named_bar_sync(1, 128);
+        for (int dc = tid; dc < d; dc += 128) {
+          const float nuv = p.nu ? bf16lo(p.nu[dc]) : 0.f;
+          for (int n = 0; n < nq_out; ++n) {
+            float acc = wnull[n] * nuv;
+            for (int s2 = 0; s2 < nsp; ++s2)
+              acc = fmaf(wsc[s2 * NQ + n], __ldcg(part_g + ((size_t)s2 * NQ + n) * part_stride + 4 + dc), acc);
+            store_bf16(out_g + (size_t)n * d + dc, acc);
+          }
+        }
+        if (tid == 0) p.counters[g] = 0u;
+      }
+    }
+  }
+  tc::fence_before();
+  __syncthreads();
+  if (warp == 4 && nt > 0) {
+    tc::fence_after();
+    tc::dealloc(tmem, ncols);
+  }
+}
+
+namespace {
+
+int encode3d(CUtensorMap* map, const void* ptr, uint64_t d0, uint64_t d1, uint64_t d2, uint32_t b1) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  if (!encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return -1;
+    encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {d0 * 2, d0 * d1 * 2};
+  const cuuint32_t box[3] = {64, b1, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, estr,
+                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : (int)r;
+}
+
+// Shared-memory plan of a launch: Q' chunks, the ring, two P tiles,
+// barriers, scratch. Returns the dynamic shared-memory bytes.
+int mu_smem_plan(MuParams& P, int nq, int d) {
+  const int qbytes = (d / 64) * nq * 128;
+  const int fixed = 2 * nq * 128 + 4096 + 1024;
+  int ns = (kMuSmemBudget - qbytes - fixed) / kMuBox;
+  ns &= ~1;
+  if (ns > 16) ns = 16;
+  if (ns < 4) return -1;
+  P.ns = ns;
+  P.off_ring = (qbytes + 1023) / 1024 * 1024;
+  P.off_p = P.off_ring + ns * kMuBox;
+  P.off_bar = P.off_p + 2 * nq * 128;
+  const int nbars = 1 + 2 * ns + 9;
+  P.off_misc = (P.off_bar + nbars * 8 + 15) / 16 * 16;
+  // misc: 16 B words + red[2][4][NQ] + alpha[2][NQ] + lsum[4][NQ] + mfin[NQ]
+  const int misc = 16 + (8 + 2 + 4 + 1) * nq * 4;
+  return P.off_misc + misc + 1024;
+}
+
+template <int NQ>
+cudaError_t launch_mu_nq(const MuParams& P, int smem, cudaStream_t st) {
+  cudaError_t e = ensure_smem_limit<3000 + NQ>(mu_attention_kernel<NQ>, kMuSmemBudget + 2048);
+  if (e != cudaSuccess) return e;
+  mu_attention_kernel<NQ><<<P.n_units, kMuThreads, smem, st>>>(P);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int mu_query_tile(int nq_total, int d) {
+  // the widest query tile whose accumulators fit TMEM: NQ (2 + d/128) <= 512
+  for (int nq : {64, 32, 16}) {
+    if (nq * (2 + d / 128) > 512) continue;
+    if (nq <= 16 || nq_total > nq / 2) return nq;
+  }
+  return 0;
+}
+
+int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity) {
+  return encode3d(map, pool, (uint64_t)d, (uint64_t)kRows, (uint64_t)capacity, 64);
+}
+
+cudaError_t launch_mu_attention(MuParams& P, int nq, cudaStream_t st) {
+  if (P.n_units == 0) return cudaSuccess;
+  if (encode3d(&P.q, P.qptr, (uint64_t)P.d, (uint64_t)P.nrows, (uint64_t)P.n_qg, (uint32_t)nq)) return cudaErrorInvalidValue;
+  const int smem = mu_smem_plan(P, nq, P.d);
+  if (smem < 0 || smem > kMuSmemBudget + 2048) return cudaErrorInvalidValue;
+  if (nq == 64) return launch_mu_nq<64>(P, smem, st);
+  if (nq == 32) return launch_mu_nq<32>(P, smem, st);
+  if (nq == 16) return launch_mu_nq<16>(P, smem, st);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace smem

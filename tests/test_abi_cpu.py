@@ -28,7 +28,7 @@ def test_exports_every_declared_symbol():
     for n in names:
         assert hasattr(L, n), n
     assert set(names) == set(smem.EXPORTED)
-    assert smem.smem_abi_version() == 2
+    assert smem.smem_abi_version() == 3
 
 
 def test_required_bytes_validation():
@@ -145,5 +145,25 @@ def test_layer_entry_points_on_a_bookkeeping_cache():
         seq = (ctypes.c_int32 * 1)(0)
         assert L.smem_reader_layer_decode(h, 0, 1, seq, seq, seq, arr, None, None, 0, None) == smem.ERR_NO_DEVICE
         assert smem.smem_get_table(h, 0) == ([], [])
+    finally:
+        smem.smem_cache_destroy(h)
+
+
+def test_recompute_geometry():
+    """A recompute cache's slot holds R*d bf16 memory rows instead of the
+    L*H*2*R*d_h of the materialized K/V; unsupported widths are refused."""
+    mat = smem.make_config(4, 4, 64, 2, 8, 64)
+    rec = smem.make_config(4, 4, 64, 2, 8, 64, recompute_kv=True)
+    diff = smem.smem_cache_required_bytes(mat) - smem.smem_cache_required_bytes(rec)
+    assert abs(diff - 64 * (4 * 4 * 2 * 64 * 64 * 2 - 64 * 256 * 2)) < 8192
+    assert smem.smem_cache_required_bytes(smem.make_config(1, 1, 64, 1, 4, 4, recompute_kv=True)) == 0  # d = 64
+    h = smem.smem_cache_create(rec, None)
+    try:
+        d = 4 * 64
+        w0 = smem.smem_layer_workspace_bytes(h, 0)
+        w2 = smem.smem_layer_workspace_bytes(h, 2)
+        # per row: the dense buffers, q' and O' [H][d] bf16, split partials
+        dense = 6 * d * 2 + 4 * d * 4 + 4 * d * 2
+        assert w2 - w0 >= 2 * (dense + 2 * 4 * d * 2)
     finally:
         smem.smem_cache_destroy(h)

@@ -30,10 +30,10 @@ class LayerCache:
     """A device cache filled through the reader-layer entry points."""
 
     def __init__(self, model: LayerModel, H, D, max_seqs, max_blocks, capacity, has_null=True, free_order=None,
-                 max_batch=None):
+                 max_batch=None, recompute=False):
         self.m, self.H, self.D, self.d = model, H, D, H * D
         self.cfg = smem.make_config(model.L, H, D, max_seqs, max_blocks, capacity, has_null_row=has_null,
-                                    max_decode_batch=max_batch, free_order=free_order)
+                                    max_decode_batch=max_batch, free_order=free_order, recompute_kv=recompute)
         self.cache = smem.SmemCache(self.cfg, device="cuda")
         self.h = self.cache.h
         self.mirror = CacheMirror(capacity, max_seqs, max_blocks, free_order=free_order)
@@ -118,14 +118,15 @@ def test_layer_block_skip_equals_full_pass():
         assert_layer_close(_np(x), full[sl], X[sl], f"block {i}")
 
 
-def _decode_setup(model, H, D, ctx, free_order=None, history=False):
+def _decode_setup(model, H, D, ctx, free_order=None, history=False, recompute=False):
     """Sequences with the given contexts; each sequence's current block
     (index ctx[s]) runs the layer prefill on all layers first, leaving its
     in-block rows. history=True reaches the same block set by another edit
     path (extra blocks appended and deleted, a delete/re-append)."""
     S = len(ctx)
     cap = sum(ctx) + 4 * S + 8
-    lc = LayerCache(model, H, D, max_seqs=S, max_blocks=max(ctx) + 8, capacity=cap, free_order=free_order)
+    lc = LayerCache(model, H, D, max_seqs=S, max_blocks=max(ctx) + 8, capacity=cap, free_order=free_order,
+                    recompute=recompute)
     for s, n in enumerate(ctx):
         order = list(range(n))
         if history:

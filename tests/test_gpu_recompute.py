@@ -1,0 +1,139 @@
+"""GPU parity of the recompute-K/V regime (the pool holds only the memory rows
+mu; every reader-layer call re-derives the layer's cross-attention from them,
+arXiv 2609.32395, Sec. 3.1 and App. "Serving") against the same fp64 layer
+oracle as the materialized path -- keys mu W_kc and values mu W_vc are the
+oracle's definition; the kernel's re-association is checked against it:
+
+* one-block prefill and batched decode per layer, with and without the null
+  row, d_h 64/128, at test shapes and at the 160M / 410M / 1.5B widths;
+* bitwise edit-path independence (Theorem 1) of prefill and decode outputs;
+* agreement with the materialized cache on the same inputs;
+* entry points that take projected K/V refuse a recompute cache.
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle.reader_layer import reader_layer_decode, reader_layer_prefill
+from paper_2609_32395_gb300 import smem
+from tests.layer_helpers import B_TOK, LayerModel, assert_layer_close, bits_dev, mu_bits
+from tests.test_gpu_layer import LayerCache, _decode_setup, _np, x_rows
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("D,H,has_null", [(64, 4, True), (64, 4, False), (128, 2, True)])
+def test_recompute_layer_prefill_matches_oracle(D, H, has_null):
+    model = LayerModel(2, H * D, seed=601 + D)
+    lc = LayerCache(model, H, D, max_seqs=1, max_blocks=16, capacity=24, has_null=has_null,
+                    free_order=synth.slot_permutation(3, 24), recompute=True)
+    for j in (5, 0, 7, 2, 6, 1, 4, 3):
+        lc.append(0, j)
+    for q_idx in (8, 3, 0):
+        x = torch.from_numpy(x_rows(model.seed, 0, q_idx, lc.d)).cuda()
+        for layer in range(model.L):
+            x_in = _np(x)
+            lc.prefill(0, layer, q_idx, x)
+            ref, _, _ = lc.oracle_prefill(0, layer, q_idx, x_in)
+            assert_layer_close(_np(x), ref, x_in, f"layer {layer} q_idx {q_idx}")
+    assert smem.smem_check_device_error(lc.h) == smem.OK
+
+
+@pytest.mark.parametrize("H,D,nblk", [(12, 64, 64), (16, 64, 40), (16, 128, 24)])
+def test_recompute_prefill_at_model_widths(H, D, nblk):
+    """d = 768 / 1024 / 2048 (the 160M / 410M / 1.5B reader widths): every
+    query-tile width of the kernel (64, 32, 16 queries per CTA)."""
+    d = H * D
+    model = LayerModel(1, d, seed=701 + d)
+    lc = LayerCache(model, H, D, max_seqs=1, max_blocks=nblk + 4, capacity=nblk + 4, recompute=True)
+    for j in range(nblk):
+        lc.append(0, j)
+    x = torch.from_numpy(x_rows(model.seed, 0, nblk, d)).cuda()
+    x_in = _np(x)
+    lc.prefill(0, 0, nblk, x)
+    ref, _, _ = lc.oracle_prefill(0, 0, nblk, x_in)
+    assert_layer_close(_np(x), ref, x_in, f"d {d}")
+
+
+def _decode_check(model, lc, xs, ctx, pos, H, D):
+    x = torch.from_numpy(np.stack([xs[s][0][0][pos[s]] for s in range(len(ctx))]).astype(np.float32)).cuda()
+    for layer in range(model.L):
+        x_in = _np(x)
+        lc.decode(layer, list(range(len(ctx))), pos, ctx, x)
+        got = _np(x)
+        for s in range(len(ctx)):
+            ids, mu = lc.memory(s, ctx[s])
+            _, ks, vs = reader_layer_prefill(xs[s][0][layer], ids, mu, ctx[s], model.oracle[layer], H, D, lc.nu)
+            ref, _, _ = reader_layer_decode(x_in[s], ids, mu, ctx[s], pos[s], ks[:pos[s]], vs[:pos[s]],
+                                            model.oracle[layer], H, D, lc.nu)
+            assert_layer_close(got[s], ref, x_in[s], f"decode layer {layer} seq {s}")
+    return _np(x)
+
+
+@pytest.mark.parametrize("H,D", [(4, 64), (16, 64), (12, 128)])
+def test_recompute_decode_after_prefill_matches_oracle(H, D):
+    """Batched decode (contexts 5, 0, 9, 30 blocks; offsets 17, 0, 63, 5)
+    after each sequence's layer prefill."""
+    model = LayerModel(2, H * D, seed=809 + H)
+    ctx, pos = [5, 0, 9, 30], [17, 0, 63, 5]
+    lc, xs = _decode_setup(model, H, D, ctx, recompute=True)
+    _decode_check(model, lc, xs, ctx, pos, H, D)
+    assert smem.smem_check_device_error(lc.h) == smem.OK
+
+
+def test_recompute_outputs_are_edit_path_independent():
+    H, D, L = 4, 64, 2
+    model = LayerModel(L, H * D, seed=907)
+    ctx = [20, 3]
+    a, xa = _decode_setup(model, H, D, ctx, recompute=True)
+    b, xb = _decode_setup(model, H, D, ctx, free_order=synth.slot_permutation(5, sum(ctx) + 16), history=True,
+                          recompute=True)
+    assert a.mirror.table(0)[1] != b.mirror.table(0)[1]
+    for s in range(2):
+        np.testing.assert_array_equal(xa[s][1], xb[s][1])
+    pos = [11, 40]
+    x0 = np.stack([xa[s][0][0][pos[s]] for s in range(2)]).astype(np.float32)
+    outs = []
+    for lc in (a, b):
+        x = torch.from_numpy(x0).cuda()
+        for layer in range(L):
+            lc.decode(layer, [0, 1], pos, ctx, x)
+        outs.append(_np(x))
+    np.testing.assert_array_equal(outs[0], outs[1])
+
+
+def test_recompute_agrees_with_materialized_cache():
+    """The same blocks, weights and inputs through both regimes: the outputs
+    agree within the layer tolerance (they round at different places)."""
+    H, D = 4, 64
+    model = LayerModel(1, H * D, seed=1009)
+    ctx = [12]
+    m, xm = _decode_setup(model, H, D, ctx)
+    r, xr = _decode_setup(model, H, D, ctx, recompute=True)
+    assert_layer_close(xr[0][1], xm[0][1].astype(np.float64), xm[0][0][0], "prefill: recompute vs materialized")
+
+
+def test_recompute_cache_refuses_projected_kv_entries():
+    H, D = 4, 64
+    d = H * D
+    model = LayerModel(2, d, seed=1103)
+    mat = smem.make_config(2, H, D, 2, 8, 8, has_null_row=True)
+    rec = smem.make_config(2, H, D, 2, 8, 8, has_null_row=True, recompute_kv=True)
+    # the pool shrinks from L*H*2*R*d_h to R*d elements per slot (2L = 4 times)
+    pool_m = 8 * 2 * H * 2 * 64 * D * 2
+    pool_r = 8 * 64 * d * 2
+    assert smem.smem_cache_required_bytes(mat) - smem.smem_cache_required_bytes(rec) >= pool_m - pool_r - (1 << 20)
+    lc = LayerCache(model, H, D, max_seqs=2, max_blocks=8, capacity=8, recompute=True)
+    t = torch.zeros(B_TOK, H, D, dtype=torch.bfloat16, device="cuda")
+    kv = torch.zeros(2, H, 64, D, dtype=torch.bfloat16, device="cuda")
+    for call in (lambda: smem.smem_append_block(lc.h, 0, 0, kv, kv),
+                 lambda: smem.smem_set_null_row(lc.h, t[0], t[0]),
+                 lambda: smem.smem_prefill_block(lc.h, 0, 0, 0, t, t, t, t, t, t),
+                 lambda: smem.smem_decode(lc.h, 0, [0], [0], [0], t[:1], t[:1], t[:1], t[:1], t[:1], t[:1])):
+        with pytest.raises(smem.SmemError) as e:
+            call()
+        assert e.value.code == smem.ERR_UNSUPPORTED
+    # memory rows need no weights on a recompute cache
+    slot = smem.smem_append_block_rows(lc.h, 1, 0, bits_dev(mu_bits(1, 1, 0, d)), [], lc.ws)
+    assert slot == lc.mirror.append(1, 0)[1]
