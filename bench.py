@@ -46,6 +46,7 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-serve", action="store_true")
     ap.add_argument("--no-layer", action="store_true", help="skip the full-reader-layer cells")
+    ap.add_argument("--no-recompute", action="store_true", help="skip the recompute-K/V cells")
     ap.add_argument("--workload", default="decode", choices=["decode", "long"],
                     help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
     ap.add_argument("--long-batches", default="1,16", help="batches of the long-context cells")
@@ -392,6 +393,118 @@ def measure_layer_decode(wl, steps, warmup, device):
             "timing": "CUDA events around the layer calls of each step (appends excluded), inputs resident"}
 
 
+class RecomputeDecode:
+    """The 410M-shaped decode workload on a recompute-K/V cache: the pool
+    holds only each block's memory rows mu [R][d] (d = H*d_h, shared by the
+    24 layers); every layer re-derives its cross-attention from them. Same
+    sequences, contexts and in-block offsets as the materialized workload."""
+
+    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None):
+        import torch
+
+        import synth
+        from paper_2609_32395_gb300 import smem
+
+        W = WORKLOAD
+        self.L, self.H, self.D = (layers or W["L"]), W["H"], W["D"]
+        self.d = self.H * self.D
+        self.S = seqs
+        self.seed = rank_seed(seed, rank)
+        self.nblk = synth.ragged_contexts(self.seed, seqs, W["ctx_lo"], W["ctx_hi"]).astype(np.int64)
+        self.pos = synth.inblock_positions(self.seed, seqs, B_TOK).astype(np.int64)
+        n_new = [(int(p) + steps_total) // B_TOK + 1 for p in self.pos]
+        capacity = int(self.nblk.sum()) + sum(n_new)
+        max_blocks = int(self.nblk.max()) + max(n_new) + 1
+        perm = synth.slot_permutation(self.seed, capacity)
+        self.cfg = smem.make_config(self.L, self.H, self.D, seqs, max_blocks, capacity, free_order=perm,
+                                    recompute_kv=True)
+        self.cache = smem.SmemCache(self.cfg, device=device)
+        self.h = self.cache.h
+        self.ws = torch.empty(smem.smem_layer_workspace_bytes(self.h, seqs), dtype=torch.uint8, device=device)
+        for s in range(seqs):
+            n = int(self.nblk[s])
+            mu = synth.tensor_torch(self.seed, synth.KIND_MU, (n * R, self.d), s, device=device)
+            for j in range(n):
+                smem.smem_append_block_rows(self.h, s, j, mu[j * R:(j + 1) * R], [], self.ws)
+            del mu
+        for s in range(seqs):
+            p = int(self.pos[s])
+            for layer in range(self.L):
+                if p:
+                    Kb = synth.tensor_torch(self.seed, synth.KIND_KIN, (p, self.H, self.D), s, layer, 0,
+                                            device=device)
+                    Vb = synth.tensor_torch(self.seed, synth.KIND_VIN, (p, self.H, self.D), s, layer, 0,
+                                            device=device)
+                    smem.smem_write_inblock(self.h, s, layer, p, Kb, Vb)
+        self.seq_ids = np.arange(seqs, dtype=np.int32)
+        self.new_used = [0] * seqs
+        self.step_no = 0
+        torch.cuda.synchronize()
+
+    def rows_read(self):
+        return int(self.nblk.sum()) * R
+
+
+def measure_recompute(steps, warmup, device, seqs, layers=None):
+    """Recompute-K/V regime at the 410M decode shape: the memory-row
+    attention kernel alone (CUDA events per launch; algorithmic bytes = 2d
+    per memory row read + the folded queries and outputs) and the full
+    reader layer's decode tok/s on the same cache."""
+    import torch
+
+    import synth
+    from paper_2609_32395_gb300 import smem
+
+    rw = RecomputeDecode(seqs, warmup + steps + 4 + (warmup + steps), WORKLOAD["seed"], device, layers=layers)
+    d, H = rw.d, rw.H
+    qp = (synth.tensor_torch(rw.seed, synth.KIND_QDEC_C, (seqs, H, d), 7, device=device).float() / math.sqrt(d)
+          ).to(torch.bfloat16)
+    op = torch.empty(seqs, H, d, dtype=torch.bfloat16, device=device)
+    st = torch.cuda.current_stream()
+    ctx = rw.nblk.astype(np.int32)
+    for _ in range(warmup):
+        smem.smem_mu_decode(rw.h, rw.seq_ids, ctx, qp, op, rw.ws)
+    torch.cuda.synchronize()
+    n_launch = steps * 2
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(n_launch)]
+    for i in range(n_launch):
+        ev[i][0].record(st)
+        smem.smem_mu_decode(rw.h, rw.seq_ids, ctx, qp, op, rw.ws)
+        ev[i][1].record(st)
+    torch.cuda.synchronize()
+    if smem.smem_check_device_error(rw.h) != smem.OK:
+        raise RuntimeError("device error recorded during the memory-row attention")
+    kern_ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+    rows = rw.rows_read()
+    alg = rows * 2 * d + 2 * seqs * H * d * 2
+    kernel = {"kernel": "mu_attention_kernel<16> (memory-row cross-attention, tcgen05)", "launches": n_launch,
+              "kernel_ms_mean": kern_ms, "rows_per_launch": rows, "alg_bytes_per_launch": alg,
+              "achieved_gbs": alg / (kern_ms / 1e3) / 1e9,
+              "materialized_bytes_per_launch": rows * 4 * H * rw.D}
+    # full reader layer on the recompute cache (appends take memory rows)
+    stack = LayerStack(rw.L, d, 5, device)
+    x0 = synth.tensor_torch(rw.seed, synth.KIND_X, (seqs, d), 0, device=device).float()
+    x = x0.clone()
+    mu = synth.tensor_torch(rw.seed, synth.KIND_MU, (R, d), 1 << 20, device=device)
+    for _ in range(warmup):
+        layer_decode_step(rw, stack, x, rw.ws, mu)
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+    for i in range(steps):
+        x.copy_(x0)
+        layer_decode_step(rw, stack, x, rw.ws, mu, events=evs[i])
+    torch.cuda.synchronize()
+    if smem.smem_check_device_error(rw.h) != smem.OK:
+        raise RuntimeError("device error recorded during the recompute decode")
+    step_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    out = {"workload": WORKLOAD["name"] + ", recompute-K/V cache", "pool_bytes": int(rw.cache.nbytes),
+           "memory_row_kernel": kernel,
+           "layer_decode": {"tok_per_s": seqs / (step_ms / 1e3), "step_ms": step_ms, "steps": steps,
+                            "timing": "CUDA events around each step's layer calls (appends excluded)"}}
+    rw.cache.close()
+    return out
+
+
 # ----------------------------------------------------------------------------- prefill workload
 SERVE = dict(name="160M-shaped one-block cached-context prefill", L=12, H=12, D=64, contexts=(16, 64, 256), seed=1)
 
@@ -401,7 +514,7 @@ class PrefillWorkload:
     shuffled slots) served by running the reader's attention on the final
     block alone: 12 one-block prefill launches, one per layer."""
 
-    def __init__(self, nblk, device, L=None, H=None, D=None, seed=None):
+    def __init__(self, nblk, device, L=None, H=None, D=None, seed=None, recompute=False):
         import torch
 
         import synth
@@ -414,9 +527,19 @@ class PrefillWorkload:
         seed = SERVE["seed"] if seed is None else seed
         cap = nblk + 2
         self.cfg = smem.make_config(self.L, self.H, self.D, 1, nblk + 1, cap,
-                                    free_order=synth.slot_permutation(seed + nblk, cap))
+                                    free_order=synth.slot_permutation(seed + nblk, cap), recompute_kv=recompute)
         self.cache = smem.SmemCache(self.cfg, device=device)
         self.h = self.cache.h
+        if recompute:  # the pool keeps memory rows only; attention-only launches do not apply
+            import torch
+
+            d = self.H * self.D
+            ws = torch.empty(smem.smem_layer_workspace_bytes(self.h, 0), dtype=torch.uint8, device=device)
+            mu = synth.tensor_torch(seed, synth.KIND_MU, (max(nblk, 1) * R, d), 0, device=device)
+            for j in range(nblk):
+                smem.smem_append_block_rows(self.h, 0, j, mu[j * R:(j + 1) * R], [], ws)
+            torch.cuda.synchronize()
+            return
         for b0 in range(0, nblk, 16):
             ids = list(range(b0, min(nblk, b0 + 16)))
             K, V = synth.block_rows_torch(seed, 0, ids, self.L, self.H, R, self.D, device)
@@ -496,7 +619,7 @@ def measure_serve(nblk, device, iters=30, flush_bytes=512 << 20):
     return out
 
 
-def measure_layer_serve(nblk, device, iters=30, flush_bytes=512 << 20):
+def measure_layer_serve(nblk, device, iters=30, flush_bytes=512 << 20, recompute=False):
     """Latency of one cached-context serve through the full reader layer
     (12 layers of LayerNorm, projections, attention and FFN over the final
     block's 64 tokens), replayed from a CUDA graph with L2 flushed before
@@ -506,7 +629,7 @@ def measure_layer_serve(nblk, device, iters=30, flush_bytes=512 << 20):
     import synth
     from paper_2609_32395_gb300 import smem
 
-    wl = PrefillWorkload(nblk, device)
+    wl = PrefillWorkload(nblk, device, recompute=recompute)
     d = wl.H * wl.D
     stack = LayerStack(wl.L, d, 6, device)
     ws = torch.empty(smem.smem_layer_workspace_bytes(wl.h, B_TOK), dtype=torch.uint8, device=device)
@@ -541,7 +664,7 @@ def measure_layer_serve(nblk, device, iters=30, flush_bytes=512 << 20):
         raise RuntimeError("device error recorded during the full-layer serve")
     lat = sorted(a.elapsed_time(b) for a, b in zip(e0, e1))
     del g
-    kv = nblk * R * 4 * d * wl.L
+    kv = nblk * R * (2 * d if recompute else 4 * d) * wl.L  # memory rows (recompute) or K/V read per layer
     w = stack.bytes_per_layer() * wl.L
     alg = kv + w
     med = lat[len(lat) // 2]
@@ -927,7 +1050,10 @@ def run_ours(args):
     layer_dec = measure_layer_decode(wl, layer_steps, args.warmup, device) if layer_steps else None
 
     # --- one-block cached-context serve (prefill), the metric's second half
-    serve = layer_serve = None
+    serve = layer_serve = rec_serve = None
+    recompute = None
+    if not args.no_recompute and rank == 0:
+        recompute = measure_recompute(min(args.steps, 64), args.warmup, device, args.seqs, layers=args.layers)
     if not args.no_serve:
         wl.cache.close()
         wl.cache.buf = None
@@ -935,6 +1061,8 @@ def run_ours(args):
         torch.cuda.empty_cache()
         serve = [measure_serve(n, device) for n in SERVE["contexts"]]
         layer_serve = None if args.no_layer else [measure_layer_serve(n, device) for n in SERVE["contexts"]]
+        if not args.no_layer and not args.no_recompute:
+            rec_serve = [measure_layer_serve(n, device, recompute=True) for n in SERVE["contexts"]]
     edit = None if args.no_serve else [measure_edit_latency(n, device) for n in EDIT["contexts"]]
 
     if rank != 0:
@@ -991,6 +1119,15 @@ def run_ours(args):
             layer["serve"] = {"workload": SERVE["name"], "unit": "ms", "cells": layer_serve,
                               "timing": "CUDA graph of the 12 layer calls, L2 flushed before each"}
         line["layer"] = layer
+    if recompute:
+        k = recompute["memory_row_kernel"]
+        k["hbm_frac"] = k["achieved_gbs"] / peak
+        if rec_serve:
+            for c in rec_serve:
+                c["hbm_frac"] = c["achieved_gbs"] / peak
+            recompute["layer_serve"] = {"workload": SERVE["name"] + ", recompute-K/V cache", "unit": "ms",
+                                        "cells": rec_serve}
+        line["recompute"] = recompute
     if edit:
         line["edit"] = {"workload": EDIT["name"], "unit": "us",
                         "note": "host = whole C ABI call; device = table-edit kernel; no row moves", "cells": edit}
@@ -1013,7 +1150,11 @@ def run_serve_only(args):
     torch.cuda.set_device(0)
     smem.lib()
     cells = [measure_serve(n, torch.device("cuda", 0)) for n in SERVE["contexts"]]
-    print(json.dumps({"serve_only": True, "workload": SERVE["name"], "cells": cells}), flush=True)
+    out = {"serve_only": True, "workload": SERVE["name"], "cells": cells}
+    if not args.no_recompute:  # the full reader layer on a recompute-K/V cache
+        out["recompute_layer_cells"] = [measure_layer_serve(n, torch.device("cuda", 0), recompute=True)
+                                        for n in SERVE["contexts"]]
+    print(json.dumps(out), flush=True)
 
 
 def main():

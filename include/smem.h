@@ -295,6 +295,25 @@ int smem_reader_layer_decode(smem_cache *c, int32_t layer, int32_t nb, const int
                              const smem_layer_weights *w, float *x, void *ws, size_t ws_bytes,
                              void *stream);
 
+/* The memory-row cross-attention of a recompute_kv cache on its own (the
+ * step between the two per-head maps of the reader layer): for every query
+ * vector q' (d wide, already multiplied by W_kc,h and by the softmax scale
+ * log2(e)/sqrt(d_h) -- scores are base-2 exponents)
+ *   O'[q] = sum_r softmax_r(q' . mu_r) mu_r
+ * over the null row nu (if any) and the memory rows of the table blocks with
+ * index < the query block index, ascending. bf16 in and out, fp32
+ * accumulation. ws as for the layer calls (smem_layer_workspace_bytes with
+ * n_rows = nb, or b for the prefill form).
+ * smem_mu_decode: item i reads sequence seq_ids[i] (distinct) below block
+ *   q_block_idx[i] (host arrays [nb]); qp, op device [nb][H][d].
+ * smem_mu_prefill: the b queries of every head of block q_block_idx of seq;
+ *   qp, op device [H][b][d].
+ * SMEM_ERR_UNSUPPORTED on a cache without recompute_kv. */
+int smem_mu_decode(smem_cache *c, int32_t nb, const int32_t *seq_ids, const int32_t *q_block_idx,
+                   const void *qp, void *op, void *ws, size_t ws_bytes, void *stream);
+int smem_mu_prefill(smem_cache *c, int32_t seq, int32_t q_block_idx, const void *qp, void *op, void *ws,
+                    size_t ws_bytes, void *stream);
+
 /* Introspection for bit-exact bookkeeping checks (host state, no CUDA).
  * smem_get_table: the table of `seq` in ascending block index; up to `cap`
  * entries into idx_out / slot_out (either may be NULL); *n_out = length.

@@ -107,8 +107,6 @@ int make_layout(const smem_config* c, Layout* L) {
   off = align_up(off + (size_t)L->H * L->pf_max_splits * smem::kBlockTok * (D + 4) * 4, A);
   L->off_pf_cnt = off;
   off = align_up(off + (size_t)L->H * 4, A);
-  L->off_mu_cnt = off;
-  off = align_up(off + (size_t)smem::kMaxMuGroups * 4, A);
   L->off_err = off;
   off = align_up(off + 256, A);
   L->total = off;
@@ -817,32 +815,18 @@ struct LayerRun {
   }
 };
 
-// Cross-attention of a layer call on a recompute cache (the memory rows mu
-// in the pool): q'_h = scale W_kc,h q_h, O'_h = attention of q'_h over the
-// rows, att_h = O'_h W_vc,h. Prefill: one row set, groups (head, query
-// tile); decode: one group per sequence holding all its heads.
-int mu_cross_attention(LayerRun& r, int layer, int nb, const int32_t* seq_ids, const int32_t* q_block_idx,
-                       bool prefill, int seq, int q_idx) {
-  smem_cache* c = r.c;
+// The memory-row attention launch(es): O' of every query in qp (prefill:
+// [H][b][d], one row set; decode: [nb][H][d], one row set per item).
+int mu_attend(smem_cache* c, uint8_t* ws, const LayerWs& o, bool prefill, int nb, const int32_t* seq_ids,
+              const int32_t* q_block_idx, int seq, int q_idx, const uint16_t* qp, uint16_t* op, cudaStream_t st) {
   const Layout& L = c->lay;
-  const int d = r.d, H = L.H, D = L.D;
-  const float scale = (float)(1.4426950408889634 / std::sqrt((double)D));
-  const uint16_t* wkc = static_cast<const uint16_t*>(r.w->w_kc);
-  const uint16_t* wvc = static_cast<const uint16_t*>(r.w->w_vc);
-  uint16_t* qp = reinterpret_cast<uint16_t*>(r.ws + r.o.qp);
-  uint16_t* op = reinterpret_cast<uint16_t*>(r.ws + r.o.op);
-  const int nq = prefill ? smem::kBlockTok : nb;  // queries per head
-  // q'[.][h][i] = scale sum_j qc[.][h][j] W_kc[i][h D + j]; prefill stores [h][q][d], decode [s][h][d]
-  int rc = blas_rc(smem::blas_gemm_sb(c->blas, true, false, d, nq, D, scale, wkc, d, D, r.qc(), d, D, qp,
-                                      prefill ? d : H * d, prefill ? (long long)smem::kBlockTok * d : d, H, g_detail,
-                                      sizeof(g_detail)));
-  if (rc) return rc;
+  const int d = L.H * L.D, H = L.H;
+  int rc = SMEM_OK;
   static thread_local smem::MuParams P;
   P.pool = c->pool_map_mu;
   P.table = reinterpret_cast<const int*>(c->dev + L.off_table);
   P.nu = L.has_null ? reinterpret_cast<const uint16_t*>(c->dev + L.off_null) : nullptr;
-  P.part = reinterpret_cast<float*>(r.ws + r.o.part);
-  P.counters = reinterpret_cast<unsigned*>(c->dev + L.off_mu_cnt);
+  P.part = reinterpret_cast<float*>(ws + o.part);
   P.err = reinterpret_cast<int*>(c->dev + L.off_err);
   P.d = d;
   P.max_blocks = L.max_blocks;
@@ -869,7 +853,7 @@ int mu_cross_attention(LayerRun& r, int layer, int nb, const int32_t* seq_ids, c
       }
     P.n_units = u;
     if (injected_failure(c)) return SMEM_ERR_CUDA;
-    rc = cuda_rc(smem::launch_mu_attention(P, nqt, r.st), "memory-row attention");
+    rc = cuda_rc(smem::launch_mu_attention(P, nqt, st), "memory-row attention");
   } else {
     const int nqt = smem::mu_query_tile(H, d);
     for (int i0 = 0; i0 < nb && !rc; i0 += smem::kMaxMuGroups) {
@@ -890,9 +874,33 @@ int mu_cross_attention(LayerRun& r, int layer, int nb, const int32_t* seq_ids, c
       }
       P.n_units = u;
       if (injected_failure(c)) return SMEM_ERR_CUDA;
-      rc = cuda_rc(smem::launch_mu_attention(P, nqt, r.st), "memory-row attention");
+      rc = cuda_rc(smem::launch_mu_attention(P, nqt, st), "memory-row attention");
     }
   }
+  return rc;
+}
+
+// Cross-attention of a layer call on a recompute cache (the memory rows mu
+// in the pool): q'_h = scale W_kc,h q_h, O'_h = attention of q'_h over the
+// rows, att_h = O'_h W_vc,h. Prefill: one row set, groups (head, query
+// tile); decode: one group per sequence holding all its heads.
+int mu_cross_attention(LayerRun& r, int layer, int nb, const int32_t* seq_ids, const int32_t* q_block_idx,
+                       bool prefill, int seq, int q_idx) {
+  smem_cache* c = r.c;
+  const Layout& L = c->lay;
+  const int d = r.d, H = L.H, D = L.D;
+  const float scale = (float)(1.4426950408889634 / std::sqrt((double)D));
+  const uint16_t* wkc = static_cast<const uint16_t*>(r.w->w_kc);
+  const uint16_t* wvc = static_cast<const uint16_t*>(r.w->w_vc);
+  uint16_t* qp = reinterpret_cast<uint16_t*>(r.ws + r.o.qp);
+  uint16_t* op = reinterpret_cast<uint16_t*>(r.ws + r.o.op);
+  const int nq = prefill ? smem::kBlockTok : nb;  // queries per head
+  // q'[.][h][i] = scale sum_j qc[.][h][j] W_kc[i][h D + j]; prefill stores [h][q][d], decode [s][h][d]
+  int rc = blas_rc(smem::blas_gemm_sb(c->blas, true, false, d, nq, D, scale, wkc, d, D, r.qc(), d, D, qp,
+                                      prefill ? d : H * d, prefill ? (long long)smem::kBlockTok * d : d, H, g_detail,
+                                      sizeof(g_detail)));
+  if (rc) return rc;
+  rc = mu_attend(c, r.ws, r.o, prefill, nb, seq_ids, q_block_idx, seq, q_idx, qp, op, r.st);
   if (rc) return rc;
   // att[.][h][e] = sum_i O'[h-row][i] W_vc[i][h D + e]
   return blas_rc(smem::blas_gemm_sb(c->blas, false, false, D, nq, d, 1.f, wvc, d, D, op,
@@ -969,6 +977,47 @@ int smem_reader_layer_decode(smem_cache* c, int32_t layer, int32_t nb, const int
   }
   if (!rc) rc = r.after_ca();
   return rc;
+}
+
+int smem_mu_decode(smem_cache* c, int32_t nb, const int32_t* seq_ids, const int32_t* q_block_idx, const void* qp,
+                   void* op, void* ws, size_t ws_bytes, void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (!c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
+  if (nb < 1 || nb > c->lay.max_batch || !seq_ids || !q_block_idx || !qp || !op) return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(qp) || !aligned16(op)) return SMEM_ERR_ALIGN;
+  if (++c->seen_epoch == 0) {
+    std::fill(c->seen.begin(), c->seen.end(), 0u);
+    c->seen_epoch = 1;
+  }
+  for (int i = 0; i < nb; ++i) {
+    const int s = seq_ids[i];
+    if (s < 0 || s >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
+    if (c->seen[s] == c->seen_epoch || q_block_idx[i] < 0) return SMEM_ERR_INVALID_ARG;
+    c->seen[s] = c->seen_epoch;
+  }
+  DeviceGuard g(c->device);
+  const cudaStream_t st = as_stream(stream);
+  const int rc = layer_begin(c, ws, ws_bytes, nb, st);
+  if (rc) return rc;
+  return mu_attend(c, static_cast<uint8_t*>(ws), layer_ws(c->lay, nb), false, nb, seq_ids, q_block_idx, 0, 0,
+                   static_cast<const uint16_t*>(qp), static_cast<uint16_t*>(op), st);
+}
+
+int smem_mu_prefill(smem_cache* c, int32_t seq, int32_t q_block_idx, const void* qp, void* op, void* ws,
+                    size_t ws_bytes, void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (!c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
+  if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
+  if (q_block_idx < 0 || !qp || !op) return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(qp) || !aligned16(op)) return SMEM_ERR_ALIGN;
+  DeviceGuard g(c->device);
+  const cudaStream_t st = as_stream(stream);
+  const int rc = layer_begin(c, ws, ws_bytes, smem::kBlockTok, st);
+  if (rc) return rc;
+  return mu_attend(c, static_cast<uint8_t*>(ws), layer_ws(c->lay, smem::kBlockTok), true, 0, nullptr, nullptr, seq,
+                   q_block_idx, static_cast<const uint16_t*>(qp), static_cast<uint16_t*>(op), st);
 }
 
 int smem_get_table(const smem_cache* c, int32_t seq, int32_t* idx_out, int32_t* slot_out, int32_t cap,

@@ -28,7 +28,7 @@ struct Layout {
   int pf_max_splits;   // split-K partial slots per prefill head
   size_t slot_elems;   // bf16 elements per pool slot: L*H*2*R*D, or R*d (recompute)
   size_t off_pool, off_inblock, off_null, off_table, off_dec_part, off_dec_cnt, off_pf_part, off_pf_cnt,
-      off_mu_cnt, off_err, total;
+      off_err, total;
 };
 
 // Split-K plan of the decode cross-attention: the number of memory blocks a
@@ -151,7 +151,8 @@ int blas_gemm_sb(void* blas, bool ta, bool tb, int m, int n, int k, float alpha,
 // ---------------------------------------------------------------------------
 constexpr int kMaxMuGroups = 512;   // groups (row set x query tile) per launch
 constexpr int kMuMaxSplits = 16;    // splits of one group's blocks
-constexpr int kMuSmemBudget = 200 * 1024;
+constexpr int kMuSmemBudget = 200 * 1024;  // one CTA per SM
+constexpr int kMuSmemHalf = 110 * 1024;    // two CTAs per SM
 // One group: NQ queries (rows n0.. of query set qg) that read the same row
 // set (the first nblk table blocks of `seq`), cut into nsplit units of
 // split_blks blocks; units of a group are consecutive from unit_begin.
@@ -166,7 +167,6 @@ struct MuParams {
   const uint16_t* nu;         // null row [d] or nullptr
   uint16_t* out;              // O' [n_qg][nrows][d] bf16, normalized
   float* part;                // [unit][NQ][d + 4]: m, l, pad, pad, O'[d]
-  unsigned* counters;         // [kMaxMuGroups], zero between launches
   int* err;
   int d, nrows, n_qg, max_blocks, capacity, n_groups, n_units;
   int ns, off_ring, off_p, off_bar, off_misc;  // shared-memory plan (set by the launcher)
@@ -178,14 +178,18 @@ int mu_query_tile(int nq_total, int d);
 int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity);
 cudaError_t launch_mu_attention(MuParams& P, int nq, cudaStream_t st);
 // Split plans (functions of the block count and the cache geometry only).
+// A split reads at least kMuMinSplitBlocks blocks: its partial (NQ x d fp32)
+// and fixed costs stay small next to the rows it streams.
+constexpr int kMuMinSplitBlocks = 8;
 SMEM_HD inline int mu_decode_split_blocks(int nblk) {
   const int s = (nblk + kMuMaxSplits - 1) / kMuMaxSplits;
-  return s > 8 ? s : 8;
+  return s > kMuMinSplitBlocks ? s : kMuMinSplitBlocks;
 }
 SMEM_HD inline int mu_prefill_split_blocks(int nblk, int groups) {
   int ns = (304 + groups - 1) / groups;
   if (ns > kMuMaxSplits) ns = kMuMaxSplits;
-  if (ns > nblk) ns = nblk;
+  const int cap = (nblk + 3) / 4;  // at least 4 blocks per split
+  if (ns > cap) ns = cap;
   if (ns < 1) ns = 1;
   return (nblk + ns - 1) / ns;
 }

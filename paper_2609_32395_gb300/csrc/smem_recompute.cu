@@ -22,10 +22,11 @@
 // for P.V (the second pass normally hits L2) -- so any d fits in shared
 // memory. Softmax runs column-wise (one query per column) with the same
 // conditional rescale as the prefill kernel (raise the running maximum only
-// when it grows by more than 2^8). Splits of a row set write (m, l, O') and
-// the CTA holding the last ticket merges them in split order, null row first
-// (the null row nu is just one more d-wide row). Reduction orders depend only
-// on the block count, so outputs are bitwise independent of the edit path.
+// when it grows by more than 2^8). Every unit (a split of a row set) writes
+// its partial (m, l, O'); a second kernel, one CTA per (group, 128 columns),
+// merges the splits in split order, null row first (the null row nu is just
+// one more d-wide row). Reduction orders depend only on the block count, so
+// outputs are bitwise independent of the edit path.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -65,7 +66,7 @@ __device__ __forceinline__ void store_bf16(uint16_t* p, float v) {
 }  // namespace
 
 template <int NQ>
-__global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __grid_constant__ MuParams p) {
+__global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_kernel(const __grid_constant__ MuParams p) {
   using C = MuCfg<NQ>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -87,7 +88,6 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __gri
   uint8_t* misc = base + p.off_misc;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 4);
-  volatile unsigned* ticket = reinterpret_cast<volatile unsigned*>(misc + 8);
   float* red = reinterpret_cast<float*>(misc + 16);  // [2][4][NQ] column maxima per warp
   float* alpha = red + 2 * 4 * NQ;                   // [2][NQ] rescale factors
   float* lsum = alpha + 2 * NQ;                      // [4][NQ] column sums per warp
@@ -142,8 +142,7 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __gri
       int k = 0;
       bool ok = true;
       // one pass = the NC chunks of tile t; order S(0), S(1), PV(0), S(2), PV(1), ...
-      auto pass = [&](int t) {
-        const int slot = trow[b0 + t];
+      auto pass = [&](int slot) {
         const bool good = slot >= 0 && slot < p.capacity;
         if (!good) record_error(p.err, kDevErrBounds);
         for (int c = 0; c < NC && ok; ++c, ++k) {
@@ -162,10 +161,17 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __gri
           }
         }
       };
-      pass(0);
+      // slots of tiles t and t+1 in registers; the load of t+2 is issued one
+      // iteration before its use, so its latency hides behind two passes
+      int s_cur = trow[b0];
+      int s_nxt = nt > 1 ? trow[b0 + 1] : 0;
+      pass(s_cur);
       for (int t = 0; t < nt && ok; ++t) {
-        if (t + 1 < nt) pass(t + 1);
-        if (ok) pass(t);
+        const int s_nn = t + 2 < nt ? trow[b0 + t + 2] : 0;
+        if (t + 1 < nt) pass(s_nxt);
+        if (ok) pass(s_cur);
+        s_cur = s_nxt;
+        s_nxt = s_nn;
       }
       if (!ok) {
         // let every copy already issued land before the CTA can exit
@@ -367,70 +373,6 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __gri
           part_u[(size_t)tid * part_stride] = mfin[tid];
           part_u[(size_t)tid * part_stride + 1] = lsum[tid] + lsum[NQ + tid] + lsum[2 * NQ + tid] + lsum[3 * NQ + tid];
         }
-        __threadfence();
-      }
-      ok = all_ok;
-    }
-    // ---------------------------------------------------------- merge
-    const int nq_out = min(NQ, p.nrows - G.n0);  // queries of this group that exist
-    uint16_t* out_g = p.out + ((size_t)G.qg * p.nrows + G.n0) * d;
-    if (nt == 0) {
-      // no readable memory block: the null row's value (nu) or zero
-      for (int i = tid; i < nq_out * d; i += 128) {
-        const int dc = i % d;
-        out_g[i] = p.nu ? p.nu[dc] : (uint16_t)0;
-      }
-    } else if (ok) {
-      if (tid == 0) *ticket = atomicAdd(&p.counters[g], 1u);
-      named_bar_sync(1, 128);
-      if (*ticket == (unsigned)(G.nsplit - 1)) {
-        __threadfence();
-        const int nsp = G.nsplit;
-        const float* part_g = p.part + (size_t)G.unit_begin * NQ * part_stride;
-        float* wsc = reinterpret_cast<float*>(ring);  // [nsp][NQ] split weights, then [NQ] null weights
-        float* wnull = wsc + kMuMaxSplits * NQ;
-        float* snull = wnull + NQ;  // [4][NQ] partial null scores
-        // null scores q'_n . nu (q' carries the softmax scale)
-        if (p.nu) {
-          for (int n = 0; n < NQ; ++n) {
-            float dot = 0.f;
-            if (n < nq_out) {
-              const uint16_t* qrow = p.qptr + ((size_t)G.qg * p.nrows + G.n0 + n) * d;
-              for (int dc = tid; dc < d; dc += 128) dot = fmaf(bf16lo(qrow[dc]), bf16lo(p.nu[dc]), dot);
-            }
-#pragma unroll
-            for (int o = 16; o; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-            if (lane == 0) snull[warp * NQ + n] = dot;
-          }
-        }
-        named_bar_sync(1, 128);
-        if (tid < NQ) {
-          const int n = tid;
-          const float sn = p.nu ? snull[n] + snull[NQ + n] + snull[2 * NQ + n] + snull[3 * NQ + n] : -INFINITY;
-          float M = sn;
-          for (int s2 = 0; s2 < nsp; ++s2) M = fmaxf(M, __ldcg(part_g + ((size_t)s2 * NQ + n) * part_stride));
-          float L = p.nu ? exp2f(sn - M) : 0.f;
-          for (int s2 = 0; s2 < nsp; ++s2) {
-            const float* pr = part_g + ((size_t)s2 * NQ + n) * part_stride;
-            const float f = exp2f(__ldcg(pr) - M);
-            wsc[s2 * NQ + n] = f;
-            L = fmaf(f, __ldcg(pr + 1), L);
-          }
-          const float inv = 1.f / L;
-          for (int s2 = 0; s2 < nsp; ++s2) wsc[s2 * NQ + n] *= inv;
-          wnull[n] = p.nu ? exp2f(sn - M) * inv : 0.f;
-        }
-        named_bar_sync(1, 128);
-        for (int dc = tid; dc < d; dc += 128) {
-          const float nuv = p.nu ? bf16lo(p.nu[dc]) : 0.f;
-          for (int n = 0; n < nq_out; ++n) {
-            float acc = wnull[n] * nuv;
-            for (int s2 = 0; s2 < nsp; ++s2)
-              acc = fmaf(wsc[s2 * NQ + n], __ldcg(part_g + ((size_t)s2 * NQ + n) * part_stride + 4 + dc), acc);
-            store_bf16(out_g + (size_t)n * d + dc, acc);
-          }
-        }
-        if (tid == 0) p.counters[g] = 0u;
       }
     }
   }
@@ -439,6 +381,81 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __gri
   if (warp == 4 && nt > 0) {
     tc::fence_after();
     tc::dealloc(tmem, ncols);
+  }
+}
+
+// Merge of the split partials of every group: CTA (column block, group),
+// thread = one of 128 columns of O'. Splits in split order, null row first.
+template <int NQ>
+__global__ void __launch_bounds__(128) mu_merge_kernel(const __grid_constant__ MuParams p) {
+  __shared__ float snull[4][NQ];
+  __shared__ float wsc[kMuMaxSplits + 1][NQ];  // split weights, then the null row's
+  const int g = blockIdx.y;
+  const MuGroup& G = p.groups[g];
+  const int d = p.d;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int dc = blockIdx.x * 128 + tid;
+  const int nq_out = min(NQ, p.nrows - G.n0);
+  const size_t ps = (size_t)d + 4;
+  uint16_t* out = p.out + ((size_t)G.qg * p.nrows + G.n0) * d;
+  const float nuv = p.nu ? bf16lo(p.nu[dc]) : 0.f;
+  if (G.nblk == 0) {  // no readable memory block: the null row's value or zero
+    for (int n = 0; n < nq_out; ++n) out[(size_t)n * d + dc] = p.nu ? p.nu[dc] : (uint16_t)0;
+    return;
+  }
+  // null scores q'_n . nu (q' carries the softmax scale)
+  if (p.nu) {
+    for (int n = 0; n < NQ; ++n) {
+      float dot = 0.f;
+      if (n < nq_out) {
+        const uint16_t* qrow = p.qptr + ((size_t)G.qg * p.nrows + G.n0 + n) * d;
+        for (int c = tid; c < d; c += 128) dot = fmaf(bf16lo(qrow[c]), bf16lo(p.nu[c]), dot);
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+      if (lane == 0) snull[warp][n] = dot;
+    }
+  }
+  __syncthreads();
+  const int nsp = G.nsplit;
+  const float* part_g = p.part + (size_t)G.unit_begin * NQ * ps;
+  if (tid < NQ) {
+    const int n = tid;
+    const float sn = p.nu ? snull[0][n] + snull[1][n] + snull[2][n] + snull[3][n] : -INFINITY;
+    float ms[kMuMaxSplits], ls[kMuMaxSplits];
+#pragma unroll
+    for (int s2 = 0; s2 < kMuMaxSplits; ++s2) {
+      const float2 v = s2 < nsp ? __ldcg(reinterpret_cast<const float2*>(part_g + ((size_t)s2 * NQ + n) * ps))
+                                : make_float2(-INFINITY, 0.f);
+      ms[s2] = v.x;
+      ls[s2] = v.y;
+    }
+    float M = sn;
+#pragma unroll
+    for (int s2 = 0; s2 < kMuMaxSplits; ++s2) M = fmaxf(M, ms[s2]);
+    float L = p.nu ? exp2f(sn - M) : 0.f;
+    float f[kMuMaxSplits];
+#pragma unroll
+    for (int s2 = 0; s2 < kMuMaxSplits; ++s2) {
+      f[s2] = s2 < nsp ? exp2f(ms[s2] - M) : 0.f;
+      L = fmaf(f[s2], ls[s2], L);
+    }
+    const float inv = 1.f / L;
+#pragma unroll
+    for (int s2 = 0; s2 < kMuMaxSplits; ++s2) wsc[s2][n] = f[s2] * inv;
+    wsc[kMuMaxSplits][n] = p.nu ? exp2f(sn - M) * inv : 0.f;
+  }
+  __syncthreads();
+  for (int n = 0; n < nq_out; ++n) {
+    float v[kMuMaxSplits];
+#pragma unroll
+    for (int s2 = 0; s2 < kMuMaxSplits; ++s2)
+      v[s2] = s2 < nsp ? __ldcg(part_g + ((size_t)s2 * NQ + n) * ps + 4 + dc) : 0.f;
+    float acc = wsc[kMuMaxSplits][n] * nuv;
+#pragma unroll
+    for (int s2 = 0; s2 < kMuMaxSplits; ++s2)
+      if (s2 < nsp) acc = fmaf(wsc[s2][n], v[s2], acc);
+    store_bf16(out + (size_t)n * d + dc, acc);
   }
 }
 
@@ -469,7 +486,9 @@ int encode3d(CUtensorMap* map, const void* ptr, uint64_t d0, uint64_t d1, uint64
 int mu_smem_plan(MuParams& P, int nq, int d) {
   const int qbytes = (d / 64) * nq * 128;
   const int fixed = 2 * nq * 128 + 4096 + 1024;
-  int ns = (kMuSmemBudget - qbytes - fixed) / kMuBox;
+  // two CTAs per SM when the queries leave room for an 8-stage ring in half the SM
+  const int budget = qbytes + fixed + 8 * kMuBox <= kMuSmemHalf ? kMuSmemHalf : kMuSmemBudget;
+  int ns = (budget - qbytes - fixed) / kMuBox;
   ns &= ~1;
   if (ns > 16) ns = 16;
   if (ns < 4) return -1;
@@ -489,6 +508,9 @@ cudaError_t launch_mu_nq(const MuParams& P, int smem, cudaStream_t st) {
   cudaError_t e = ensure_smem_limit<3000 + NQ>(mu_attention_kernel<NQ>, kMuSmemBudget + 2048);
   if (e != cudaSuccess) return e;
   mu_attention_kernel<NQ><<<P.n_units, kMuThreads, smem, st>>>(P);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  mu_merge_kernel<NQ><<<dim3((unsigned)(P.d / 128), (unsigned)P.n_groups), 128, 0, st>>>(P);
   return cudaGetLastError();
 }
 

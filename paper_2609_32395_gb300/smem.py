@@ -37,7 +37,7 @@ EXPORTED = [
     "smem_decode", "smem_decode_static_scratch", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table", "smem_check_device_error",
     "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
     "smem_layer_workspace_bytes", "smem_append_block_rows", "smem_set_null_vector", "smem_reader_layer_prefill",
-    "smem_reader_layer_decode",
+    "smem_reader_layer_decode", "smem_mu_decode", "smem_mu_prefill",
 ]
 
 
@@ -115,6 +115,8 @@ def lib():
                                                          _vp]),
             "smem_reader_layer_decode": (ctypes.c_int, [_vp, _i32, _i32, _i32p, _i32p, _i32p, _wp, _vp, _vp,
                                                         ctypes.c_size_t, _vp]),
+            "smem_mu_decode": (ctypes.c_int, [_vp, _i32, _i32p, _i32p, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
+            "smem_mu_prefill": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -334,6 +336,22 @@ def smem_reader_layer_decode(h, layer, seq_ids, pos, q_block_idx, weights, x, ws
     wp, wn = _ws(ws)
     return _check(lib().smem_reader_layer_decode(h, layer, len(s), sp, pp, qp, arr, _ptr(x), wp, wn,
                                                  _stream(stream)), "smem_reader_layer_decode")
+
+
+def smem_mu_decode(h, seq_ids, q_block_idx, qp, op, ws, stream=None):
+    """Memory-row cross-attention of a recompute cache: qp, op [nb][H][d]."""
+    s, sp = _i32arr(seq_ids)
+    q, qptr = _i32arr(q_block_idx)
+    wp, wn = _ws(ws)
+    return _check(lib().smem_mu_decode(h, len(s), sp, qptr, _ptr(qp), _ptr(op), wp, wn, _stream(stream)),
+                  "smem_mu_decode")
+
+
+def smem_mu_prefill(h, seq, q_block_idx, qp, op, ws, stream=None):
+    """Memory-row cross-attention of one block's queries: qp, op [H][b][d]."""
+    wp, wn = _ws(ws)
+    return _check(lib().smem_mu_prefill(h, seq, q_block_idx, _ptr(qp), _ptr(op), wp, wn, _stream(stream)),
+                  "smem_mu_prefill")
 
 
 class SmemCache:

@@ -137,3 +137,75 @@ def test_recompute_cache_refuses_projected_kv_entries():
     # memory rows need no weights on a recompute cache
     slot = smem.smem_append_block_rows(lc.h, 1, 0, bits_dev(mu_bits(1, 1, 0, d)), [], lc.ws)
     assert slot == lc.mirror.append(1, 0)[1]
+
+
+def _qprime(seed, shape, d, fields):
+    """Folded queries q' (bf16): N(0, 1/d), so that base-2 scores q'.mu have
+    unit spread over N(0,1) memory rows."""
+    z = torch.from_numpy(bits_f64_arr(synth.tensor_np(seed, synth.KIND_QDEC_C, shape, *fields)))
+    return (z.float() * float(np.float32(1.0 / np.sqrt(d)))).to(torch.bfloat16)
+
+
+def bits_f64_arr(bits):
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def _oracle_mu(q, mus, nu):
+    """The oracle's attention with every query reading the same rows: keys =
+    values = the memory rows (broadcast over the queries), scale chosen so
+    that the oracle's exp(q.k / sqrt(d)) equals the kernel's 2^(q'.mu)."""
+    import oracle
+    nq, d = q.shape
+    qo = q * (np.log(2.0) * np.sqrt(d))
+    n = len(mus)
+    bk = np.broadcast_to(np.asarray(mus)[:, None], (n, nq, 64, d)) if n else None
+    kn = np.broadcast_to(nu, (nq, d)) if nu is not None else None
+    zero = np.zeros((nq, d))
+    _, oca = oracle.reader_decode(np.arange(n), bk, bk, n, 0, None, None, zero, zero, zero, qo, kn, kn)
+    return oca
+
+
+@pytest.mark.parametrize("has_null", [True, False])
+def test_mu_decode_kernel_matches_oracle(has_null):
+    """The memory-row attention primitive alone: items with 0, 3, 9 and 300
+    blocks (one to sixteen splits), H = 4 queries of width d = 256 each."""
+    from tests.gpu_helpers import MAX_ABS, MEAN_ABS
+    H, D = 4, 64
+    d = H * D
+    model = LayerModel(1, d, seed=1201)
+    ctx = [0, 3, 9, 300]
+    lc = LayerCache(model, H, D, max_seqs=4, max_blocks=310, capacity=320, has_null=has_null, recompute=True)
+    for s, n in enumerate(ctx):
+        for j in range(n):
+            lc.append(s, j)
+    qp = _qprime(1201, (4, H, d), d, (0,))
+    op = torch.empty(4, H, d, dtype=torch.bfloat16, device="cuda")
+    smem.smem_mu_decode(lc.h, [0, 1, 2, 3], ctx, qp.cuda(), op, lc.ws)
+    got = op.float().cpu().numpy().astype(np.float64)
+    for s, n in enumerate(ctx):
+        _, mus = lc.memory(s, n)
+        ref = _oracle_mu(qp[s].double().numpy(), list(mus), lc.nu)
+        err = np.abs(got[s] - ref)
+        assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (s, err.max(), err.mean())
+    assert smem.smem_check_device_error(lc.h) == smem.OK
+
+
+@pytest.mark.parametrize("H,D,nblk", [(4, 64, 7), (12, 64, 40), (16, 64, 20), (16, 128, 12)])
+def test_mu_prefill_kernel_matches_oracle(H, D, nblk):
+    """The block form: H x 64 queries over one row set, every query-tile
+    width (64, 32, 16)."""
+    from tests.gpu_helpers import MAX_ABS, MEAN_ABS
+    d = H * D
+    model = LayerModel(1, d, seed=1301 + d)
+    lc = LayerCache(model, H, D, max_seqs=1, max_blocks=nblk + 2, capacity=nblk + 2, recompute=True)
+    for j in range(nblk):
+        lc.append(0, j)
+    qp = _qprime(1301, (H, B_TOK, d), d, (1,))
+    op = torch.empty(H, B_TOK, d, dtype=torch.bfloat16, device="cuda")
+    smem.smem_mu_prefill(lc.h, 0, nblk, qp.cuda(), op, lc.ws)
+    got = op.float().cpu().numpy().astype(np.float64)
+    _, mus = lc.memory(0, nblk)
+    for h in range(H):
+        ref = _oracle_mu(qp[h].double().numpy(), list(mus), lc.nu)
+        err = np.abs(got[h] - ref)
+        assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (h, err.max(), err.mean())
