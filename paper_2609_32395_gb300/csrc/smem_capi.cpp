@@ -832,9 +832,9 @@ int mu_attend(smem_cache* c, uint8_t* ws, const LayerWs& o, bool prefill, int nb
   P.max_blocks = L.max_blocks;
   P.capacity = L.capacity;
   if (prefill) {
-    const int nqt = smem::mu_query_tile(smem::kBlockTok, d);
     const std::vector<int32_t>& ix = c->idx[seq];
     const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_idx) - ix.begin());
+    const int nqt = smem::mu_prefill_query_tile(nblk, H, d);
     const int tiles = smem::kBlockTok / nqt;
     const int groups = H * tiles;
     const int sb = nblk ? smem::mu_prefill_split_blocks(nblk, groups) : 1;

@@ -151,8 +151,9 @@ int blas_gemm_sb(void* blas, bool ta, bool tb, int m, int n, int k, float alpha,
 // ---------------------------------------------------------------------------
 constexpr int kMaxMuGroups = 512;   // groups (row set x query tile) per launch
 constexpr int kMuMaxSplits = 16;    // splits of one group's blocks
-constexpr int kMuSmemBudget = 200 * 1024;  // one CTA per SM
+constexpr int kMuSmemBudget = 220 * 1024;  // one CTA per SM
 constexpr int kMuSmemHalf = 110 * 1024;    // two CTAs per SM
+constexpr int kMuMaxStages = 32;           // ring stages of 8 KB
 // One group: NQ queries (rows n0.. of query set qg) that read the same row
 // set (the first nblk table blocks of `seq`), cut into nsplit units of
 // split_blks blocks; units of a group are consecutive from unit_begin.
@@ -169,12 +170,15 @@ struct MuParams {
   float* part;                // [unit][NQ][d + 4]: m, l, pad, pad, O'[d]
   int* err;
   int d, nrows, n_qg, max_blocks, capacity, n_groups, n_units;
-  int ns, off_ring, off_p, off_bar, off_misc;  // shared-memory plan (set by the launcher)
+  int ns, hold, off_ring, off_p, off_bar, off_misc;  // shared-memory plan (set by the launcher)
   MuGroup groups[kMaxMuGroups];
 };
 // Widest query tile (16, 32 or 64) for nq_total queries per row set at width
 // d whose accumulators fit tensor memory; 0 if none does.
 int mu_query_tile(int nq_total, int d);
+// Query tile of the one-block form for nblk readable blocks (a function of
+// the block count and the geometry only).
+int mu_prefill_query_tile(int nblk, int H, int d);
 int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity);
 cudaError_t launch_mu_attention(MuParams& P, int nq, cudaStream_t st);
 // Split plans (functions of the block count and the cache geometry only).

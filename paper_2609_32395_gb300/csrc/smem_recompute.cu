@@ -165,13 +165,23 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
       // iteration before its use, so its latency hides behind two passes
       int s_cur = trow[b0];
       int s_nxt = nt > 1 ? trow[b0 + 1] : 0;
-      pass(s_cur);
-      for (int t = 0; t < nt && ok; ++t) {
-        const int s_nn = t + 2 < nt ? trow[b0 + t + 2] : 0;
-        if (t + 1 < nt) pass(s_nxt);
-        if (ok) pass(s_cur);
-        s_cur = s_nxt;
-        s_nxt = s_nn;
+      if (p.hold) {
+        // hold mode: each tile is loaded once and stays until its P.V is done
+        for (int t = 0; t < nt && ok; ++t) {
+          const int s_nn = t + 2 < nt ? trow[b0 + t + 2] : 0;
+          pass(s_cur);
+          s_cur = s_nxt;
+          s_nxt = s_nn;
+        }
+      } else {
+        pass(s_cur);
+        for (int t = 0; t < nt && ok; ++t) {
+          const int s_nn = t + 2 < nt ? trow[b0 + t + 2] : 0;
+          if (t + 1 < nt) pass(s_nxt);
+          if (ok) pass(s_cur);
+          s_cur = s_nxt;
+          s_nxt = s_nn;
+        }
       }
       if (!ok) {
         // let every copy already issued land before the CTA can exit
@@ -226,10 +236,64 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
         }
         if (ok) tc::commit(&o_done[pb]);
       };
-      issue_s(0);
-      for (int t = 0; t < nt && ok; ++t) {
-        if (t + 1 < nt) issue_s(t + 1);
-        issue_pv(t);
+      if (p.hold) {
+        // Hold mode: a tile's chunks stay in the ring from its S to its P.V,
+        // so the issuer polls two queues -- the next S chunk (data landed,
+        // S buffer free) and the P.V of the oldest tile whose P is ready --
+        // and never blocks one on the other.
+        int kS = 0, tS = 0, cS = 0, tP = 0;
+        unsigned long long t_last = global_timer_ns();
+        while (ok && tP < nt) {
+          bool prog = false;
+          if (tP < tS && mbar_test_wait(&p_full[tP & 1], (tP >> 1) & 1)) {
+            tc::fence_after();
+            const uint32_t b = smem_u32(pt + (tP & 1) * C::PBYTES);
+            for (int cp = 0; cp < NC / 2; ++cp) {
+              const int st = (tP * NC + 2 * cp) % ns;  // even: the pair sits in slots st, st + 1
+              const uint32_t a = ra + st * kMuBox;
+#pragma unroll
+              for (int kk = 0; kk < 4; ++kk)
+                tc::mma_bf16(tmem + colO + cp * NQ, tc::sdesc_sw128(a + kk * 2048, kMuBox, 1024),
+                             tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_PV, (tP > 0 || kk > 0));
+              tc::commit(&empty[st]);
+              tc::commit(&empty[st + 1]);
+            }
+            tc::commit(&o_done[tP & 1]);
+            ++tP;
+            prog = true;
+          }
+          if (tS < nt) {
+            const int sb = tS & 1;
+            const bool sfree = cS > 0 || tS < 2 || mbar_test_wait(&s_free[sb], ((tS >> 1) - 1) & 1);
+            const int st = kS % ns;
+            if (sfree && mbar_test_wait(&full[st], (kS / ns) & 1)) {
+              tc::fence_after();
+              const uint32_t a = ra + st * kMuBox, b = qa + cS * C::PBYTES;
+#pragma unroll
+              for (int kk = 0; kk < 4; ++kk)
+                tc::mma_bf16(tmem + sb * NQ, tc::sdesc_sw128(a + kk * 32, 16, 1024),
+                             tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_S, (cS | kk) > 0);
+              ++kS;
+              if (++cS == NC) {
+                tc::commit(&s_full[sb]);
+                ++tS;
+                cS = 0;
+              }
+              prog = true;
+            }
+          }
+          if (prog) {
+            t_last = global_timer_ns();
+          } else if (*abort_flag || global_timer_ns() - t_last > kWaitLimitNs) {
+            ok = false;
+          }
+        }
+      } else {
+        issue_s(0);
+        for (int t = 0; t < nt && ok; ++t) {
+          if (t + 1 < nt) issue_s(t + 1);
+          issue_pv(t);
+        }
       }
       if (!ok) {
         if (!*abort_flag) record_error(p.err, kDevErrWaitMma);
@@ -486,17 +550,31 @@ int encode3d(CUtensorMap* map, const void* ptr, uint64_t d0, uint64_t d1, uint64
 int mu_smem_plan(MuParams& P, int nq, int d) {
   const int qbytes = (d / 64) * nq * 128;
   const int fixed = 2 * nq * 128 + 4096 + 1024;
-  // two CTAs per SM when the queries leave room for an 8-stage ring in half the SM
-  const int budget = qbytes + fixed + 8 * kMuBox <= kMuSmemHalf ? kMuSmemHalf : kMuSmemBudget;
-  int ns = (budget - qbytes - fixed) / kMuBox;
-  ns &= ~1;
-  if (ns > 16) ns = 16;
+  const int nc = d / 64;
+  // Two CTAs per SM streaming every tile twice (the second pass from L2)
+  // when the queries leave room for an 8-stage ring in half the SM; else one
+  // CTA per SM holding whole tiles from S to P.V (hold mode) when a tile and
+  // four chunks of lookahead fit; else one CTA per SM streaming twice.
+  // Two interleaved CTAs measured faster than one CTA holding its tiles.
+  int ns_full = ((kMuSmemBudget - qbytes - fixed) / kMuBox) & ~1;
+  if (ns_full > kMuMaxStages) ns_full = kMuMaxStages;
+  const int ns_half = ((kMuSmemHalf - qbytes - fixed) / kMuBox) & ~1;
+  int ns;
+  P.hold = 0;
+  if (ns_half >= 8) {
+    ns = ns_half;
+  } else if (ns_full >= nc + 4) {
+    ns = ns_full;
+    P.hold = 1;
+  } else {
+    ns = ns_full;
+  }
   if (ns < 4) return -1;
   P.ns = ns;
   P.off_ring = (qbytes + 1023) / 1024 * 1024;
   P.off_p = P.off_ring + ns * kMuBox;
   P.off_bar = P.off_p + 2 * nq * 128;
-  const int nbars = 1 + 2 * ns + 9;
+  const int nbars = 1 + 2 * ns + 9;  // q_full, full/empty rings, s_full/s_free/p_full/o_done pairs, drain
   P.off_misc = (P.off_bar + nbars * 8 + 15) / 16 * 16;
   // misc: 16 B words + red[2][4][NQ] + alpha[2][NQ] + lsum[4][NQ] + mfin[NQ]
   const int misc = 16 + (8 + 2 + 4 + 1) * nq * 4;
@@ -523,6 +601,18 @@ int mu_query_tile(int nq_total, int d) {
     if (nq <= 16 || nq_total > nq / 2) return nq;
   }
   return 0;
+}
+
+int mu_prefill_query_tile(int nblk, int H, int d) {
+  // the widest tile (fewest re-reads of the rows from L2) that still gives
+  // every SM a unit; the narrowest otherwise
+  for (int nq : {64, 32}) {
+    if (nq * (2 + d / 128) > 512) continue;
+    const int groups = H * (kBlockTok / nq);
+    const int sb = mu_prefill_split_blocks(nblk, groups);
+    if (groups * ((nblk + sb - 1) / sb) >= 152) return nq;
+  }
+  return 16;
 }
 
 int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity) {

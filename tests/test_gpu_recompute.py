@@ -40,10 +40,11 @@ def test_recompute_layer_prefill_matches_oracle(D, H, has_null):
     assert smem.smem_check_device_error(lc.h) == smem.OK
 
 
-@pytest.mark.parametrize("H,D,nblk", [(12, 64, 64), (16, 64, 40), (16, 128, 24)])
+@pytest.mark.parametrize("H,D,nblk", [(12, 64, 256), (12, 64, 64), (16, 64, 40), (16, 128, 24)])
 def test_recompute_prefill_at_model_widths(H, D, nblk):
     """d = 768 / 1024 / 2048 (the 160M / 410M / 1.5B reader widths): every
-    query-tile width of the kernel (64, 32, 16 queries per CTA)."""
+    query-tile width of the kernel (64 queries per CTA at 256 blocks, 32 at
+    64 and 40, 16 at d = 2048)."""
     d = H * D
     model = LayerModel(1, d, seed=701 + d)
     lc = LayerCache(model, H, D, max_seqs=1, max_blocks=nblk + 4, capacity=nblk + 4, recompute=True)
