@@ -59,7 +59,7 @@
 extern "C" {
 #endif
 
-#define SMEM_ABI_VERSION 3
+#define SMEM_ABI_VERSION 4
 
 enum {
     SMEM_OK = 0,
@@ -102,6 +102,19 @@ typedef struct smem_config {
                                    each layer's keys and values from them
                                    (the recompute regime, App. "Serving").
                                    The pool is then 2L times smaller.          */
+    int32_t rope_window;        /* 0: no rotary phases. W in 1..63: the
+                                   SMem+RoPE composite (Sec. 4, App. "Training
+                                   recipes"): self-attention queries/keys turn
+                                   by their in-block offset, a cross-attention
+                                   query by its block index i and a memory
+                                   row's key by max(j, i - W) (the null row's
+                                   by max(0, i - W); App. "Needle", saturating
+                                   offsets, W = 15 in the paper); values never
+                                   turn. Pairs (2m, 2m+1) turn by
+                                   phase * base^(-2m/d_h). All inputs are
+                                   given UNROTATED; stored in-block keys are
+                                   kept turned. Not with recompute_kv.          */
+    float rope_base;            /* rotary base (10000 in the paper)           */
 } smem_config;
 
 typedef struct smem_cache smem_cache;

@@ -84,47 +84,65 @@ def null_kv(nu, w: LayerWeights, H: int, D: int):
     return (nu @ w.w_kc).reshape(H, D), (nu @ w.w_vc).reshape(H, D)
 
 
-def reader_layer_prefill(x, block_idx, mu_blocks, q_idx, w: LayerWeights, H: int, D: int, nu=None):
+def _attn_prefill(rope_window):
+    if rope_window:
+        from .rope import reader_prefill_rope
+        return lambda *a: reader_prefill_rope(*a, window=rope_window)
+    return reader_prefill
+
+
+def _attn_decode(rope_window):
+    if rope_window:
+        from .rope import reader_decode_rope
+        return lambda *a: reader_decode_rope(*a, window=rope_window)
+    return reader_decode
+
+
+def reader_layer_prefill(x, block_idx, mu_blocks, q_idx, w: LayerWeights, H: int, D: int, nu=None, rope_window=0):
     """One-block pass of one reader layer.
     x: [b][d] residual stream of the query block; block_idx: [n] memory block
-    indices (any order); mu_blocks: [n][R][d] their memory rows.
-    Returns (x_out [b][d], k_s [b][H][D], v_s [b][H][D])."""
+    indices (any order); mu_blocks: [n][R][d] their memory rows. rope_window
+    W > 0: the SMem+RoPE composite's rotary phases (oracle.rope).
+    Returns (x_out [b][d], k_s [b][H][D], v_s [b][H][D]); k_s unrotated."""
+    attn = _attn_prefill(rope_window)
     b, d = x.shape
     h1 = layer_norm(x, w.ln1_g, w.ln1_b)
     qkv = h1 @ w.w_qkv
     qs, ks, vs = (qkv[:, i * d:(i + 1) * d].reshape(b, H, D) for i in range(3))
     zero = np.zeros((b, H, D))
-    osa, _ = reader_prefill([], None, None, 0, qs, ks, vs, zero)
+    osa, _ = attn([], None, None, 0, qs, ks, vs, zero)
     x1 = x + osa.reshape(b, d) @ w.w_os
     h2 = layer_norm(x1, w.ln2_g, w.ln2_b)
     qc = (h2 @ w.w_qc).reshape(b, H, D)
     n = len(block_idx)
     mk, mv = memory_kv(np.asarray(mu_blocks), w, H, D) if n else (None, None)
     kn, vn = null_kv(nu, w, H, D) if nu is not None else (None, None)
-    _, oca = reader_prefill(block_idx, mk, mv, q_idx, zero, zero, zero, qc, kn, vn)
+    _, oca = attn(block_idx, mk, mv, q_idx, zero, zero, zero, qc, kn, vn)
     x2 = x1 + oca.reshape(b, d) @ w.w_oc
     h3 = layer_norm(x2, w.ln3_g, w.ln3_b)
     x3 = x2 + gelu(h3 @ w.w_1) @ w.w_2
     return x3, ks, vs
 
 
-def reader_layer_decode(x, block_idx, mu_blocks, q_idx, p, kin, vin, w: LayerWeights, H: int, D: int, nu=None):
+def reader_layer_decode(x, block_idx, mu_blocks, q_idx, p, kin, vin, w: LayerWeights, H: int, D: int, nu=None,
+                        rope_window=0):
     """One decode step of one reader layer for one sequence.
-    x: [d]; kin/vin: [p][H][D] in-block rows of earlier tokens.
+    x: [d]; kin/vin: [p][H][D] in-block rows of earlier tokens (unrotated).
     Returns (x_out [d], k_new [H][D], v_new [H][D])."""
+    attn = _attn_decode(rope_window)
     d = x.shape[0]
     h1 = layer_norm(x[None], w.ln1_g, w.ln1_b)[0]
     qkv = h1 @ w.w_qkv
     qs, kn_, vn_ = (qkv[i * d:(i + 1) * d].reshape(H, D) for i in range(3))
     zero = np.zeros((H, D))
-    osa, _ = reader_decode([], None, None, 0, p, kin, vin, qs, kn_, vn_, zero)
+    osa, _ = attn([], None, None, 0, p, kin, vin, qs, kn_, vn_, zero)
     x1 = x + osa.reshape(d) @ w.w_os
     h2 = layer_norm(x1[None], w.ln2_g, w.ln2_b)[0]
     qc = (h2 @ w.w_qc).reshape(H, D)
     n = len(block_idx)
     mk, mv = memory_kv(np.asarray(mu_blocks), w, H, D) if n else (None, None)
     knull, vnull = null_kv(nu, w, H, D) if nu is not None else (None, None)
-    _, oca = reader_decode(block_idx, mk, mv, q_idx, 0, None, None, zero, zero, zero, qc, knull, vnull)
+    _, oca = attn(block_idx, mk, mv, q_idx, 0, None, None, zero, zero, zero, qc, knull, vnull)
     x2 = x1 + oca.reshape(d) @ w.w_oc
     h3 = layer_norm(x2[None], w.ln3_g, w.ln3_b)[0]
     x3 = x2 + gelu(h3 @ w.w_1) @ w.w_2

@@ -69,6 +69,9 @@ int make_layout(const smem_config* c, Layout* L) {
   if (c->block_tokens != smem::kBlockTok || c->rows_per_block != smem::kRows) return SMEM_ERR_UNSUPPORTED;
   if (c->has_null_row != 0 && c->has_null_row != 1) return SMEM_ERR_INVALID_ARG;
   if (c->recompute_kv != 0 && c->recompute_kv != 1) return SMEM_ERR_INVALID_ARG;
+  if (c->rope_window < 0 || c->rope_window >= smem::kRopePhases) return SMEM_ERR_INVALID_ARG;
+  if (c->rope_window > 0 && !(c->rope_base > 1.0f && c->rope_base < 1e30f)) return SMEM_ERR_INVALID_ARG;
+  if (c->rope_window > 0 && c->recompute_kv) return SMEM_ERR_UNSUPPORTED;
   // recompute caches: rows of d = H*d_h in 128-column pairs, at most 64 heads per query tile
   if (c->recompute_kv && ((c->n_heads * c->head_dim) % 128 != 0 || c->n_heads > 64 ||
                           smem::mu_query_tile(c->n_heads, c->n_heads * c->head_dim) == 0))
@@ -82,6 +85,8 @@ int make_layout(const smem_config* c, Layout* L) {
   L->has_null = c->has_null_row;
   L->max_batch = c->max_decode_batch;
   L->recompute = c->recompute_kv;
+  L->rope_w = c->rope_window;
+  L->rope_base = c->rope_base;
   int ms = 1;
   for (int n = 1; n <= c->max_blocks_per_seq; ++n)
     ms = std::max(ms, smem::ceil_div(n, smem::decode_split_blocks(n)));
@@ -99,6 +104,12 @@ int make_layout(const smem_config* c, Layout* L) {
   off = align_up(off + (!L->has_null ? 0 : L->recompute ? (size_t)L->H * D * 2 : (size_t)L->L * L->H * 2 * D * 2), A);
   L->off_table = off;
   off = align_up(off + (size_t)L->max_seqs * L->max_blocks * 4, A);
+  L->off_bidx = off;
+  off = align_up(off + (size_t)L->max_seqs * L->max_blocks * 4, A);
+  L->off_rope = off;
+  off = align_up(off + (L->rope_w ? (size_t)smem::kRopePhases * (D / 2) * 8 : 0), A);
+  L->off_rope_scr = off;  // rotated copies of Qs and Ks for smem_prefill_block
+  off = align_up(off + (L->rope_w ? (size_t)2 * smem::kBlockTok * L->H * D * 2 : 0), A);
   L->off_dec_part = off;
   off = align_up(off + (size_t)L->max_batch * L->H * L->dec_max_splits * (D + 4) * 4, A);
   L->off_dec_cnt = off;
@@ -156,6 +167,12 @@ inline uint16_t* inblock_layer(smem_cache* c, int seq, int layer) {
   const Layout& L = c->lay;
   return reinterpret_cast<uint16_t*>(c->dev + L.off_inblock) +
          ((size_t)seq * L.L + layer) * L.H * 2 * smem::kBlockTok * L.D;
+}
+inline int* bidx_row(smem_cache* c, int seq) {
+  return reinterpret_cast<int*>(c->dev + c->lay.off_bidx) + (size_t)seq * c->lay.max_blocks;
+}
+inline const float2* rope_tab(smem_cache* c) {
+  return c->lay.rope_w ? reinterpret_cast<const float2*>(c->dev + c->lay.off_rope) : nullptr;
 }
 inline const uint16_t* null_kv(smem_cache* c) {
   return c->lay.has_null ? reinterpret_cast<const uint16_t*>(c->dev + c->lay.off_null) : nullptr;
@@ -284,6 +301,10 @@ int prefill_impl(smem_cache* c, int seq, int layer, int q_block_idx, const void*
   a.tok_s = tok_s;
   a.tok_c = tok_c;
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->lay.D));
+  a.rope_tab = rope_tab(c);
+  a.bidx_row = bidx_row(c, seq);
+  a.rope_w = c->lay.rope_w;
+  a.q_blk = q_block_idx;
   if (injected_failure(c)) return SMEM_ERR_CUDA;
   return check_launch(c, smem::launch_prefill(a, st), "prefill");
 }
@@ -348,6 +369,9 @@ int decode_impl(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const 
     P.s_stride = s_stride;
     P.c_stride = c_stride;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
+    P.rope_tab = rope_tab(c);
+    P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);
+    P.rope_w = L.rope_w;
     int pairs = 0;
     for (int i = 0; i < n; ++i) {
       const int s = seq_ids[i0 + i];
@@ -357,6 +381,7 @@ int decode_impl(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const 
       P.items[i].nblk = nblk;
       P.items[i].pos = pos[i0 + i];
       P.items[i].pair_begin = pairs;
+      P.items[i].qblk = q_block_idx[i0 + i];
       if (nblk && (mode & 2)) pairs += smem::ceil_div(nblk, smem::decode_split_blocks(nblk));
     }
     P.n_pairs = pairs;
@@ -417,6 +442,17 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
     // zero everything but the pool: in-block rows, null rows, tables,
     // workspace, counters and the error word
     if (e == cudaSuccess) e = smem::launch_zero(c->dev + L.off_inblock, L.total - L.off_inblock, nullptr);
+    if (e == cudaSuccess && L.rope_w) {
+      // rotary table: (cos, sin) of phase * base^(-2m/D), phases 0..63, pairs m < D/2
+      std::vector<float> tab((size_t)smem::kRopePhases * L.D);
+      for (int ph = 0; ph < smem::kRopePhases; ++ph)
+        for (int m = 0; m < L.D / 2; ++m) {
+          const double ang = ph * std::pow((double)L.rope_base, -2.0 * m / L.D);
+          tab[((size_t)ph * (L.D / 2) + m) * 2] = (float)std::cos(ang);
+          tab[((size_t)ph * (L.D / 2) + m) * 2 + 1] = (float)std::sin(ang);
+        }
+      e = cudaMemcpy(c->dev + L.off_rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice);
+    }
     if (e == cudaSuccess) e = cudaStreamSynchronize(nullptr);
     if (e != cudaSuccess) {
       set_detail("create", e);
@@ -491,7 +527,8 @@ int smem_append_block(smem_cache* c, int32_t seq, int32_t block_idx, const void*
     const int rc = check_launch(c,
                                 smem::launch_append(pool_slot(c, s), static_cast<const uint16_t*>(K),
                                                     static_cast<const uint16_t*>(V), c->lay.L, c->lay.H, c->lay.D,
-                                                    table_row(c, seq), pos, (int)ix.size(), s, as_stream(stream)),
+                                                    table_row(c, seq), bidx_row(c, seq), pos, (int)ix.size(), s,
+                                                    block_idx, as_stream(stream)),
                                 "append");
     if (rc) return rc;
   }
@@ -513,7 +550,8 @@ int smem_delete_block(smem_cache* c, int32_t seq, int32_t block_idx, void* strea
   if (c->dev) {
     DeviceGuard g(c->device);
     if (injected_failure(c)) return SMEM_ERR_CUDA;
-    const int rc = check_launch(c, smem::launch_table_remove(table_row(c, seq), pos, (int)ix.size(), as_stream(stream)),
+    const int rc = check_launch(c, smem::launch_table_remove(table_row(c, seq), bidx_row(c, seq), pos, (int)ix.size(),
+                                                              as_stream(stream)),
                                 "delete");
     if (rc) return rc;
   }
@@ -548,7 +586,7 @@ int smem_write_inblock(smem_cache* c, int32_t seq, int32_t layer, int32_t n_rows
   return check_launch(c,
                       smem::launch_inblock_write(inblock_layer(c, seq, layer), static_cast<const uint16_t*>(K),
                                                  static_cast<const uint16_t*>(V), n_rows, c->lay.H, c->lay.D,
-                                                 as_stream(stream)),
+                                                 as_stream(stream), 0, rope_tab(c)),
                       "in-block write");
 }
 
@@ -565,7 +603,23 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
     if (!aligned16(p)) return SMEM_ERR_ALIGN;
   }
   DeviceGuard g(c->device);
-  return prefill_impl(c, seq, layer, q_block_idx, Qs, Ks, Vs, Qc, Osa, Oca, 3, 0, 0, as_stream(stream));
+  const cudaStream_t st = as_stream(stream);
+  if (c->lay.rope_w) {
+    // self-attention queries and keys turn by their in-block offsets first
+    const Layout& L = c->lay;
+    uint16_t* qr = reinterpret_cast<uint16_t*>(c->dev + L.off_rope_scr);
+    uint16_t* kr = qr + (size_t)smem::kBlockTok * L.H * L.D;
+    const int tok = L.H * L.D;
+    if (injected_failure(c)) return SMEM_ERR_CUDA;
+    int rc = check_launch(c, smem::launch_rope_rows(static_cast<const uint16_t*>(Qs), tok, qr, tok, smem::kBlockTok,
+                                                    L.H, L.D, rope_tab(c), st), "rotary");
+    if (!rc)
+      rc = check_launch(c, smem::launch_rope_rows(static_cast<const uint16_t*>(Ks), tok, kr, tok, smem::kBlockTok, L.H,
+                                                  L.D, rope_tab(c), st), "rotary");
+    if (rc) return rc;
+    return prefill_impl(c, seq, layer, q_block_idx, qr, kr, Vs, Qc, Osa, Oca, 3, 0, 0, st);
+  }
+  return prefill_impl(c, seq, layer, q_block_idx, Qs, Ks, Vs, Qc, Osa, Oca, 3, 0, 0, st);
 }
 
 int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,
@@ -664,12 +718,16 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     P.mode = 3;
     P.s_stride = P.c_stride = L.H * L.D;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
+    P.rope_tab = rope_tab(c);
+    P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);
+    P.rope_w = L.rope_w;
     int pairs = 0;
     for (int i = 0; i < n; ++i) {
       P.items[i].seq = seq_ids[i0 + i];
       P.items[i].nblk = nblk[i0 + i];
       P.items[i].pos = pos[i0 + i];
       P.items[i].pair_begin = pairs;
+      P.items[i].qblk = q_block_idx[i0 + i];
       if (nblk[i0 + i]) pairs += smem::ceil_div(nblk[i0 + i], smem::decode_split_blocks(nblk[i0 + i]));
     }
     P.n_pairs = pairs;
@@ -731,7 +789,8 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
                                             static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc),
                                             slot + ((size_t)l * L.H * 2 + kv) * smem::kRows * L.D,
                                             (long long)head_stride, g_detail, sizeof(g_detail)));
-  if (!rc) rc = cuda_rc(smem::launch_table_insert(table_row(c, seq), pos, (int)ix.size(), s, st), "append rows");
+  if (!rc) rc = cuda_rc(smem::launch_table_insert(table_row(c, seq), bidx_row(c, seq), pos, (int)ix.size(), s,
+                                                          block_idx, st), "append rows");
   if (rc) return rc;
   c->fifo.pop_front();
   ix.insert(ix.begin() + pos, block_idx);
@@ -928,7 +987,13 @@ int smem_reader_layer_prefill(smem_cache* c, int32_t seq, int32_t layer, int32_t
   LayerRun r{c, w, x, static_cast<uint8_t*>(ws), layer_ws(L, n), n, L.H * L.D, st};
   const int d = r.d;
   rc = r.qkv_proj();
-  // the block's self-attention keys/values become its in-block rows
+  if (!rc && L.rope_w) {  // self-attention queries and keys turn by their in-block offsets
+    rc = cuda_rc(smem::launch_rope_rows(r.qkv(), 3 * d, r.qkv(), 3 * d, n, L.H, L.D, rope_tab(c), st), "rotary");
+    if (!rc)
+      rc = cuda_rc(smem::launch_rope_rows(r.qkv() + d, 3 * d, r.qkv() + d, 3 * d, n, L.H, L.D, rope_tab(c), st),
+                   "rotary");
+  }
+  // the block's self-attention keys/values become its in-block rows (already turned)
   if (!rc)
     rc = cuda_rc(smem::launch_inblock_write(inblock_layer(c, seq, layer), r.qkv() + d, r.qkv() + 2 * d, n, L.H, L.D,
                                             st, 3 * d),

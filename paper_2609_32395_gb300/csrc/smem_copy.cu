@@ -11,6 +11,7 @@
 // overwrites an unread entry.
 #include <cuda_runtime.h>
 
+#include "smem_device.cuh"
 #include "smem_internal.h"
 
 namespace smem {
@@ -44,12 +45,15 @@ __device__ void table_remove_cta(int* row, int pos, int n) {
 }
 
 // Grid: n_copy CTAs copy K and V [L][H][R][D] into the slot laid out as
-// [L][H][2][R][D]; one extra CTA edits the table.
+// [L][H][2][R][D]; one extra CTA edits the table and the block-index row.
 __global__ void __launch_bounds__(kCopyThreads) append_kernel(uint4* slot_base, const uint4* K, const uint4* V,
                                                               long long heads, int chunks_per_head, int* table_row,
-                                                              int pos, int n_old, int slot, int n_copy) {
+                                                              int* bidx_row, int pos, int n_old, int slot,
+                                                              int block_idx, int n_copy) {
   if ((int)blockIdx.x == n_copy) {
     table_insert_cta(table_row, pos, n_old, slot);
+    __syncthreads();
+    table_insert_cta(bidx_row, pos, n_old, block_idx);
     return;
   }
   const long long per_kv = heads * chunks_per_head;
@@ -65,13 +69,45 @@ __global__ void __launch_bounds__(kCopyThreads) append_kernel(uint4* slot_base, 
   }
 }
 
-__global__ void __launch_bounds__(kCopyThreads) table_remove_kernel(int* row, int pos, int n) {
+__global__ void __launch_bounds__(kCopyThreads) table_remove_kernel(int* row, int* bidx_row, int pos, int n) {
   table_remove_cta(row, pos, n);
+  __syncthreads();
+  table_remove_cta(bidx_row, pos, n);
+}
+
+// (x[2m], x[2m+1]) turned by the table row's angle for pair m (8 values =
+// pairs m0 .. m0+3).
+__device__ __forceinline__ uint4 rotate8(const uint4 v, const float2* cs) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t o[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float x0 = bf16lo(w[e]), x1 = bf16hi(w[e]);
+    const float2 c = cs[e];
+    o[e] = pack_bf16x2(x0 * c.x - x1 * c.y, x0 * c.y + x1 * c.x);
+  }
+  return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// src rows [n][H][D] (token stride src16 16-byte chunks) -> dst, token t
+// turned by phase t (tab: [kRopePhases][D/2] float2).
+__global__ void rope_rows_kernel(const uint4* src, int src16, uint4* dst, int dst16, int n, int H, int cpr,
+                                 const float2* tab) {
+  const int total = n * H * cpr;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    const int t = i / (H * cpr);
+    const int h = (i / cpr) % H;
+    const int c = i % cpr;
+    const uint4 v = src[(size_t)t * src16 + (size_t)h * cpr + c];
+    dst[(size_t)t * dst16 + (size_t)h * cpr + c] = rotate8(v, tab + (size_t)t * (cpr * 4) + c * 4);
+  }
 }
 
 // rows [n][H][D] (K and V, token stride `tok16` chunks of 16 bytes) ->
-// in-block layout [H][2][b][D] of one layer
-__global__ void inblock_write_kernel(uint4* ib, const uint4* K, const uint4* V, int n, int H, int cpr, int tok16) {
+// in-block layout [H][2][b][D] of one layer; keys turned by their offset
+// when a rotary table is given
+__global__ void inblock_write_kernel(uint4* ib, const uint4* K, const uint4* V, int n, int H, int cpr, int tok16,
+                                     const float2* tab) {
   const int total = 2 * n * H * cpr;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
     const int kv = i >= n * H * cpr;
@@ -80,7 +116,9 @@ __global__ void inblock_write_kernel(uint4* ib, const uint4* K, const uint4* V, 
     const int h = (j / cpr) % H;
     const int c = j % cpr;
     const size_t src = (size_t)t * tok16 + (size_t)h * cpr + c;
-    ib[((h * 2 + kv) * kBlockTok + t) * cpr + c] = kv ? V[src] : K[src];
+    uint4 v = kv ? V[src] : K[src];
+    if (tab && !kv) v = rotate8(v, tab + (size_t)t * (cpr * 4) + c * 4);
+    ib[((h * 2 + kv) * kBlockTok + t) * cpr + c] = v;
   }
 }
 
@@ -101,7 +139,8 @@ __global__ void zero_kernel(uint4* p, long long n16) {
 }
 
 cudaError_t launch_append(uint16_t* slot_base, const uint16_t* K, const uint16_t* V, int L, int H, int D,
-                          int* table_row, int pos, int n_old, int slot, cudaStream_t st) {
+                          int* table_row, int* bidx_row, int pos, int n_old, int slot, int block_idx,
+                          cudaStream_t st) {
   const int chunks_per_head = kRows * D * 2 / 16;
   const long long heads = (long long)L * H;
   const long long total = 2 * heads * chunks_per_head;
@@ -109,22 +148,35 @@ cudaError_t launch_append(uint16_t* slot_base, const uint16_t* K, const uint16_t
   if (n_copy > 1184) n_copy = 1184;
   append_kernel<<<(int)n_copy + 1, kCopyThreads, 0, st>>>(
       reinterpret_cast<uint4*>(slot_base), reinterpret_cast<const uint4*>(K), reinterpret_cast<const uint4*>(V),
-      heads, chunks_per_head, table_row, pos, n_old, slot, (int)n_copy);
+      heads, chunks_per_head, table_row, bidx_row, pos, n_old, slot, block_idx, (int)n_copy);
   return cudaGetLastError();
 }
 
-cudaError_t launch_table_insert(int* table_row, int pos, int n_old, int slot, cudaStream_t st) {
-  append_kernel<<<1, kCopyThreads, 0, st>>>(nullptr, nullptr, nullptr, 0, 0, table_row, pos, n_old, slot, 0);
+cudaError_t launch_table_insert(int* table_row, int* bidx_row, int pos, int n_old, int slot, int block_idx,
+                                cudaStream_t st) {
+  append_kernel<<<1, kCopyThreads, 0, st>>>(nullptr, nullptr, nullptr, 0, 0, table_row, bidx_row, pos, n_old, slot,
+                                            block_idx, 0);
   return cudaGetLastError();
 }
 
-cudaError_t launch_table_remove(int* table_row, int pos, int n_old, cudaStream_t st) {
-  table_remove_kernel<<<1, kCopyThreads, 0, st>>>(table_row, pos, n_old);
+cudaError_t launch_table_remove(int* table_row, int* bidx_row, int pos, int n_old, cudaStream_t st) {
+  table_remove_kernel<<<1, kCopyThreads, 0, st>>>(table_row, bidx_row, pos, n_old);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_rows(const uint16_t* src, int src_tok, uint16_t* dst, int dst_tok, int n, int H, int D,
+                             const float2* rope_tab, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  const int cpr = D / 8;
+  const int total = n * H * cpr;
+  rope_rows_kernel<<<(total + 255) / 256, 256, 0, st>>>(reinterpret_cast<const uint4*>(src), src_tok / 8,
+                                                        reinterpret_cast<uint4*>(dst), dst_tok / 8, n, H, cpr,
+                                                        rope_tab);
   return cudaGetLastError();
 }
 
 cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
-                                 int D, cudaStream_t st, int tok) {
+                                 int D, cudaStream_t st, int tok, const float2* rope_tab) {
   if (n == 0) return cudaSuccess;
   const int cpr = D * 2 / 16;
   const int tok16 = (tok ? tok : H * D) * 2 / 16;
@@ -132,7 +184,7 @@ cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, con
   const int blocks = (total + 255) / 256;
   inblock_write_kernel<<<blocks, 256, 0, st>>>(reinterpret_cast<uint4*>(ib_layer_base),
                                                reinterpret_cast<const uint4*>(K),
-                                               reinterpret_cast<const uint4*>(V), n, H, cpr, tok16);
+                                               reinterpret_cast<const uint4*>(V), n, H, cpr, tok16, rope_tab);
   return cudaGetLastError();
 }
 

@@ -125,6 +125,18 @@ __device__ __forceinline__ void store_bf16x8(uint16_t* dst, const float* v, floa
   *reinterpret_cast<uint4*>(dst) = o;
 }
 
+// Rotary phase: the 8 values t (pairs (0,1) .. (6,7)) turned by the angles
+// of pairs cs[0..3] of a table row.
+__device__ __forceinline__ void rot8f(float* t, const float2* cs) {
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 c = cs[e];
+    const float x0 = t[2 * e], x1 = t[2 * e + 1];
+    t[2 * e] = x0 * c.x - x1 * c.y;
+    t[2 * e + 1] = x0 * c.y + x1 * c.x;
+  }
+}
+
 // Issue side of one warp's chunk stream over dynamically fetched CA units.
 // Lane 0 only. Units come from a launch-wide atomic counter, one unit ahead
 // of the unit being issued; each fetched unit is pushed on the warp's unit
@@ -193,7 +205,7 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
 // Self-attention unit: in-block rows 0..p-1 and the new token's row, read
 // directly from global memory. Writes osa, stores the new row, and writes
 // oca for a sequence that has no readable memory block.
-template <int D>
+template <int D, bool ROPE>
 __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int lane) {
   constexpr int LPR = Dec<D>::LPR;
   constexpr int RPP = 32 / LPR;  // rows per pass
@@ -203,12 +215,15 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
   const size_t soff = (size_t)U.item * p.s_stride + (size_t)U.h * D;  // qs, k_new, v_new
   const uint16_t* ib = p.inblock + (((size_t)it.seq * p.L + p.layer) * p.H + U.h) * (size_t)2 * kBlockTok * D;
   const int hh = lane % LPR;  // which 64 columns of the row
+  // with rotary phases the new token's query and key turn by its offset p
+  const float2* rp = ROPE ? p.rope_tab + (size_t)it.pos * (D / 2) + hh * 32 : nullptr;
   if (p.mode & 1) {
     float q[64];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       float t[8];
       unpack8(ld_nc16(p.qs + soff + hh * 64 + j * 8), t);
+      if (ROPE) rot8f(t, rp + j * 4);
 #pragma unroll
       for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
     }
@@ -225,6 +240,7 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
         for (int j = 0; j < 8; ++j) {
           float t[8];
           unpack8(ld_nc16(row + hh * 64 + j * 8), t);
+          if (ROPE && r == it.pos) rot8f(t, rp + j * 4);  // stored rows are already turned
 #pragma unroll
           for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
         }
@@ -276,7 +292,15 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
     if (lane < 2 * CPL) {
       const int kv = lane / CPL, cc = lane % CPL;
       uint16_t* dst = (uint16_t*)ib + (size_t)kv * kBlockTok * D + (size_t)it.pos * D + cc * 8;
-      *reinterpret_cast<uint4*>(dst) = ld_nc16((kv ? p.v_new : p.k_new) + soff + cc * 8);
+      uint4 w = ld_nc16((kv ? p.v_new : p.k_new) + soff + cc * 8);
+      if (ROPE && !kv) {
+        float t[8];
+        unpack8(w, t);
+        rot8f(t, p.rope_tab + (size_t)it.pos * (D / 2) + cc * 4);
+        w = make_uint4(pack_bf16x2(t[0], t[1]), pack_bf16x2(t[2], t[3]), pack_bf16x2(t[4], t[5]),
+                       pack_bf16x2(t[6], t[7]));
+      }
+      *reinterpret_cast<uint4*>(dst) = w;
     }
   }  // self-attention half
   // no readable memory block: oca is the null row's value or zero
@@ -299,7 +323,7 @@ struct Pending {
   unsigned ticket;  // lane 0
 };
 
-template <int D>
+template <int D, bool ROPE>
 __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane) {
   constexpr int CPT = D / 32;  // columns per lane
   const size_t qoff = ((size_t)pd.item * p.H + pd.h) * D;
@@ -308,10 +332,24 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
   if (p.null_kv) {
     // null-row score with the same scaled-query dot product as the rows
     const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + pd.h) * 2 * D;
+    float qv[CPT];
+#pragma unroll
+    for (int e = 0; e < CPT; ++e) qv[e] = bf16lo(p.qc[qcoff + lane * CPT + e]);
+    if (ROPE) {
+      // the null row's key phase is max(0, i - W): the query turns by min(i, W)
+      const int qb = p.items[pd.item].qblk;
+      const float2* cs = p.rope_tab + (size_t)min(qb, p.rope_w) * (D / 2) + lane * (CPT / 2);
+#pragma unroll
+      for (int e = 0; e < CPT; e += 2) {
+        const float2 c = cs[e / 2];
+        const float x0 = qv[e], x1 = qv[e + 1];
+        qv[e] = x0 * c.x - x1 * c.y;
+        qv[e + 1] = x0 * c.y + x1 * c.x;
+      }
+    }
     float dot = 0.f;
 #pragma unroll
-    for (int e = 0; e < CPT; ++e)
-      dot = fmaf(bf16lo(p.qc[qcoff + lane * CPT + e]) * p.scale_log2, bf16lo(kn[lane * CPT + e]), dot);
+    for (int e = 0; e < CPT; ++e) dot = fmaf(qv[e] * p.scale_log2, bf16lo(kn[lane * CPT + e]), dot);
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
     nscore = dot;
@@ -368,13 +406,13 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
 }
 
 // pend2: read its ticket; the warp that completed the last split merges.
-template <int D>
+template <int D, bool ROPE>
 __device__ __forceinline__ void settle(const DecodeParams& p, Pending& pd, int lane) {
   if (!pd.valid) return;
   const unsigned t = __shfl_sync(0xffffffffu, pd.ticket, 0);
   if (t == (unsigned)(pd.nsplit - 1)) {
     __threadfence();
-    merge_splits<D>(p, pd, lane);
+    merge_splits<D, ROPE>(p, pd, lane);
   }
   pd.valid = 0;
 }
@@ -388,7 +426,7 @@ __device__ __forceinline__ void announce(const DecodeParams& p, Pending& from, P
   from.valid = 0;
 }
 
-template <int D>
+template <int D, bool ROPE>
 __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid_constant__ DecodeParams p) {
   using C = Dec<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -426,7 +464,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     U.sa = 1;
     U.item = u / p.H;
     U.h = u - U.item * p.H;
-    sa_unit<D>(p, U, pbuf, lane);
+    sa_unit<D, ROPE>(p, U, pbuf, lane);
   }
   __syncwarp();
 
@@ -453,6 +491,17 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     float m = -INFINITY, l = 0.f, acc[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+    // Rotary phases (CA): the query turns by W once; a block j read from query
+    // block i needs the relative phase min(i - j, W), so only the last W table
+    // entries can differ from W -- their keys turn by W - (i - j) on the fly.
+    // Their block indices are fetched here, while the first chunk is in flight.
+    int near0 = 0x7fffffff, jv0 = 0, jv1 = 0;
+    if (ROPE) {
+      near0 = max(U.b0, it.nblk - p.rope_w);
+      const int* brow = p.bidx + (size_t)it.seq * p.max_blocks;
+      if (near0 + lane < U.b0 + U.nt) jv0 = brow[near0 + lane];
+      if (near0 + 32 + lane < U.b0 + U.nt) jv1 = brow[near0 + 32 + lane];
+    }
 
     const int nch = U.nt * C::CHUNKS;
     for (int ch = 0; ch < nch; ++ch, ++k) {
@@ -470,8 +519,18 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
         for (int j = 0; j < 8; ++j) {
           float t[8];
           unpack8(*reinterpret_cast<const uint4*>(qs + j * 8), t);
+          if (ROPE) rot8f(t, p.rope_tab + (size_t)p.rope_w * (D / 2) + hh * 32 + j * 4);
 #pragma unroll
           for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
+        }
+      }
+      int dk = 0;  // extra key phase of this chunk's block (0: none)
+      if (ROPE) {
+        const int bp = U.b0 + ch / C::CHUNKS;
+        if (bp >= near0) {
+          const int o = bp - near0;
+          const int j = __shfl_sync(0xffffffffu, o < 32 ? jv0 : jv1, o & 31);
+          dk = max(0, p.rope_w - (it.qblk - j));
         }
       }
       const uint8_t* kb = ring + s * C::STAGE;
@@ -479,15 +538,32 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       // scores: lane-per-row (two lanes per row at d_h = 128)
       float dot0 = 0.f, dot1 = 0.f;
       const uint8_t* krow = kb + hh * C::BOX_BYTES + rr * 128;
+      if (ROPE && dk > 0) {
+        const float2* cs = p.rope_tab + (size_t)dk * (D / 2) + hh * 32;
 #pragma unroll
-      for (int j = 0; j < 8; j += 2) {
-        float t0[8], t1[8];
-        unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
-        unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
+        for (int j = 0; j < 8; j += 2) {
+          float t0[8], t1[8];
+          unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
+          unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
+          rot8f(t0, cs + j * 4);
+          rot8f(t1, cs + j * 4 + 4);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
-          dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
+          for (int e = 0; e < 8; ++e) {
+            dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
+            dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; j += 2) {
+          float t0[8], t1[8];
+          unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
+          unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
+            dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
+          }
         }
       }
       float sc = dot0 + dot1;
@@ -541,7 +617,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       if (g == 0) store_bf16x8(p.oca + qoff + c * 8, acc, 1.f / l);
       continue;
     }
-    settle<D>(p, pend2, lane);
+    settle<D, ROPE>(p, pend2, lane);
     announce(p, pend1, pend2, lane);
     float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h) * (D + 4);
     if (g == 0) {
@@ -560,9 +636,9 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
   }
 
   if (!failed) {
-    settle<D>(p, pend2, lane);
+    settle<D, ROPE>(p, pend2, lane);
     announce(p, pend1, pend2, lane);
-    settle<D>(p, pend2, lane);
+    settle<D, ROPE>(p, pend2, lane);
   }
   if (lane == 0) {
     if (failed) {
@@ -632,21 +708,20 @@ int decode_max_grid(int D, int num_sms) {
 
 int decode_warps_per_cta() { return Dec<64>::NW; }
 
-cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st) {
-  if (D == 64) {
-    using C = Dec<64>;
-    cudaError_t e = ensure_smem_limit<64>(decode_kernel<64>, C::SMEM);
-    if (e != cudaSuccess) return e;
-    decode_kernel<64><<<grid, C::THREADS, C::SMEM, st>>>(p);
-  } else if (D == 128) {
-    using C = Dec<128>;
-    cudaError_t e = ensure_smem_limit<128>(decode_kernel<128>, C::SMEM);
-    if (e != cudaSuccess) return e;
-    decode_kernel<128><<<grid, C::THREADS, C::SMEM, st>>>(p);
-  } else {
-    return cudaErrorInvalidValue;
-  }
+template <int D, bool ROPE>
+static cudaError_t launch_decode_d(const DecodeParams& p, int grid, cudaStream_t st) {
+  using C = Dec<D>;
+  cudaError_t e = ensure_smem_limit<D + (ROPE ? 1 : 0)>(decode_kernel<D, ROPE>, C::SMEM);
+  if (e != cudaSuccess) return e;
+  decode_kernel<D, ROPE><<<grid, C::THREADS, C::SMEM, st>>>(p);
   return cudaGetLastError();
+}
+
+cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st) {
+  const bool rope = p.rope_tab != nullptr;
+  if (D == 64) return rope ? launch_decode_d<64, true>(p, grid, st) : launch_decode_d<64, false>(p, grid, st);
+  if (D == 128) return rope ? launch_decode_d<128, true>(p, grid, st) : launch_decode_d<128, false>(p, grid, st);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace smem

@@ -24,11 +24,13 @@ constexpr int kBlockTok = 64; // b: query tokens per block
 struct Layout {
   int L, H, D, max_seqs, max_blocks, capacity, has_null, max_batch;
   int recompute;       // 1: slots hold memory rows mu [R][d] instead of per-layer K/V
+  int rope_w;          // 0: no rotary phases; else the saturating window W of the RoPE composite
+  float rope_base;
   int dec_max_splits;  // split-K partial slots per (decode item, head)
   int pf_max_splits;   // split-K partial slots per prefill head
   size_t slot_elems;   // bf16 elements per pool slot: L*H*2*R*D, or R*d (recompute)
-  size_t off_pool, off_inblock, off_null, off_table, off_dec_part, off_dec_cnt, off_pf_part, off_pf_cnt,
-      off_err, total;
+  size_t off_pool, off_inblock, off_null, off_table, off_bidx, off_rope, off_rope_scr, off_dec_part, off_dec_cnt,
+      off_pf_part, off_pf_cnt, off_err, total;
 };
 
 // Split-K plan of the decode cross-attention: the number of memory blocks a
@@ -65,7 +67,14 @@ struct DecodeItem {
   int nblk;        // memory blocks read (table prefix with index < q_block_idx)
   int pos;         // in-block offset p of the new token
   int pair_begin;  // first (item, split) pair of this item
+  int qblk;        // the token's block index (rotary phase of its cross-attention query)
 };
+
+// Rotary phases of the SMem+RoPE composite: a table of (cos, sin) of
+// phase * theta_m for phases 0 .. kRopePhases-1 and pairs m < D/2
+// (theta_m = base^(-2m/D)); self-attention phases are in-block offsets,
+// cross-attention phase differences are clamped to the window W < 64.
+constexpr int kRopePhases = 64;
 
 struct DecodeParams {
   CUtensorMap tmap;          // pool viewed as [C][L*H*2*R][D] bf16, 128-byte swizzle
@@ -89,6 +98,9 @@ struct DecodeParams {
   int mode;                  // bit 0: in-block self-attention, bit 1: cross-attention
   int s_stride, c_stride;    // elements between items of qs/k_new/v_new and of qc
   float scale_log2;          // log2(e) / sqrt(D)
+  const float2* rope_tab;    // [kRopePhases][D/2] (cos, sin), or nullptr: no rotary phases
+  const int* bidx;           // [max_seqs][max_blocks] block index of each table entry
+  int rope_w;                // saturating window W
   DecodeItem items[kMaxDecodeItems];
 };
 
@@ -108,21 +120,30 @@ int decode_stage_rows(int D);
 // ---------------------------------------------------------------------------
 // Appends: copy K, V [L][H][R][D] into a pool slot and insert `slot` at
 // table position `pos` of `seq` (n_old entries before the insert).
+// The block index is inserted at the same position of the block-index row.
 cudaError_t launch_append(uint16_t* slot_base, const uint16_t* K, const uint16_t* V, int L, int H, int D,
-                          int* table_row, int pos, int n_old, int slot, cudaStream_t st);
-// Removes table position `pos` of a row holding n_old entries.
-cudaError_t launch_table_remove(int* table_row, int pos, int n_old, cudaStream_t st);
+                          int* table_row, int* bidx_row, int pos, int n_old, int slot, int block_idx,
+                          cudaStream_t st);
+// Removes table position `pos` of a row (and of its block-index row) holding n_old entries.
+cudaError_t launch_table_remove(int* table_row, int* bidx_row, int pos, int n_old, cudaStream_t st);
 // In-block write: rows [n][H][D] (token stride `tok` elements, 0: H*D) ->
-// inblock[seq][layer][h][2][b][D].
+// inblock[seq][layer][h][2][b][D]; with a rotary table the keys are stored
+// turned by their in-block offset.
 cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
-                                 int D, cudaStream_t st, int tok = 0);
+                                 int D, cudaStream_t st, int tok = 0, const float2* rope_tab = nullptr);
+// Rotary phases by in-block offset: row t of src (n tokens x H heads x D,
+// token stride src_tok) turned by phase t into dst (token stride dst_tok;
+// dst may equal src).
+cudaError_t launch_rope_rows(const uint16_t* src, int src_tok, uint16_t* dst, int dst_tok, int n, int H, int D,
+                             const float2* rope_tab, cudaStream_t st);
 // Null row: k,v [L][H][D] -> null_kv [L][H][2][D].
 cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
                               cudaStream_t st);
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st);
 
 // Table insert alone (the slot's rows written by other kernels before it).
-cudaError_t launch_table_insert(int* table_row, int pos, int n_old, int slot, cudaStream_t st);
+cudaError_t launch_table_insert(int* table_row, int* bidx_row, int pos, int n_old, int slot, int block_idx,
+                                cudaStream_t st);
 
 // ---------------------------------------------------------------------------
 // dense parts of the reader layer (LayerNorm, GELU, cuBLAS projections)
@@ -214,6 +235,9 @@ struct PrefillArgs {
   long long slot_elems;
   int L, H, D, layer, nblk, split_blks, n_splits, capacity;
   int cluster;                // 1: cluster mode (one cluster of n_splits + 1 CTAs per head)
+  const float2* rope_tab;     // rotary table or nullptr (Qs/Ks then arrive already turned by offset)
+  const int* bidx_row;        // block index of each table entry of this sequence
+  int rope_w, q_blk;          // saturating window, the query block's index
   int mode;                   // bit 0: self-attention, bit 1: cross-attention (0: both)
   int tok_s, tok_c;           // elements between tokens of Qs/Ks/Vs and of Qc (0: H*D)
   float scale_log2;

@@ -81,14 +81,70 @@ struct PrefillParams {
   int n_sa;            // self-attention CTAs of the cluster-free grid (0 or H)
   int tok_c;           // elements between consecutive tokens of Qc
   float scale_log2;
+  const float2* rope_tab;  // rotary table [kRopePhases][D/2] (ROPE kernels only)
+  const int* bidx_row;     // block index of each table entry of the sequence
+  int rope_w, q_blk;       // saturating window W, the query block's index
+  int rope_half;           // D/2: pairs per table row
 };
+
+// (x[2m], x[2m+1]) of 8 values turned by table pairs cs[0..3].
+__device__ __forceinline__ void rot8(float* t, const float2* cs) {
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 c = cs[e];
+    const float x0 = t[2 * e], x1 = t[2 * e + 1];
+    t[2 * e] = x0 * c.x - x1 * c.y;
+    t[2 * e + 1] = x0 * c.y + x1 * c.x;
+  }
+}
+
+// Turns a [64 rows][D] bf16 tile (D/64 boxes of [64][128 B], 128-byte
+// swizzle) in place by one table row; one warp, then a proxy fence so that
+// the tensor cores see the new values.
+template <int D>
+__device__ void rotate_tile(uint8_t* tile, const float2* cs_row, int lane) {
+  constexpr int CH = D / 8;  // 16-byte chunks per row
+  for (int i = lane; i < 64 * CH; i += 32) {
+    const int r = i / CH, c = i % CH;
+    uint8_t* ptr = tile + (c >> 3) * (64 * 128) + r * 128 + ((((c & 7) ^ (r & 7))) << 4);
+    float t[8];
+    unpack8(*reinterpret_cast<const uint4*>(ptr), t);
+    rot8(t, cs_row + c * 4);
+    *reinterpret_cast<uint4*>(ptr) = make_uint4(pack_bf16x2(t[0], t[1]), pack_bf16x2(t[2], t[3]),
+                                                pack_bf16x2(t[4], t[5]), pack_bf16x2(t[6], t[7]));
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+}
+
+// A query row's cross-attention null-row score (its columns col0 ..
+// col0+n-1): with rotary phases the null row's key sits at phase
+// max(0, i - W), so the query turns by min(i, W).
+template <bool ROPE>
+__device__ __forceinline__ float null_dot(const PrefillParams& p, const uint16_t* q, const uint16_t* kn, int col0,
+                                          int n) {
+  float dot = 0.f;
+  const float2* cs = ROPE ? p.rope_tab + (size_t)min(p.q_blk, p.rope_w) * (p.rope_half) + col0 / 2 : nullptr;
+  for (int c = 0; c < n; c += 2) {
+    float x0 = bf16lo(q[col0 + c]), x1 = bf16lo(q[col0 + c + 1]);
+    if (ROPE) {
+      const float2 r = cs[c / 2];
+      const float y0 = x0 * r.x - x1 * r.y;
+      x1 = x0 * r.y + x1 * r.x;
+      x0 = y0;
+    }
+    dot = fmaf(x0, bf16lo(kn[col0 + c]), dot);
+    dot = fmaf(x1, bf16lo(kn[col0 + c + 1]), dot);
+  }
+  return dot;
+}
 
 // Cluster mode (d_h = 64): one cluster of n_splits + 1 CTAs per head, rank 0
 // the in-block SA tile and rank k the split k-1. Each split CTA parks its
 // partial rows (m, l, O) in its own shared memory; after a cluster barrier
 // every CTA merges a slice of the 64 rows by reading the others' partials
 // over distributed shared memory, in split order (null row first).
-template <int D>
+template <int D, bool ROPE>
 __device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint32_t cs, uint32_t stage_saddr,
                               int warp, int lane) {
   constexpr int CPL = D / 32;  // columns per lane
@@ -101,10 +157,7 @@ __device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint
     float nscore = -INFINITY;
     if (p.null_kv) {
       const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
-      float dot = 0.f;
-#pragma unroll
-      for (int e = 0; e < CPL; ++e)
-        dot = fmaf(bf16lo(p.qc_ptr[qcoff + lane * CPL + e]), bf16lo(kn[lane * CPL + e]), dot);
+      float dot = null_dot<ROPE>(p, p.qc_ptr + qcoff, kn, lane * CPL, CPL);
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
       nscore = dot * p.scale_log2;
@@ -157,7 +210,7 @@ __device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint
   }
 }
 
-template <int D, bool CL>
+template <int D, bool CL, bool ROPE>
 __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kernel(const __grid_constant__ PrefillParams p) {
   using C = Pf<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -263,6 +316,77 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         mbar_wait_bounded(q_full, 0, nullptr);
         for (int j = 0; j < issued; ++j) mbar_wait_bounded(&full[j % C::NS], (j / C::NS) & 1, nullptr);
       }
+    }
+  } else if (warp == 5 && ROPE && !sa) {
+    // ------------------------------------------- MMA issuer, rotary phases (CA)
+    // The whole warp runs the loop: it turns the query tile by W once and the
+    // key tile of every near block j (the last W table entries) by
+    // W - (i - j), so that each score sees the relative phase min(i - j, W);
+    // lane 0 issues the MMAs.
+    if (work) {
+      bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(q_full, 0, abort_flag));
+      const int near0 = max(b0, p.nblk - p.rope_w);
+      int jv0 = 0, jv1 = 0;
+      if (near0 + lane < b0 + nt) jv0 = p.bidx_row[near0 + lane];
+      if (near0 + 32 + lane < b0 + nt) jv1 = p.bidx_row[near0 + 32 + lane];
+      if (ok) {
+        tc::fence_after();
+        rotate_tile<D>(qt, p.rope_tab + (size_t)p.rope_w * (D / 2), lane);
+      }
+      const uint32_t qa = smem_u32(qt);
+      for (int jj = 0; ok && jj <= nt; ++jj) {
+        if (jj < nt) {  // S[jj%2] = Q . K^T
+          const int st = jj % C::NS, sb = jj & 1;
+          ok = __all_sync(0xffffffffu, mbar_wait_bounded(&full[st], (jj / C::NS) & 1, abort_flag));
+          if (ok && jj >= 2)
+            ok = __all_sync(0xffffffffu, mbar_wait_bounded(&s_free[sb], ((jj >> 1) - 1) & 1, abort_flag));
+          if (!ok) break;
+          tc::fence_after();
+          if (b0 + jj >= near0) {
+            const int o = b0 + jj - near0;
+            const int j = __shfl_sync(0xffffffffu, o < 32 ? jv0 : jv1, o & 31);
+            const int dk = max(0, p.rope_w - (p.q_blk - j));
+            if (dk > 0) rotate_tile<D>(ring + st * C::STAGE, p.rope_tab + (size_t)dk * (D / 2), lane);
+          }
+          if (lane == 0) {
+            const uint32_t ka = smem_u32(ring + st * C::STAGE);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k) {
+              const uint32_t off = (k >> 2) * C::BOX + (k & 3) * 32;
+              tc::mma_bf16(tmem + 64 * sb, tc::sdesc_sw128(qa + off, 16, 1024), tc::sdesc_sw128(ka + off, 16, 1024),
+                           C::ID_QK, k > 0);
+            }
+            tc::commit(&s_full[sb]);
+          }
+          __syncwarp();
+        }
+        if (jj >= 1) {  // O += P . V for tile jj-1
+          const int j = jj - 1, st = j % C::NS, pb = j & 1;
+          ok = __all_sync(0xffffffffu, mbar_wait_bounded(&p_full[pb], (j >> 1) & 1, abort_flag));
+          if (!ok) break;
+          tc::fence_after();
+          if (lane == 0) {
+            const uint32_t pa = smem_u32(pt + pb * C::PBYTES);
+            const uint32_t va = smem_u32(ring + st * C::STAGE + C::TILE);
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024),
+                           tc::sdesc_sw128(va + k * 2048, C::BOX, 1024), C::ID_PV, (j > 0 || k > 0));
+            tc::commit(&empty[st]);
+            tc::commit(&o_done[pb]);
+          }
+          __syncwarp();
+        }
+      }
+      if (!ok) {
+        if (lane == 0 && !*abort_flag) record_error(p.err, kDevErrWaitMma);
+        *abort_flag = 1;
+      }
+      if (lane == 0) {
+        tc::commit(drain);
+        mbar_wait_bounded(drain, 0, nullptr);
+      }
+      __syncwarp();
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------- MMA issuer
@@ -462,9 +586,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         float nscore = -INFINITY;
         if (p.null_kv) {
           const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
-          float dot = 0.f;
-          for (int c = 0; c < D / 2; ++c)
-            dot = fmaf(bf16lo(p.qc_ptr[qcoff + col0 + c]), bf16lo(kn[col0 + c]), dot);
+          float dot = null_dot<ROPE>(p, p.qc_ptr + qcoff, kn, col0, D / 2);
           dot += __shfl_xor_sync(0xffffffffu, dot, 16);
           nscore = dot * p.scale_log2;
         }
@@ -546,7 +668,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   __syncthreads();
   if (CL && p.n_splits > 0) {
     tc::cluster_sync();  // every split's partial rows are parked
-    cluster_merge<D>(p, h, crank, cs, smem_u32(ring), warp, lane);
+    cluster_merge<D, ROPE>(p, h, crank, cs, smem_u32(ring), warp, lane);
     tc::cluster_sync();  // no CTA leaves while others read its shared memory
   }
   if (warp == 4) {
@@ -555,23 +677,26 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   }
 }
 
-template <int D>
+template <int D, bool ROPE>
 static cudaError_t launch_prefill_d(const PrefillParams& p, int grid, cudaStream_t st) {
   using C = Pf<D>;
-  cudaError_t e = ensure_smem_limit<1000 + D>(prefill_kernel<D, false>, C::SMEM);
+  cudaError_t e = ensure_smem_limit<1000 + D + (ROPE ? 1 : 0)>(prefill_kernel<D, false, ROPE>, C::SMEM);
   if (e != cudaSuccess) return e;
-  prefill_kernel<D, false><<<grid, C::THREADS, C::SMEM, st>>>(p);
+  prefill_kernel<D, false, ROPE><<<grid, C::THREADS, C::SMEM, st>>>(p);
   return cudaGetLastError();
 }
 
+template <bool ROPE>
 static cudaError_t cluster_kernel_setup() {
-  cudaError_t e = ensure_smem_limit<2064>(prefill_kernel<64, true>, Pf<64>::SMEM);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(prefill_kernel<64, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaError_t e = ensure_smem_limit<2064 + (ROPE ? 1 : 0)>(prefill_kernel<64, true, ROPE>, Pf<64>::SMEM);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(prefill_kernel<64, true, ROPE>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   return e;
 }
 
+template <bool ROPE>
 static cudaError_t launch_prefill_cluster(const PrefillParams& p, cudaStream_t st) {
-  cudaError_t e = cluster_kernel_setup();
+  cudaError_t e = cluster_kernel_setup<ROPE>();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   const unsigned cs = (unsigned)p.n_splits + 1;
@@ -586,7 +711,7 @@ static cudaError_t launch_prefill_cluster(const PrefillParams& p, cudaStream_t s
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, prefill_kernel<64, true>, p);
+  e = cudaLaunchKernelEx(&cfg, prefill_kernel<64, true, ROPE>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -605,7 +730,7 @@ int prefill_cluster_max(int H, int D) {
   // the largest cluster (at most 16 CTAs) of which one per head can be
   // resident at once on the current device; 0: cluster mode unavailable
   if (D != 64) return 0;
-  if (cluster_kernel_setup() != cudaSuccess ||
+  if (cluster_kernel_setup<false>() != cudaSuccess || cluster_kernel_setup<true>() != cudaSuccess ||
       cudaFuncSetAttribute(prefill_footprint_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, Pf<64>::SMEM) !=
           cudaSuccess ||
       cudaFuncSetAttribute(prefill_footprint_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
@@ -688,9 +813,16 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   P.scale_log2 = a.scale_log2;
   P.n_sa = ((mode & 1) || ((mode & 2) && a.nblk == 0)) ? a.H : 0;
   const int grid = P.n_splits * a.H + P.n_sa;
-  if (a.D == 64 && a.cluster && P.n_splits > 0) return launch_prefill_cluster(P, st);
-  if (a.D == 64) return launch_prefill_d<64>(P, grid, st);
-  if (a.D == 128) return launch_prefill_d<128>(P, grid, st);
+  P.rope_tab = a.rope_tab;
+  P.bidx_row = a.bidx_row;
+  P.rope_w = a.rope_w;
+  P.q_blk = a.q_blk;
+  P.rope_half = a.D / 2;
+  const bool rope = a.rope_tab != nullptr;
+  if (a.D == 64 && a.cluster && P.n_splits > 0)
+    return rope ? launch_prefill_cluster<true>(P, st) : launch_prefill_cluster<false>(P, st);
+  if (a.D == 64) return rope ? launch_prefill_d<64, true>(P, grid, st) : launch_prefill_d<64, false>(P, grid, st);
+  if (a.D == 128) return rope ? launch_prefill_d<128, true>(P, grid, st) : launch_prefill_d<128, false>(P, grid, st);
   return cudaErrorInvalidValue;
 }
 

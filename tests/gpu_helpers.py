@@ -43,11 +43,12 @@ class DeviceCache:
     """A device cache plus a host record of what each slot holds."""
 
     def __init__(self, L, H, D, max_seqs, max_blocks, capacity, seed=0, free_order=None, has_null=False,
-                 max_batch=None):
+                 max_batch=None, rope_window=0):
         self.L, self.H, self.D = L, H, D
         self.seed = seed
+        self.rope_window = rope_window
         self.cfg = smem.make_config(L, H, D, max_seqs, max_blocks, capacity, has_null_row=has_null,
-                                    max_decode_batch=max_batch, free_order=free_order)
+                                    max_decode_batch=max_batch, free_order=free_order, rope_window=rope_window)
         self.cache = smem.SmemCache(self.cfg, device="cuda")
         self.h = self.cache.h
         self.mirror = CacheMirror(capacity, max_seqs, max_blocks, free_order=free_order)
@@ -124,6 +125,10 @@ class DeviceCache:
     def oracle_prefill(self, seq, layer, q_idx, qs, ks, vs, qc):
         idx, mk, mv = self.oracle_memory(seq, layer)
         kn0, vn0 = self.null(layer)
+        if self.rope_window:
+            from oracle.rope import reader_prefill_rope
+            return reader_prefill_rope(idx, mk, mv, q_idx, f64(qs), f64(ks), f64(vs), f64(qc), kn0, vn0,
+                                       window=self.rope_window)
         return oracle.reader_prefill(idx, mk, mv, q_idx, f64(qs), f64(ks), f64(vs), f64(qc), kn0, vn0)
 
     # -------------------------------------------------------------- decode
@@ -154,4 +159,8 @@ class DeviceCache:
         kin = f64(Kb[:p]) if p else None
         vin = f64(Vb[:p]) if p else None
         kn0, vn0 = self.null(layer)
+        if self.rope_window:
+            from oracle.rope import reader_decode_rope
+            return reader_decode_rope(idx, mk, mv, qidx, p, kin, vin, f64(qs), f64(kn), f64(vn), f64(qc), kn0, vn0,
+                                      window=self.rope_window)
         return oracle.reader_decode(idx, mk, mv, qidx, p, kin, vin, f64(qs), f64(kn), f64(vn), f64(qc), kn0, vn0)

@@ -85,7 +85,8 @@ def test_one_block_layer_equals_full_pass(with_null):
         np.testing.assert_allclose(out, full[sl], rtol=0, atol=1e-11)
 
 
-def test_decode_step_equals_one_block_row():
+@pytest.mark.parametrize("rope_window", [0, 2])
+def test_decode_step_equals_one_block_row(rope_window):
     rng = np.random.default_rng(37)
     b, H, D, nblk = 8, 2, 8, 3
     d = H * D
@@ -93,9 +94,10 @@ def test_decode_step_equals_one_block_row():
     X = rng.standard_normal((b, d))
     mu = rng.standard_normal((nblk, b, d))
     nu = rng.standard_normal(d)
-    out, ks, vs = reader_layer_prefill(X, np.arange(nblk), mu, nblk, w, H, D, nu)
+    out, ks, vs = reader_layer_prefill(X, np.arange(nblk), mu, nblk, w, H, D, nu, rope_window=rope_window)
     for p in (0, 3, b - 1):
-        xo, kn, vn = reader_layer_decode(X[p], np.arange(nblk), mu, nblk, p, ks[:p], vs[:p], w, H, D, nu)
+        xo, kn, vn = reader_layer_decode(X[p], np.arange(nblk), mu, nblk, p, ks[:p], vs[:p], w, H, D, nu,
+                                         rope_window=rope_window)
         np.testing.assert_allclose(xo, out[p], rtol=0, atol=1e-12)
         np.testing.assert_allclose(kn, ks[p], rtol=0, atol=1e-12)
 
