@@ -47,6 +47,7 @@ def parse_args():
     ap.add_argument("--no-serve", action="store_true")
     ap.add_argument("--no-layer", action="store_true", help="skip the full-reader-layer cells")
     ap.add_argument("--no-recompute", action="store_true", help="skip the recompute-K/V cells")
+    ap.add_argument("--no-rope", action="store_true", help="skip the rotary-phase (RoPE composite) cells")
     ap.add_argument("--workload", default="decode", choices=["decode", "long"],
                     help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
     ap.add_argument("--long-batches", default="1,16", help="batches of the long-context cells")
@@ -189,7 +190,7 @@ def rank_seed(seed: int, rank: int) -> int:
 class DecodeWorkload:
     """Device state of the 410M-shaped batched-decode workload."""
 
-    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None):
+    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None, rope_window=0):
         import torch
 
         import synth
@@ -207,7 +208,8 @@ class DecodeWorkload:
         capacity = int(self.nblk.sum()) + sum(self.n_new)
         max_blocks = int(self.nblk.max()) + max(self.n_new) + 1
         perm = synth.slot_permutation(self.seed, capacity)
-        self.cfg = smem.make_config(self.L, self.H, self.D, seqs, max_blocks, capacity, free_order=perm)
+        self.cfg = smem.make_config(self.L, self.H, self.D, seqs, max_blocks, capacity, free_order=perm,
+                                    rope_window=rope_window)
         self.cache = smem.SmemCache(self.cfg, device=device)
         self.h = self.cache.h
         torch.cuda.synchronize()
@@ -393,6 +395,43 @@ def measure_layer_decode(wl, steps, warmup, device):
             "timing": "CUDA events around the layer calls of each step (appends excluded), inputs resident"}
 
 
+ROPE_WINDOW = 15  # the paper's saturating window (trained range of 16 blocks)
+
+
+def measure_rope_decode(steps, warmup, device, seqs, layers=None):
+    """The headline decode workload on a cache with the SMem+RoPE composite's
+    rotary phases (window 15): decode tok/s and the decode kernel's HBM
+    fraction, timed like the headline (CUDA events per launch)."""
+    import torch
+
+    from paper_2609_32395_gb300 import smem
+
+    wl = DecodeWorkload(seqs, warmup + steps + 2, WORKLOAD["seed"], device, layers=layers, rope_window=ROPE_WINDOW)
+    for _ in range(warmup):
+        wl.step()
+    torch.cuda.synchronize()
+    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(wl.L)] for _ in range(2)] for _ in range(steps)]
+    st = torch.cuda.current_stream()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    rows = []
+    start.record(st)
+    for i in range(steps):
+        rows.append(wl.rows_read())
+        wl.step(events=ev[i])
+    end.record(st)
+    torch.cuda.synchronize()
+    if smem.smem_check_device_error(wl.h) != smem.OK:
+        raise RuntimeError("device error recorded during the rotary decode")
+    elapsed = start.elapsed_time(end) / 1e3
+    kern_ms = [ev[i][0][l].elapsed_time(ev[i][1][l]) for i in range(steps) for l in range(wl.L)]
+    alg = [r * 4 * wl.H * wl.D for r in rows for _ in range(wl.L)]
+    out = {"window": ROPE_WINDOW, "tok_per_s": steps * seqs / elapsed, "steps": steps,
+           "kernel_ms_mean": float(np.mean(kern_ms)),
+           "achieved_gbs": sum(alg) / (sum(kern_ms) / 1e3) / 1e9}
+    wl.cache.close()
+    return out
+
+
 class RecomputeDecode:
     """The 410M-shaped decode workload on a recompute-K/V cache: the pool
     holds only each block's memory rows mu [R][d] (d = H*d_h, shared by the
@@ -514,7 +553,7 @@ class PrefillWorkload:
     shuffled slots) served by running the reader's attention on the final
     block alone: 12 one-block prefill launches, one per layer."""
 
-    def __init__(self, nblk, device, L=None, H=None, D=None, seed=None, recompute=False):
+    def __init__(self, nblk, device, L=None, H=None, D=None, seed=None, recompute=False, rope_window=0):
         import torch
 
         import synth
@@ -527,7 +566,8 @@ class PrefillWorkload:
         seed = SERVE["seed"] if seed is None else seed
         cap = nblk + 2
         self.cfg = smem.make_config(self.L, self.H, self.D, 1, nblk + 1, cap,
-                                    free_order=synth.slot_permutation(seed + nblk, cap), recompute_kv=recompute)
+                                    free_order=synth.slot_permutation(seed + nblk, cap), recompute_kv=recompute,
+                                    rope_window=rope_window)
         self.cache = smem.SmemCache(self.cfg, device=device)
         self.h = self.cache.h
         if recompute:  # the pool keeps memory rows only; attention-only launches do not apply
@@ -575,14 +615,14 @@ class PrefillWorkload:
         return ca + sa
 
 
-def measure_serve(nblk, device, iters=30, flush_bytes=512 << 20):
+def measure_serve(nblk, device, iters=30, flush_bytes=512 << 20, rope_window=0):
     """Latency of one cached-context serve (12 layers) replayed from a CUDA
     graph, and the mean duration of one prefill launch; L2 is flushed before
     each timed iteration (the flush also keeps the stream busy while the
     timed work is enqueued)."""
     import torch
 
-    wl = PrefillWorkload(nblk, device)
+    wl = PrefillWorkload(nblk, device, rope_window=rope_window)
     flush = torch.empty(flush_bytes, dtype=torch.uint8, device=device)
     st = torch.cuda.current_stream()
     for _ in range(3):
@@ -1054,6 +1094,12 @@ def run_ours(args):
     recompute = None
     if not args.no_recompute and rank == 0:
         recompute = measure_recompute(min(args.steps, 64), args.warmup, device, args.seqs, layers=args.layers)
+    rope = None
+    if not args.no_rope and rank == 0:
+        wl.cache.close()
+        wl.cache.buf = None
+        torch.cuda.empty_cache()
+        rope = {"decode": measure_rope_decode(min(args.steps, 64), args.warmup, device, args.seqs, layers=args.layers)}
     if not args.no_serve:
         wl.cache.close()
         wl.cache.buf = None
@@ -1063,6 +1109,8 @@ def run_ours(args):
         layer_serve = None if args.no_layer else [measure_layer_serve(n, device) for n in SERVE["contexts"]]
         if not args.no_layer and not args.no_recompute:
             rec_serve = [measure_layer_serve(n, device, recompute=True) for n in SERVE["contexts"]]
+        if rope is not None:
+            rope["serve"] = [measure_serve(n, device, rope_window=ROPE_WINDOW) for n in SERVE["contexts"]]
     edit = None if args.no_serve else [measure_edit_latency(n, device) for n in EDIT["contexts"]]
 
     if rank != 0:
@@ -1119,6 +1167,10 @@ def run_ours(args):
             layer["serve"] = {"workload": SERVE["name"], "unit": "ms", "cells": layer_serve,
                               "timing": "CUDA graph of the 12 layer calls, L2 flushed before each"}
         line["layer"] = layer
+    if rope:
+        rope["decode"]["hbm_frac"] = rope["decode"]["achieved_gbs"] / peak
+        rope["workload"] = WORKLOAD["name"] + " and " + SERVE["name"] + ", SMem+RoPE composite (window 15)"
+        line["rope"] = rope
     if recompute:
         k = recompute["memory_row_kernel"]
         k["hbm_frac"] = k["achieved_gbs"] / peak

@@ -611,11 +611,10 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
     uint16_t* kr = qr + (size_t)smem::kBlockTok * L.H * L.D;
     const int tok = L.H * L.D;
     if (injected_failure(c)) return SMEM_ERR_CUDA;
-    int rc = check_launch(c, smem::launch_rope_rows(static_cast<const uint16_t*>(Qs), tok, qr, tok, smem::kBlockTok,
-                                                    L.H, L.D, rope_tab(c), st), "rotary");
-    if (!rc)
-      rc = check_launch(c, smem::launch_rope_rows(static_cast<const uint16_t*>(Ks), tok, kr, tok, smem::kBlockTok, L.H,
-                                                  L.D, rope_tab(c), st), "rotary");
+    const int rc = check_launch(c, smem::launch_rope_rows(static_cast<const uint16_t*>(Qs), qr,
+                                                          static_cast<const uint16_t*>(Ks), kr, tok, tok,
+                                                          smem::kBlockTok, L.H, L.D, rope_tab(c), st),
+                                "rotary");
     if (rc) return rc;
     return prefill_impl(c, seq, layer, q_block_idx, qr, kr, Vs, Qc, Osa, Oca, 3, 0, 0, st);
   }
@@ -988,10 +987,9 @@ int smem_reader_layer_prefill(smem_cache* c, int32_t seq, int32_t layer, int32_t
   const int d = r.d;
   rc = r.qkv_proj();
   if (!rc && L.rope_w) {  // self-attention queries and keys turn by their in-block offsets
-    rc = cuda_rc(smem::launch_rope_rows(r.qkv(), 3 * d, r.qkv(), 3 * d, n, L.H, L.D, rope_tab(c), st), "rotary");
-    if (!rc)
-      rc = cuda_rc(smem::launch_rope_rows(r.qkv() + d, 3 * d, r.qkv() + d, 3 * d, n, L.H, L.D, rope_tab(c), st),
-                   "rotary");
+    rc = cuda_rc(smem::launch_rope_rows(r.qkv(), r.qkv(), r.qkv() + d, r.qkv() + d, 3 * d, 3 * d, n, L.H, L.D,
+                                        rope_tab(c), st),
+                 "rotary");
   }
   // the block's self-attention keys/values become its in-block rows (already turned)
   if (!rc)

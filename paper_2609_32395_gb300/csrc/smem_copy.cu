@@ -89,10 +89,13 @@ __device__ __forceinline__ uint4 rotate8(const uint4 v, const float2* cs) {
   return make_uint4(o[0], o[1], o[2], o[3]);
 }
 
-// src rows [n][H][D] (token stride src16 16-byte chunks) -> dst, token t
-// turned by phase t (tab: [kRopePhases][D/2] float2).
-__global__ void rope_rows_kernel(const uint4* src, int src16, uint4* dst, int dst16, int n, int H, int cpr,
-                                 const float2* tab) {
+// Two row sets (blockIdx.y: 0 -> a, 1 -> b) of [n][H][D] (token stride
+// src16 16-byte chunks) -> dst, token t turned by phase t (tab:
+// [kRopePhases][D/2] float2).
+__global__ void rope_rows_kernel(const uint4* src_a, uint4* dst_a, const uint4* src_b, uint4* dst_b, int src16,
+                                 int dst16, int n, int H, int cpr, const float2* tab) {
+  const uint4* src = blockIdx.y ? src_b : src_a;
+  uint4* dst = blockIdx.y ? dst_b : dst_a;
   const int total = n * H * cpr;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
     const int t = i / (H * cpr);
@@ -164,14 +167,14 @@ cudaError_t launch_table_remove(int* table_row, int* bidx_row, int pos, int n_ol
   return cudaGetLastError();
 }
 
-cudaError_t launch_rope_rows(const uint16_t* src, int src_tok, uint16_t* dst, int dst_tok, int n, int H, int D,
-                             const float2* rope_tab, cudaStream_t st) {
+cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, const uint16_t* src_b, uint16_t* dst_b,
+                             int src_tok, int dst_tok, int n, int H, int D, const float2* rope_tab, cudaStream_t st) {
   if (n == 0) return cudaSuccess;
   const int cpr = D / 8;
   const int total = n * H * cpr;
-  rope_rows_kernel<<<(total + 255) / 256, 256, 0, st>>>(reinterpret_cast<const uint4*>(src), src_tok / 8,
-                                                        reinterpret_cast<uint4*>(dst), dst_tok / 8, n, H, cpr,
-                                                        rope_tab);
+  rope_rows_kernel<<<dim3((total + 255) / 256, 2), 256, 0, st>>>(
+      reinterpret_cast<const uint4*>(src_a), reinterpret_cast<uint4*>(dst_a), reinterpret_cast<const uint4*>(src_b),
+      reinterpret_cast<uint4*>(dst_b), src_tok / 8, dst_tok / 8, n, H, cpr, rope_tab);
   return cudaGetLastError();
 }
 

@@ -131,11 +131,11 @@ cudaError_t launch_table_remove(int* table_row, int* bidx_row, int pos, int n_ol
 // turned by their in-block offset.
 cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
                                  int D, cudaStream_t st, int tok = 0, const float2* rope_tab = nullptr);
-// Rotary phases by in-block offset: row t of src (n tokens x H heads x D,
-// token stride src_tok) turned by phase t into dst (token stride dst_tok;
-// dst may equal src).
-cudaError_t launch_rope_rows(const uint16_t* src, int src_tok, uint16_t* dst, int dst_tok, int n, int H, int D,
-                             const float2* rope_tab, cudaStream_t st);
+// Rotary phases by in-block offset, for two row sets at once (queries and
+// keys): row t of src (n tokens x H heads x D, token stride src_tok) turned
+// by phase t into dst (token stride dst_tok; dst may equal src).
+cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, const uint16_t* src_b, uint16_t* dst_b,
+                             int src_tok, int dst_tok, int n, int H, int D, const float2* rope_tab, cudaStream_t st);
 // Null row: k,v [L][H][D] -> null_kv [L][H][2][D].
 cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
                               cudaStream_t st);
