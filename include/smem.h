@@ -59,7 +59,7 @@
 extern "C" {
 #endif
 
-#define SMEM_ABI_VERSION 4
+#define SMEM_ABI_VERSION 5
 
 enum {
     SMEM_OK = 0,
@@ -156,8 +156,27 @@ int smem_append_block(smem_cache *c, int32_t seq, int32_t block_idx, const void 
 /* Deletes block `block_idx` of `seq` (Theorem 1: the result is exactly the
  * memory in which the block was never encoded; other blocks keep their
  * indices): removes the table entry and puts the slot at the back of the
- * free FIFO. No memory row moves. */
+ * free FIFO (once no other table entry shares it). No memory row moves. */
 int smem_delete_block(smem_cache *c, int32_t seq, int32_t block_idx, void *stream);
+
+/* Shares a cached block (exact composition, Sec. 2: a block encoded once is
+ * reusable under any surrounding content): the table of dst_seq gains an
+ * entry (dst_idx -> the slot of src_seq's block src_idx); no row is copied.
+ * Slots count the table entries naming them; smem_delete_block and
+ * smem_release_seq drop one reference each, and a slot returns to the back of
+ * the free FIFO when its last reference goes. Without rotary phases the
+ * block keeps its index (dst_idx must equal src_idx, SMEM_ERR_INVALID_ARG
+ * otherwise: moving a block needs a re-encode); on a rope_window cache its
+ * rows carry no position and dst_idx is free. Errors, checked in this order:
+ * SMEM_ERR_NO_SUCH_SEQ (either id), SMEM_ERR_INVALID_ARG (negative index),
+ * SMEM_ERR_NO_SUCH_BLOCK, SMEM_ERR_INVALID_ARG (index rule),
+ * SMEM_ERR_DUPLICATE_BLOCK, SMEM_ERR_TABLE_FULL. *slot_out (may be NULL)
+ * receives the shared slot. */
+int smem_share_block(smem_cache *c, int32_t src_seq, int32_t src_idx, int32_t dst_seq, int32_t dst_idx,
+                     void *stream, int32_t *slot_out);
+
+/* Number of table entries naming `slot` (0: free). */
+int smem_slot_refs(const smem_cache *c, int32_t slot, int32_t *n_out);
 
 /* Deletes every block of `seq`; slots go to the back of the free FIFO in
  * ascending block order. */

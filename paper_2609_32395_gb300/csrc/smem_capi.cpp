@@ -36,6 +36,7 @@ struct smem_cache {
   std::vector<std::vector<int32_t>> idx;   // per sequence, ascending block index
   std::vector<std::vector<int32_t>> slot;  // per sequence, same order
   std::deque<int32_t> fifo;                // free slots, front = next to use
+  std::vector<int32_t> refs;               // table entries naming each slot (0: free)
   std::vector<uint32_t> seen;              // decode: duplicate-sequence check
   uint32_t seen_epoch = 0;
   int fail_after = 0;                      // test hook: n-th next launch fails
@@ -434,6 +435,7 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
   c->idx.assign(L.max_seqs, {});
   c->slot.assign(L.max_seqs, {});
   c->fifo.assign(order.begin(), order.end());
+  c->refs.assign(L.capacity, 0);
   c->seen.assign(L.max_seqs, 0);
   if (device) {
     c->dev = static_cast<uint8_t*>(dev_buf);
@@ -533,6 +535,7 @@ int smem_append_block(smem_cache* c, int32_t seq, int32_t block_idx, const void*
     if (rc) return rc;
   }
   c->fifo.pop_front();
+  c->refs[s] = 1;
   ix.insert(ix.begin() + pos, block_idx);
   c->slot[seq].insert(c->slot[seq].begin() + pos, s);
   if (slot_out) *slot_out = s;
@@ -558,7 +561,46 @@ int smem_delete_block(smem_cache* c, int32_t seq, int32_t block_idx, void* strea
   const int32_t s = c->slot[seq][pos];
   ix.erase(ix.begin() + pos);
   c->slot[seq].erase(c->slot[seq].begin() + pos);
-  c->fifo.push_back(s);
+  if (--c->refs[s] == 0) c->fifo.push_back(s);
+  return SMEM_OK;
+}
+
+int smem_share_block(smem_cache* c, int32_t src_seq, int32_t src_idx, int32_t dst_seq, int32_t dst_idx,
+                     void* stream, int32_t* slot_out) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (src_seq < 0 || src_seq >= c->lay.max_seqs || dst_seq < 0 || dst_seq >= c->lay.max_seqs)
+    return SMEM_ERR_NO_SUCH_SEQ;
+  if (src_idx < 0 || dst_idx < 0) return SMEM_ERR_INVALID_ARG;
+  const std::vector<int32_t>& sx = c->idx[src_seq];
+  const auto si = std::lower_bound(sx.begin(), sx.end(), src_idx);
+  if (si == sx.end() || *si != src_idx) return SMEM_ERR_NO_SUCH_BLOCK;
+  // rows that carry no block position (rotary phases) may be reused at any index
+  if (!c->lay.rope_w && dst_idx != src_idx) return SMEM_ERR_INVALID_ARG;
+  const int32_t s = c->slot[src_seq][si - sx.begin()];
+  std::vector<int32_t>& dx = c->idx[dst_seq];
+  const auto di = std::lower_bound(dx.begin(), dx.end(), dst_idx);
+  const int pos = (int)(di - dx.begin());
+  if (di != dx.end() && *di == dst_idx) return SMEM_ERR_DUPLICATE_BLOCK;
+  if ((int)dx.size() >= c->lay.max_blocks) return SMEM_ERR_TABLE_FULL;
+  if (c->dev) {
+    DeviceGuard g(c->device);
+    if (injected_failure(c)) return SMEM_ERR_CUDA;
+    const int rc = check_launch(c,
+                                smem::launch_table_insert(table_row(c, dst_seq), bidx_row(c, dst_seq), pos,
+                                                          (int)dx.size(), s, dst_idx, as_stream(stream)),
+                                "share");
+    if (rc) return rc;
+  }
+  dx.insert(dx.begin() + pos, dst_idx);
+  c->slot[dst_seq].insert(c->slot[dst_seq].begin() + pos, s);
+  ++c->refs[s];
+  if (slot_out) *slot_out = s;
+  return SMEM_OK;
+}
+
+int smem_slot_refs(const smem_cache* c, int32_t slot, int32_t* n_out) {
+  if (!c || !n_out || slot < 0 || slot >= c->lay.capacity) return SMEM_ERR_INVALID_ARG;
+  *n_out = c->refs[slot];
   return SMEM_OK;
 }
 
@@ -566,7 +608,8 @@ int smem_release_seq(smem_cache* c, int32_t seq, void* stream) {
   (void)stream;  // the device row needs no edit: its length lives on the host
   if (!c) return SMEM_ERR_INVALID_ARG;
   if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
-  for (int32_t s : c->slot[seq]) c->fifo.push_back(s);
+  for (int32_t s : c->slot[seq])
+    if (--c->refs[s] == 0) c->fifo.push_back(s);
   c->idx[seq].clear();
   c->slot[seq].clear();
   return SMEM_OK;
@@ -792,6 +835,7 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
                                                           block_idx, st), "append rows");
   if (rc) return rc;
   c->fifo.pop_front();
+  c->refs[s] = 1;
   ix.insert(ix.begin() + pos, block_idx);
   c->slot[seq].insert(c->slot[seq].begin() + pos, s);
   if (slot_out) *slot_out = s;

@@ -37,7 +37,7 @@ EXPORTED = [
     "smem_decode", "smem_decode_static_scratch", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table", "smem_check_device_error",
     "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
     "smem_layer_workspace_bytes", "smem_append_block_rows", "smem_set_null_vector", "smem_reader_layer_prefill",
-    "smem_reader_layer_decode", "smem_mu_decode", "smem_mu_prefill",
+    "smem_reader_layer_decode", "smem_mu_decode", "smem_mu_prefill", "smem_share_block", "smem_slot_refs",
 ]
 
 
@@ -118,6 +118,8 @@ def lib():
                                                         ctypes.c_size_t, _vp]),
             "smem_mu_decode": (ctypes.c_int, [_vp, _i32, _i32p, _i32p, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
             "smem_mu_prefill": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
+            "smem_share_block": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32, _vp, _i32p]),
+            "smem_slot_refs": (ctypes.c_int, [_vp, _i32, _i32p]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -196,6 +198,20 @@ def smem_append_block(h, seq, block_idx, K=None, V=None, stream=None) -> int:
     st = _stream(stream) if K is not None else None
     _check(lib().smem_append_block(h, seq, block_idx, _ptr(K), _ptr(V), st, ctypes.byref(slot)), "smem_append_block")
     return slot.value
+
+
+def smem_share_block(h, src_seq, src_idx, dst_seq, dst_idx, stream=None, device=True) -> int:
+    """dst_seq's table gains (dst_idx -> the slot of src_seq's src_idx); returns the slot."""
+    slot = ctypes.c_int32(-1)
+    st = _stream(stream) if device else None
+    _check(lib().smem_share_block(h, src_seq, src_idx, dst_seq, dst_idx, st, ctypes.byref(slot)), "smem_share_block")
+    return slot.value
+
+
+def smem_slot_refs(h, slot) -> int:
+    n = ctypes.c_int32(0)
+    _check(lib().smem_slot_refs(h, slot, ctypes.byref(n)), "smem_slot_refs")
+    return n.value
 
 
 def smem_delete_block(h, seq, block_idx, stream=None, device=True):

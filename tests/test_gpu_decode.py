@@ -143,3 +143,59 @@ def test_decode_rejects_bad_arguments():
     with pytest.raises(smem.SmemError) as e:
         smem.smem_decode(dc.h, 1, [0], [0], [1], x, x, x, x, x, x)  # no such layer
     assert e.value.code == smem.ERR_INVALID_ARG
+
+
+@pytest.mark.gpu
+def test_shared_blocks_read_like_private_copies():
+    """Exact reuse (Sec. 2): sequence 1 shares sequence 0's cached blocks by
+    reference, sequence 2 holds private copies of the same rows; prefill and
+    decode outputs of 1 and 2 are bitwise equal. Deleting 0's references
+    keeps 1 unchanged and frees no shared slot; releasing 1 frees them."""
+    import torch
+
+    import synth
+    from paper_2609_32395_gb300 import smem
+    from tests.gpu_helpers import DeviceCache, to_dev
+
+    dc = DeviceCache(L=2, H=4, D=64, max_seqs=3, max_blocks=16, capacity=40)
+    for j in range(10):
+        dc.append(0, j)
+        dc.append(2, j, content_seq=0)            # private copy of the same rows
+    for j in range(10):
+        smem.smem_share_block(dc.h, 0, j, 1, j)
+        assert dc.mirror.share(0, j, 1, j)[0] == 0
+    fifo0 = smem.smem_get_free_fifo(dc.h)
+    assert fifo0 == dc.mirror.free_list()
+
+    def outputs():
+        res = []
+        for s in (1, 2):
+            _, sa, ca = dc.prefill(s, 1, 10, tag=3)
+            res.append((sa, ca))
+        return res
+
+    (sa1, ca1), (sa2, ca2) = outputs()
+    assert torch.equal(sa1, sa2) and torch.equal(ca1, ca2)
+    for j in range(10):
+        smem.smem_delete_block(dc.h, 0, j)
+        assert dc.mirror.delete(0, j) == 0
+    assert smem.smem_get_free_fifo(dc.h) == fifo0   # no shared slot came free
+    (_, ca1b), (_, ca2b) = outputs()
+    assert torch.equal(ca1b, ca1) and torch.equal(ca2b, ca2)
+    # a decode step of each with identical inputs and identical in-block rows
+    Kb = to_dev(synth.tensor_np(7, synth.KIND_KIN, (5, 4, 64), 0))
+    Vb = to_dev(synth.tensor_np(7, synth.KIND_VIN, (5, 4, 64), 0))
+    q = [to_dev(synth.tensor_np(7, k, (1, 4, 64), 1)) for k in (synth.KIND_QDEC_S, synth.KIND_KNEW,
+                                                               synth.KIND_VNEW, synth.KIND_QDEC_C)]
+    outs = []
+    for s in (1, 2):
+        smem.smem_write_inblock(dc.h, s, 0, 5, Kb, Vb)
+        osa = torch.empty(1, 4, 64, dtype=torch.bfloat16, device="cuda")
+        oca = torch.empty_like(osa)
+        smem.smem_decode(dc.h, 0, [s], [5], [10], *q, osa, oca)
+        outs.append((osa, oca))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+    smem.smem_release_seq(dc.h, 1)
+    assert dc.mirror.release(1) == 0
+    assert smem.smem_get_free_fifo(dc.h) == dc.mirror.free_list()
+    assert len(dc.mirror.free_list()) == len(fifo0) + 10
