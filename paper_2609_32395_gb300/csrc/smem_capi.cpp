@@ -66,7 +66,7 @@ int make_layout(const smem_config* c, Layout* L) {
   if (c->n_layers > 4096 || c->n_heads > 1024 || c->max_seqs > (1 << 20) || c->max_blocks_per_seq > (1 << 22) ||
       c->capacity_slots > (1 << 26))
     return SMEM_ERR_INVALID_ARG;
-  if (c->head_dim != 64 && c->head_dim != 128) return SMEM_ERR_UNSUPPORTED;
+  if (c->head_dim != 32 && c->head_dim != 64 && c->head_dim != 128) return SMEM_ERR_UNSUPPORTED;
   if (c->block_tokens != smem::kBlockTok || c->rows_per_block != smem::kRows) return SMEM_ERR_UNSUPPORTED;
   if (c->has_null_row != 0 && c->has_null_row != 1) return SMEM_ERR_INVALID_ARG;
   if (c->recompute_kv != 0 && c->recompute_kv != 1) return SMEM_ERR_INVALID_ARG;

@@ -43,16 +43,19 @@ constexpr int kUnitQueue = 8;  // fetched-but-unconsumed units of a warp (<= NS 
 template <int D>
 struct Dec {
   static constexpr int R = kRows;
-  static constexpr int SROWS = D == 64 ? 32 : 16;  // rows per stage
+  static constexpr int SROWS = D == 32 ? 64 : (D == 64 ? 32 : 16);  // rows per stage
   static constexpr int CHUNKS = R / SROWS;         // stages per memory block
   static constexpr int HALF = SROWS * D * 2;       // K (or V) bytes of a stage
   static constexpr int STAGE = 2 * HALF;           // 8 KB
-  static constexpr int BOXES = D / 64;             // 128-byte-wide TMA boxes per row
-  static constexpr int BOX_BYTES = SROWS * 128;
+  static constexpr int BOXES = D < 64 ? 1 : D / 64;  // TMA boxes per row (64 or 128 bytes wide)
+  static constexpr int ROWB = D < 64 ? D * 2 : 128;  // bytes of a row within a box
+  static constexpr int BOX_BYTES = SROWS * ROWB;
+  static constexpr int QW = D < 64 ? D : 64;       // query columns a lane holds
+  static constexpr int RPL = D == 32 ? 2 : 1;      // K rows a lane scores per stage
   static constexpr int NW = 8;                     // worker warps per CTA
   static constexpr int NS = 3;                     // stages per warp
   static constexpr int THREADS = NW * 32;
-  static constexpr int LPR = D / 64;               // lanes per row in the score phase
+  static constexpr int LPR = D < 64 ? 1 : D / 64;  // lanes per row in the score phase
   static constexpr int OFF_BAR = NW * NS * STAGE;
   static constexpr int OFF_P = OFF_BAR + NW * NS * 8;
   static constexpr int OFF_Q = OFF_P + NW * 64 * 4;            // per stage: the unit's query
@@ -60,6 +63,14 @@ struct Dec {
   static constexpr int OFF_END = OFF_UQ + NW * kUnitQueue * 4;
   static constexpr int SMEM = OFF_END + 1024;      // + slack to align the base to 1 KB
 };
+
+// Byte offset of 16-byte chunk c of row r in a stage half: 128-byte swizzle
+// over boxes of 64 columns, or the 64-byte swizzle of 32-column rows.
+template <int D>
+__device__ __forceinline__ int chunk_off(int r, int c) {
+  if constexpr (D == 32) return r * 64 + ((c ^ ((r >> 1) & 3)) << 4);
+  else return (c >> 3) * Dec<D>::BOX_BYTES + r * 128 + (((c & 7) ^ (r & 7)) << 4);
+}
 
 struct Unit {
   int sa;     // 1: self-attention unit
@@ -214,15 +225,16 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
   const size_t qoff = ((size_t)U.item * p.H + U.h) * D;           // outputs
   const size_t soff = (size_t)U.item * p.s_stride + (size_t)U.h * D;  // qs, k_new, v_new
   const uint16_t* ib = p.inblock + (((size_t)it.seq * p.L + p.layer) * p.H + U.h) * (size_t)2 * kBlockTok * D;
-  const int hh = lane % LPR;  // which 64 columns of the row
+  constexpr int QW = Dec<D>::QW;  // columns of a row per lane
+  const int hh = lane % LPR;  // which QW columns of the row
   // with rotary phases the new token's query and key turn by its offset p
-  const float2* rp = ROPE ? p.rope_tab + (size_t)it.pos * (D / 2) + hh * 32 : nullptr;
+  const float2* rp = ROPE ? p.rope_tab + (size_t)it.pos * (D / 2) + hh * (QW / 2) : nullptr;
   if (p.mode & 1) {
-    float q[64];
+    float q[QW];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < QW / 8; ++j) {
       float t[8];
-      unpack8(ld_nc16(p.qs + soff + hh * 64 + j * 8), t);
+      unpack8(ld_nc16(p.qs + soff + hh * QW + j * 8), t);
       if (ROPE) rot8f(t, rp + j * 4);
 #pragma unroll
       for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
@@ -237,9 +249,9 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
       if (r < n) {
         const uint16_t* row = r == it.pos ? p.k_new + soff : ib + (size_t)r * D;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < QW / 8; ++j) {
           float t[8];
-          unpack8(ld_nc16(row + hh * 64 + j * 8), t);
+          unpack8(ld_nc16(row + hh * QW + j * 8), t);
           if (ROPE && r == it.pos) rot8f(t, rp + j * 4);  // stored rows are already turned
 #pragma unroll
           for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
@@ -338,13 +350,22 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
     if (ROPE) {
       // the null row's key phase is max(0, i - W): the query turns by min(i, W)
       const int qb = p.items[pd.item].qblk;
-      const float2* cs = p.rope_tab + (size_t)min(qb, p.rope_w) * (D / 2) + lane * (CPT / 2);
+      const float2* tab = p.rope_tab + (size_t)min(qb, p.rope_w) * (D / 2);
+      if constexpr (CPT == 1) {
+        // one column per lane: the pair (2m, 2m+1) spans lanes 2m and 2m+1
+        const float xe = __shfl_sync(0xffffffffu, qv[0], lane & ~1);
+        const float xo = __shfl_sync(0xffffffffu, qv[0], lane | 1);
+        const float2 c = tab[lane >> 1];
+        qv[0] = (lane & 1) ? xe * c.y + xo * c.x : xe * c.x - xo * c.y;
+      } else {
+        const float2* cs = tab + lane * (CPT / 2);
 #pragma unroll
-      for (int e = 0; e < CPT; e += 2) {
-        const float2 c = cs[e / 2];
-        const float x0 = qv[e], x1 = qv[e + 1];
-        qv[e] = x0 * c.x - x1 * c.y;
-        qv[e + 1] = x0 * c.y + x1 * c.x;
+        for (int e = 0; e < CPT; e += 2) {
+          const float2 c = cs[e / 2];
+          const float x0 = qv[e], x1 = qv[e + 1];
+          qv[e] = x0 * c.x - x1 * c.y;
+          qv[e + 1] = x0 * c.y + x1 * c.x;
+        }
       }
     }
     float dot = 0.f;
@@ -399,9 +420,14 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
     }
   }
   const float inv = 1.f / Lsum;
-  uint32_t* o32 = reinterpret_cast<uint32_t*>(p.oca + qoff) + lane * (CPT / 2);
+  if constexpr (CPT == 1) {
+    const __nv_bfloat16 b = __float2bfloat16_rn(A[0] * inv);
+    p.oca[qoff + lane] = *reinterpret_cast<const uint16_t*>(&b);
+  } else {
+    uint32_t* o32 = reinterpret_cast<uint32_t*>(p.oca + qoff) + lane * (CPT / 2);
 #pragma unroll
-  for (int e = 0; e < CPT; e += 2) o32[e / 2] = pack_bf16x2(A[e] * inv, A[e + 1] * inv);
+    for (int e = 0; e < CPT; e += 2) o32[e / 2] = pack_bf16x2(A[e] * inv, A[e + 1] * inv);
+  }
   if (lane == 0) p.counters[pd.item * p.H + pd.h] = 0u;
 }
 
@@ -487,7 +513,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     const Unit U = unit_of(p, u);
     const DecodeItem& it = p.items[U.item];
     const size_t qoff = ((size_t)U.item * p.H + U.h) * D;
-    float q[64];
+    float q[C::QW];
     float m = -INFINITY, l = 0.f, acc[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] = 0.f;
@@ -514,12 +540,12 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
         break;
       }
       if (ch == 0) {
-        const uint16_t* qs = qarea + s * D + hh * 64;
+        const uint16_t* qs = qarea + s * D + hh * C::QW;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < C::QW / 8; ++j) {
           float t[8];
           unpack8(*reinterpret_cast<const uint4*>(qs + j * 8), t);
-          if (ROPE) rot8f(t, p.rope_tab + (size_t)p.rope_w * (D / 2) + hh * 32 + j * 4);
+          if (ROPE) rot8f(t, p.rope_tab + (size_t)p.rope_w * (D / 2) + hh * (C::QW / 2) + j * 4);
 #pragma unroll
           for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
         }
@@ -535,54 +561,83 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       }
       const uint8_t* kb = ring + s * C::STAGE;
       const uint8_t* vb = kb + C::HALF;
-      // scores: lane-per-row (two lanes per row at d_h = 128)
-      float dot0 = 0.f, dot1 = 0.f;
-      const uint8_t* krow = kb + hh * C::BOX_BYTES + rr * 128;
-      if (ROPE && dk > 0) {
-        const float2* cs = p.rope_tab + (size_t)dk * (D / 2) + hh * 32;
+      if constexpr (D == 32) {
+        // scores: two rows per lane (rows lane and lane + 32), 64-byte rows
+        float sc2[2];
 #pragma unroll
-        for (int j = 0; j < 8; j += 2) {
-          float t0[8], t1[8];
-          unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
-          unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
-          rot8f(t0, cs + j * 4);
-          rot8f(t1, cs + j * 4 + 4);
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const int r = lane + 32 * h2;
+          float dot = 0.f;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
-            dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
+          for (int j = 0; j < 4; ++j) {
+            float t[8];
+            unpack8(*reinterpret_cast<const uint4*>(kb + chunk_off<D>(r, j)), t);
+            if (ROPE && dk > 0) rot8f(t, p.rope_tab + (size_t)dk * (D / 2) + j * 4);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
           }
+          sc2[h2] = dot;
         }
+        float mx = fmaxf(sc2[0], sc2[1]);
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        const float m_new = fmaxf(m, mx);
+        const float alpha = exp2f(m - m_new);
+        const float p0 = exp2f(sc2[0] - m_new), p1 = exp2f(sc2[1] - m_new);
+        l = l * alpha + p0 + p1;
+        pbuf[lane] = p0;
+        pbuf[lane + 32] = p1;
+        m = m_new;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] *= alpha;
       } else {
-#pragma unroll
-        for (int j = 0; j < 8; j += 2) {
-          float t0[8], t1[8];
-          unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
-          unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
-            dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
+        // scores: lane-per-row (two lanes per row at d_h = 128)
+        float dot0 = 0.f, dot1 = 0.f;
+        const uint8_t* krow = kb + hh * C::BOX_BYTES + rr * 128;
+        if (ROPE && dk > 0) {
+          const float2* cs = p.rope_tab + (size_t)dk * (D / 2) + hh * 32;
+  #pragma unroll
+          for (int j = 0; j < 8; j += 2) {
+            float t0[8], t1[8];
+            unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
+            unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
+            rot8f(t0, cs + j * 4);
+            rot8f(t1, cs + j * 4 + 4);
+  #pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
+              dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
+            }
+          }
+        } else {
+  #pragma unroll
+          for (int j = 0; j < 8; j += 2) {
+            float t0[8], t1[8];
+            unpack8(*reinterpret_cast<const uint4*>(krow + ((j ^ (rr & 7)) << 4)), t0);
+            unpack8(*reinterpret_cast<const uint4*>(krow + (((j + 1) ^ (rr & 7)) << 4)), t1);
+  #pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              dot0 = fmaf(q[j * 8 + e], t0[e], dot0);
+              dot1 = fmaf(q[j * 8 + 8 + e], t1[e], dot1);
+            }
           }
         }
+        float sc = dot0 + dot1;
+        if (C::LPR == 2) sc += __shfl_xor_sync(0xffffffffu, sc, 1);
+        float mx = sc;
+  #pragma unroll
+        for (int o = C::LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        const float m_new = fmaxf(m, mx);
+        const float alpha = exp2f(m - m_new);
+        const float pr = exp2f(sc - m_new);
+        l = l * alpha + (hh == 0 ? pr : 0.f);
+        if (hh == 0) pbuf[rr] = pr;
+        m = m_new;
+  #pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] *= alpha;
       }
-      float sc = dot0 + dot1;
-      if (C::LPR == 2) sc += __shfl_xor_sync(0xffffffffu, sc, 1);
-      float mx = sc;
-#pragma unroll
-      for (int o = C::LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      const float m_new = fmaxf(m, mx);
-      const float alpha = exp2f(m - m_new);
-      const float pr = exp2f(sc - m_new);
-      l = l * alpha + (hh == 0 ? pr : 0.f);
-      if (hh == 0) pbuf[rr] = pr;
-      m = m_new;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] *= alpha;
       __syncwarp();
       // P.V: lane (g, c), rows g*RG .. g*RG+RG-1, columns c*8 .. c*8+7
-      const uint8_t* vcol = vb + (c >> 3) * C::BOX_BYTES;
-      const int cc = c & 7;
       const float4 p0 = *reinterpret_cast<const float4*>(pbuf + g * RG);
       const float4 p1 = *reinterpret_cast<const float4*>(pbuf + g * RG + 4);
       const float pv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
@@ -590,7 +645,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       for (int i = 0; i < RG; ++i) {
         const int r = g * RG + i;
         float t[8];
-        unpack8(*reinterpret_cast<const uint4*>(vcol + r * 128 + ((cc ^ (r & 7)) << 4)), t);
+        unpack8(*reinterpret_cast<const uint4*>(vb + chunk_off<D>(r, c)), t);
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc[e] = fmaf(pv[i], t[e], acc[e]);
       }
@@ -679,7 +734,7 @@ int static_scratch_address(void** out) {
   return 0;
 }
 
-int decode_stage_rows(int D) { return D == 64 ? Dec<64>::SROWS : Dec<128>::SROWS; }
+int decode_stage_rows(int D) { return D == 32 ? Dec<32>::SROWS : D == 64 ? Dec<64>::SROWS : Dec<128>::SROWS; }
 
 int encode_pool_map(CUtensorMap* map, void* pool, int L, int H, int D, int capacity, int rows_per_box) {
   static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
@@ -693,10 +748,12 @@ int encode_pool_map(CUtensorMap* map, void* pool, int L, int H, int D, int capac
   }
   const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)L * H * 2 * kRows, (cuuint64_t)capacity};
   const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)D * 2 * L * H * 2 * kRows};
-  const cuuint32_t box[3] = {64, (cuuint32_t)rows_per_box, 1};
+  // rows of 64 columns (128 bytes, 128-byte swizzle) or of 32 (64 bytes, 64-byte swizzle)
+  const cuuint32_t box[3] = {(cuuint32_t)(D < 64 ? D : 64), (cuuint32_t)rows_per_box, 1};
   const cuuint32_t estr[3] = {1, 1, 1};
   const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, pool, dims, strides, box, estr,
-                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_INTERLEAVE_NONE,
+                            D < 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? 0 : (int)r;
 }
@@ -719,6 +776,7 @@ static cudaError_t launch_decode_d(const DecodeParams& p, int grid, cudaStream_t
 
 cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st) {
   const bool rope = p.rope_tab != nullptr;
+  if (D == 32) return rope ? launch_decode_d<32, true>(p, grid, st) : launch_decode_d<32, false>(p, grid, st);
   if (D == 64) return rope ? launch_decode_d<64, true>(p, grid, st) : launch_decode_d<64, false>(p, grid, st);
   if (D == 128) return rope ? launch_decode_d<128, true>(p, grid, st) : launch_decode_d<128, false>(p, grid, st);
   return cudaErrorInvalidValue;

@@ -49,7 +49,7 @@ SMEM_HD inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 // two blocks per split.
 constexpr int kPrefillMaxSplits = 16;
 SMEM_HD inline int prefill_split_blocks(int nblk, int H, int D) {
-  const int target = D == 64 ? 304 : 152;
+  const int target = D <= 64 ? 304 : 152;
   int ns = target / H;
   if (ns > kPrefillMaxSplits) ns = kPrefillMaxSplits;
   if (ns > (nblk + 1) / 2) ns = (nblk + 1) / 2;

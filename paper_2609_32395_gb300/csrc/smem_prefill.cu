@@ -39,11 +39,11 @@ template <int D>
 struct Pf {
   static constexpr int R = kRows;
   static constexpr int B = kBlockTok;
-  static constexpr int BOXES = D / 64;            // 128-byte-wide column boxes
-  static constexpr int BOX = 64 * 128;            // one [64 rows][128 B] box
+  static constexpr int BOXES = D < 64 ? 1 : D / 64;  // column boxes (128 bytes wide; one of 64 bytes at d_h = 32)
+  static constexpr int BOX = 64 * (D < 64 ? D * 2 : 128);  // one [64 rows][box width] box
   static constexpr int TILE = BOXES * BOX;        // K or V of one block and head
   static constexpr int STAGE = 2 * TILE;
-  static constexpr int NS = D == 64 ? 5 : 4;      // ring stages (2 CTAs per SM fit at d_h = 64)
+  static constexpr int NS = D == 32 ? 8 : (D == 64 ? 5 : 4);  // ring stages (2 CTAs per SM fit at d_h <= 64)
   static constexpr int PBYTES = 64 * 64 * 2;      // P tile [64 queries][64 keys] bf16
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_RING = TILE;
@@ -54,7 +54,7 @@ struct Pf {
   static constexpr int OFF_MISC = OFF_BAR + NBARS * 8;
   static constexpr int SMEM = OFF_MISC + 64 + 1024;
   static constexpr int THREADS = 192;             // 4 softmax warps, producer, MMA
-  static constexpr int MIN_CTAS = D == 64 ? 2 : 1; // resident CTAs per SM (smem and TMEM allow it)
+  static constexpr int MIN_CTAS = D <= 64 ? 2 : 1; // resident CTAs per SM (smem and TMEM allow it)
   static constexpr uint32_t TMEM_COLS = 256;      // S0 | S1 | O
   static constexpr uint32_t COL_O = 128;
   static constexpr uint32_t ID_QK = tc::idesc_bf16(64, 64, 0, 0);
@@ -62,6 +62,49 @@ struct Pf {
   static constexpr int PART_BYTES = B * (D + 4) * 4;          // one split's partial rows
   static constexpr int MERGE_SPR = NS * STAGE / PART_BYTES;   // split partials staged per round
 };
+
+// Shared-memory descriptors of the K-major Q/K tiles (k-th step of 16
+// columns) and of the MN-major V tile (k-th step of 16 rows).
+template <int D>
+__device__ __forceinline__ uint64_t qk_desc(uint32_t base, int k) {
+  if constexpr (D == 32) return tc::sdesc_sw64(base + k * 32, 16, 512);
+  else return tc::sdesc_sw128(base + (k >> 2) * Pf<D>::BOX + (k & 3) * 32, 16, 1024);
+}
+template <int D>
+__device__ __forceinline__ uint64_t v_desc(uint32_t base, int k) {
+  if constexpr (D == 32) return tc::sdesc_sw64(base + k * 1024, Pf<D>::BOX, 512);
+  else return tc::sdesc_sw128(base + k * 2048, Pf<D>::BOX, 1024);
+}
+
+// O columns of a softmax thread (its half of the row), read or written in TMEM.
+template <int D>
+__device__ __forceinline__ void ld_o(uint32_t trow, uint32_t (&o)[D / 2]) {
+  if constexpr (D == 32) {
+    tc::ld_16x32bx2_x16<16>(trow, o);
+  } else {
+#pragma unroll
+    for (int cb = 0; cb < D / 64; ++cb) {
+      uint32_t t[32];
+      tc::ld_16x32bx2_x32<D / 2>(trow + 32 * cb, t);
+#pragma unroll
+      for (int c = 0; c < 32; ++c) o[cb * 32 + c] = t[c];
+    }
+  }
+}
+template <int D>
+__device__ __forceinline__ void st_o(uint32_t trow, const uint32_t (&o)[D / 2]) {
+  if constexpr (D == 32) {
+    tc::st_16x32bx2_x16<16>(trow, o);
+  } else {
+#pragma unroll
+    for (int cb = 0; cb < D / 64; ++cb) {
+      uint32_t t[32];
+#pragma unroll
+      for (int c = 0; c < 32; ++c) t[c] = o[cb * 32 + c];
+      tc::st_16x32bx2_x32<D / 2>(trow + 32 * cb, t);
+    }
+  }
+}
 
 constexpr float kRescaleLog2 = 8.0f;  // raise the running max when it grows by more than 2^8
 
@@ -106,7 +149,8 @@ __device__ void rotate_tile(uint8_t* tile, const float2* cs_row, int lane) {
   constexpr int CH = D / 8;  // 16-byte chunks per row
   for (int i = lane; i < 64 * CH; i += 32) {
     const int r = i / CH, c = i % CH;
-    uint8_t* ptr = tile + (c >> 3) * (64 * 128) + r * 128 + ((((c & 7) ^ (r & 7))) << 4);
+    uint8_t* ptr = D == 32 ? tile + r * 64 + ((c ^ ((r >> 1) & 3)) << 4)
+                           : tile + (c >> 3) * (64 * 128) + r * 128 + ((((c & 7) ^ (r & 7))) << 4);
     float t[8];
     unpack8(*reinterpret_cast<const uint4*>(ptr), t);
     rot8(t, cs_row + c * 4);
@@ -351,11 +395,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           if (lane == 0) {
             const uint32_t ka = smem_u32(ring + st * C::STAGE);
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k) {
-              const uint32_t off = (k >> 2) * C::BOX + (k & 3) * 32;
-              tc::mma_bf16(tmem + 64 * sb, tc::sdesc_sw128(qa + off, 16, 1024), tc::sdesc_sw128(ka + off, 16, 1024),
-                           C::ID_QK, k > 0);
-            }
+            for (int k = 0; k < D / 16; ++k)
+              tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k), qk_desc<D>(ka, k), C::ID_QK, k > 0);
             tc::commit(&s_full[sb]);
           }
           __syncwarp();
@@ -370,8 +411,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
             const uint32_t va = smem_u32(ring + st * C::STAGE + C::TILE);
 #pragma unroll
             for (int k = 0; k < 4; ++k)
-              tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024),
-                           tc::sdesc_sw128(va + k * 2048, C::BOX, 1024), C::ID_PV, (j > 0 || k > 0));
+              tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024), v_desc<D>(va, k), C::ID_PV,
+                           (j > 0 || k > 0));
             tc::commit(&empty[st]);
             tc::commit(&o_done[pb]);
           }
@@ -403,11 +444,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           tc::fence_after();
           const uint32_t ka = smem_u32(ring + st * C::STAGE);
 #pragma unroll
-          for (int k = 0; k < D / 16; ++k) {
-            const uint32_t off = (k >> 2) * C::BOX + (k & 3) * 32;
-            tc::mma_bf16(tmem + 64 * sb, tc::sdesc_sw128(qa + off, 16, 1024), tc::sdesc_sw128(ka + off, 16, 1024),
-                         C::ID_QK, k > 0);
-          }
+          for (int k = 0; k < D / 16; ++k)
+            tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k), qk_desc<D>(ka, k), C::ID_QK, k > 0);
           tc::commit(&s_full[sb]);
         }
         if (jj >= 1) {  // O += P . V for tile jj-1
@@ -419,8 +457,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           const uint32_t va = smem_u32(ring + st * C::STAGE + C::TILE);
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024),
-                         tc::sdesc_sw128(va + k * 2048, C::BOX, 1024), C::ID_PV, (j > 0 || k > 0));
+            tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024), v_desc<D>(va, k), C::ID_PV,
+                         (j > 0 || k > 0));
           tc::commit(&empty[st]);
           tc::commit(&o_done[pb]);
         }
@@ -468,14 +506,13 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         if (!ok) break;
         tc::fence_after();
         const float alpha = need ? exp2f(m_used - m_new) : 1.f;
-#pragma unroll
-        for (int cb = 0; cb < D / 64; ++cb) {
-          uint32_t o[32];
-          tc::ld_16x32bx2_x32<D / 2>(trow + C::COL_O + 32 * cb, o);
+        {
+          uint32_t o[D / 2];
+          ld_o<D>(trow + C::COL_O, o);
           tc::wait_ld();
 #pragma unroll
-          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
-          tc::st_16x32bx2_x32<D / 2>(trow + C::COL_O + 32 * cb, o);
+          for (int c = 0; c < D / 2; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+          st_o<D>(trow + C::COL_O, o);
         }
         tc::wait_st();
       }
@@ -517,13 +554,12 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
     float o[D / 2];
     if (ok && work) {
       tc::fence_after();
-#pragma unroll
-      for (int cb = 0; cb < D / 64; ++cb) {
-        uint32_t t[32];
-        tc::ld_16x32bx2_x32<D / 2>(trow + C::COL_O + 32 * cb, t);
+      {
+        uint32_t t[D / 2];
+        ld_o<D>(trow + C::COL_O, t);
         tc::wait_ld();
 #pragma unroll
-        for (int c = 0; c < 32; ++c) o[cb * 32 + c] = __uint_as_float(t[c]);
+        for (int c = 0; c < D / 2; ++c) o[c] = __uint_as_float(t[c]);
       }
     }
     const float lrow = l + __shfl_xor_sync(0xffffffffu, l, 16);
@@ -666,10 +702,12 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   }
   tc::fence_before();
   __syncthreads();
-  if (CL && p.n_splits > 0) {
-    tc::cluster_sync();  // every split's partial rows are parked
-    cluster_merge<D, ROPE>(p, h, crank, cs, smem_u32(ring), warp, lane);
-    tc::cluster_sync();  // no CTA leaves while others read its shared memory
+  if constexpr (CL) {
+    if (p.n_splits > 0) {
+      tc::cluster_sync();  // every split's partial rows are parked
+      cluster_merge<D, ROPE>(p, h, crank, cs, smem_u32(ring), warp, lane);
+      tc::cluster_sync();  // no CTA leaves while others read its shared memory
+    }
   }
   if (warp == 4) {
     tc::fence_after();
@@ -769,10 +807,11 @@ static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D, int tok_s
   }
   const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)kBlockTok};
   const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)tok_stride * 2};
-  const cuuint32_t box[3] = {64, 1, (cuuint32_t)kBlockTok};
+  const cuuint32_t box[3] = {(cuuint32_t)(D < 64 ? D : 64), 1, (cuuint32_t)kBlockTok};
   const cuuint32_t estr[3] = {1, 1, 1};
   const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
-                            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                            D < 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? 0 : (int)r;
 }
@@ -821,6 +860,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   const bool rope = a.rope_tab != nullptr;
   if (a.D == 64 && a.cluster && P.n_splits > 0)
     return rope ? launch_prefill_cluster<true>(P, st) : launch_prefill_cluster<false>(P, st);
+  if (a.D == 32) return rope ? launch_prefill_d<32, true>(P, grid, st) : launch_prefill_d<32, false>(P, grid, st);
   if (a.D == 64) return rope ? launch_prefill_d<64, true>(P, grid, st) : launch_prefill_d<64, false>(P, grid, st);
   if (a.D == 128) return rope ? launch_prefill_d<128, true>(P, grid, st) : launch_prefill_d<128, false>(P, grid, st);
   return cudaErrorInvalidValue;

@@ -7,7 +7,7 @@
 //   N >> 3 (bits 17-22), M >> 4 (bits 24-28);
 //   shared memory descriptor: start >> 4 (bits 0-13), leading byte offset
 //   >> 4 (16-29), stride byte offset >> 4 (32-45), version 1 (46-47),
-//   layout 128-byte swizzle (bits 61-63 = 2).
+//   layout 128-byte swizzle (bits 61-63 = 2; 4 for the 64-byte swizzle).
 // With M = 64 the accumulator row r lives in TMEM lane 32*(r/16) + r%16;
 // the 16x32bx2 load gives thread t < 16 lane t, columns [c, c+n) and thread
 // t >= 16 lane t-16, columns [c+off, c+off+n).
@@ -29,6 +29,17 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, ui
   d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
   d |= (uint64_t)1 << 46;
   d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// The same for the 64-byte swizzle (rows of 64 bytes, 8-row atoms of 512 B).
+__device__ __forceinline__ uint64_t sdesc_sw64(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFF);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)4 << 61;
   return d;
 }
 
@@ -120,6 +131,16 @@ __device__ __forceinline__ void ld_16x32bx2_x16(uint32_t taddr, uint32_t (&r)[16
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
         "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
       : "r"(taddr), "n"(OFF)
+      : "memory");
+}
+
+template <int OFF>
+__device__ __forceinline__ void st_16x32bx2_x16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x32bx2.x16.b32 [%0], %17, {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "n"(OFF)
       : "memory");
 }
 

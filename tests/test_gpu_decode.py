@@ -45,7 +45,7 @@ def test_tiny_config_decode_and_delete_reappend():
     assert smem.smem_check_device_error(dc.h) == smem.OK
 
 
-@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("D", [32, 64, 128])
 @pytest.mark.parametrize("has_null", [False, True])
 def test_ragged_batch(D, has_null):
     """Ragged contexts spanning one to many splits with a ragged last split,

@@ -80,7 +80,7 @@ def _np(t):
     return t.detach().cpu().numpy().astype(np.float64)
 
 
-@pytest.mark.parametrize("D,H,has_null", [(64, 4, True), (64, 4, False), (128, 2, True)])
+@pytest.mark.parametrize("D,H,has_null", [(64, 4, True), (64, 4, False), (128, 2, True), (32, 8, True)])
 def test_layer_prefill_matches_oracle(D, H, has_null):
     """Two chained layers, 8 memory blocks appended out of order into a
     shuffled pool; blocks 8 (all readable), 3 and 0 (null row only)."""

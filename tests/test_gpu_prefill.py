@@ -47,7 +47,7 @@ def test_tiny_config_prefill_and_delete_reappend(cluster_mode):
     assert smem.smem_check_device_error(dc.h) == smem.OK
 
 
-@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("D", [32, 64, 128])
 @pytest.mark.parametrize("has_null", [False, True])
 def test_ragged_contexts(D, has_null, cluster_mode):
     """Contexts from empty to many splits with a ragged last split, and a
@@ -79,7 +79,7 @@ def test_160m_shape_one_layer(nblk, cluster_mode):
     assert smem.smem_check_device_error(dc.h) == smem.OK
 
 
-@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("D", [32, 64, 128])
 def test_path_independence_bitwise(D):
     outs = []
     target = list(range(0, 40, 2)) + [41, 45]

@@ -23,7 +23,7 @@ from tests.test_gpu_layer import LayerCache, _decode_setup, _np, x_rows
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("D,H,has_null", [(64, 4, True), (64, 4, False), (128, 2, True)])
+@pytest.mark.parametrize("D,H,has_null", [(64, 4, True), (64, 4, False), (128, 2, True), (32, 8, True)])
 def test_recompute_layer_prefill_matches_oracle(D, H, has_null):
     model = LayerModel(2, H * D, seed=601 + D)
     lc = LayerCache(model, H, D, max_seqs=1, max_blocks=16, capacity=24, has_null=has_null,
