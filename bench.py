@@ -48,6 +48,7 @@ def parse_args():
     ap.add_argument("--no-layer", action="store_true", help="skip the full-reader-layer cells")
     ap.add_argument("--no-recompute", action="store_true", help="skip the recompute-K/V cells")
     ap.add_argument("--no-rope", action="store_true", help="skip the rotary-phase (RoPE composite) cells")
+    ap.add_argument("--no-d32", action="store_true", help="skip the d_h = 32 decode cell")
     ap.add_argument("--workload", default="decode", choices=["decode", "long"],
                     help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
     ap.add_argument("--long-batches", default="1,16", help="batches of the long-context cells")
@@ -190,7 +191,7 @@ def rank_seed(seed: int, rank: int) -> int:
 class DecodeWorkload:
     """Device state of the 410M-shaped batched-decode workload."""
 
-    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None, rope_window=0):
+    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None, rope_window=0, heads=None):
         import torch
 
         import synth
@@ -198,6 +199,8 @@ class DecodeWorkload:
 
         W = WORKLOAD
         self.L, self.H, self.D = (layers or W["L"]), W["H"], W["D"]
+        if heads is not None:  # same width d = H * d_h, other head count
+            self.H, self.D = heads, W["H"] * W["D"] // heads
         self.S = seqs
         self.seed = rank_seed(seed, rank)
         self.device = device
@@ -398,15 +401,19 @@ def measure_layer_decode(wl, steps, warmup, device):
 ROPE_WINDOW = 15  # the paper's saturating window (trained range of 16 blocks)
 
 
-def measure_rope_decode(steps, warmup, device, seqs, layers=None):
-    """The headline decode workload on a cache with the SMem+RoPE composite's
-    rotary phases (window 15): decode tok/s and the decode kernel's HBM
-    fraction, timed like the headline (CUDA events per launch)."""
+def measure_decode_variant(steps, warmup, device, seqs, layers=None, window=None, heads=None):
+    """The headline decode workload on a cache variant -- the SMem+RoPE
+    composite's rotary phases (window 15 by default; 0: none) and/or another
+    head count at the same width (heads=32: d_h = 32): decode tok/s and the
+    decode kernel's HBM fraction, timed like the headline (CUDA events per
+    launch)."""
     import torch
 
     from paper_2609_32395_gb300 import smem
 
-    wl = DecodeWorkload(seqs, warmup + steps + 2, WORKLOAD["seed"], device, layers=layers, rope_window=ROPE_WINDOW)
+    win = ROPE_WINDOW if window is None else window
+    wl = DecodeWorkload(seqs, warmup + steps + 2, WORKLOAD["seed"], device, layers=layers, rope_window=win,
+                        heads=heads)
     for _ in range(warmup):
         wl.step()
     torch.cuda.synchronize()
@@ -425,7 +432,7 @@ def measure_rope_decode(steps, warmup, device, seqs, layers=None):
     elapsed = start.elapsed_time(end) / 1e3
     kern_ms = [ev[i][0][l].elapsed_time(ev[i][1][l]) for i in range(steps) for l in range(wl.L)]
     alg = [r * 4 * wl.H * wl.D for r in rows for _ in range(wl.L)]
-    out = {"window": ROPE_WINDOW, "tok_per_s": steps * seqs / elapsed, "steps": steps,
+    out = {"window": win, "heads": wl.H, "head_dim": wl.D, "tok_per_s": steps * seqs / elapsed, "steps": steps,
            "kernel_ms_mean": float(np.mean(kern_ms)),
            "achieved_gbs": sum(alg) / (sum(kern_ms) / 1e3) / 1e9}
     wl.cache.close()
@@ -1099,7 +1106,12 @@ def run_ours(args):
         wl.cache.close()
         wl.cache.buf = None
         torch.cuda.empty_cache()
-        rope = {"decode": measure_rope_decode(min(args.steps, 64), args.warmup, device, args.seqs, layers=args.layers)}
+        rope = {"decode": measure_decode_variant(min(args.steps, 64), args.warmup, device, args.seqs, layers=args.layers)}
+    d32 = None
+    if not args.no_d32 and rank == 0:
+        # the paper's head width: 32 heads of d_h = 32 at the same d = 1024
+        d32 = measure_decode_variant(min(args.steps, 32), args.warmup, device, args.seqs, layers=args.layers, window=0,
+                                  heads=WORKLOAD["H"] * WORKLOAD["D"] // 32)
     if not args.no_serve:
         wl.cache.close()
         wl.cache.buf = None
@@ -1167,6 +1179,10 @@ def run_ours(args):
             layer["serve"] = {"workload": SERVE["name"], "unit": "ms", "cells": layer_serve,
                               "timing": "CUDA graph of the 12 layer calls, L2 flushed before each"}
         line["layer"] = layer
+    if d32:
+        d32["hbm_frac"] = d32["achieved_gbs"] / peak
+        d32["workload"] = WORKLOAD["name"] + " with 32 heads of d_h = 32 (the same d)"
+        line["d32"] = d32
     if rope:
         rope["decode"]["hbm_frac"] = rope["decode"]["achieved_gbs"] / peak
         rope["workload"] = WORKLOAD["name"] + " and " + SERVE["name"] + ", SMem+RoPE composite (window 15)"

@@ -59,7 +59,7 @@
 extern "C" {
 #endif
 
-#define SMEM_ABI_VERSION 5
+#define SMEM_ABI_VERSION 6
 
 enum {
     SMEM_OK = 0,
@@ -115,6 +115,16 @@ typedef struct smem_config {
                                    given UNROTATED; stored in-block keys are
                                    kept turned. Not with recompute_kv.          */
     float rope_base;            /* rotary base (10000 in the paper)           */
+    int32_t n_kv_heads;         /* grouped-query attention (Sec. 3.1: it
+                                   composes with the KV saving): key/value
+                                   heads of the memory rows and the in-block
+                                   rows, H % n_kv_heads == 0; query head h
+                                   reads key/value head h / (H / n_kv_heads).
+                                   Slots, in-block rows, null rows and every
+                                   K/V argument then have n_kv_heads heads
+                                   (and W_qkv is [d][d + 2 n_kv_heads d_h],
+                                   W_kc/W_vc [d][n_kv_heads d_h]). 0: = H.
+                                   Not with recompute_kv.                      */
 } smem_config;
 
 typedef struct smem_cache smem_cache;

@@ -69,19 +69,28 @@ class LayerWeights:
     w_2: np.ndarray
 
 
+def _group(w: LayerWeights, H: int, D: int) -> int:
+    """Query heads per key/value head (grouped-query attention: W_kc has
+    H_kv * D columns and query head h reads key/value head h // G)."""
+    return H // (w.w_kc.shape[1] // D)
+
+
 def memory_kv(mu, w: LayerWeights, H: int, D: int):
     """Per-layer cross-attention K/V of memory rows mu [..][R][d] ->
-    ([..][H][R][D], [..][H][R][D])."""
+    ([..][H][R][D], [..][H][R][D]), key/value heads repeated over their group."""
+    G = _group(w, H, D)
     k = mu @ w.w_kc
     v = mu @ w.w_vc
-    shp = mu.shape[:-1] + (H, D)
-    k = np.moveaxis(k.reshape(shp), -2, -3)
-    v = np.moveaxis(v.reshape(shp), -2, -3)
+    shp = mu.shape[:-1] + (H // G, D)
+    k = np.repeat(np.moveaxis(k.reshape(shp), -2, -3), G, axis=-3)
+    v = np.repeat(np.moveaxis(v.reshape(shp), -2, -3), G, axis=-3)
     return k, v
 
 
 def null_kv(nu, w: LayerWeights, H: int, D: int):
-    return (nu @ w.w_kc).reshape(H, D), (nu @ w.w_vc).reshape(H, D)
+    G = _group(w, H, D)
+    return (np.repeat((nu @ w.w_kc).reshape(H // G, D), G, axis=0),
+            np.repeat((nu @ w.w_vc).reshape(H // G, D), G, axis=0))
 
 
 def _attn_prefill(rope_window):
@@ -103,14 +112,18 @@ def reader_layer_prefill(x, block_idx, mu_blocks, q_idx, w: LayerWeights, H: int
     x: [b][d] residual stream of the query block; block_idx: [n] memory block
     indices (any order); mu_blocks: [n][R][d] their memory rows. rope_window
     W > 0: the SMem+RoPE composite's rotary phases (oracle.rope).
-    Returns (x_out [b][d], k_s [b][H][D], v_s [b][H][D]); k_s unrotated."""
+    Returns (x_out [b][d], k_s [b][H_kv][D], v_s [b][H_kv][D]); k_s unrotated."""
     attn = _attn_prefill(rope_window)
     b, d = x.shape
+    G = _group(w, H, D)
+    kvd = d // G
     h1 = layer_norm(x, w.ln1_g, w.ln1_b)
     qkv = h1 @ w.w_qkv
-    qs, ks, vs = (qkv[:, i * d:(i + 1) * d].reshape(b, H, D) for i in range(3))
+    qs = qkv[:, :d].reshape(b, H, D)
+    ks = qkv[:, d:d + kvd].reshape(b, H // G, D)
+    vs = qkv[:, d + kvd:].reshape(b, H // G, D)
     zero = np.zeros((b, H, D))
-    osa, _ = attn([], None, None, 0, qs, ks, vs, zero)
+    osa, _ = attn([], None, None, 0, qs, np.repeat(ks, G, axis=1), np.repeat(vs, G, axis=1), zero)
     x1 = x + osa.reshape(b, d) @ w.w_os
     h2 = layer_norm(x1, w.ln2_g, w.ln2_b)
     qc = (h2 @ w.w_qc).reshape(b, H, D)
@@ -127,15 +140,19 @@ def reader_layer_prefill(x, block_idx, mu_blocks, q_idx, w: LayerWeights, H: int
 def reader_layer_decode(x, block_idx, mu_blocks, q_idx, p, kin, vin, w: LayerWeights, H: int, D: int, nu=None,
                         rope_window=0):
     """One decode step of one reader layer for one sequence.
-    x: [d]; kin/vin: [p][H][D] in-block rows of earlier tokens (unrotated).
-    Returns (x_out [d], k_new [H][D], v_new [H][D])."""
+    x: [d]; kin/vin: [p][H_kv][D] in-block rows of earlier tokens (unrotated).
+    Returns (x_out [d], k_new [H_kv][D], v_new [H_kv][D])."""
     attn = _attn_decode(rope_window)
     d = x.shape[0]
+    G = _group(w, H, D)
+    kvd = d // G
     h1 = layer_norm(x[None], w.ln1_g, w.ln1_b)[0]
     qkv = h1 @ w.w_qkv
-    qs, kn_, vn_ = (qkv[i * d:(i + 1) * d].reshape(H, D) for i in range(3))
+    qs = qkv[:d].reshape(H, D)
+    kn_, vn_ = qkv[d:d + kvd].reshape(H // G, D), qkv[d + kvd:].reshape(H // G, D)
     zero = np.zeros((H, D))
-    osa, _ = attn([], None, None, 0, p, kin, vin, qs, kn_, vn_, zero)
+    rep = lambda a, ax: np.repeat(a, G, axis=ax) if a is not None and len(a) else a  # noqa: E731
+    osa, _ = attn([], None, None, 0, p, rep(kin, 1), rep(vin, 1), qs, rep(kn_, 0), rep(vn_, 0), zero)
     x1 = x + osa.reshape(d) @ w.w_os
     h2 = layer_norm(x1[None], w.ln2_g, w.ln2_b)[0]
     qc = (h2 @ w.w_qc).reshape(H, D)

@@ -70,6 +70,9 @@ int make_layout(const smem_config* c, Layout* L) {
   if (c->block_tokens != smem::kBlockTok || c->rows_per_block != smem::kRows) return SMEM_ERR_UNSUPPORTED;
   if (c->has_null_row != 0 && c->has_null_row != 1) return SMEM_ERR_INVALID_ARG;
   if (c->recompute_kv != 0 && c->recompute_kv != 1) return SMEM_ERR_INVALID_ARG;
+  const int hkv = c->n_kv_heads ? c->n_kv_heads : c->n_heads;
+  if (hkv < 1 || hkv > c->n_heads || c->n_heads % hkv) return SMEM_ERR_INVALID_ARG;
+  if (hkv != c->n_heads && c->recompute_kv) return SMEM_ERR_UNSUPPORTED;
   if (c->rope_window < 0 || c->rope_window >= smem::kRopePhases) return SMEM_ERR_INVALID_ARG;
   if (c->rope_window > 0 && !(c->rope_base > 1.0f && c->rope_base < 1e30f)) return SMEM_ERR_INVALID_ARG;
   if (c->rope_window > 0 && c->recompute_kv) return SMEM_ERR_UNSUPPORTED;
@@ -86,6 +89,7 @@ int make_layout(const smem_config* c, Layout* L) {
   L->has_null = c->has_null_row;
   L->max_batch = c->max_decode_batch;
   L->recompute = c->recompute_kv;
+  L->Hkv = hkv;
   L->rope_w = c->rope_window;
   L->rope_base = c->rope_base;
   int ms = 1;
@@ -94,15 +98,16 @@ int make_layout(const smem_config* c, Layout* L) {
   L->dec_max_splits = ms;
   L->pf_max_splits = smem::kPrefillMaxSplits;
   const size_t D = (size_t)L->D;
-  L->slot_elems = L->recompute ? (size_t)smem::kRows * L->H * D : (size_t)L->L * L->H * 2 * smem::kRows * D;
+  L->slot_elems = L->recompute ? (size_t)smem::kRows * L->H * D : (size_t)L->L * L->Hkv * 2 * smem::kRows * D;
   size_t off = 0;
   const size_t A = 1024;
   L->off_pool = off;
   off = align_up(off + (size_t)L->capacity * L->slot_elems * 2, A);
   L->off_inblock = off;
-  off = align_up(off + (size_t)L->max_seqs * L->L * L->H * 2 * smem::kBlockTok * D * 2, A);
+  off = align_up(off + (size_t)L->max_seqs * L->L * L->Hkv * 2 * smem::kBlockTok * D * 2, A);
   L->off_null = off;
-  off = align_up(off + (!L->has_null ? 0 : L->recompute ? (size_t)L->H * D * 2 : (size_t)L->L * L->H * 2 * D * 2), A);
+  off = align_up(off + (!L->has_null ? 0 : L->recompute ? (size_t)L->H * D * 2 : (size_t)L->L * L->Hkv * 2 * D * 2),
+                 A);
   L->off_table = off;
   off = align_up(off + (size_t)L->max_seqs * L->max_blocks * 4, A);
   L->off_bidx = off;
@@ -167,7 +172,7 @@ inline int* table_row(smem_cache* c, int seq) {
 inline uint16_t* inblock_layer(smem_cache* c, int seq, int layer) {
   const Layout& L = c->lay;
   return reinterpret_cast<uint16_t*>(c->dev + L.off_inblock) +
-         ((size_t)seq * L.L + layer) * L.H * 2 * smem::kBlockTok * L.D;
+         ((size_t)seq * L.L + layer) * L.Hkv * 2 * smem::kBlockTok * L.D;
 }
 inline int* bidx_row(smem_cache* c, int seq) {
   return reinterpret_cast<int*>(c->dev + c->lay.off_bidx) + (size_t)seq * c->lay.max_blocks;
@@ -288,6 +293,7 @@ int prefill_impl(smem_cache* c, int seq, int layer, int q_block_idx, const void*
   a.slot_elems = (long long)c->lay.slot_elems;
   a.L = c->lay.L;
   a.H = c->lay.H;
+  a.Hkv = c->lay.Hkv;
   a.D = c->lay.D;
   a.layer = layer;
   a.nblk = nblk;
@@ -337,7 +343,7 @@ int check_decode_args(smem_cache* c, int layer, int nb, const int32_t* seq_ids, 
 // qs/k_new/v_new and of qc. Outputs are [nb][H][D].
 int decode_impl(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const int32_t* pos,
                 const int32_t* q_block_idx, const void* qs, const void* k_new, const void* v_new, const void* qc,
-                void* osa, void* oca, int mode, int s_stride, int c_stride, cudaStream_t st) {
+                void* osa, void* oca, int mode, int s_stride, int c_stride, cudaStream_t st, int kv_stride) {
   const Layout& L = c->lay;
   const size_t tok = (size_t)L.H * L.D;  // output elements per item
   static thread_local smem::DecodeParams P;
@@ -354,8 +360,8 @@ int decode_impl(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const 
                                                     ((size_t)L.max_batch * L.H * 4 + 15) / 16 * 16);
     P.err = reinterpret_cast<int*>(c->dev + L.off_err);
     P.qs = static_cast<const uint16_t*>(qs) + (size_t)i0 * s_stride;
-    P.k_new = static_cast<const uint16_t*>(k_new) + (size_t)i0 * s_stride;
-    P.v_new = static_cast<const uint16_t*>(v_new) + (size_t)i0 * s_stride;
+    P.k_new = static_cast<const uint16_t*>(k_new) + (size_t)i0 * kv_stride;
+    P.v_new = static_cast<const uint16_t*>(v_new) + (size_t)i0 * kv_stride;
     P.qc = static_cast<const uint16_t*>(qc) + (size_t)i0 * c_stride;
     P.osa = static_cast<uint16_t*>(osa) + i0 * tok;
     P.oca = static_cast<uint16_t*>(oca) + i0 * tok;
@@ -369,6 +375,8 @@ int decode_impl(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const 
     P.mode = mode;
     P.s_stride = s_stride;
     P.c_stride = c_stride;
+    P.Hkv = L.Hkv;
+    P.kv_stride = kv_stride;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
     P.rope_tab = rope_tab(c);
     P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);
@@ -465,10 +473,10 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
     if (L.recompute) {
       er = smem::encode_mu_pool_map(&c->pool_map_mu, c->dev + L.off_pool, L.H * L.D, L.capacity);
     } else {
-      er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity,
+      er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.Hkv, L.D, L.capacity,
                                  smem::decode_stage_rows(L.D));
       if (er == 0)
-        er = smem::encode_pool_map(&c->pool_map_pf, c->dev + L.off_pool, L.L, L.H, L.D, L.capacity, smem::kRows);
+        er = smem::encode_pool_map(&c->pool_map_pf, c->dev + L.off_pool, L.L, L.Hkv, L.D, L.capacity, smem::kRows);
     }
     if (er != 0) {
       std::snprintf(g_detail, sizeof(g_detail), "tensor map encode failed (%d)", er);
@@ -499,7 +507,7 @@ int smem_set_null_row(smem_cache* c, const void* k_null, const void* v_null, voi
   return check_launch(c,
                       smem::launch_null_write(reinterpret_cast<uint16_t*>(c->dev + c->lay.off_null),
                                               static_cast<const uint16_t*>(k_null),
-                                              static_cast<const uint16_t*>(v_null), c->lay.L, c->lay.H, c->lay.D,
+                                              static_cast<const uint16_t*>(v_null), c->lay.L, c->lay.Hkv, c->lay.D,
                                               as_stream(stream)),
                       "null row");
 }
@@ -528,7 +536,7 @@ int smem_append_block(smem_cache* c, int32_t seq, int32_t block_idx, const void*
     if (injected_failure(c)) return SMEM_ERR_CUDA;
     const int rc = check_launch(c,
                                 smem::launch_append(pool_slot(c, s), static_cast<const uint16_t*>(K),
-                                                    static_cast<const uint16_t*>(V), c->lay.L, c->lay.H, c->lay.D,
+                                                    static_cast<const uint16_t*>(V), c->lay.L, c->lay.Hkv, c->lay.D,
                                                     table_row(c, seq), bidx_row(c, seq), pos, (int)ix.size(), s,
                                                     block_idx, as_stream(stream)),
                                 "append");
@@ -628,7 +636,7 @@ int smem_write_inblock(smem_cache* c, int32_t seq, int32_t layer, int32_t n_rows
   if (injected_failure(c)) return SMEM_ERR_CUDA;
   return check_launch(c,
                       smem::launch_inblock_write(inblock_layer(c, seq, layer), static_cast<const uint16_t*>(K),
-                                                 static_cast<const uint16_t*>(V), n_rows, c->lay.H, c->lay.D,
+                                                 static_cast<const uint16_t*>(V), n_rows, c->lay.Hkv, c->lay.D,
                                                  as_stream(stream), 0, rope_tab(c)),
                       "in-block write");
 }
@@ -652,11 +660,11 @@ int smem_prefill_block(smem_cache* c, int32_t seq, int32_t layer, int32_t q_bloc
     const Layout& L = c->lay;
     uint16_t* qr = reinterpret_cast<uint16_t*>(c->dev + L.off_rope_scr);
     uint16_t* kr = qr + (size_t)smem::kBlockTok * L.H * L.D;
-    const int tok = L.H * L.D;
+    const int tq = L.H * L.D, tk = L.Hkv * L.D;
     if (injected_failure(c)) return SMEM_ERR_CUDA;
-    const int rc = check_launch(c, smem::launch_rope_rows(static_cast<const uint16_t*>(Qs), qr,
-                                                          static_cast<const uint16_t*>(Ks), kr, tok, tok,
-                                                          smem::kBlockTok, L.H, L.D, rope_tab(c), st),
+    const int rc = check_launch(c, smem::launch_rope_rows(static_cast<const uint16_t*>(Qs), qr, tq, tq, L.H,
+                                                          static_cast<const uint16_t*>(Ks), kr, tk, tk, L.Hkv,
+                                                          smem::kBlockTok, L.D, rope_tab(c), st),
                                 "rotary");
     if (rc) return rc;
     return prefill_impl(c, seq, layer, q_block_idx, qr, kr, Vs, Qc, Osa, Oca, 3, 0, 0, st);
@@ -678,7 +686,7 @@ int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids
   DeviceGuard g(c->device);
   const int tok = c->lay.H * c->lay.D;
   return decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, qs, k_new, v_new, qc, osa, oca, 3, tok, tok,
-                     as_stream(stream));
+                     as_stream(stream), c->lay.Hkv * c->lay.D);
 }
 
 int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,
@@ -745,8 +753,8 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     P.part = reinterpret_cast<float*>(sb + 256 + ticket_bytes);
     P.err = reinterpret_cast<int*>(c->dev + L.off_err);
     P.qs = static_cast<const uint16_t*>(qs) + i0 * tok;
-    P.k_new = static_cast<const uint16_t*>(k_new) + i0 * tok;
-    P.v_new = static_cast<const uint16_t*>(v_new) + i0 * tok;
+    P.k_new = static_cast<const uint16_t*>(k_new) + (size_t)i0 * L.Hkv * L.D;
+    P.v_new = static_cast<const uint16_t*>(v_new) + (size_t)i0 * L.Hkv * L.D;
     P.qc = static_cast<const uint16_t*>(qc) + i0 * tok;
     P.osa = static_cast<uint16_t*>(osa) + i0 * tok;
     P.oca = static_cast<uint16_t*>(oca) + i0 * tok;
@@ -759,6 +767,8 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     P.n_items = n;
     P.mode = 3;
     P.s_stride = P.c_stride = L.H * L.D;
+    P.Hkv = L.Hkv;
+    P.kv_stride = L.Hkv * L.D;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
     P.rope_tab = rope_tab(c);
     P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);
@@ -827,9 +837,9 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
     rc = cuda_rc(cudaMemcpyAsync(slot, mu, (size_t)smem::kRows * d * 2, cudaMemcpyDeviceToDevice, st), "append rows");
   for (int l = 0; l < L.L && !rc && !L.recompute; ++l)
     for (int kv = 0; kv < 2 && !rc; ++kv)
-      rc = blas_rc(smem::blas_project_heads(c->blas, smem::kRows, d, L.H, L.D, static_cast<const uint16_t*>(mu),
-                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc),
-                                            slot + ((size_t)l * L.H * 2 + kv) * smem::kRows * L.D,
+      rc = blas_rc(smem::blas_project_heads(c->blas, smem::kRows, d, L.Hkv, L.D, static_cast<const uint16_t*>(mu),
+                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc), L.Hkv * L.D,
+                                            slot + ((size_t)l * L.Hkv * 2 + kv) * smem::kRows * L.D,
                                             (long long)head_stride, g_detail, sizeof(g_detail)));
   if (!rc) rc = cuda_rc(smem::launch_table_insert(table_row(c, seq), bidx_row(c, seq), pos, (int)ix.size(), s,
                                                           block_idx, st), "append rows");
@@ -863,9 +873,9 @@ int smem_set_null_vector(smem_cache* c, const void* nu, const smem_layer_weights
     return cuda_rc(cudaMemcpyAsync(nk, nu, (size_t)d * 2, cudaMemcpyDeviceToDevice, as_stream(stream)), "null vector");
   for (int l = 0; l < L.L && !rc; ++l)
     for (int kv = 0; kv < 2 && !rc; ++kv)
-      rc = blas_rc(smem::blas_project_heads(c->blas, 1, d, L.H, L.D, static_cast<const uint16_t*>(nu),
-                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc),
-                                            nk + ((size_t)l * L.H * 2 + kv) * L.D, (long long)2 * L.D, g_detail,
+      rc = blas_rc(smem::blas_project_heads(c->blas, 1, d, L.Hkv, L.D, static_cast<const uint16_t*>(nu),
+                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc), L.Hkv * L.D,
+                                            nk + ((size_t)l * L.Hkv * 2 + kv) * L.D, (long long)2 * L.D, g_detail,
                                             sizeof(g_detail)));
   return rc;
 }
@@ -883,6 +893,8 @@ struct LayerRun {
   LayerWs o;
   int n, d;
   cudaStream_t st;
+  int kvd() const { return c->lay.Hkv * c->lay.D; }  // key (or value) width of a token
+  int w3() const { return d + 2 * kvd(); }            // q|k|v width of a token
   uint16_t* h() const { return reinterpret_cast<uint16_t*>(ws + o.h); }
   uint16_t* qkv() const { return reinterpret_cast<uint16_t*>(ws + o.qkv); }
   uint16_t* att() const { return reinterpret_cast<uint16_t*>(ws + o.att); }
@@ -899,7 +911,7 @@ struct LayerRun {
   // h1 = LN1(x); qkv = h1 W_qkv
   int qkv_proj() {
     int rc = ln(w->ln1_g, w->ln1_b);
-    return rc ? rc : gemm(3 * d, d, h(), w->w_qkv, qkv(), false, false);
+    return rc ? rc : gemm(w3(), d, h(), w->w_qkv, qkv(), false, false);
   }
   // x += att W_os; h2 = LN2(x); qc = h2 W_qc
   int after_sa() {
@@ -1028,21 +1040,21 @@ int smem_reader_layer_prefill(smem_cache* c, int32_t seq, int32_t layer, int32_t
   if (rc) return rc;
   const Layout& L = c->lay;
   LayerRun r{c, w, x, static_cast<uint8_t*>(ws), layer_ws(L, n), n, L.H * L.D, st};
-  const int d = r.d;
+  const int d = r.d, kvd = r.kvd(), w3 = r.w3();
   rc = r.qkv_proj();
   if (!rc && L.rope_w) {  // self-attention queries and keys turn by their in-block offsets
-    rc = cuda_rc(smem::launch_rope_rows(r.qkv(), r.qkv(), r.qkv() + d, r.qkv() + d, 3 * d, 3 * d, n, L.H, L.D,
-                                        rope_tab(c), st),
+    rc = cuda_rc(smem::launch_rope_rows(r.qkv(), r.qkv(), w3, w3, L.H, r.qkv() + d, r.qkv() + d, w3, w3, L.Hkv, n,
+                                        L.D, rope_tab(c), st),
                  "rotary");
   }
   // the block's self-attention keys/values become its in-block rows (already turned)
   if (!rc)
-    rc = cuda_rc(smem::launch_inblock_write(inblock_layer(c, seq, layer), r.qkv() + d, r.qkv() + 2 * d, n, L.H, L.D,
-                                            st, 3 * d),
+    rc = cuda_rc(smem::launch_inblock_write(inblock_layer(c, seq, layer), r.qkv() + d, r.qkv() + d + kvd, n, L.Hkv,
+                                            L.D, st, w3),
                  "in-block write");
   if (!rc)
-    rc = prefill_impl(c, seq, layer, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + 2 * d, r.qkv(), r.att(), r.att(), 1,
-                      3 * d, 3 * d, st);
+    rc = prefill_impl(c, seq, layer, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + d + kvd, r.qkv(), r.att(), r.att(),
+                      1, w3, w3, st);
   if (!rc) rc = r.after_sa();
   if (!rc) {
     if (L.recompute)
@@ -1069,18 +1081,18 @@ int smem_reader_layer_decode(smem_cache* c, int32_t layer, int32_t nb, const int
   if (rc) return rc;
   const Layout& L = c->lay;
   LayerRun r{c, w, x, static_cast<uint8_t*>(ws), layer_ws(L, nb), nb, L.H * L.D, st};
-  const int d = r.d;
+  const int d = r.d, kvd = r.kvd(), w3 = r.w3();
   rc = r.qkv_proj();
   if (!rc)
-    rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + 2 * d, r.qkv(), r.att(),
-                     r.att(), 1, 3 * d, 3 * d, st);
+    rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + d + kvd, r.qkv(),
+                     r.att(), r.att(), 1, w3, w3, st, w3);
   if (!rc) rc = r.after_sa();
   if (!rc) {
     if (L.recompute)
       rc = mu_cross_attention(r, layer, nb, seq_ids, q_block_idx, false, 0, 0);
     else
       rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qc(), r.qc(), r.qc(), r.qc(), r.att(), r.att(), 2,
-                       d, d, st);
+                       d, d, st, d);
   }
   if (!rc) rc = r.after_ca();
   return rc;

@@ -92,10 +92,13 @@ __device__ __forceinline__ uint4 rotate8(const uint4 v, const float2* cs) {
 // Two row sets (blockIdx.y: 0 -> a, 1 -> b) of [n][H][D] (token stride
 // src16 16-byte chunks) -> dst, token t turned by phase t (tab:
 // [kRopePhases][D/2] float2).
-__global__ void rope_rows_kernel(const uint4* src_a, uint4* dst_a, const uint4* src_b, uint4* dst_b, int src16,
-                                 int dst16, int n, int H, int cpr, const float2* tab) {
+__global__ void rope_rows_kernel(const uint4* src_a, uint4* dst_a, int src16_a, int dst16_a, int H_a,
+                                 const uint4* src_b, uint4* dst_b, int src16_b, int dst16_b, int H_b, int n, int cpr,
+                                 const float2* tab) {
   const uint4* src = blockIdx.y ? src_b : src_a;
   uint4* dst = blockIdx.y ? dst_b : dst_a;
+  const int src16 = blockIdx.y ? src16_b : src16_a, dst16 = blockIdx.y ? dst16_b : dst16_a;
+  const int H = blockIdx.y ? H_b : H_a;
   const int total = n * H * cpr;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
     const int t = i / (H * cpr);
@@ -167,14 +170,16 @@ cudaError_t launch_table_remove(int* table_row, int* bidx_row, int pos, int n_ol
   return cudaGetLastError();
 }
 
-cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, const uint16_t* src_b, uint16_t* dst_b,
-                             int src_tok, int dst_tok, int n, int H, int D, const float2* rope_tab, cudaStream_t st) {
+cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, int src_tok_a, int dst_tok_a, int H_a,
+                             const uint16_t* src_b, uint16_t* dst_b, int src_tok_b, int dst_tok_b, int H_b, int n,
+                             int D, const float2* rope_tab, cudaStream_t st) {
   if (n == 0) return cudaSuccess;
   const int cpr = D / 8;
-  const int total = n * H * cpr;
+  const int total = n * (H_a > H_b ? H_a : H_b) * cpr;
   rope_rows_kernel<<<dim3((total + 255) / 256, 2), 256, 0, st>>>(
-      reinterpret_cast<const uint4*>(src_a), reinterpret_cast<uint4*>(dst_a), reinterpret_cast<const uint4*>(src_b),
-      reinterpret_cast<uint4*>(dst_b), src_tok / 8, dst_tok / 8, n, H, cpr, rope_tab);
+      reinterpret_cast<const uint4*>(src_a), reinterpret_cast<uint4*>(dst_a), src_tok_a / 8, dst_tok_a / 8, H_a,
+      reinterpret_cast<const uint4*>(src_b), reinterpret_cast<uint4*>(dst_b), src_tok_b / 8, dst_tok_b / 8, H_b, n,
+      cpr, rope_tab);
   return cudaGetLastError();
 }
 

@@ -200,7 +200,7 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
     record_error(p.err, kDevErrBounds);
     mbar_arrive(bar);  // the stage keeps stale rows; the error is flagged
   } else {
-    const int y = ((p.layer * p.H + is.h) * 2) * C::R + row0;
+    const int y = ((p.layer * p.Hkv + is.h / (p.H / p.Hkv)) * 2) * C::R + row0;
     mbar_arrive_expect_tx(bar, C::STAGE + qbytes);
 #pragma unroll
     for (int bx = 0; bx < C::BOXES; ++bx) {
@@ -222,9 +222,12 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
   constexpr int RPP = 32 / LPR;  // rows per pass
   const DecodeItem& it = p.items[U.item];
   const int n = it.pos + 1;
-  const size_t qoff = ((size_t)U.item * p.H + U.h) * D;           // outputs
-  const size_t soff = (size_t)U.item * p.s_stride + (size_t)U.h * D;  // qs, k_new, v_new
-  const uint16_t* ib = p.inblock + (((size_t)it.seq * p.L + p.layer) * p.H + U.h) * (size_t)2 * kBlockTok * D;
+  const int grp = p.H / p.Hkv;  // query heads per key/value head (grouped-query attention)
+  const int kvh = U.h / grp;
+  const size_t qoff = ((size_t)U.item * p.H + U.h) * D;               // outputs
+  const size_t soff = (size_t)U.item * p.s_stride + (size_t)U.h * D;   // qs
+  const size_t koff = (size_t)U.item * p.kv_stride + (size_t)kvh * D;  // k_new, v_new
+  const uint16_t* ib = p.inblock + (((size_t)it.seq * p.L + p.layer) * p.Hkv + kvh) * (size_t)2 * kBlockTok * D;
   constexpr int QW = Dec<D>::QW;  // columns of a row per lane
   const int hh = lane % LPR;  // which QW columns of the row
   // with rotary phases the new token's query and key turn by its offset p
@@ -247,7 +250,7 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
       const int r = k * RPP + lane / LPR;
       float dot = 0.f;
       if (r < n) {
-        const uint16_t* row = r == it.pos ? p.k_new + soff : ib + (size_t)r * D;
+        const uint16_t* row = r == it.pos ? p.k_new + koff : ib + (size_t)r * D;
 #pragma unroll
         for (int j = 0; j < QW / 8; ++j) {
           float t[8];
@@ -288,7 +291,7 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
       const int r = g * RG + i;
       if (r < n) {
         const float pr = pbuf[r];
-        const uint16_t* row = r == it.pos ? p.v_new + soff : ib + (size_t)kBlockTok * D + (size_t)r * D;
+        const uint16_t* row = r == it.pos ? p.v_new + koff : ib + (size_t)kBlockTok * D + (size_t)r * D;
         float t[8];
         unpack8(ld_nc16(row + c * 8), t);
 #pragma unroll
@@ -300,11 +303,12 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
 #pragma unroll
       for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
     if (g == 0) store_bf16x8(p.osa + qoff + c * 8, acc, 1.f / l);
-    // the new token's k and v become in-block row p for later steps
-    if (lane < 2 * CPL) {
+    // the new token's k and v become in-block row p for later steps (one
+    // query head of the group writes the shared row)
+    if (U.h % grp == 0 && lane < 2 * CPL) {
       const int kv = lane / CPL, cc = lane % CPL;
       uint16_t* dst = (uint16_t*)ib + (size_t)kv * kBlockTok * D + (size_t)it.pos * D + cc * 8;
-      uint4 w = ld_nc16((kv ? p.v_new : p.k_new) + soff + cc * 8);
+      uint4 w = ld_nc16((kv ? p.v_new : p.k_new) + koff + cc * 8);
       if (ROPE && !kv) {
         float t[8];
         unpack8(w, t);
@@ -320,7 +324,7 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
     float v[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) v[e] = 0.f;
-    if (p.null_kv) unpack8(ld_nc16(p.null_kv + ((size_t)p.layer * p.H + U.h) * 2 * D + D + lane * 8), v);
+    if (p.null_kv) unpack8(ld_nc16(p.null_kv + ((size_t)p.layer * p.Hkv + kvh) * 2 * D + D + lane * 8), v);
     store_bf16x8(p.oca + qoff + lane * 8, v, 1.f);
   }
   __syncwarp();
@@ -343,7 +347,7 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
   float nscore = -INFINITY;
   if (p.null_kv) {
     // null-row score with the same scaled-query dot product as the rows
-    const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + pd.h) * 2 * D;
+    const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.Hkv + pd.h / (p.H / p.Hkv)) * 2 * D;
     float qv[CPT];
 #pragma unroll
     for (int e = 0; e < CPT; ++e) qv[e] = bf16lo(p.qc[qcoff + lane * CPT + e]);
@@ -393,7 +397,7 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
   if (p.null_kv) {
     const float f = exp2f(nscore - M);
     Lsum = f;
-    const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.H + pd.h) * 2 * D + D;
+    const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.Hkv + pd.h / (p.H / p.Hkv)) * 2 * D + D;
 #pragma unroll
     for (int e = 0; e < CPT; ++e) A[e] = f * bf16lo(vn[lane * CPT + e]);
   }

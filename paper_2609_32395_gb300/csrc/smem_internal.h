@@ -23,12 +23,13 @@ constexpr int kBlockTok = 64; // b: query tokens per block
 // ---------------------------------------------------------------------------
 struct Layout {
   int L, H, D, max_seqs, max_blocks, capacity, has_null, max_batch;
+  int Hkv;             // key/value heads of the memory rows and in-block rows (H % Hkv == 0)
   int recompute;       // 1: slots hold memory rows mu [R][d] instead of per-layer K/V
   int rope_w;          // 0: no rotary phases; else the saturating window W of the RoPE composite
   float rope_base;
   int dec_max_splits;  // split-K partial slots per (decode item, head)
   int pf_max_splits;   // split-K partial slots per prefill head
-  size_t slot_elems;   // bf16 elements per pool slot: L*H*2*R*D, or R*d (recompute)
+  size_t slot_elems;   // bf16 elements per pool slot: L*Hkv*2*R*D, or R*d (recompute)
   size_t off_pool, off_inblock, off_null, off_table, off_bidx, off_rope, off_rope_scr, off_dec_part, off_dec_cnt,
       off_pf_part, off_pf_cnt, off_err, total;
 };
@@ -96,7 +97,8 @@ struct DecodeParams {
   int L, H, layer, max_blocks, capacity;
   int n_items, n_pairs;      // items and CA (item, split) pairs in this launch
   int mode;                  // bit 0: in-block self-attention, bit 1: cross-attention
-  int s_stride, c_stride;    // elements between items of qs/k_new/v_new and of qc
+  int s_stride, c_stride;    // elements between items of qs and of qc
+  int Hkv, kv_stride;        // key/value heads; elements between items of k_new/v_new
   float scale_log2;          // log2(e) / sqrt(D)
   const float2* rope_tab;    // [kRopePhases][D/2] (cos, sin), or nullptr: no rotary phases
   const int* bidx;           // [max_seqs][max_blocks] block index of each table entry
@@ -132,10 +134,11 @@ cudaError_t launch_table_remove(int* table_row, int* bidx_row, int pos, int n_ol
 cudaError_t launch_inblock_write(uint16_t* ib_layer_base, const uint16_t* K, const uint16_t* V, int n, int H,
                                  int D, cudaStream_t st, int tok = 0, const float2* rope_tab = nullptr);
 // Rotary phases by in-block offset, for two row sets at once (queries and
-// keys): row t of src (n tokens x H heads x D, token stride src_tok) turned
+// keys): row t of a set (n tokens x H heads x D, token stride src_tok) turned
 // by phase t into dst (token stride dst_tok; dst may equal src).
-cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, const uint16_t* src_b, uint16_t* dst_b,
-                             int src_tok, int dst_tok, int n, int H, int D, const float2* rope_tab, cudaStream_t st);
+cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, int src_tok_a, int dst_tok_a, int H_a,
+                             const uint16_t* src_b, uint16_t* dst_b, int src_tok_b, int dst_tok_b, int H_b, int n,
+                             int D, const float2* rope_tab, cudaStream_t st);
 // Null row: k,v [L][H][D] -> null_kv [L][H][2][D].
 cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
                               cudaStream_t st);
@@ -161,7 +164,7 @@ void blas_destroy(void* blas);
 int blas_bind(void* blas, cudaStream_t st, void* ws, size_t ws_bytes, char* detail, size_t detail_len);
 int blas_gemm(void* blas, int m, int n, int k, const uint16_t* A, const uint16_t* W, void* C, bool c_f32,
               bool accumulate, char* detail, size_t detail_len);
-int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t* X, const uint16_t* W,
+int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t* X, const uint16_t* W, int ldw,
                        uint16_t* out, long long head_stride, char* detail, size_t detail_len);
 int blas_gemm_sb(void* blas, bool ta, bool tb, int m, int n, int k, float alpha, const uint16_t* A, int lda,
                  long long sA, const uint16_t* B, int ldb, long long sB, uint16_t* C, int ldc, long long sC, int batch,
@@ -239,7 +242,8 @@ struct PrefillArgs {
   const int* bidx_row;        // block index of each table entry of this sequence
   int rope_w, q_blk;          // saturating window, the query block's index
   int mode;                   // bit 0: self-attention, bit 1: cross-attention (0: both)
-  int tok_s, tok_c;           // elements between tokens of Qs/Ks/Vs and of Qc (0: H*D)
+  int tok_s, tok_c;           // elements between tokens of Qs and of Qc (0: H*D)
+  int Hkv, tok_kv;            // key/value heads; elements between tokens of Ks/Vs (0: tok_s or Hkv*D)
   float scale_log2;
 };
 cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);

@@ -135,12 +135,13 @@ int blas_gemm(void* blas, int m, int n, int k, const uint16_t* A, const uint16_t
 }
 
 // Per-head projection of rows: for every head h, out + h * head_stride holds
-// [rows][D] = X[rows][d] W[:, h*D : (h+1)*D], bf16 (one batched GEMM).
-int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t* X, const uint16_t* W,
+// [rows][D] = X[rows][d] W[:, h*D : (h+1)*D], bf16 (one batched GEMM); W is
+// [d][ldw] row-major.
+int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t* X, const uint16_t* W, int ldw,
                        uint16_t* out, long long head_stride, char* detail, size_t detail_len) {
   const float one = 1.f, zero = 0.f;
   return blas_status(cublasGemmStridedBatchedEx(handle(blas), CUBLAS_OP_N, CUBLAS_OP_N, D, rows, d, &one, W, CUDA_R_16BF,
-                                                d, (long long)D, X, CUDA_R_16BF, d, 0LL, &zero, out, CUDA_R_16BF, D,
+                                                ldw, (long long)D, X, CUDA_R_16BF, d, 0LL, &zero, out, CUDA_R_16BF, D,
                                                 head_stride, H, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT),
                      "head projection", detail, detail_len);
 }

@@ -120,6 +120,7 @@ struct PrefillParams {
   unsigned* counters;
   int* err;
   int L, H, layer, nblk, split_blks, n_splits, capacity, max_splits;
+  int Hkv;             // key/value heads (H / Hkv query heads share one)
   int mode;            // bit 0: in-block self-attention, bit 1: cross-attention
   int n_sa;            // self-attention CTAs of the cluster-free grid (0 or H)
   int tok_c;           // elements between consecutive tokens of Qc
@@ -200,7 +201,7 @@ __device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint
     const size_t qcoff = (size_t)row * p.tok_c + (size_t)h * D;
     float nscore = -INFINITY;
     if (p.null_kv) {
-      const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
+      const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D;
       float dot = null_dot<ROPE>(p, p.qc_ptr + qcoff, kn, lane * CPL, CPL);
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
@@ -224,7 +225,7 @@ __device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint
     if (p.null_kv) {
       const float f = exp2f(nscore - M);
       Lsum = f;
-      const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D + D;
+      const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D + D;
 #pragma unroll
       for (int e = 0; e < CPL; ++e) A[e] = f * bf16lo(vn[lane * CPL + e]);
     }
@@ -336,8 +337,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           mbar_arrive_expect_tx(&full[st], C::STAGE);
 #pragma unroll
           for (int bx = 0; bx < C::BOXES; ++bx) {
-            tc::tma_load_3d(kd + bx * C::BOX, &p.ks, bx * 64, h, 0, &full[st]);
-            tc::tma_load_3d(vd + bx * C::BOX, &p.vs, bx * 64, h, 0, &full[st]);
+            tc::tma_load_3d(kd + bx * C::BOX, &p.ks, bx * 64, h / (p.H / p.Hkv), 0, &full[st]);
+            tc::tma_load_3d(vd + bx * C::BOX, &p.vs, bx * 64, h / (p.H / p.Hkv), 0, &full[st]);
           }
         } else {
           const int slot = p.table_row[b0 + j];
@@ -346,7 +347,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
             mbar_arrive(&full[st]);
           } else {
             mbar_arrive_expect_tx(&full[st], C::STAGE);
-            const int y = ((p.layer * p.H + h) * 2) * C::R;
+            const int y = ((p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2) * C::R;
 #pragma unroll
             for (int bx = 0; bx < C::BOXES; ++bx) {
               tc::tma_load_3d(kd + bx * C::BOX, &p.pool, bx * 64, y, slot, &full[st]);
@@ -581,7 +582,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
     if (ok && sa && p.nblk == 0 && (p.mode & 2)) {
       // no readable memory block: oca is the null row's value or zero
       uint16_t* out = p.oca + ((size_t)r * p.H + h) * D + col0;
-      const uint16_t* vn = p.null_kv ? p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D + D + col0 : nullptr;
+      const uint16_t* vn =
+          p.null_kv ? p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D + D + col0 : nullptr;
 #pragma unroll
       for (int c = 0; c < D / 2; c += 8)
         *reinterpret_cast<uint4*>(out + c) = vn ? *reinterpret_cast<const uint4*>(vn + c) : make_uint4(0, 0, 0, 0);
@@ -621,7 +623,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         const size_t qcoff = (size_t)r * p.tok_c + (size_t)h * D;
         float nscore = -INFINITY;
         if (p.null_kv) {
-          const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D;
+          const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D;
           float dot = null_dot<ROPE>(p, p.qc_ptr + qcoff, kn, col0, D / 2);
           dot += __shfl_xor_sync(0xffffffffu, dot, 16);
           nscore = dot * p.scale_log2;
@@ -646,7 +648,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         if (p.null_kv) {
           const float f = exp2f(nscore - M);
           Lsum = f;
-          const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.H + h) * 2 * D + D + col0;
+          const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D + D + col0;
 #pragma unroll
           for (int c = 0; c < D / 2; ++c) A[c] = f * bf16lo(vn[c]);
         }
@@ -819,7 +821,9 @@ static int encode_bhd(CUtensorMap* map, const void* ptr, int H, int D, int tok_s
 cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   static thread_local PrefillParams P;
   P.pool = *a.pool_map;
+  const int Hkv = a.Hkv ? a.Hkv : a.H;
   const int tok_s = a.tok_s ? a.tok_s : a.H * a.D;
+  const int tok_kv = a.tok_kv ? a.tok_kv : (a.tok_s ? a.tok_s : Hkv * a.D);
   const int tok_c = a.tok_c ? a.tok_c : a.H * a.D;
   const int mode = a.mode ? a.mode : 3;
   // a half that is not requested keeps a harmless map (its pointer is valid)
@@ -828,9 +832,11 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   const void* vs = (mode & 1) ? a.vs : a.qc;
   const void* qc = (mode & 2) ? a.qc : a.qs;
   const int ts = (mode & 1) ? tok_s : tok_c, tc2 = (mode & 2) ? tok_c : tok_s;
-  if (encode_bhd(&P.qs, qs, a.H, a.D, ts) || encode_bhd(&P.ks, ks, a.H, a.D, ts) ||
-      encode_bhd(&P.vs, vs, a.H, a.D, ts) || encode_bhd(&P.qc, qc, a.H, a.D, tc2))
+  const int tkv = (mode & 1) ? tok_kv : tok_c, hkv = (mode & 1) ? Hkv : a.H;
+  if (encode_bhd(&P.qs, qs, a.H, a.D, ts) || encode_bhd(&P.ks, ks, hkv, a.D, tkv) ||
+      encode_bhd(&P.vs, vs, hkv, a.D, tkv) || encode_bhd(&P.qc, qc, a.H, a.D, tc2))
     return cudaErrorInvalidValue;
+  P.Hkv = Hkv;
   P.mode = mode;
   P.tok_c = tok_c;
   P.table_row = a.table_row;

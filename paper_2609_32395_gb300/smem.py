@@ -57,7 +57,7 @@ class SmemConfig(ctypes.Structure):
         ("max_blocks_per_seq", ctypes.c_int32), ("capacity_slots", ctypes.c_int32),
         ("has_null_row", ctypes.c_int32), ("max_decode_batch", ctypes.c_int32),
         ("free_order", ctypes.POINTER(ctypes.c_int32)), ("recompute_kv", ctypes.c_int32),
-        ("rope_window", ctypes.c_int32), ("rope_base", ctypes.c_float),
+        ("rope_window", ctypes.c_int32), ("rope_base", ctypes.c_float), ("n_kv_heads", ctypes.c_int32),
     ]
 
 
@@ -160,11 +160,11 @@ def _i32arr(a):
 
 def make_config(n_layers, n_heads, head_dim, max_seqs, max_blocks_per_seq, capacity_slots, has_null_row=False,
                 max_decode_batch=None, free_order=None, block_tokens=64, rows_per_block=64,
-                recompute_kv=False, rope_window=0, rope_base=1e4) -> SmemConfig:
+                recompute_kv=False, rope_window=0, rope_base=1e4, n_kv_heads=0) -> SmemConfig:
     cfg = SmemConfig(n_layers, n_heads, head_dim, block_tokens, rows_per_block, max_seqs, max_blocks_per_seq,
                      capacity_slots, int(bool(has_null_row)),
                      max_seqs if max_decode_batch is None else max_decode_batch, None, int(bool(recompute_kv)),
-                     int(rope_window), float(rope_base))
+                     int(rope_window), float(rope_base), int(n_kv_heads))
     if free_order is not None:
         arr, p = _i32arr(free_order)
         cfg._free_order_keep = arr

@@ -231,12 +231,20 @@ def _matrix_scale(fan_in: int) -> np.float32:
     return np.float32(1.0 / np.sqrt(fan_in))
 
 
-def reader_layer_weights_np(seed: int, layer: int, d: int) -> dict:
+def _fan_out(name: str, fo: int, d: int, kvd) -> int:
+    """Columns of a matrix; with grouped key/value heads (kvd = their width)
+    W_qkv is [d][d + 2 kvd] and W_kc, W_vc are [d][kvd]."""
+    if kvd is None:
+        return fo * d
+    return d + 2 * kvd if name == "w_qkv" else (kvd if name in ("w_kc", "w_vc") else fo * d)
+
+
+def reader_layer_weights_np(seed: int, layer: int, d: int, kvd=None) -> dict:
     """One layer's weights: matrices as bf16 bits (uint16 [fan_in][fan_out]),
     LayerNorm parameters as float32 [d]."""
     out = {}
     for i, (name, fi, fo) in enumerate(LAYER_MATRICES):
-        z = tensor_np(seed, KIND_WEIGHT, (fi * d, fo * d), layer, i)
+        z = tensor_np(seed, KIND_WEIGHT, (fi * d, _fan_out(name, fo, d, kvd)), layer, i)
         f = (z.astype(np.uint32) << 16).view(np.float32) * _matrix_scale(fi * d)
         out[name] = _round_f32_bits_to_bf16(f.view(np.uint32).astype(np.int64)).astype(np.uint16)
     for i, name in enumerate(LAYER_NORMS):
@@ -247,14 +255,14 @@ def reader_layer_weights_np(seed: int, layer: int, d: int) -> dict:
     return out
 
 
-def reader_layer_weights_torch(seed: int, layer: int, d: int, device=None) -> dict:
+def reader_layer_weights_torch(seed: int, layer: int, d: int, device=None, kvd=None) -> dict:
     """Same values as :func:`reader_layer_weights_np`, as torch tensors
     (bfloat16 matrices, float32 LayerNorm parameters) on `device`."""
     import torch
 
     out = {}
     for i, (name, fi, fo) in enumerate(LAYER_MATRICES):
-        z = tensor_torch(seed, KIND_WEIGHT, (fi * d, fo * d), layer, i, device=device)
+        z = tensor_torch(seed, KIND_WEIGHT, (fi * d, _fan_out(name, fo, d, kvd)), layer, i, device=device)
         f = z.to(torch.float32) * torch.tensor(float(_matrix_scale(fi * d)), dtype=torch.float32, device=z.device)
         bits = f.view(torch.int32).to(torch.int64) & M32
         r = _round_f32_bits_to_bf16(bits)

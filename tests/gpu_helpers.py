@@ -43,12 +43,15 @@ class DeviceCache:
     """A device cache plus a host record of what each slot holds."""
 
     def __init__(self, L, H, D, max_seqs, max_blocks, capacity, seed=0, free_order=None, has_null=False,
-                 max_batch=None, rope_window=0):
+                 max_batch=None, rope_window=0, n_kv_heads=0):
         self.L, self.H, self.D = L, H, D
+        self.Hkv = n_kv_heads or H          # key/value heads (grouped-query attention)
+        self.G = H // self.Hkv
         self.seed = seed
         self.rope_window = rope_window
         self.cfg = smem.make_config(L, H, D, max_seqs, max_blocks, capacity, has_null_row=has_null,
-                                    max_decode_batch=max_batch, free_order=free_order, rope_window=rope_window)
+                                    max_decode_batch=max_batch, free_order=free_order, rope_window=rope_window,
+                                    n_kv_heads=n_kv_heads)
         self.cache = smem.SmemCache(self.cfg, device="cuda")
         self.h = self.cache.h
         self.mirror = CacheMirror(capacity, max_seqs, max_blocks, free_order=free_order)
@@ -56,13 +59,13 @@ class DeviceCache:
         self.inblock = {}  # (seq, layer) -> (K bits, V bits) [b][H][D], rows written so far
         self.k_null = self.v_null = None
         if has_null:
-            self.k_null = synth.tensor_np(seed, synth.KIND_KNULL, (L, H, D))
-            self.v_null = synth.tensor_np(seed, synth.KIND_VNULL, (L, H, D))
+            self.k_null = synth.tensor_np(seed, synth.KIND_KNULL, (L, self.Hkv, D))
+            self.v_null = synth.tensor_np(seed, synth.KIND_VNULL, (L, self.Hkv, D))
             smem.smem_set_null_row(self.h, to_dev(self.k_null), to_dev(self.v_null))
 
     def block_bits(self, seq, idx, content_seq=None):
         cs = seq if content_seq is None else content_seq
-        return synth.block_rows_np(self.seed, cs, idx, self.L, self.H, R, self.D)
+        return synth.block_rows_np(self.seed, cs, idx, self.L, self.Hkv, R, self.D)
 
     def append(self, seq, idx, content_seq=None):
         K, V = self.block_bits(seq, idx, content_seq)
@@ -78,8 +81,8 @@ class DeviceCache:
         del self.blocks[(seq, idx)]
 
     def write_inblock(self, seq, layer, n, tag=0):
-        Kb = synth.tensor_np(self.seed, synth.KIND_KIN, (B_TOK, self.H, self.D), seq, layer, tag)
-        Vb = synth.tensor_np(self.seed, synth.KIND_VIN, (B_TOK, self.H, self.D), seq, layer, tag)
+        Kb = synth.tensor_np(self.seed, synth.KIND_KIN, (B_TOK, self.Hkv, self.D), seq, layer, tag)
+        Vb = synth.tensor_np(self.seed, synth.KIND_VIN, (B_TOK, self.Hkv, self.D), seq, layer, tag)
         smem.smem_write_inblock(self.h, seq, layer, n, to_dev(Kb[:n]), to_dev(Vb[:n]))
         self.inblock[(seq, layer)] = (Kb.copy(), Vb.copy())
 
@@ -101,18 +104,20 @@ class DeviceCache:
             return idx, None, None
         mk = np.stack([f64(self.blocks[k][0][layer]) for k in keys])
         mv = np.stack([f64(self.blocks[k][1][layer]) for k in keys])
-        return idx, mk, mv
+        # query head h reads key/value head h // G
+        return idx, np.repeat(mk, self.G, axis=1), np.repeat(mv, self.G, axis=1)
 
     def null(self, layer):
         if self.k_null is None:
             return None, None
-        return f64(self.k_null[layer]), f64(self.v_null[layer])
+        return np.repeat(f64(self.k_null[layer]), self.G, axis=0), np.repeat(f64(self.v_null[layer]), self.G, axis=0)
 
     # -------------------------------------------------------------- prefill
     def prefill_inputs(self, layer, tag=0):
-        shape = (B_TOK, self.H, self.D)
-        return [synth.tensor_np(self.seed, k, shape, layer, tag)
-                for k in (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+        shape, kvs = (B_TOK, self.H, self.D), (B_TOK, self.Hkv, self.D)
+        return [synth.tensor_np(self.seed, k, sh, layer, tag)
+                for k, sh in ((synth.KIND_QS, shape), (synth.KIND_KS, kvs), (synth.KIND_VS, kvs),
+                              (synth.KIND_QC, shape))]
 
     def prefill(self, seq, layer, q_idx, tag=0):
         qs, ks, vs, qc = self.prefill_inputs(layer, tag)
@@ -125,17 +130,18 @@ class DeviceCache:
     def oracle_prefill(self, seq, layer, q_idx, qs, ks, vs, qc):
         idx, mk, mv = self.oracle_memory(seq, layer)
         kn0, vn0 = self.null(layer)
+        ks, vs = (np.repeat(f64(a), self.G, axis=1) for a in (ks, vs))
         if self.rope_window:
             from oracle.rope import reader_prefill_rope
-            return reader_prefill_rope(idx, mk, mv, q_idx, f64(qs), f64(ks), f64(vs), f64(qc), kn0, vn0,
+            return reader_prefill_rope(idx, mk, mv, q_idx, f64(qs), ks, vs, f64(qc), kn0, vn0,
                                        window=self.rope_window)
-        return oracle.reader_prefill(idx, mk, mv, q_idx, f64(qs), f64(ks), f64(vs), f64(qc), kn0, vn0)
+        return oracle.reader_prefill(idx, mk, mv, q_idx, f64(qs), ks, vs, f64(qc), kn0, vn0)
 
     # -------------------------------------------------------------- decode
     def decode_inputs(self, nb, layer, step):
-        H, D = self.H, self.D
-        t = [synth.tensor_np(self.seed, k, (nb, H, D), layer, step)
-             for k in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
+        H, D, Hk = self.H, self.D, self.Hkv
+        t = [synth.tensor_np(self.seed, k, (nb, h, D), layer, step)
+             for k, h in ((synth.KIND_QDEC_S, H), (synth.KIND_KNEW, Hk), (synth.KIND_VNEW, Hk), (synth.KIND_QDEC_C, H))]
         return t  # qs, k_new, v_new, qc bits
 
     def decode(self, layer, seqs, pos, qidx, step=0):
@@ -147,8 +153,8 @@ class DeviceCache:
         torch.cuda.synchronize()
         # the step stored the new token's k, v at in-block row pos
         for i, (s, p) in enumerate(zip(seqs, pos)):
-            Kb, Vb = self.inblock.setdefault((s, layer), (np.zeros((B_TOK, self.H, self.D), np.uint16),
-                                                          np.zeros((B_TOK, self.H, self.D), np.uint16)))
+            Kb, Vb = self.inblock.setdefault((s, layer), (np.zeros((B_TOK, self.Hkv, self.D), np.uint16),
+                                                          np.zeros((B_TOK, self.Hkv, self.D), np.uint16)))
             Kb[p] = kn[i]
             Vb[p] = vn[i]
         return (qs, kn, vn, qc), osa, oca
@@ -156,11 +162,12 @@ class DeviceCache:
     def oracle_decode(self, layer, seq, p, qidx, qs, kn, vn, qc):
         idx, mk, mv = self.oracle_memory(seq, layer)
         Kb, Vb = self.inblock[(seq, layer)]
-        kin = f64(Kb[:p]) if p else None
-        vin = f64(Vb[:p]) if p else None
+        kin = np.repeat(f64(Kb[:p]), self.G, axis=1) if p else None
+        vin = np.repeat(f64(Vb[:p]), self.G, axis=1) if p else None
         kn0, vn0 = self.null(layer)
+        kn, vn = (np.repeat(f64(a), self.G, axis=0) for a in (kn, vn))
         if self.rope_window:
             from oracle.rope import reader_decode_rope
-            return reader_decode_rope(idx, mk, mv, qidx, p, kin, vin, f64(qs), f64(kn), f64(vn), f64(qc), kn0, vn0,
+            return reader_decode_rope(idx, mk, mv, qidx, p, kin, vin, f64(qs), kn, vn, f64(qc), kn0, vn0,
                                       window=self.rope_window)
-        return oracle.reader_decode(idx, mk, mv, qidx, p, kin, vin, f64(qs), f64(kn), f64(vn), f64(qc), kn0, vn0)
+        return oracle.reader_decode(idx, mk, mv, qidx, p, kin, vin, f64(qs), kn, vn, f64(qc), kn0, vn0)

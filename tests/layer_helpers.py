@@ -43,9 +43,9 @@ class LayerModel:
     """L reader layers of width d: host fp64 weights for the oracle, device
     tensors and their SmemLayerWeights for the library."""
 
-    def __init__(self, L: int, d: int, seed: int, device="cuda"):
+    def __init__(self, L: int, d: int, seed: int, device="cuda", kvd=None):
         self.L, self.d, self.seed = L, d, seed
-        self.host = [synth.reader_layer_weights_np(seed, l, d) for l in range(L)]
+        self.host = [synth.reader_layer_weights_np(seed, l, d, kvd) for l in range(L)]
         self.oracle = []
         self.dev = []
         self.sw = []

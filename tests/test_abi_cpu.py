@@ -28,7 +28,7 @@ def test_exports_every_declared_symbol():
     for n in names:
         assert hasattr(L, n), n
     assert set(names) == set(smem.EXPORTED)
-    assert smem.smem_abi_version() == 5
+    assert smem.smem_abi_version() == 6
 
 
 def test_required_bytes_validation():

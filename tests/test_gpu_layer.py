@@ -30,11 +30,11 @@ class LayerCache:
     """A device cache filled through the reader-layer entry points."""
 
     def __init__(self, model: LayerModel, H, D, max_seqs, max_blocks, capacity, has_null=True, free_order=None,
-                 max_batch=None, recompute=False, rope_window=0):
+                 max_batch=None, recompute=False, rope_window=0, n_kv_heads=0):
         self.m, self.H, self.D, self.d = model, H, D, H * D
         self.cfg = smem.make_config(model.L, H, D, max_seqs, max_blocks, capacity, has_null_row=has_null,
                                     max_decode_batch=max_batch, free_order=free_order, recompute_kv=recompute,
-                                    rope_window=rope_window)
+                                    rope_window=rope_window, n_kv_heads=n_kv_heads)
         self.cache = smem.SmemCache(self.cfg, device="cuda")
         self.h = self.cache.h
         self.mirror = CacheMirror(capacity, max_seqs, max_blocks, free_order=free_order)

@@ -134,3 +134,33 @@ def test_zero_branches_leave_the_stream_unchanged():
     X = rng.standard_normal((b, d))
     out, _, _ = reader_layer_prefill(X, np.arange(nblk), rng.standard_normal((nblk, b, d)), nblk, w, H, D)
     np.testing.assert_array_equal(out, X)
+
+
+def test_grouped_kv_heads_equal_repeated_full_heads():
+    """Grouped-query attention (H_kv key/value heads, query head h reading
+    head h // G) equals ordinary multi-head attention whose key/value maps
+    repeat each grouped head's columns G times."""
+    rng = np.random.default_rng(47)
+    b, H, D, nblk, G = 8, 4, 8, 3, 2
+    d, kvd = H * D, H * D // G
+    w = rand_weights(rng, d)
+    w.w_qkv = rng.standard_normal((d, d + 2 * kvd)) / np.sqrt(d)
+    w.w_kc = rng.standard_normal((d, kvd)) / np.sqrt(d)
+    w.w_vc = rng.standard_normal((d, kvd)) / np.sqrt(d)
+
+    def expand(m):  # [d][H_kv*D] -> [d][H*D], head h = grouped head h // G
+        return np.repeat(m.reshape(m.shape[0], H // G, D), G, axis=1).reshape(m.shape[0], d)
+
+    full = LayerWeights(**{**w.__dict__})
+    full.w_qkv = np.concatenate([w.w_qkv[:, :d], expand(w.w_qkv[:, d:d + kvd]), expand(w.w_qkv[:, d + kvd:])], axis=1)
+    full.w_kc, full.w_vc = expand(w.w_kc), expand(w.w_vc)
+    X = rng.standard_normal((b, d))
+    mu = rng.standard_normal((nblk, b, d))
+    nu = rng.standard_normal(d)
+    a, ks, vs = reader_layer_prefill(X, np.arange(nblk), mu, nblk, w, H, D, nu)
+    c, ks_full, _ = reader_layer_prefill(X, np.arange(nblk), mu, nblk, full, H, D, nu)
+    np.testing.assert_allclose(a, c, rtol=0, atol=1e-12)
+    assert ks.shape == (b, H // G, D)
+    np.testing.assert_allclose(np.repeat(ks, G, axis=1), ks_full, rtol=0, atol=1e-12)
+    xo, _, _ = reader_layer_decode(X[3], np.arange(nblk), mu, nblk, 3, ks[:3], vs[:3], w, H, D, nu)
+    np.testing.assert_allclose(xo, a[3], rtol=0, atol=1e-12)
