@@ -49,6 +49,7 @@ def parse_args():
     ap.add_argument("--no-recompute", action="store_true", help="skip the recompute-K/V cells")
     ap.add_argument("--no-rope", action="store_true", help="skip the rotary-phase (RoPE composite) cells")
     ap.add_argument("--no-d32", action="store_true", help="skip the d_h = 32 decode cell")
+    ap.add_argument("--no-gqa", action="store_true", help="skip the grouped-query decode cell")
     ap.add_argument("--workload", default="decode", choices=["decode", "long"],
                     help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
     ap.add_argument("--long-batches", default="1,16", help="batches of the long-context cells")
@@ -191,7 +192,7 @@ def rank_seed(seed: int, rank: int) -> int:
 class DecodeWorkload:
     """Device state of the 410M-shaped batched-decode workload."""
 
-    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None, rope_window=0, heads=None):
+    def __init__(self, seqs, steps_total, seed, device, rank=0, layers=None, rope_window=0, heads=None, kv_heads=0):
         import torch
 
         import synth
@@ -201,6 +202,7 @@ class DecodeWorkload:
         self.L, self.H, self.D = (layers or W["L"]), W["H"], W["D"]
         if heads is not None:  # same width d = H * d_h, other head count
             self.H, self.D = heads, W["H"] * W["D"] // heads
+        self.Hkv = kv_heads or self.H  # key/value heads (grouped-query attention)
         self.S = seqs
         self.seed = rank_seed(seed, rank)
         self.device = device
@@ -212,7 +214,7 @@ class DecodeWorkload:
         max_blocks = int(self.nblk.max()) + max(self.n_new) + 1
         perm = synth.slot_permutation(self.seed, capacity)
         self.cfg = smem.make_config(self.L, self.H, self.D, seqs, max_blocks, capacity, free_order=perm,
-                                    rope_window=rope_window)
+                                    rope_window=rope_window, n_kv_heads=kv_heads)
         self.cache = smem.SmemCache(self.cfg, device=device)
         self.h = self.cache.h
         torch.cuda.synchronize()
@@ -222,7 +224,7 @@ class DecodeWorkload:
             n = int(self.nblk[s])
             for b0 in range(0, n, chunk):
                 ids = list(range(b0, min(n, b0 + chunk)))
-                K, V = synth.block_rows_torch(self.seed, s, ids, self.L, self.H, R, self.D, device)
+                K, V = synth.block_rows_torch(self.seed, s, ids, self.L, self.Hkv, R, self.D, device)
                 for i, j in enumerate(ids):
                     smem.smem_append_block(self.h, s, j, K[i], V[i])
                 del K, V
@@ -230,7 +232,7 @@ class DecodeWorkload:
         self.new_K, self.new_V = [], []
         for s in range(seqs):
             ids = [int(self.nblk[s]) + k for k in range(self.n_new[s])]
-            K, V = synth.block_rows_torch(self.seed, s, ids, self.L, self.H, R, self.D, device)
+            K, V = synth.block_rows_torch(self.seed, s, ids, self.L, self.Hkv, R, self.D, device)
             self.new_K.append(K)
             self.new_V.append(V)
         self.new_used = [0] * seqs
@@ -239,9 +241,9 @@ class DecodeWorkload:
             p = int(self.pos[s])
             for layer in range(self.L):
                 if p:
-                    Kb = synth.tensor_torch(self.seed, synth.KIND_KIN, (p, self.H, self.D), s, layer, 0,
+                    Kb = synth.tensor_torch(self.seed, synth.KIND_KIN, (p, self.Hkv, self.D), s, layer, 0,
                                             device=device)
-                    Vb = synth.tensor_torch(self.seed, synth.KIND_VIN, (p, self.H, self.D), s, layer, 0,
+                    Vb = synth.tensor_torch(self.seed, synth.KIND_VIN, (p, self.Hkv, self.D), s, layer, 0,
                                             device=device)
                     smem.smem_write_inblock(self.h, s, layer, p, Kb, Vb)
         # per-layer decode inputs (a few distinct sets, cycled)
@@ -251,9 +253,10 @@ class DecodeWorkload:
         for k in range(self.n_sets):
             per_layer = []
             for layer in range(self.L):
-                per_layer.append([synth.tensor_torch(self.seed, kind, shape, layer, k, device=device)
-                                  for kind in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW,
-                                               synth.KIND_QDEC_C)])
+                kv_shape = (seqs, self.Hkv, self.D)
+                per_layer.append([synth.tensor_torch(self.seed, kind, sh, layer, k, device=device)
+                                  for kind, sh in ((synth.KIND_QDEC_S, shape), (synth.KIND_KNEW, kv_shape),
+                                                   (synth.KIND_VNEW, kv_shape), (synth.KIND_QDEC_C, shape))])
             self.inputs.append(per_layer)
         self.osa = torch.empty(shape, dtype=torch.bfloat16, device=device)
         self.oca = torch.empty(shape, dtype=torch.bfloat16, device=device)
@@ -401,7 +404,7 @@ def measure_layer_decode(wl, steps, warmup, device):
 ROPE_WINDOW = 15  # the paper's saturating window (trained range of 16 blocks)
 
 
-def measure_decode_variant(steps, warmup, device, seqs, layers=None, window=None, heads=None):
+def measure_decode_variant(steps, warmup, device, seqs, layers=None, window=None, heads=None, kv_heads=0):
     """The headline decode workload on a cache variant -- the SMem+RoPE
     composite's rotary phases (window 15 by default; 0: none) and/or another
     head count at the same width (heads=32: d_h = 32): decode tok/s and the
@@ -413,7 +416,7 @@ def measure_decode_variant(steps, warmup, device, seqs, layers=None, window=None
 
     win = ROPE_WINDOW if window is None else window
     wl = DecodeWorkload(seqs, warmup + steps + 2, WORKLOAD["seed"], device, layers=layers, rope_window=win,
-                        heads=heads)
+                        heads=heads, kv_heads=kv_heads)
     for _ in range(warmup):
         wl.step()
     torch.cuda.synchronize()
@@ -431,8 +434,9 @@ def measure_decode_variant(steps, warmup, device, seqs, layers=None, window=None
         raise RuntimeError("device error recorded during the rotary decode")
     elapsed = start.elapsed_time(end) / 1e3
     kern_ms = [ev[i][0][l].elapsed_time(ev[i][1][l]) for i in range(steps) for l in range(wl.L)]
-    alg = [r * 4 * wl.H * wl.D for r in rows for _ in range(wl.L)]
-    out = {"window": win, "heads": wl.H, "head_dim": wl.D, "tok_per_s": steps * seqs / elapsed, "steps": steps,
+    alg = [r * 4 * wl.Hkv * wl.D for r in rows for _ in range(wl.L)]  # each key/value row once
+    out = {"window": win, "heads": wl.H, "kv_heads": wl.Hkv, "head_dim": wl.D, "pool_bytes": int(wl.cache.nbytes),
+           "tok_per_s": steps * seqs / elapsed, "steps": steps,
            "kernel_ms_mean": float(np.mean(kern_ms)),
            "achieved_gbs": sum(alg) / (sum(kern_ms) / 1e3) / 1e9}
     wl.cache.close()
@@ -1107,6 +1111,10 @@ def run_ours(args):
         wl.cache.buf = None
         torch.cuda.empty_cache()
         rope = {"decode": measure_decode_variant(min(args.steps, 64), args.warmup, device, args.seqs, layers=args.layers)}
+    gqa = None
+    if not args.no_gqa and rank == 0:
+        gqa = measure_decode_variant(min(args.steps, 32), args.warmup, device, args.seqs, layers=args.layers, window=0,
+                                     kv_heads=WORKLOAD["H"] // 4)
     d32 = None
     if not args.no_d32 and rank == 0:
         # the paper's head width: 32 heads of d_h = 32 at the same d = 1024
@@ -1179,6 +1187,10 @@ def run_ours(args):
             layer["serve"] = {"workload": SERVE["name"], "unit": "ms", "cells": layer_serve,
                               "timing": "CUDA graph of the 12 layer calls, L2 flushed before each"}
         line["layer"] = layer
+    if gqa:
+        gqa["hbm_frac"] = gqa["achieved_gbs"] / peak
+        gqa["workload"] = WORKLOAD["name"] + " with 4 key/value heads shared by groups of 4 query heads"
+        line["gqa"] = gqa
     if d32:
         d32["hbm_frac"] = d32["achieved_gbs"] / peak
         d32["workload"] = WORKLOAD["name"] + " with 32 heads of d_h = 32 (the same d)"

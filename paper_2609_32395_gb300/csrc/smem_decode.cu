@@ -157,6 +157,7 @@ struct Issue {
   int c;       // next chunk of that unit
   int nc;      // chunks of that unit
   int item, h, b0;
+  int ybase;   // pool-map row of the unit's (layer, key/value head) K tile
   int next_u;  // unit fetched for after this one
   int pushed;  // queue entries pushed
 };
@@ -177,6 +178,7 @@ __device__ __forceinline__ void issue_begin_unit(const DecodeParams& p, Issue& i
     is.item = U.item;
     is.h = U.h;
     is.b0 = U.b0;
+    is.ybase = ((p.layer * p.Hkv + U.h / (p.H / p.Hkv)) * 2) * Dec<D>::R;
     is.next_u = fetch_unit(p);
   } else {
     is.nc = 0;
@@ -200,7 +202,7 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
     record_error(p.err, kDevErrBounds);
     mbar_arrive(bar);  // the stage keeps stale rows; the error is flagged
   } else {
-    const int y = ((p.layer * p.Hkv + is.h / (p.H / p.Hkv)) * 2) * C::R + row0;
+    const int y = is.ybase + row0;
     mbar_arrive_expect_tx(bar, C::STAGE + qbytes);
 #pragma unroll
     for (int bx = 0; bx < C::BOXES; ++bx) {
@@ -645,11 +647,14 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       const float4 p0 = *reinterpret_cast<const float4*>(pbuf + g * RG);
       const float4 p1 = *reinterpret_cast<const float4*>(pbuf + g * RG + 4);
       const float pv[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+      const uint8_t* vcol = vb + (D == 32 ? 0 : (c >> 3) * C::BOX_BYTES);
+      const int cc = D == 32 ? c : (c & 7);
 #pragma unroll
       for (int i = 0; i < RG; ++i) {
         const int r = g * RG + i;
         float t[8];
-        unpack8(*reinterpret_cast<const uint4*>(vb + chunk_off<D>(r, c)), t);
+        const int off = D == 32 ? r * 64 + ((cc ^ ((r >> 1) & 3)) << 4) : r * 128 + ((cc ^ (r & 7)) << 4);
+        unpack8(*reinterpret_cast<const uint4*>(vcol + off), t);
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc[e] = fmaf(pv[i], t[e], acc[e]);
       }
