@@ -40,7 +40,7 @@ namespace smem {
 
 constexpr int kUnitQueue = 8;  // fetched-but-unconsumed units of a warp (<= NS + 1 used)
 
-template <int D>
+template <int D, int QN = 1>
 struct Dec {
   static constexpr int R = kRows;
   static constexpr int SROWS = D == 32 ? 64 : (D == 64 ? 32 : 16);  // rows per stage
@@ -57,9 +57,10 @@ struct Dec {
   static constexpr int THREADS = NW * 32;
   static constexpr int LPR = D < 64 ? 1 : D / 64;  // lanes per row in the score phase
   static constexpr int OFF_BAR = NW * NS * STAGE;
-  static constexpr int OFF_P = OFF_BAR + NW * NS * 8;
-  static constexpr int OFF_Q = OFF_P + NW * 64 * 4;            // per stage: the unit's query
-  static constexpr int OFF_UQ = OFF_Q + NW * NS * D * 2;         // per warp: unit queue
+  static constexpr int OFF_P = OFF_BAR + NW * NS * 8;               // per warp: P of QN queries
+  static constexpr int OFF_Q = OFF_P + NW * QN * 64 * 4;            // per stage: the unit's queries
+  static constexpr int OFF_QB = OFF_Q + NW * NS * QN * D * 2;       // per warp: fp32 queries (QN > 1)
+  static constexpr int OFF_UQ = OFF_QB + (QN > 1 ? NW * QN * D * 4 : 0);  // per warp: unit queue
   static constexpr int OFF_END = OFF_UQ + NW * kUnitQueue * 4;
   static constexpr int SMEM = OFF_END + 1024;      // + slack to align the base to 1 KB
 };
@@ -83,11 +84,12 @@ struct Unit {
 
 __device__ __forceinline__ Unit unit_of(const DecodeParams& p, int u) {
   Unit U;
-  const int nca = p.n_pairs * p.H;
+  const int upp = p.H / p.qn;  // CA units per (item, split): one per group of qn query heads
+  const int nca = p.n_pairs * upp;
   if (u < nca) {
-    const int pair = u / p.H;
+    const int pair = u / upp;
     U.sa = 0;
-    U.h = u - pair * p.H;
+    U.h = (u - pair * upp) * p.qn;  // first query head of the unit
     int lo = 0, hi = p.n_items - 1;  // last item with pair_begin <= pair
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
@@ -164,7 +166,7 @@ struct Issue {
 
 __device__ __forceinline__ int fetch_unit(const DecodeParams& p) {
   const unsigned long long u = atomicAdd(p.sched, 1ull);
-  const int nca = p.n_pairs * p.H;
+  const int nca = p.n_pairs * (p.H / p.qn);
   return u < (unsigned long long)nca ? (int)u : -1;
 }
 
@@ -197,7 +199,7 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
   const int blk = is.b0 + is.c / C::CHUNKS;
   const int row0 = (is.c % C::CHUNKS) * C::SROWS;
   const int slot = p.table[(size_t)p.items[is.item].seq * p.max_blocks + blk];
-  const uint32_t qbytes = is.c == 0 ? D * 2 : 0;
+  const uint32_t qbytes = is.c == 0 ? p.qn * D * 2 : 0;  // the unit's qn query heads (contiguous)
   if (slot < 0 || slot >= p.capacity) {
     record_error(p.err, kDevErrBounds);
     mbar_arrive(bar);  // the stage keeps stale rows; the error is flagged
@@ -458,17 +460,18 @@ __device__ __forceinline__ void announce(const DecodeParams& p, Pending& from, P
   from.valid = 0;
 }
 
-template <int D, bool ROPE>
+template <int D, bool ROPE, int QN>
 __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid_constant__ DecodeParams p) {
-  using C = Dec<D>;
+  using C = Dec<D, QN>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   uint8_t* ring = base + warp * C::NS * C::STAGE;
   uint64_t* full = reinterpret_cast<uint64_t*>(base + C::OFF_BAR) + warp * C::NS;
-  float* pbuf = reinterpret_cast<float*>(base + C::OFF_P) + warp * 64;
-  uint16_t* qarea = reinterpret_cast<uint16_t*>(base + C::OFF_Q) + warp * C::NS * D;
+  float* pbuf = reinterpret_cast<float*>(base + C::OFF_P) + warp * QN * 64;
+  uint16_t* qarea = reinterpret_cast<uint16_t*>(base + C::OFF_Q) + warp * C::NS * QN * D;
+  float* qbuf = reinterpret_cast<float*>(base + C::OFF_QB) + warp * QN * D;  // QN > 1 only
   int* uq = reinterpret_cast<int*>(base + C::OFF_UQ) + warp * kUnitQueue;
 
   if (lane == 0) {
@@ -487,7 +490,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     is.pushed = 0;
     issue_begin_unit<D>(p, is, fetch_unit(p), uq);
     for (int s = 0; s < C::NS; ++s)
-      if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * D, &full[s], uq)) ++issued;
+      if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * QN * D, &full[s], uq)) ++issued;
   }
 
   // self-attention units (static, while the first tiles are in flight)
@@ -518,6 +521,162 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     if (u < 0) break;
     const Unit U = unit_of(p, u);
     const DecodeItem& it = p.items[U.item];
+    if constexpr (QN > 1) {
+      // ---- grouped unit: the p.qn query heads U.h .. U.h+qn-1 read one
+      // key/value head; every chunk is scored against all of them (queries
+      // in shared memory, fp32, pre-scaled), so the rows stream once per group
+      const int ng = p.qn;
+      float gm[QN], gl[QN], gacc[QN][8];
+#pragma unroll
+      for (int j = 0; j < QN; ++j) {
+        gm[j] = -INFINITY;
+        gl[j] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) gacc[j][e] = 0.f;
+      }
+      const int nch = U.nt * C::CHUNKS;
+      for (int ch = 0; ch < nch; ++ch, ++k) {
+        const int s = k % C::NS;
+        const uint32_t par = (k / C::NS) & 1;
+        if (!__all_sync(0xffffffffu, mbar_wait_bounded(&full[s], par, nullptr))) {
+          if (lane == 0) record_error(p.err, kDevErrWaitFull);
+          failed = true;
+          break;
+        }
+        if (ch == 0) {
+          const uint16_t* qs = qarea + s * QN * D;
+          for (int i = lane; i < ng * (D / 8); i += 32) {
+            float t[8];
+            unpack8(*reinterpret_cast<const uint4*>(qs + i * 8), t);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) qbuf[i * 8 + e] = t[e] * p.scale_log2;
+          }
+          __syncwarp();
+        }
+        const uint8_t* kb = ring + s * C::STAGE;
+        const uint8_t* vb = kb + C::HALF;
+        // scores of this lane's row(s) against every query of the group
+        float sc[QN][C::RPL];
+#pragma unroll
+        for (int h2 = 0; h2 < C::RPL; ++h2) {
+          const int r = C::RPL == 2 ? lane + 32 * h2 : rr;
+          float kr[C::QW];
+#pragma unroll
+          for (int j = 0; j < C::QW / 8; ++j)
+            unpack8(*reinterpret_cast<const uint4*>(kb + chunk_off<D>(r, hh * 8 + j)), &kr[j * 8]);
+#pragma unroll
+          for (int j = 0; j < QN; ++j) {
+            float dot = 0.f;
+            if (j < ng) {
+              const float4* qv = reinterpret_cast<const float4*>(qbuf + j * D + hh * C::QW);
+#pragma unroll
+              for (int e4 = 0; e4 < C::QW / 4; ++e4) {
+                const float4 q4 = qv[e4];
+                dot = fmaf(q4.x, kr[4 * e4], dot);
+                dot = fmaf(q4.y, kr[4 * e4 + 1], dot);
+                dot = fmaf(q4.z, kr[4 * e4 + 2], dot);
+                dot = fmaf(q4.w, kr[4 * e4 + 3], dot);
+              }
+            }
+            if (C::LPR == 2) dot += __shfl_xor_sync(0xffffffffu, dot, 1);
+            sc[j][h2] = dot;
+          }
+        }
+        float galpha[QN];
+#pragma unroll
+        for (int j = 0; j < QN; ++j) {
+          float mx = C::RPL == 2 ? fmaxf(sc[j][0], sc[j][C::RPL - 1]) : sc[j][0];
+#pragma unroll
+          for (int o = C::LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+          const float m_new = fmaxf(gm[j], mx);
+          galpha[j] = exp2f(gm[j] - m_new);
+          gm[j] = m_new;
+          if (j < ng) {
+            if (C::RPL == 2) {
+              const float p0 = exp2f(sc[j][0] - m_new), p1 = exp2f(sc[j][C::RPL - 1] - m_new);
+              gl[j] = gl[j] * galpha[j] + p0 + p1;
+              pbuf[j * 64 + lane] = p0;
+              pbuf[j * 64 + lane + 32] = p1;
+            } else {
+              const float pr = exp2f(sc[j][0] - m_new);
+              gl[j] = gl[j] * galpha[j] + (hh == 0 ? pr : 0.f);
+              if (hh == 0) pbuf[j * 64 + rr] = pr;
+            }
+          }
+#pragma unroll
+          for (int e = 0; e < 8; ++e) gacc[j][e] *= galpha[j];
+        }
+        __syncwarp();
+        // P.V: lane (g, c), rows g*RG .. g*RG+RG-1, columns c*8 .. c*8+7, every query
+        float pv[QN][8];
+#pragma unroll
+        for (int j = 0; j < QN; ++j) {
+          const float4 a = *reinterpret_cast<const float4*>(pbuf + j * 64 + g * RG);
+          const float4 b = *reinterpret_cast<const float4*>(pbuf + j * 64 + g * RG + 4);
+          pv[j][0] = a.x; pv[j][1] = a.y; pv[j][2] = a.z; pv[j][3] = a.w;
+          pv[j][4] = b.x; pv[j][5] = b.y; pv[j][6] = b.z; pv[j][7] = b.w;
+        }
+#pragma unroll
+        for (int i = 0; i < RG; ++i) {
+          const int r = g * RG + i;
+          float t[8];
+          unpack8(*reinterpret_cast<const uint4*>(vb + chunk_off<D>(r, c)), t);
+#pragma unroll
+          for (int j = 0; j < QN; ++j)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) gacc[j][e] = fmaf(pv[j][i], t[e], gacc[j][e]);
+        }
+        __syncwarp();
+        if (lane == 0) {
+          fence_proxy_async_smem();
+          if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * QN * D, &full[s], uq)) ++issued;
+        }
+        __syncwarp();
+      }
+      if (failed) break;
+      const int nsplit = ceil_div(it.nblk, decode_split_blocks(it.nblk));
+      unsigned last = 0;  // bit j: this unit completed query j's last split
+#pragma unroll
+      for (int j = 0; j < QN; ++j) {
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) gl[j] += __shfl_xor_sync(0xffffffffu, gl[j], o);
+#pragma unroll
+        for (int o = CPL; o < 32; o <<= 1)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) gacc[j][e] += __shfl_xor_sync(0xffffffffu, gacc[j][e], o);
+        if (j >= ng) continue;
+        if (nsplit == 1 && !p.null_kv) {
+          if (g == 0) store_bf16x8(p.oca + ((size_t)U.item * p.H + U.h + j) * D + c * 8, gacc[j], 1.f / gl[j]);
+          continue;
+        }
+        float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h + j) * (D + 4);
+        if (g == 0) {
+          *reinterpret_cast<float4*>(pp + 4 + c * 8) = make_float4(gacc[j][0], gacc[j][1], gacc[j][2], gacc[j][3]);
+          *reinterpret_cast<float4*>(pp + 8 + c * 8) = make_float4(gacc[j][4], gacc[j][5], gacc[j][6], gacc[j][7]);
+        }
+        if (lane == 0) {
+          pp[0] = gm[j];
+          pp[1] = gl[j];
+        }
+      }
+      if (nsplit == 1 && !p.null_kv) continue;
+      __threadfence();
+      // one ticket per query head, taken by lanes 0 .. ng-1 at once
+      const bool mine = lane < ng && atomicAdd(&p.counters[U.item * p.H + U.h + lane], 1u) == (unsigned)(nsplit - 1);
+      last = __ballot_sync(0xffffffffu, mine);
+      for (int j = 0; j < ng; ++j) {
+        if (!(last >> j & 1u)) continue;
+        __threadfence();
+        Pending pd;
+        pd.valid = 1;
+        pd.item = U.item;
+        pd.h = U.h + j;
+        pd.nsplit = nsplit;
+        pd.pair_begin = it.pair_begin;
+        merge_splits<D, ROPE>(p, pd, lane);
+      }
+      continue;
+    }
     const size_t qoff = ((size_t)U.item * p.H + U.h) * D;
     float q[C::QW];
     float m = -INFINITY, l = 0.f, acc[8];
@@ -546,7 +705,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
         break;
       }
       if (ch == 0) {
-        const uint16_t* qs = qarea + s * D + hh * C::QW;
+        const uint16_t* qs = qarea + s * QN * D + hh * C::QW;
 #pragma unroll
         for (int j = 0; j < C::QW / 8; ++j) {
           float t[8];
@@ -662,7 +821,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       // refill this stage with the chunk NS ahead
       if (lane == 0) {
         fence_proxy_async_smem();
-        if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * D, &full[s], uq)) ++issued;
+        if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * QN * D, &full[s], uq)) ++issued;
       }
       __syncwarp();
     }
@@ -774,20 +933,37 @@ int decode_max_grid(int D, int num_sms) {
 
 int decode_warps_per_cta() { return Dec<64>::NW; }
 
-template <int D, bool ROPE>
+template <int D, bool ROPE, int QN>
 static cudaError_t launch_decode_d(const DecodeParams& p, int grid, cudaStream_t st) {
-  using C = Dec<D>;
-  cudaError_t e = ensure_smem_limit<D + (ROPE ? 1 : 0)>(decode_kernel<D, ROPE>, C::SMEM);
+  using C = Dec<D, QN>;
+  cudaError_t e = ensure_smem_limit<D + (ROPE ? 1 : 0) + 4 * QN>(decode_kernel<D, ROPE, QN>, C::SMEM);
   if (e != cudaSuccess) return e;
-  decode_kernel<D, ROPE><<<grid, C::THREADS, C::SMEM, st>>>(p);
+  decode_kernel<D, ROPE, QN><<<grid, C::THREADS, C::SMEM, st>>>(p);
   return cudaGetLastError();
+}
+
+int decode_group_width(int D, int G, bool rope) {
+  // query heads per grouped unit: the largest of 4 (2 at d_h = 128, whose
+  // rings leave less shared memory) dividing the group; 1 with rotary phases
+  if (rope || G < 2) return 1;
+  const int qmax = D == 128 ? 2 : 4;
+  for (int q = qmax; q >= 2; q >>= 1)
+    if (G % q == 0) return q;
+  return 1;
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st) {
   const bool rope = p.rope_tab != nullptr;
-  if (D == 32) return rope ? launch_decode_d<32, true>(p, grid, st) : launch_decode_d<32, false>(p, grid, st);
-  if (D == 64) return rope ? launch_decode_d<64, true>(p, grid, st) : launch_decode_d<64, false>(p, grid, st);
-  if (D == 128) return rope ? launch_decode_d<128, true>(p, grid, st) : launch_decode_d<128, false>(p, grid, st);
+  if (p.qn > 1) {
+    if (rope) return cudaErrorInvalidValue;
+    if (D == 32) return launch_decode_d<32, false, 4>(p, grid, st);
+    if (D == 64) return launch_decode_d<64, false, 4>(p, grid, st);
+    if (D == 128) return launch_decode_d<128, false, 2>(p, grid, st);
+    return cudaErrorInvalidValue;
+  }
+  if (D == 32) return rope ? launch_decode_d<32, true, 1>(p, grid, st) : launch_decode_d<32, false, 1>(p, grid, st);
+  if (D == 64) return rope ? launch_decode_d<64, true, 1>(p, grid, st) : launch_decode_d<64, false, 1>(p, grid, st);
+  if (D == 128) return rope ? launch_decode_d<128, true, 1>(p, grid, st) : launch_decode_d<128, false, 1>(p, grid, st);
   return cudaErrorInvalidValue;
 }
 

@@ -99,6 +99,7 @@ struct DecodeParams {
   int mode;                  // bit 0: in-block self-attention, bit 1: cross-attention
   int s_stride, c_stride;    // elements between items of qs and of qc
   int Hkv, kv_stride;        // key/value heads; elements between items of k_new/v_new
+  int qn;                    // query heads per cross-attention unit (grouped-query decode; 1: one)
   float scale_log2;          // log2(e) / sqrt(D)
   const float2* rope_tab;    // [kRopePhases][D/2] (cos, sin), or nullptr: no rotary phases
   const int* bidx;           // [max_seqs][max_blocks] block index of each table entry
@@ -107,6 +108,9 @@ struct DecodeParams {
 };
 
 cudaError_t launch_decode(const DecodeParams& p, int D, int grid, cudaStream_t st);
+// Query heads a grouped decode unit scores together for a group of G query
+// heads per key/value head (1: one unit per query head).
+int decode_group_width(int D, int G, bool rope);
 // Device address of the fixed scratch array of smem_decode_static_scratch on
 // the current device (looked up once per device). Returns a cudaError_t.
 int static_scratch_address(void** out);

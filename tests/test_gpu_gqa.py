@@ -41,7 +41,7 @@ def _cache(Hkv, D=64, H=8, rope=0, seed=17, perm_seed=4):
     return dc, nblks
 
 
-@pytest.mark.parametrize("Hkv,D", [(2, 64), (1, 64), (4, 128)])
+@pytest.mark.parametrize("Hkv,D", [(2, 64), (1, 64), (2, 128)])
 def test_gqa_prefill_matches_oracle(Hkv, D, cluster_mode):
     if D != 64 and cluster_mode == "clusters":
         pytest.skip("cluster mode is a d_h = 64 kernel")
@@ -54,9 +54,13 @@ def test_gqa_prefill_matches_oracle(Hkv, D, cluster_mode):
     assert smem.smem_check_device_error(dc.h) == smem.OK
 
 
-@pytest.mark.parametrize("Hkv,rope", [(2, 0), (1, 0), (2, 15)])
-def test_gqa_decode_consecutive_steps(Hkv, rope):
-    dc, nblks = _cache(Hkv, rope=rope)
+@pytest.mark.parametrize("Hkv,rope,D,H", [(2, 0, 64, 8), (1, 0, 64, 8), (2, 15, 64, 8), (2, 0, 128, 4),
+                                          (4, 0, 128, 4), (2, 0, 32, 8), (4, 0, 64, 12)])
+def test_gqa_decode_consecutive_steps(Hkv, rope, D, H):
+    """Groups of 4 (one grouped unit of four queries), 8 (two units), 2 at
+    d_h 128 and 32, 3 (one query per unit), and 1; with and without rotary
+    phases."""
+    dc, nblks = _cache(Hkv, rope=rope, D=D, H=H)
     pos0 = [0, 30, 61, 5]
     for s, p in enumerate(pos0):
         dc.write_inblock(s, 1, p, tag=s)
