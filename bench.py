@@ -527,7 +527,10 @@ def measure_recompute(steps, warmup, device, seqs, layers=None):
     kern_ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
     rows = rw.rows_read()
     alg = rows * 2 * d + 2 * seqs * H * d * 2
-    kernel = {"kernel": "mu_attention_kernel<16> (memory-row cross-attention, tcgen05)", "launches": n_launch,
+    nq, cl, wsl = smem.smem_mu_decode_plan(rw.h)
+    name = (f"mu_slice_kernel<{nq}> (memory-row cross-attention, tcgen05; clusters of {cl} CTAs x {wsl} columns)"
+            if cl else f"mu_attention_kernel<{nq}> (memory-row cross-attention, tcgen05; two-pass)")
+    kernel = {"kernel": name, "launches": n_launch,
               "kernel_ms_mean": kern_ms, "rows_per_launch": rows, "alg_bytes_per_launch": alg,
               "achieved_gbs": alg / (kern_ms / 1e3) / 1e9,
               "materialized_bytes_per_launch": rows * 4 * H * rw.D}

@@ -59,7 +59,7 @@
 extern "C" {
 #endif
 
-#define SMEM_ABI_VERSION 6
+#define SMEM_ABI_VERSION 7
 
 enum {
     SMEM_OK = 0,
@@ -98,7 +98,8 @@ typedef struct smem_config {
                                    for every layer (materialized, Sec. 3.1).
                                    1: a slot holds only the block's memory
                                    rows mu [R][d] (d = H*d_h, shared by all
-                                   layers); the reader-layer calls re-derive
+                                   layers; stored as d/64 contiguous chunks
+                                   of [R][64]); the reader-layer calls re-derive
                                    each layer's keys and values from them
                                    (the recompute regime, App. "Serving").
                                    The pool is then 2L times smaller.          */
@@ -297,8 +298,9 @@ size_t smem_layer_workspace_bytes(const smem_cache *c, int32_t n_rows);
  * w_kc and w_vc are read. The slot receives, for every layer l and head h,
  * K = mu W_kc^l[:, h d_h : (h+1) d_h] and V likewise (bf16), then the table
  * insert follows as in smem_append_block (same validation, errors and
- * FIFO order). On a recompute_kv cache the slot receives mu itself and w
- * is not read (may be NULL). */
+ * FIFO order). On a recompute_kv cache the slot receives mu itself (in
+ * 64-column chunks, each [R][64] contiguous) and w is not read (may be
+ * NULL). */
 int smem_append_block_rows(smem_cache *c, int32_t seq, int32_t block_idx, const void *mu,
                            const smem_layer_weights *w, void *ws, size_t ws_bytes, void *stream,
                            int32_t *slot_out);
@@ -355,6 +357,17 @@ int smem_mu_decode(smem_cache *c, int32_t nb, const int32_t *seq_ids, const int3
                    const void *qp, void *op, void *ws, size_t ws_bytes, void *stream);
 int smem_mu_prefill(smem_cache *c, int32_t seq, int32_t q_block_idx, const void *qp, void *op, void *ws,
                     size_t ws_bytes, void *stream);
+
+/* Decode kernel of a recompute_kv cache's memory-row attention, chosen at
+ * create time from H, d and the device (host state, no CUDA): *nq queries
+ * per CTA; *cluster > 0: the column-slice form, each cluster of *cluster
+ * CTAs streaming one row set once with *slice_cols columns per CTA (taken
+ * only when the environment variable SMEM_MU_CLUSTERS is "1" at create
+ * time); *cluster = 0: the two-pass form (one CTA reads each tile twice,
+ * the second time normally from L2).
+ * Any out pointer may be NULL. SMEM_ERR_UNSUPPORTED without recompute_kv,
+ * SMEM_ERR_NO_DEVICE on a bookkeeping-only cache. */
+int smem_mu_decode_plan(const smem_cache *c, int32_t *nq, int32_t *cluster, int32_t *slice_cols);
 
 /* Introspection for bit-exact bookkeeping checks (host state, no CUDA).
  * smem_get_table: the table of `seq` in ascending block index; up to `cap`

@@ -27,7 +27,7 @@ using smem::Layout;
 struct smem_cache {
   CUtensorMap pool_map{};     // decode kernel's view of the pool (device caches)
   CUtensorMap pool_map_pf{};  // prefill kernel's view (whole 64-row tiles)
-  CUtensorMap pool_map_mu{};  // memory-row view [C][R][d] (recompute caches)
+  CUtensorMap pool_map_mu{};  // memory-row view [C][d/64][R][64] (recompute caches)
   smem_config cfg{};
   Layout lay{};
   uint8_t* dev = nullptr;  // nullptr: bookkeeping-only
@@ -41,6 +41,7 @@ struct smem_cache {
   uint32_t seen_epoch = 0;
   int fail_after = 0;                      // test hook: n-th next launch fails
   int pf_cluster_max = 0;                  // prefill cluster limit on this device (0: no clusters)
+  smem::MuDecodePlan mu_plan{};            // recompute caches: decode kernel and query tile on this device
   void* blas = nullptr;                    // cuBLAS handle of the reader-layer calls (created on first use)
   ~smem_cache() { smem::blas_destroy(blas); }
 };
@@ -219,7 +220,10 @@ LayerWs layer_ws(const Layout& L, int n) {
     w.op = off;
     off = align_up(off + (size_t)n * L.H * d * 2, 256);
     w.part = off;
-    const size_t rows = std::max((size_t)std::min(n, smem::kMaxMuGroups) * nqd,
+    // decode: at most kMaxMuGroups groups per launch, each item ceil(H / nq)
+    // tiles of nq (two-pass) or one tile of H rounded up to 16 (column slices)
+    const size_t per_item = std::max((size_t)smem::ceil_div(L.H, nqd) * nqd, (size_t)(L.H + 15) / 16 * 16);
+    const size_t rows = std::max((size_t)std::min(n, smem::kMaxMuGroups) * per_item,
                                  n >= smem::kBlockTok ? (size_t)smem::kBlockTok * L.H : (size_t)0);
     off = align_up(off + rows * smem::kMuMaxSplits * (d + 4) * 4, 256);
   }
@@ -486,6 +490,14 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
     }
     const char* knob = std::getenv("SMEM_PREFILL_CLUSTERS");
     c->pf_cluster_max = (knob && knob[0] == '0') ? 0 : smem::prefill_cluster_max(L.H, L.D);
+    if (L.recompute) {
+      // the column-slice decode kernel is opt-in (SMEM_MU_CLUSTERS=1): at the
+      // model shapes its per-slice softmax and cluster exchange cost more
+      // than the two-pass kernel's second read of each tile from L2
+      const char* mk = std::getenv("SMEM_MU_CLUSTERS");
+      c->mu_plan = (mk && mk[0] == '1') ? smem::mu_decode_plan(L.H, L.H * L.D)
+                                        : smem::MuDecodePlan{smem::mu_query_tile(L.H, L.H * L.D), 0, 0};
+    }
   }
   *out = c;
   return SMEM_OK;
@@ -835,8 +847,8 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
   uint16_t* slot = pool_slot(c, s);
   const int d = L.H * L.D;
   const size_t head_stride = (size_t)2 * smem::kRows * L.D;
-  if (L.recompute)  // the slot keeps the memory rows themselves
-    rc = cuda_rc(cudaMemcpyAsync(slot, mu, (size_t)smem::kRows * d * 2, cudaMemcpyDeviceToDevice, st), "append rows");
+  if (L.recompute)  // the slot keeps the memory rows themselves, one 64-column chunk after another
+    rc = cuda_rc(smem::launch_mu_tile(slot, static_cast<const uint16_t*>(mu), d, st), "append rows");
   for (int l = 0; l < L.L && !rc && !L.recompute; ++l)
     for (int kv = 0; kv < 2 && !rc; ++kv)
       rc = blas_rc(smem::blas_project_heads(c->blas, smem::kRows, d, L.Hkv, L.D, static_cast<const uint16_t*>(mu),
@@ -971,26 +983,33 @@ int mu_attend(smem_cache* c, uint8_t* ws, const LayerWs& o, bool prefill, int nb
     if (injected_failure(c)) return SMEM_ERR_CUDA;
     rc = cuda_rc(smem::launch_mu_attention(P, nqt, st), "memory-row attention");
   } else {
-    const int nqt = smem::mu_query_tile(H, d);
-    for (int i0 = 0; i0 < nb && !rc; i0 += smem::kMaxMuGroups) {
-      const int n = std::min(nb - i0, smem::kMaxMuGroups);
+    // one group per (item, tile of nq heads); the column-slice kernel when planned
+    const smem::MuDecodePlan& pl = c->mu_plan;
+    const int nqt = pl.nq;
+    const int qtiles = smem::ceil_div(H, nqt);
+    const int per_launch = smem::kMaxMuGroups / qtiles;
+    for (int i0 = 0; i0 < nb && !rc; i0 += per_launch) {
+      const int n = std::min(nb - i0, per_launch);
       P.qptr = qp + (size_t)i0 * H * d;
       P.out = op + (size_t)i0 * H * d;
       P.nrows = H;
       P.n_qg = n;
-      P.n_groups = n;
+      P.n_groups = n * qtiles;
       int u = 0;
       for (int i = 0; i < n; ++i) {
         const std::vector<int32_t>& ix = c->idx[seq_ids[i0 + i]];
         const int nblk = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx[i0 + i]) - ix.begin());
-        const int sb = nblk ? smem::mu_decode_split_blocks(nblk) : 1;
+        const int sb = nblk ? smem::mu_decode_split_blocks(nblk, pl.cl) : 1;
         const int nsplit = nblk ? smem::ceil_div(nblk, sb) : 1;
-        P.groups[i] = {seq_ids[i0 + i], i, 0, nblk, sb, nsplit, u, 0};
-        u += nsplit;
+        for (int q = 0; q < qtiles; ++q) {
+          P.groups[i * qtiles + q] = {seq_ids[i0 + i], i, q * nqt, nblk, sb, nsplit, u, 0};
+          u += nsplit;
+        }
       }
       P.n_units = u;
       if (injected_failure(c)) return SMEM_ERR_CUDA;
-      rc = cuda_rc(smem::launch_mu_attention(P, nqt, st), "memory-row attention");
+      rc = cuda_rc(pl.cl > 0 ? smem::launch_mu_slice(P, pl, st) : smem::launch_mu_attention(P, nqt, st),
+                   "memory-row attention");
     }
   }
   return rc;
@@ -1235,6 +1254,16 @@ const char* smem_strerror(int code) {
     case SMEM_ERR_SCRATCH_LIMIT: return "request exceeds the fixed scratch array";
     default: return "unknown error";
   }
+}
+
+int smem_mu_decode_plan(const smem_cache* c, int32_t* nq, int32_t* cluster, int32_t* slice_cols) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (nq) *nq = c->mu_plan.nq;
+  if (cluster) *cluster = c->mu_plan.cl;
+  if (slice_cols) *slice_cols = c->mu_plan.wsl;
+  return SMEM_OK;
 }
 
 int smem_abi_version(void) { return SMEM_ABI_VERSION; }

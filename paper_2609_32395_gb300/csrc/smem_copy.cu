@@ -206,6 +206,23 @@ cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16
   return cudaGetLastError();
 }
 
+// Memory rows mu [R][d] -> the slot's chunk-tiled form [d/64][R][64]: thread
+// i moves source 16-byte unit i (row r, chunk c, part e), so reads are
+// coalesced and writes go in 128-byte runs.
+__global__ void mu_tile_kernel(uint4* dst, const uint4* src, int nc) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= kRows * nc * 8) return;
+  const int r = i / (nc * 8), c = (i / 8) % nc, e = i % 8;
+  dst[((size_t)c * kRows + r) * 8 + e] = src[i];
+}
+
+cudaError_t launch_mu_tile(uint16_t* slot, const uint16_t* mu, int d, cudaStream_t st) {
+  const int total = kRows * (d / 64) * 8;
+  mu_tile_kernel<<<(total + 255) / 256, 256, 0, st>>>(reinterpret_cast<uint4*>(slot),
+                                                       reinterpret_cast<const uint4*>(mu), d / 64);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st) {
   const long long n16 = (long long)(bytes / 16);
   if (n16 == 0) return cudaSuccess;

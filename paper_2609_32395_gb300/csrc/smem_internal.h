@@ -24,7 +24,7 @@ constexpr int kBlockTok = 64; // b: query tokens per block
 struct Layout {
   int L, H, D, max_seqs, max_blocks, capacity, has_null, max_batch;
   int Hkv;             // key/value heads of the memory rows and in-block rows (H % Hkv == 0)
-  int recompute;       // 1: slots hold memory rows mu [R][d] instead of per-layer K/V
+  int recompute;       // 1: slots hold memory rows mu ([d/64][R][64]) instead of per-layer K/V
   int rope_w;          // 0: no rotary phases; else the saturating window W of the RoPE composite
   float rope_base;
   int dec_max_splits;  // split-K partial slots per (decode item, head)
@@ -147,6 +147,9 @@ cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, int src_tok
 cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
                               cudaStream_t st);
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st);
+// Memory rows of a recompute cache: mu [R][d] (d a multiple of 64) -> slot
+// [d/64][R][64], each 64-column chunk of the block contiguous (8 KB).
+cudaError_t launch_mu_tile(uint16_t* slot, const uint16_t* mu, int d, cudaStream_t st);
 
 // Table insert alone (the slot's rows written by other kernels before it).
 cudaError_t launch_table_insert(int* table_row, int* bidx_row, int pos, int n_old, int slot, int block_idx,
@@ -189,7 +192,7 @@ struct MuGroup {
   int seq, qg, n0, nblk, split_blks, nsplit, unit_begin, pad;
 };
 struct MuParams {
-  CUtensorMap pool;           // memory rows [C][R][d], box 64 x 64 x 1
+  CUtensorMap pool;           // memory rows [C][d/64 chunks][R][64], box 64 x 64 x 1
   CUtensorMap q;              // Q' [n_qg][nrows][d], box 64 x NQ x 1 (set by the launcher)
   const int* table;           // [max_seqs][max_blocks]
   const uint16_t* qptr;       // Q' (bf16, softmax scale log2(e)/sqrt(d_h) folded in)
@@ -199,8 +202,18 @@ struct MuParams {
   int* err;
   int d, nrows, n_qg, max_blocks, capacity, n_groups, n_units;
   int ns, hold, off_ring, off_p, off_bar, off_misc;  // shared-memory plan (set by the launcher)
+  int cl, wsl, off_x;  // column-slice kernel: cluster size, slice width, exchange offset
   MuGroup groups[kMaxMuGroups];
 };
+// Decode plan of a recompute cache: nq queries per CTA (a multiple of 16,
+// covering ceil(H / nq) query tiles per item); cl > 0 selects the
+// column-slice kernel on clusters of cl CTAs of wsl = d / cl columns, cl = 0
+// the two-pass kernel. A function of H, d and the current device only.
+struct MuDecodePlan {
+  int nq, cl, wsl;
+};
+MuDecodePlan mu_decode_plan(int H, int d);
+cudaError_t launch_mu_slice(MuParams& P, const MuDecodePlan& pl, cudaStream_t st);
 // Widest query tile (16, 32 or 64) for nq_total queries per row set at width
 // d whose accumulators fit tensor memory; 0 if none does.
 int mu_query_tile(int nq_total, int d);
@@ -212,10 +225,14 @@ cudaError_t launch_mu_attention(MuParams& P, int nq, cudaStream_t st);
 // Split plans (functions of the block count and the cache geometry only).
 // A split reads at least kMuMinSplitBlocks blocks: its partial (NQ x d fp32)
 // and fixed costs stay small next to the rows it streams.
+// The column-slice kernel streams a tile in a fraction of the time of one
+// CTA, so its splits are longer (kMuSliceMinSplitBlocks).
 constexpr int kMuMinSplitBlocks = 8;
-SMEM_HD inline int mu_decode_split_blocks(int nblk) {
+constexpr int kMuSliceMinSplitBlocks = 32;
+SMEM_HD inline int mu_decode_split_blocks(int nblk, int cl) {
   const int s = (nblk + kMuMaxSplits - 1) / kMuMaxSplits;
-  return s > kMuMinSplitBlocks ? s : kMuMinSplitBlocks;
+  const int lo = cl > 0 ? kMuSliceMinSplitBlocks : kMuMinSplitBlocks;
+  return s > lo ? s : lo;
 }
 SMEM_HD inline int mu_prefill_split_blocks(int nblk, int groups) {
   int ns = (304 + groups - 1) / groups;

@@ -155,7 +155,7 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
           }
           if (good) {
             mbar_arrive_expect_tx(&full[st], kMuBox);
-            tc::tma_load_3d(ring + st * kMuBox, &p.pool, c * 64, 0, slot, &full[st]);
+            tc::tma_load_3d(ring + st * kMuBox, &p.pool, 0, c * kRows, slot, &full[st]);
           } else {
             mbar_arrive(&full[st]);
           }
@@ -448,6 +448,354 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
   }
 }
 
+// Decode form on a cluster of CL CTAs that cut the row width d into column
+// slices of wsl = d / CL: CTA `rank` streams only its slice of every tile
+// (64 rows x wsl), once, and keeps it in shared memory from its score MMA to
+// its P.V MMA (no second pass). The tile's scores are the sum of the CL slice
+// partials; every CTA sends its fp32 partial S^T [64][NQ] to every peer with
+// st.async (completing on the peer's exchange barrier), sums the CL partials
+// in rank order -- the same fp32 sum in every CTA -- and runs the identical
+// softmax, so P, m and l agree bitwise across the cluster and each CTA
+// accumulates its own slice of O'. The exchange is double-buffered by tile
+// parity; a CTA sends tile t+2's partial only after it consumed every
+// peer's tile t+1 partial, which each peer sent only after it finished
+// reading tile t's partials, so a buffer is never overwritten while read.
+template <int NQ>
+__global__ void __launch_bounds__(kMuThreads, 1) mu_slice_kernel(const __grid_constant__ MuParams p) {
+  using C = MuCfg<NQ>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const int CL = p.cl;
+  const int NCS = p.wsl / 64;  // 64-column chunks of a slice (even)
+  const int nslot = p.ns;      // tile slots of the ring
+  const uint32_t rank = tc::cluster_ctarank();
+  const int unit = (int)blockIdx.x / CL;
+  uint8_t* qt = base;
+  uint8_t* ring = base + p.off_ring;
+  uint8_t* pt = base + p.off_p;
+  float* xb = reinterpret_cast<float*>(base + p.off_x);  // [2][CL][64 rows][NQ]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + p.off_bar);
+  uint64_t* q_full = bars;
+  uint64_t* full = bars + 1;
+  uint64_t* empty = full + nslot;
+  uint64_t* s_full = empty + nslot;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* o_done = p_full + 2;
+  uint64_t* x_full = o_done + 2;
+  uint64_t* drain = x_full + 2;
+  uint8_t* misc = base + p.off_misc;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 4);
+  float* red = reinterpret_cast<float*>(misc + 16);  // [2][4][NQ] column maxima per warp
+  float* alpha = red + 2 * 4 * NQ;                   // [2][NQ] rescale factors
+  float* lsum = alpha + 2 * NQ;                      // [4][NQ] column sums per warp
+  float* mfin = lsum + 4 * NQ;                       // [NQ]
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  int lo = 0, hi = p.n_groups - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.groups[mid].unit_begin <= unit) lo = mid;
+    else hi = mid - 1;
+  }
+  const MuGroup& G = p.groups[lo];
+  const int split = unit - G.unit_begin;
+  const int b0 = split * G.split_blks;
+  const int nt = G.nblk > 0 ? min(G.split_blks, G.nblk - b0) : 0;  // the same in every CTA of the cluster
+  const int* trow = p.table + (size_t)G.seq * p.max_blocks;
+  uint32_t ncols = 32;
+  while (ncols < (uint32_t)(NQ * (2 + NCS / 2))) ncols <<= 1;
+  const uint32_t colO = 2 * NQ;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < nslot; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_free[b], 4);
+      mbar_init(&p_full[b], 4);
+      mbar_init(&o_done[b], 1);
+      mbar_init(&x_full[b], 1);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 4 && nt > 0) tc::alloc(tslot, ncols);
+  tc::fence_before();
+  tc::cluster_sync();  // every CTA's barriers exist before any peer signals them
+  tc::fence_after();
+  const uint32_t tmem = nt > 0 ? *tslot : 0u;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0 && nt > 0) {
+      mbar_arrive_expect_tx(q_full, (uint32_t)(NCS * C::PBYTES));
+      for (int c = 0; c < NCS; ++c)
+        tc::tma_load_3d(qt + c * C::PBYTES, &p.q, (int)rank * p.wsl + c * 64, G.n0, G.qg, q_full);
+      bool ok = true;
+      int issued = 0;
+      for (int t = 0; t < nt; ++t) {
+        const int sl = t % nslot;
+        if (t >= nslot && !mbar_wait_bounded(&empty[sl], ((t / nslot) - 1) & 1, abort_flag)) {
+          if (!*abort_flag) record_error(p.err, kDevErrWaitEmpty);
+          *abort_flag = 1;
+          ok = false;
+          break;
+        }
+        const int slot = trow[b0 + t];
+        if (slot >= 0 && slot < p.capacity) {
+          mbar_arrive_expect_tx(&full[sl], (uint32_t)(NCS * kMuBox));
+          for (int c = 0; c < NCS; ++c)
+            tc::tma_load_3d(ring + (sl * NCS + c) * kMuBox, &p.pool, 0, ((int)rank * NCS + c) * kRows, slot,
+                            &full[sl]);
+        } else {
+          record_error(p.err, kDevErrBounds);
+          mbar_arrive(&full[sl]);
+        }
+        ++issued;
+      }
+      if (!ok) {
+        // let every copy already issued land before the CTA can exit
+        mbar_wait_bounded(q_full, 0, nullptr);
+        for (int j = issued > nslot ? issued - nslot : 0; j < issued; ++j)
+          mbar_wait_bounded(&full[j % nslot], (j / nslot) & 1, nullptr);
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------- MMA issuer
+    if (lane == 0 && nt > 0) {
+      bool ok = mbar_wait_bounded(q_full, 0, abort_flag);
+      tc::fence_after();
+      const uint32_t qa = smem_u32(qt);
+      const uint32_t ra = smem_u32(ring);
+      // P.V of tile t: O'^T[wsl][NQ] += slice^T P^T, one M = 128 MMA per column pair
+      auto issue_pv = [&](int t) {
+        const int pb = t & 1;
+        if (ok) ok = mbar_wait_bounded(&p_full[pb], (t >> 1) & 1, abort_flag);
+        if (!ok) return;
+        tc::fence_after();
+        const uint32_t b = smem_u32(pt + pb * C::PBYTES);
+        const uint32_t a0 = ra + (uint32_t)((t % nslot) * NCS * kMuBox);
+        for (int cp = 0; cp < NCS / 2; ++cp) {
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + colO + cp * NQ, tc::sdesc_sw128(a0 + 2 * cp * kMuBox + kk * 2048, kMuBox, 1024),
+                         tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_PV, (t > 0 || kk > 0));
+        }
+        tc::commit(&empty[t % nslot]);
+        tc::commit(&o_done[pb]);
+      };
+      for (int t = 0; t < nt && ok; ++t) {
+        const int sb = t & 1, sl = t % nslot;
+        if (t >= 2) ok = mbar_wait_bounded(&s_free[sb], ((t >> 1) - 1) & 1, abort_flag);
+        if (ok) ok = mbar_wait_bounded(&full[sl], (t / nslot) & 1, abort_flag);
+        if (!ok) break;
+        tc::fence_after();
+        // partial S^T[64][NQ] of this slice: K = wsl
+        const uint32_t a0 = ra + (uint32_t)(sl * NCS * kMuBox);
+        for (int c = 0; c < NCS; ++c) {
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + sb * NQ, tc::sdesc_sw128(a0 + c * kMuBox + kk * 32, 16, 1024),
+                         tc::sdesc_sw128(qa + c * C::PBYTES + kk * 32, 16, 1024), C::ID_S, (c | kk) > 0);
+        }
+        tc::commit(&s_full[sb]);
+        if (t > 0) issue_pv(t - 1);
+      }
+      if (ok) issue_pv(nt - 1);
+      if (!ok) {
+        if (!*abort_flag) record_error(p.err, kDevErrWaitMma);
+        *abort_flag = 1;
+      }
+      tc::commit(drain);
+      mbar_wait_bounded(drain, 0, nullptr);
+    }
+  } else {
+    // ---------------------------------------------------------- softmax warps
+    const int tid = threadIdx.x;            // 0..127: TMEM lane of O'
+    const int r = 16 * warp + (lane & 15);  // row of the tile
+    const int hf = lane >> 4;               // column half of S
+    const int col0 = hf * C::C2;
+    const uint32_t tlane = tmem + ((uint32_t)(32 * warp) << 16);
+    const uint32_t xbytes = (uint32_t)((CL - 1) * 64 * NQ * 4);
+    float m_used[C::C2], lp[C::C2];
+#pragma unroll
+    for (int c = 0; c < C::C2; ++c) {
+      m_used[c] = -INFINITY;
+      lp[c] = 0.f;
+    }
+    bool ok = true;
+    for (int t = 0; t < nt; ++t) {
+      const int sb = t & 1;
+      ok = bar_all(3, 128, mbar_wait_bounded(&s_full[sb], (t >> 1) & 1, abort_flag));
+      if (!ok) break;
+      tc::fence_after();
+      uint32_t sr[C::C2];
+      ld_s<NQ>(tlane + sb * NQ, sr);
+      tc::wait_ld();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);
+      float x[C::C2];
+      if (CL > 1) {
+        if (tid == 0) mbar_arrive_expect_tx(&x_full[sb], xbytes);
+        const uint32_t mine = smem_u32(xb + ((size_t)(sb * CL + (int)rank) * 64 + r) * NQ + col0);
+        const uint32_t xbar = smem_u32(&x_full[sb]);
+        for (int k = 1; k < CL; ++k) {
+          const uint32_t peer = (rank + (uint32_t)k) % (uint32_t)CL;
+          const uint32_t dst = tc::dsmem_addr(mine, peer);
+          const uint32_t pbar = tc::dsmem_addr(xbar, peer);
+#pragma unroll
+          for (int c = 0; c < C::C2; c += 4) tc::st_async_v4(dst + c * 4, sr[c], sr[c + 1], sr[c + 2], sr[c + 3], pbar);
+        }
+        ok = bar_all(3, 128, mbar_wait_bounded(&x_full[sb], (t >> 1) & 1, abort_flag));
+        if (!ok) break;
+        // the CL slice partials summed in rank order (identical in every CTA)
+        const float* xr = xb + ((size_t)(sb * CL) * 64 + r) * NQ + col0;
+#pragma unroll
+        for (int c = 0; c < C::C2; c += 4) {
+          float4 acc = rank == 0 ? make_float4(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1]),
+                                               __uint_as_float(sr[c + 2]), __uint_as_float(sr[c + 3]))
+                                 : *reinterpret_cast<const float4*>(xr + c);
+          for (int k = 1; k < CL; ++k) {
+            const float4 v = k == (int)rank ? make_float4(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1]),
+                                                          __uint_as_float(sr[c + 2]), __uint_as_float(sr[c + 3]))
+                                            : *reinterpret_cast<const float4*>(xr + (size_t)k * 64 * NQ + c);
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+          }
+          x[c] = acc.x;
+          x[c + 1] = acc.y;
+          x[c + 2] = acc.z;
+          x[c + 3] = acc.w;
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < C::C2; ++c) x[c] = __uint_as_float(sr[c]);
+      }
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        float v = x[c];
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+        if ((lane & 15) == 0) red[(sb * 4 + warp) * NQ + col0 + c] = v;
+      }
+      named_bar_sync(1, 128);
+      bool need_mine = false;
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        const int col = col0 + c;
+        float tmax = red[(sb * 4) * NQ + col];
+#pragma unroll
+        for (int w2 = 1; w2 < 4; ++w2) tmax = fmaxf(tmax, red[(sb * 4 + w2) * NQ + col]);
+        float a_c = 1.f;
+        if (tmax > m_used[c] + kMuRescaleLog2) {
+          a_c = exp2f(m_used[c] - tmax);
+          lp[c] *= a_c;
+          m_used[c] = tmax;
+          need_mine = true;
+        }
+        if (warp == 0 && (lane & 15) == 0) alpha[sb * NQ + col] = a_c;
+      }
+      const bool any = !bar_all(2, 128, !need_mine);
+      if (t > 0 && any) {
+        ok = bar_all(3, 128, mbar_wait_bounded(&o_done[(t - 1) & 1], ((t - 1) >> 1) & 1, abort_flag));
+        if (!ok) break;
+        tc::fence_after();
+        for (int cp = 0; cp < NCS / 2; ++cp) {
+#pragma unroll
+          for (int cb = 0; cb < NQ / 16; ++cb) {
+            uint32_t o[16];
+            const uint32_t ta = tlane + colO + cp * NQ + cb * 16;
+            tc::ld_32x32b_x16(ta, o);
+            tc::wait_ld();
+#pragma unroll
+            for (int j = 0; j < 16; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha[sb * NQ + cb * 16 + j]);
+            tc::st_32x32b_x16(ta, o);
+          }
+        }
+        tc::wait_st();
+      }
+      if (t >= 2) {  // P buffer sb was last read by P.V of tile t-2
+        ok = bar_all(3, 128, mbar_wait_bounded(&o_done[sb], ((t - 2) >> 1) & 1, abort_flag));
+        if (!ok) break;
+      }
+      uint8_t* pb = pt + sb * C::PBYTES;
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        const int col = col0 + c;
+        const float pr = exp2f(x[c] - m_used[c]);
+        lp[c] += pr;
+        store_bf16(reinterpret_cast<uint16_t*>(pb + col * 128 + ((((r >> 3) ^ (col & 7)) & 7) << 4) + (r & 7) * 2),
+                   pr);
+      }
+      fence_proxy_async_smem();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[sb]);
+    }
+    if (!ok) {
+      if (lane == 0 && !*abort_flag) record_error(p.err, kDevErrWaitFull);
+      *abort_flag = 1;
+    }
+    // ---------------------------------------------------------- epilogue
+    const size_t part_stride = (size_t)p.d + 4;
+    float* part_u = p.part + (size_t)unit * NQ * part_stride;
+    if (nt > 0) {
+      if (ok) ok = bar_all(3, 128, mbar_wait_bounded(&o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, abort_flag));
+#pragma unroll
+      for (int c = 0; c < C::C2; ++c) {
+        float v = lp[c];
+        v += __shfl_xor_sync(0xffffffffu, v, 1);
+        v += __shfl_xor_sync(0xffffffffu, v, 2);
+        v += __shfl_xor_sync(0xffffffffu, v, 4);
+        v += __shfl_xor_sync(0xffffffffu, v, 8);
+        if ((lane & 15) == 0) {
+          lsum[warp * NQ + col0 + c] = v;
+          if (warp == 0) mfin[col0 + c] = m_used[c];
+        }
+      }
+      const bool all_ok = bar_all(1, 128, ok);
+      if (all_ok) {
+        tc::fence_after();
+        for (int cp = 0; cp < NCS / 2; ++cp) {
+#pragma unroll
+          for (int cb = 0; cb < NQ / 16; ++cb) {
+            uint32_t o[16];
+            tc::ld_32x32b_x16(tlane + colO + cp * NQ + cb * 16, o);
+            tc::wait_ld();
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+              __stcg(part_u + (size_t)(cb * 16 + j) * part_stride + 4 + (int)rank * p.wsl + cp * 128 + tid,
+                     __uint_as_float(o[j]));
+          }
+        }
+        if (rank == 0 && tid < NQ) {
+          part_u[(size_t)tid * part_stride] = mfin[tid];
+          part_u[(size_t)tid * part_stride + 1] = lsum[tid] + lsum[NQ + tid] + lsum[2 * NQ + tid] + lsum[3 * NQ + tid];
+        }
+      }
+    }
+  }
+  tc::fence_before();
+  __syncthreads();
+  if (warp == 4 && nt > 0) {
+    tc::fence_after();
+    tc::dealloc(tmem, ncols);
+  }
+  tc::cluster_sync();  // no CTA leaves while a peer may still write into its shared memory
+}
+
 // Merge of the split partials of every group: CTA (column block, group),
 // thread = one of 128 columns of O'. Splits in split order, null row first.
 template <int NQ>
@@ -594,6 +942,78 @@ cudaError_t launch_mu_nq(const MuParams& P, int smem, cudaStream_t st) {
 
 }  // namespace
 
+// Shared-memory plan of the column-slice kernel: Q' slice, tile slots,
+// two P tiles, the exchange buffers, barriers, scratch. -1 if fewer than
+// three tile slots fit.
+int mu_slice_plan(MuParams& P, int nq, int wsl, int cl) {
+  const int ncs = wsl / 64;
+  const int qbytes = ncs * nq * 128;
+  const int pbytes = 2 * nq * 128;
+  const int xbytes = 2 * cl * 64 * nq * 4;
+  const int tile = ncs * kMuBox;
+  P.off_ring = (qbytes + 1023) / 1024 * 1024;
+  int nslot = (kMuSmemBudget - P.off_ring - pbytes - xbytes - 4096) / tile;
+  if (nslot > 8) nslot = 8;
+  if (nslot < 3) return -1;
+  P.ns = nslot;
+  P.hold = 1;
+  P.cl = cl;
+  P.wsl = wsl;
+  P.off_p = P.off_ring + nslot * tile;
+  P.off_x = P.off_p + pbytes;
+  P.off_bar = P.off_x + xbytes;
+  const int nbars = 1 + 2 * nslot + 11;  // q_full, full/empty, s_full/s_free/p_full/o_done/x_full pairs, drain
+  P.off_misc = (P.off_bar + nbars * 8 + 15) / 16 * 16;
+  const int misc = 16 + (8 + 2 + 4 + 1) * nq * 4;
+  return P.off_misc + misc + 1024;
+}
+
+template <int NQ>
+cudaError_t launch_slice_nq(const MuParams& P, int smem, cudaStream_t st) {
+  cudaError_t e = ensure_smem_limit<3100 + NQ>(mu_slice_kernel<NQ>, kMuSmemBudget + 2048);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[1];
+  cfg.gridDim = dim3((unsigned)(P.n_units * P.cl));
+  cfg.blockDim = dim3(kMuThreads);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = st;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)P.cl;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, mu_slice_kernel<NQ>, P);
+  if (e != cudaSuccess) return e;
+  mu_merge_kernel<NQ><<<dim3((unsigned)(P.d / 128), (unsigned)P.n_groups), 128, 0, st>>>(P);
+  return cudaGetLastError();
+}
+
+// Clusters of the column-slice kernel resident at once on the current
+// device (0: the configuration cannot run).
+template <int NQ>
+int slice_clusters(int cl, int smem) {
+  if (ensure_smem_limit<3100 + NQ>(mu_slice_kernel<NQ>, kMuSmemBudget + 2048) != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[1];
+  cfg.gridDim = dim3((unsigned)(cl * 64));
+  cfg.blockDim = dim3(kMuThreads);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)cl;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, mu_slice_kernel<NQ>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
 int mu_query_tile(int nq_total, int d) {
   // the widest query tile whose accumulators fit TMEM: NQ (2 + d/128) <= 512
   for (int nq : {64, 32, 16}) {
@@ -616,11 +1036,47 @@ int mu_prefill_query_tile(int nblk, int H, int d) {
 }
 
 int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity) {
-  return encode3d(map, pool, (uint64_t)d, (uint64_t)kRows, (uint64_t)capacity, 64);
+  // a slot is [d/64 chunks][R][64]: chunk c of a block is rows c*R .. c*R+R-1 of the view
+  return encode3d(map, pool, 64, (uint64_t)kRows * (d / 64), (uint64_t)capacity, 64);
+}
+
+MuDecodePlan mu_decode_plan(int H, int d) {
+  const MuDecodePlan two_pass{mu_query_tile(H, d), 0, 0};
+  const int nq = (H + 15) / 16 * 16;
+  if (nq > 64) return two_pass;
+  // slices of 256 columns where d allows, clusters of at most 8 CTAs, an
+  // exchange of at most 2 x 64 KB-equivalent partials (cl x nq <= 128)
+  for (int wsl : {256, 128, 384, 512}) {
+    if (d % wsl) continue;
+    const int cl = d / wsl;
+    if (cl > 8 || cl * nq > 128) continue;
+    MuParams P{};
+    const int smem = mu_slice_plan(P, nq, wsl, cl);
+    if (smem < 0) continue;
+    const int n = nq == 16 ? slice_clusters<16>(cl, smem) : nq == 32 ? slice_clusters<32>(cl, smem)
+                                                                      : slice_clusters<64>(cl, smem);
+    if (n > 0) return MuDecodePlan{nq, cl, wsl};
+  }
+  return two_pass;
+}
+
+cudaError_t launch_mu_slice(MuParams& P, const MuDecodePlan& pl, cudaStream_t st) {
+  if (P.n_units == 0) return cudaSuccess;
+  if (pl.cl < 1 || P.d != pl.cl * pl.wsl) return cudaErrorInvalidValue;
+  if (encode3d(&P.q, P.qptr, (uint64_t)P.d, (uint64_t)P.nrows, (uint64_t)P.n_qg, (uint32_t)pl.nq))
+    return cudaErrorInvalidValue;
+  const int smem = mu_slice_plan(P, pl.nq, pl.wsl, pl.cl);
+  if (smem < 0 || smem > kMuSmemBudget + 2048) return cudaErrorInvalidValue;
+  if (pl.nq == 16) return launch_slice_nq<16>(P, smem, st);
+  if (pl.nq == 32) return launch_slice_nq<32>(P, smem, st);
+  if (pl.nq == 64) return launch_slice_nq<64>(P, smem, st);
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_mu_attention(MuParams& P, int nq, cudaStream_t st) {
   if (P.n_units == 0) return cudaSuccess;
+  P.cl = 0;
+  P.wsl = 0;
   if (encode3d(&P.q, P.qptr, (uint64_t)P.d, (uint64_t)P.nrows, (uint64_t)P.n_qg, (uint32_t)nq)) return cudaErrorInvalidValue;
   const int smem = mu_smem_plan(P, nq, P.d);
   if (smem < 0 || smem > kMuSmemBudget + 2048) return cudaErrorInvalidValue;

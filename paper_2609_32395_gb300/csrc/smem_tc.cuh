@@ -196,5 +196,15 @@ __device__ __forceinline__ float2 ld_dsmem_f32x2(uint32_t addr) {
   return v;
 }
 
+// Asynchronous store of four 32-bit words (16-byte aligned) into the shared
+// memory of a CTA of the cluster; the 16 bytes complete on `remote_bar`, an
+// mbarrier of that same CTA (both addresses from dsmem_addr).
+__device__ __forceinline__ void st_async_v4(uint32_t remote_addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d,
+                                            uint32_t remote_bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];"
+               ::"r"(remote_addr), "r"(a), "r"(b), "r"(c), "r"(d), "r"(remote_bar)
+               : "memory");
+}
+
 }  // namespace tc
 }  // namespace smem

@@ -38,6 +38,7 @@ EXPORTED = [
     "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
     "smem_layer_workspace_bytes", "smem_append_block_rows", "smem_set_null_vector", "smem_reader_layer_prefill",
     "smem_reader_layer_decode", "smem_mu_decode", "smem_mu_prefill", "smem_share_block", "smem_slot_refs",
+    "smem_mu_decode_plan",
 ]
 
 
@@ -120,6 +121,7 @@ def lib():
             "smem_mu_prefill": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
             "smem_share_block": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32, _vp, _i32p]),
             "smem_slot_refs": (ctypes.c_int, [_vp, _i32, _i32p]),
+            "smem_mu_decode_plan": (ctypes.c_int, [_vp, _i32p, _i32p, _i32p]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -212,6 +214,13 @@ def smem_slot_refs(h, slot) -> int:
     n = ctypes.c_int32(0)
     _check(lib().smem_slot_refs(h, slot, ctypes.byref(n)), "smem_slot_refs")
     return n.value
+
+
+def smem_mu_decode_plan(h):
+    """(nq, cluster, slice_cols) of a recompute cache's decode kernel; cluster 0: two-pass form."""
+    v = [ctypes.c_int32(0) for _ in range(3)]
+    _check(lib().smem_mu_decode_plan(h, *[ctypes.byref(x) for x in v]), "smem_mu_decode_plan")
+    return tuple(x.value for x in v)
 
 
 def smem_delete_block(h, seq, block_idx, stream=None, device=True):

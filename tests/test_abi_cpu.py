@@ -28,7 +28,7 @@ def test_exports_every_declared_symbol():
     for n in names:
         assert hasattr(L, n), n
     assert set(names) == set(smem.EXPORTED)
-    assert smem.smem_abi_version() == 6
+    assert smem.smem_abi_version() == 7
 
 
 def test_required_bytes_validation():
@@ -165,5 +165,31 @@ def test_recompute_geometry():
         # per row: the dense buffers, q' and O' [H][d] bf16, split partials
         dense = 6 * d * 2 + 4 * d * 4 + 4 * d * 2
         assert w2 - w0 >= 2 * (dense + 2 * 4 * d * 2)
+        # the decode kernel is chosen on a device only
+        with pytest.raises(smem.SmemError) as e:
+            smem.smem_mu_decode_plan(h)
+        assert e.value.code == smem.ERR_NO_DEVICE
+    finally:
+        smem.smem_cache_destroy(h)
+    h = smem.smem_cache_create(mat, None)
+    try:
+        with pytest.raises(smem.SmemError) as e:
+            smem.smem_mu_decode_plan(h)
+        assert e.value.code == smem.ERR_UNSUPPORTED
+    finally:
+        smem.smem_cache_destroy(h)
+
+
+def test_recompute_workspace_covers_every_query_tile():
+    """H = 32 heads at d = 2048 need two 16-query tiles per decode item (the
+    two-pass kernel's accumulators fit 16 queries at that width); the
+    workspace holds the split partials of both tiles."""
+    cfg = smem.make_config(1, 32, 64, 4, 8, 16, recompute_kv=True)
+    h = smem.smem_cache_create(cfg, None)
+    try:
+        d = 32 * 64
+        w0 = smem.smem_layer_workspace_bytes(h, 0)
+        w4 = smem.smem_layer_workspace_bytes(h, 4)
+        assert w4 - w0 >= 4 * 32 * 16 * (d + 4) * 4  # 4 items x 32 query rows x 16 splits
     finally:
         smem.smem_cache_destroy(h)

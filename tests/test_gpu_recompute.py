@@ -210,3 +210,117 @@ def test_mu_prefill_kernel_matches_oracle(H, D, nblk):
         ref = _oracle_mu(qp[h].double().numpy(), list(mus), lc.nu)
         err = np.abs(got[h] - ref)
         assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (h, err.max(), err.mean())
+
+
+def _mu_cache(H, D, ctx, has_null=True, free_order=None, history=False, seed=1401):
+    d = H * D
+    model = LayerModel(1, d, seed=seed)
+    cap = sum(ctx) + 4 * len(ctx) + 8
+    lc = LayerCache(model, H, D, max_seqs=len(ctx), max_blocks=max(ctx) + 8, capacity=cap, has_null=has_null,
+                    free_order=free_order, recompute=True)
+    for s, n in enumerate(ctx):
+        order = list(range(n))[::-1] if history else list(range(n))
+        if history:
+            lc.append(s, n + 2, content_seq=77)   # appended and deleted again
+        for j in order:
+            lc.append(s, j)
+        if history:
+            lc.delete(s, n + 2)
+            if n > 3:
+                lc.delete(s, 2)
+                lc.append(s, 2)
+    return lc
+
+
+def _mu_run(lc, H, d, ctx, seed):
+    qp = _qprime(seed, (len(ctx), H, d), d, (2,))
+    op = torch.empty(len(ctx), H, d, dtype=torch.bfloat16, device="cuda")
+    smem.smem_mu_decode(lc.h, list(range(len(ctx))), ctx, qp.cuda(), op, lc.ws)
+    assert smem.smem_check_device_error(lc.h) == smem.OK
+    return qp, op
+
+
+def _check_mu_decode(lc, H, d, ctx, qp, op):
+    from tests.gpu_helpers import MAX_ABS, MEAN_ABS
+    got = op.float().cpu().numpy().astype(np.float64)
+    for s, n in enumerate(ctx):
+        _, mus = lc.memory(s, n)
+        q = qp[s].double().numpy()
+        # one query at a time keeps the oracle's broadcast rows small
+        ref = np.stack([_oracle_mu(q[i:i + 1], list(mus), lc.nu)[0] for i in range(H)])
+        err = np.abs(got[s] - ref)
+        assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (s, n, err.max(), err.mean())
+
+
+@pytest.mark.parametrize("H,D,cluster", [(4, 64, 1), (12, 64, 3), (16, 64, 4), (16, 128, 8), (32, 64, 0),
+                                         (20, 64, 0)])
+@pytest.mark.parametrize("has_null", [True, False])
+@pytest.mark.parametrize("slices", [False, True])
+def test_mu_decode_at_model_widths(H, D, cluster, has_null, slices, monkeypatch):
+    """The decode form at d = 256 .. 2048, with the two-pass kernel and with
+    the column-slice kernel switched on (clusters of 1, 3, 4 and 8 CTAs at
+    d = 256, 768 = 160M, 1024 = 410M, 2048 = 1.5B; the two-pass kernel
+    stays where the exchange would not fit). H = 32 at d = 2048 takes two
+    16-query tiles per item, H = 20 one 32-query tile. Contexts of 0, 1,
+    31, 33 and 70 blocks: no split, one short split, one split, a split
+    plus a one-block split, several splits with a ragged last."""
+    d = H * D
+    ctx = [0, 1, 31, 33, 70]
+    monkeypatch.setenv("SMEM_MU_CLUSTERS", "1" if slices else "0")
+    lc = _mu_cache(H, D, ctx, has_null=has_null)
+    nq, cl, wsl = smem.smem_mu_decode_plan(lc.h)
+    assert cl == (cluster if slices else 0)
+    if cl:
+        assert wsl * cl == d and nq == (H + 15) // 16 * 16
+    else:
+        assert nq in (16, 32) and nq * ((H + nq - 1) // nq) >= H
+    qp, op = _mu_run(lc, H, d, ctx, 1401 + d)
+    _check_mu_decode(lc, H, d, ctx, qp, op)
+
+
+@pytest.mark.parametrize("slices", [False, True])
+def test_mu_decode_sixteen_splits(slices, monkeypatch):
+    """600 blocks at d = 256: 16 splits of 38 blocks, the last ragged; 300
+    blocks: 16 splits of 19 (two-pass) or 10 of 32 (column slices, clusters
+    of one CTA)."""
+    H, D = 4, 64
+    ctx = [600, 300, 5]
+    monkeypatch.setenv("SMEM_MU_CLUSTERS", "1" if slices else "0")
+    lc = _mu_cache(H, D, ctx)
+    assert smem.smem_mu_decode_plan(lc.h)[1] == (1 if slices else 0)
+    qp, op = _mu_run(lc, H, H * D, ctx, 1501)
+    _check_mu_decode(lc, H, H * D, ctx, qp, op)
+
+
+def test_mu_decode_slice_kernel_is_edit_path_independent(monkeypatch):
+    """Theorem 1 through the column-slice kernel (d = 1024, clusters of 4):
+    the same block sets reached by different edit paths and slot orders
+    give bitwise-equal outputs."""
+    H, D = 16, 64
+    ctx = [70, 40, 9]
+    monkeypatch.setenv("SMEM_MU_CLUSTERS", "1")
+    a = _mu_cache(H, D, ctx)
+    b = _mu_cache(H, D, ctx, free_order=synth.slot_permutation(11, sum(ctx) + 4 * len(ctx) + 8), history=True)
+    assert smem.smem_mu_decode_plan(a.h)[1] == 4
+    assert a.mirror.table(0)[1] != b.mirror.table(0)[1]
+    _, oa = _mu_run(a, H, H * D, ctx, 1601)
+    _, ob = _mu_run(b, H, H * D, ctx, 1601)
+    assert torch.equal(oa.view(torch.int16), ob.view(torch.int16))
+
+
+def test_mu_decode_two_kernels_agree(monkeypatch):
+    """The two-pass kernel (clusters switched off for the cache) and the
+    column-slice kernel on the same rows and queries: both within the
+    tolerance of the oracle, and of each other."""
+    from tests.gpu_helpers import MAX_ABS
+    H, D = 16, 64
+    ctx = [45, 12]
+    monkeypatch.setenv("SMEM_MU_CLUSTERS", "1")
+    s = _mu_cache(H, D, ctx)
+    monkeypatch.setenv("SMEM_MU_CLUSTERS", "0")
+    t = _mu_cache(H, D, ctx)
+    assert smem.smem_mu_decode_plan(s.h)[1] == 4 and smem.smem_mu_decode_plan(t.h)[1] == 0
+    qs, os_ = _mu_run(s, H, H * D, ctx, 1701)
+    _, ot = _mu_run(t, H, H * D, ctx, 1701)
+    _check_mu_decode(t, H, H * D, ctx, qs, ot)
+    assert float((os_.float() - ot.float()).abs().max()) <= MAX_ABS
