@@ -27,7 +27,8 @@ using smem::Layout;
 struct smem_cache {
   CUtensorMap pool_map{};     // decode kernel's view of the pool (device caches)
   CUtensorMap pool_map_pf{};  // prefill kernel's view (whole 64-row tiles)
-  CUtensorMap pool_map_mu{};  // memory-row view [C][d/64][R][64] (recompute caches)
+  CUtensorMap pool_map_mu2{};  // memory-row view [C][d/64][R][64], two-chunk boxes (recompute caches)
+  CUtensorMap pool_map_mu4{};  // the same, four-chunk boxes (when d/64 is a multiple of 4)
   smem_config cfg{};
   Layout lay{};
   uint8_t* dev = nullptr;  // nullptr: bookkeeping-only
@@ -476,7 +477,9 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
     }
     int er = 0;
     if (L.recompute) {
-      er = smem::encode_mu_pool_map(&c->pool_map_mu, c->dev + L.off_pool, L.H * L.D, L.capacity);
+      er = smem::encode_mu_pool_map(&c->pool_map_mu2, c->dev + L.off_pool, L.H * L.D, L.capacity, 2);
+      if (er == 0 && (L.H * L.D / 64) % 4 == 0)
+        er = smem::encode_mu_pool_map(&c->pool_map_mu4, c->dev + L.off_pool, L.H * L.D, L.capacity, 4);
     } else {
       er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.Hkv, L.D, L.capacity,
                                  smem::decode_stage_rows(L.D));
@@ -951,7 +954,8 @@ int mu_attend(smem_cache* c, uint8_t* ws, const LayerWs& o, bool prefill, int nb
   const int d = L.H * L.D, H = L.H;
   int rc = SMEM_OK;
   static thread_local smem::MuParams P;
-  P.pool = c->pool_map_mu;
+  P.pool2 = c->pool_map_mu2;
+  P.pool4 = c->pool_map_mu4;
   P.table = reinterpret_cast<const int*>(c->dev + L.off_table);
   P.nu = L.has_null ? reinterpret_cast<const uint16_t*>(c->dev + L.off_null) : nullptr;
   P.part = reinterpret_cast<float*>(ws + o.part);

@@ -192,7 +192,8 @@ struct MuGroup {
   int seq, qg, n0, nblk, split_blks, nsplit, unit_begin, pad;
 };
 struct MuParams {
-  CUtensorMap pool;           // memory rows [C][d/64 chunks][R][64], box 64 x 64 x 1
+  CUtensorMap pool2;          // memory rows [C][d/64 chunks][R][64], box 64 x 2R x 1 (two chunks)
+  CUtensorMap pool4;          // the same view, box 64 x 4R x 1 (four chunks; encoded when d/64 % 4 == 0)
   CUtensorMap q;              // Q' [n_qg][nrows][d], box 64 x NQ x 1 (set by the launcher)
   const int* table;           // [max_seqs][max_blocks]
   const uint16_t* qptr;       // Q' (bf16, softmax scale log2(e)/sqrt(d_h) folded in)
@@ -201,7 +202,7 @@ struct MuParams {
   float* part;                // [unit][NQ][d + 4]: m, l, pad, pad, O'[d]
   int* err;
   int d, nrows, n_qg, max_blocks, capacity, n_groups, n_units;
-  int ns, hold, off_ring, off_p, off_bar, off_misc;  // shared-memory plan (set by the launcher)
+  int ns, nsv, cpb, nsb, off_ring, off_v, off_p, off_bar, off_misc;  // plan (set by the launcher)
   int cl, wsl, off_x;  // column-slice kernel: cluster size, slice width, exchange offset
   MuGroup groups[kMaxMuGroups];
 };
@@ -220,14 +221,16 @@ int mu_query_tile(int nq_total, int d);
 // Query tile of the one-block form for nblk readable blocks (a function of
 // the block count and the geometry only).
 int mu_prefill_query_tile(int nblk, int H, int d);
-int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity);
+int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity, int chunks_per_box);
 cudaError_t launch_mu_attention(MuParams& P, int nq, cudaStream_t st);
 // Split plans (functions of the block count and the cache geometry only).
 // A split reads at least kMuMinSplitBlocks blocks: its partial (NQ x d fp32)
 // and fixed costs stay small next to the rows it streams.
-// The column-slice kernel streams a tile in a fraction of the time of one
-// CTA, so its splits are longer (kMuSliceMinSplitBlocks).
-constexpr int kMuMinSplitBlocks = 8;
+// A unit pays a fixed start (queries, pipeline fill) and end (its O'
+// partial), so splits are at least 24 blocks long; the column-slice kernel
+// streams a tile in a fraction of the time of one CTA, so its splits are
+// longer still (kMuSliceMinSplitBlocks).
+constexpr int kMuMinSplitBlocks = 24;
 constexpr int kMuSliceMinSplitBlocks = 32;
 SMEM_HD inline int mu_decode_split_blocks(int nblk, int cl) {
   const int s = (nblk + kMuMaxSplits - 1) / kMuMaxSplits;

@@ -18,9 +18,11 @@
 // both on the tensor cores (tcgen05, fp32 accumulators in TMEM). A decode
 // step puts the H heads of one sequence in one CTA (NQ = H rounded up to 16);
 // a one-block prefill puts NQ of the block's 64 queries of one head in a
-// CTA. The row tile is streamed twice from the TMA ring -- once for S, once
-// for P.V (the second pass normally hits L2) -- so any d fits in shared
-// memory. Softmax runs column-wise (one query per column) with the same
+// CTA. The row tile is streamed twice -- once into a score ring for S,
+// once into a value ring for P.V (the second pass normally hits L2) -- so
+// any d fits in shared memory; the two rings are separate so that value
+// chunks waiting for their tile's softmax never hold up the score stream
+// from HBM. Softmax runs column-wise (one query per column) with the same
 // conditional rescale as the prefill kernel (raise the running maximum only
 // when it grows by more than 2^8). Every unit (a split of a row set) writes
 // its partial (m, l, O'); a second kernel, one CTA per (group, 128 columns),
@@ -48,6 +50,7 @@ struct MuCfg {
   static constexpr int C2 = NQ / 2;                 // S columns per thread
   static constexpr int PBYTES = NQ * 128;           // P tile [NQ][64 rows] bf16
   static constexpr uint32_t ID_S = tc::idesc_bf16(64, NQ, 0, 0);
+  static constexpr uint32_t ID_S2 = tc::idesc_bf16(128, 2 * NQ, 0, 0);  // chunk-pair scores
   static constexpr uint32_t ID_PV = tc::idesc_bf16(128, NQ, 1, 0);
 };
 
@@ -66,21 +69,29 @@ __device__ __forceinline__ void store_bf16(uint16_t* p, float v) {
 }  // namespace
 
 template <int NQ>
-__global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_kernel(const __grid_constant__ MuParams p) {
+__global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __grid_constant__ MuParams p) {
   using C = MuCfg<NQ>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int d = p.d;
-  const int NC = d / 64;  // 64-column chunks of a row (even)
-  const int ns = p.ns;
+  const int NC = d / 64;   // 64-column chunks of a row (even)
+  const int cpb = p.cpb;   // chunks per stage (2 or 4, dividing NC): one TMA box of 64 cpb rows
+  const int SPT = NC / cpb;                      // stages per tile
+  const uint32_t SB = (uint32_t)cpb * kMuBox;    // stage bytes
+  const CUtensorMap* pool = cpb == 4 ? &p.pool4 : &p.pool2;
+  const int nss = p.ns;    // score-ring stages
+  const int nsv = p.nsv;   // value-ring stages
   uint8_t* qt = base;
-  uint8_t* ring = base + p.off_ring;
+  uint8_t* sring = base + p.off_ring;
+  uint8_t* vring = base + p.off_v;
   uint8_t* pt = base + p.off_p;
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + p.off_bar);
   uint64_t* q_full = bars;
-  uint64_t* full = bars + 1;
-  uint64_t* empty = full + ns;
-  uint64_t* s_full = empty + ns;
+  uint64_t* full_s = bars + 1;
+  uint64_t* empty_s = full_s + nss;
+  uint64_t* full_v = empty_s + nss;
+  uint64_t* empty_v = full_v + nsv;
+  uint64_t* s_full = empty_v + nsv;
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
   uint64_t* o_done = p_full + 2;
@@ -92,6 +103,7 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
   float* alpha = red + 2 * 4 * NQ;                   // [2][NQ] rescale factors
   float* lsum = alpha + 2 * NQ;                      // [4][NQ] column sums per warp
   float* mfin = lsum + 4 * NQ;                       // [NQ]
+  float* xs = mfin + NQ;                             // [2][64][NQ / 2] partial-score exchange
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -108,15 +120,27 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
   const int b0 = split * G.split_blks;
   const int nt = G.nblk > 0 ? min(G.split_blks, G.nblk - b0) : 0;
   const int* trow = p.table + (size_t)G.seq * p.max_blocks;
+  // Scores: one M = 128 MMA covers a chunk pair (c, c+1) -- A = the two
+  // chunks' 128 rows, B = the queries' K-slices of both chunks (2 NQ rows) --
+  // and its diagonal blocks D[0:64][0:NQ] and D[64:128][NQ:2NQ] accumulate the
+  // even- and odd-chunk partial scores (the off-diagonal blocks are unused).
+  // Half the MMA instructions of one M = 64 MMA per chunk; the instruction
+  // rate, not the data, bounds these small shapes. NSB score buffers of
+  // 2 NQ columns (two when tensor memory allows), then O'.
+  const int NSB = p.nsb;
   uint32_t ncols = 32;
-  while (ncols < (uint32_t)(NQ * (2 + NC / 2))) ncols <<= 1;
-  const uint32_t colO = 2 * NQ;
+  while (ncols < (uint32_t)(NQ * (2 * NSB + NC / 2))) ncols <<= 1;
+  const uint32_t colO = 2 * NSB * NQ;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < ns; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+    for (int s = 0; s < nss; ++s) {
+      mbar_init(&full_s[s], 1);
+      mbar_init(&empty_s[s], 1);
+    }
+    for (int s = 0; s < nsv; ++s) {
+      mbar_init(&full_v[s], 1);
+      mbar_init(&empty_v[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&s_full[b], 1);
@@ -133,166 +157,130 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
   __syncthreads();
   tc::fence_after();
   const uint32_t tmem = nt > 0 ? *tslot : 0u;
+  const int total = nt * SPT;  // stages of the unit on each stream
 
   if (warp == 4) {
     // ------------------------------------------------------------ TMA producer
+    // Two streams: the score pass (stage k of the unit -- cpb chunks of one
+    // tile, one TMA box -- into score stage k % nss, from HBM) and the value
+    // pass of the same stages (into value stage k % nsv, normally from L2).
+    // A tile's value pass starts once all of its score stages are issued.
+    // The thread polls both rings, so a value stage held until its tile's P
+    // is ready never stalls the scores. Boxes of several chunks keep the
+    // TMA instruction rate of one thread well below its limit.
     if (lane == 0 && nt > 0) {
       mbar_arrive_expect_tx(q_full, (uint32_t)(NC * C::PBYTES));
       for (int c = 0; c < NC; ++c) tc::tma_load_3d(qt + c * C::PBYTES, &p.q, c * 64, G.n0, G.qg, q_full);
-      int k = 0;
+      int kS = 0, kV = 0, slot_s = 0, slot_v = 0;
       bool ok = true;
-      // one pass = the NC chunks of tile t; order S(0), S(1), PV(0), S(2), PV(1), ...
-      auto pass = [&](int slot) {
-        const bool good = slot >= 0 && slot < p.capacity;
-        if (!good) record_error(p.err, kDevErrBounds);
-        for (int c = 0; c < NC && ok; ++c, ++k) {
-          const int st = k % ns;
-          if (k >= ns && !mbar_wait_bounded(&empty[st], ((k / ns) - 1) & 1, abort_flag)) {
-            if (!*abort_flag) record_error(p.err, kDevErrWaitEmpty);
-            *abort_flag = 1;
-            ok = false;
-            break;
+      unsigned long long t_last = global_timer_ns();
+      while (kS < total || kV < total) {
+        bool prog = false;
+        if (kS < total && (kS < nss || mbar_test_wait(&empty_s[kS % nss], ((kS / nss) - 1) & 1))) {
+          const int j = kS % SPT, st = kS % nss;
+          if (j == 0) {
+            slot_s = trow[b0 + kS / SPT];
+            if (slot_s < 0 || slot_s >= p.capacity) record_error(p.err, kDevErrBounds);
           }
-          if (good) {
-            mbar_arrive_expect_tx(&full[st], kMuBox);
-            tc::tma_load_3d(ring + st * kMuBox, &p.pool, 0, c * kRows, slot, &full[st]);
+          if (slot_s >= 0 && slot_s < p.capacity) {
+            mbar_arrive_expect_tx(&full_s[st], SB);
+            tc::tma_load_3d(sring + st * SB, pool, 0, j * cpb * kRows, slot_s, &full_s[st]);
           } else {
-            mbar_arrive(&full[st]);
+            mbar_arrive(&full_s[st]);
           }
+          ++kS;
+          prog = true;
         }
-      };
-      // slots of tiles t and t+1 in registers; the load of t+2 is issued one
-      // iteration before its use, so its latency hides behind two passes
-      int s_cur = trow[b0];
-      int s_nxt = nt > 1 ? trow[b0 + 1] : 0;
-      if (p.hold) {
-        // hold mode: each tile is loaded once and stays until its P.V is done
-        for (int t = 0; t < nt && ok; ++t) {
-          const int s_nn = t + 2 < nt ? trow[b0 + t + 2] : 0;
-          pass(s_cur);
-          s_cur = s_nxt;
-          s_nxt = s_nn;
+        if (kV < total && (kV / SPT + 1) * SPT <= kS &&
+            (kV < nsv || mbar_test_wait(&empty_v[kV % nsv], ((kV / nsv) - 1) & 1))) {
+          const int j = kV % SPT, st = kV % nsv;
+          if (j == 0) slot_v = trow[b0 + kV / SPT];
+          if (slot_v >= 0 && slot_v < p.capacity) {
+            mbar_arrive_expect_tx(&full_v[st], SB);
+            tc::tma_load_3d(vring + st * SB, pool, 0, j * cpb * kRows, slot_v, &full_v[st]);
+          } else {
+            mbar_arrive(&full_v[st]);
+          }
+          ++kV;
+          prog = true;
         }
-      } else {
-        pass(s_cur);
-        for (int t = 0; t < nt && ok; ++t) {
-          const int s_nn = t + 2 < nt ? trow[b0 + t + 2] : 0;
-          if (t + 1 < nt) pass(s_nxt);
-          if (ok) pass(s_cur);
-          s_cur = s_nxt;
-          s_nxt = s_nn;
+        if (prog) {
+          t_last = global_timer_ns();
+        } else if (*abort_flag || global_timer_ns() - t_last > kWaitLimitNs) {
+          if (!*abort_flag) record_error(p.err, kDevErrWaitEmpty);
+          *abort_flag = 1;
+          ok = false;
+          break;
         }
       }
       if (!ok) {
         // let every copy already issued land before the CTA can exit
         mbar_wait_bounded(q_full, 0, nullptr);
-        for (int j = 0; j < k; ++j) mbar_wait_bounded(&full[j % ns], (j / ns) & 1, nullptr);
+        for (int j = kS > nss ? kS - nss : 0; j < kS; ++j) mbar_wait_bounded(&full_s[j % nss], (j / nss) & 1, nullptr);
+        for (int j = kV > nsv ? kV - nsv : 0; j < kV; ++j) mbar_wait_bounded(&full_v[j % nsv], (j / nsv) & 1, nullptr);
       }
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------- MMA issuer
+    // Polls two queues: the P.V of the oldest tile whose P is ready (value
+    // stage by stage, a column pair per MMA), and the next score stage
+    // (landed, and for a tile's first stage its S buffer free). Neither
+    // blocks the other.
     if (lane == 0 && nt > 0) {
       bool ok = mbar_wait_bounded(q_full, 0, abort_flag);
       tc::fence_after();
       const uint32_t qa = smem_u32(qt);
-      const uint32_t ra = smem_u32(ring);
-      int k = 0;
-      auto issue_s = [&](int t) {
-        const int sb = t & 1;
-        if (ok && t >= 2) ok = mbar_wait_bounded(&s_free[sb], ((t >> 1) - 1) & 1, abort_flag);
-        for (int c = 0; c < NC && ok; ++c, ++k) {
-          const int st = k % ns;
-          ok = mbar_wait_bounded(&full[st], (k / ns) & 1, abort_flag);
-          if (!ok) break;
-          tc::fence_after();
-          const uint32_t a = ra + st * kMuBox, b = qa + c * C::PBYTES;
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc::mma_bf16(tmem + sb * NQ, tc::sdesc_sw128(a + kk * 32, 16, 1024), tc::sdesc_sw128(b + kk * 32, 16, 1024),
-                         C::ID_S, (c | kk) > 0);
-          tc::commit(&empty[st]);
-        }
-        if (ok) tc::commit(&s_full[sb]);
-      };
-      auto issue_pv = [&](int t) {
-        const int pb = t & 1;
-        if (ok) ok = mbar_wait_bounded(&p_full[pb], (t >> 1) & 1, abort_flag);
-        if (!ok) return;
-        tc::fence_after();
-        const uint32_t b = smem_u32(pt + pb * C::PBYTES);
-        for (int cp = 0; cp < NC / 2 && ok; ++cp, k += 2) {
-          const int st = k % ns;  // even: the pair sits in slots st, st + 1
-          ok = mbar_wait_bounded(&full[st], (k / ns) & 1, abort_flag) &&
-               mbar_wait_bounded(&full[st + 1], ((k + 1) / ns) & 1, abort_flag);
-          if (!ok) break;
-          tc::fence_after();
-          const uint32_t a = ra + st * kMuBox;
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc::mma_bf16(tmem + colO + cp * NQ, tc::sdesc_sw128(a + kk * 2048, kMuBox, 1024),
-                         tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_PV, (t > 0 || kk > 0));
-          tc::commit(&empty[st]);
-          tc::commit(&empty[st + 1]);
-        }
-        if (ok) tc::commit(&o_done[pb]);
-      };
-      if (p.hold) {
-        // Hold mode: a tile's chunks stay in the ring from its S to its P.V,
-        // so the issuer polls two queues -- the next S chunk (data landed,
-        // S buffer free) and the P.V of the oldest tile whose P is ready --
-        // and never blocks one on the other.
-        int kS = 0, tS = 0, cS = 0, tP = 0;
-        unsigned long long t_last = global_timer_ns();
-        while (ok && tP < nt) {
-          bool prog = false;
-          if (tP < tS && mbar_test_wait(&p_full[tP & 1], (tP >> 1) & 1)) {
+      const uint32_t sa = smem_u32(sring);
+      const uint32_t va = smem_u32(vring);
+      int kS = 0, kV = 0, tP = 0;
+      unsigned long long t_last = global_timer_ns();
+      while (ok && tP < nt) {
+        bool prog = false;
+        if (tP < kS / SPT && (kV % SPT != 0 || mbar_test_wait(&p_full[tP & 1], (tP >> 1) & 1))) {
+          const int st = kV % nsv;
+          if (mbar_test_wait(&full_v[st], (kV / nsv) & 1)) {
             tc::fence_after();
+            const uint32_t a0 = va + st * SB;
             const uint32_t b = smem_u32(pt + (tP & 1) * C::PBYTES);
-            for (int cp = 0; cp < NC / 2; ++cp) {
-              const int st = (tP * NC + 2 * cp) % ns;  // even: the pair sits in slots st, st + 1
-              const uint32_t a = ra + st * kMuBox;
+            for (int q = 0; q < cpb / 2; ++q) {
+              const int cp = (kV % SPT) * (cpb / 2) + q;  // column pair of the row
 #pragma unroll
               for (int kk = 0; kk < 4; ++kk)
-                tc::mma_bf16(tmem + colO + cp * NQ, tc::sdesc_sw128(a + kk * 2048, kMuBox, 1024),
+                tc::mma_bf16(tmem + colO + cp * NQ, tc::sdesc_sw128(a0 + 2 * q * kMuBox + kk * 2048, kMuBox, 1024),
                              tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_PV, (tP > 0 || kk > 0));
-              tc::commit(&empty[st]);
-              tc::commit(&empty[st + 1]);
             }
-            tc::commit(&o_done[tP & 1]);
-            ++tP;
+            tc::commit(&empty_v[st]);
+            ++kV;
+            if (kV % SPT == 0) {
+              tc::commit(&o_done[tP & 1]);
+              ++tP;
+            }
             prog = true;
           }
-          if (tS < nt) {
-            const int sb = tS & 1;
-            const bool sfree = cS > 0 || tS < 2 || mbar_test_wait(&s_free[sb], ((tS >> 1) - 1) & 1);
-            const int st = kS % ns;
-            if (sfree && mbar_test_wait(&full[st], (kS / ns) & 1)) {
-              tc::fence_after();
-              const uint32_t a = ra + st * kMuBox, b = qa + cS * C::PBYTES;
+        }
+        if (kS < total) {
+          const int t = kS / SPT, j = kS % SPT, sb = t % NSB, st = kS % nss;
+          const bool sfree = j > 0 || t < NSB || mbar_test_wait(&s_free[sb], ((t / NSB) - 1) & 1);
+          if (sfree && mbar_test_wait(&full_s[st], (kS / nss) & 1)) {
+            tc::fence_after();
+            for (int q = 0; q < cpb / 2; ++q) {
+              const int c = j * cpb + 2 * q;  // even chunk of the pair
+              const uint32_t a = sa + st * SB + 2 * q * kMuBox, b = qa + c * C::PBYTES;
 #pragma unroll
               for (int kk = 0; kk < 4; ++kk)
-                tc::mma_bf16(tmem + sb * NQ, tc::sdesc_sw128(a + kk * 32, 16, 1024),
-                             tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_S, (cS | kk) > 0);
-              ++kS;
-              if (++cS == NC) {
-                tc::commit(&s_full[sb]);
-                ++tS;
-                cS = 0;
-              }
-              prog = true;
+                tc::mma_bf16(tmem + (uint32_t)(sb * 2 * NQ), tc::sdesc_sw128(a + kk * 32, 16, 1024),
+                             tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_S2, (c | kk) > 0);
             }
-          }
-          if (prog) {
-            t_last = global_timer_ns();
-          } else if (*abort_flag || global_timer_ns() - t_last > kWaitLimitNs) {
-            ok = false;
+            tc::commit(&empty_s[st]);
+            ++kS;
+            if (j == SPT - 1) tc::commit(&s_full[sb]);
+            prog = true;
           }
         }
-      } else {
-        issue_s(0);
-        for (int t = 0; t < nt && ok; ++t) {
-          if (t + 1 < nt) issue_s(t + 1);
-          issue_pv(t);
+        if (prog) {
+          t_last = global_timer_ns();
+        } else if (*abort_flag || global_timer_ns() - t_last > kWaitLimitNs) {
+          ok = false;
         }
       }
       if (!ok) {
@@ -304,10 +292,16 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
     }
   } else {
     // ---------------------------------------------------------- softmax warps
-    const int tid = threadIdx.x;            // 0..127: TMEM lane of O'
-    const int r = 16 * warp + (lane & 15);  // row of the tile
-    const int hf = lane >> 4;               // column half of S
-    const int col0 = hf * C::C2;
+    // Thread = TMEM lane tid of the M = 128 score tile: warps 0-1 hold the
+    // even-chunk partials of tile rows 0-63, warps 2-3 the odd-chunk ones.
+    // Each thread finishes one column half (queries hc*NQ/2 ..) of its row:
+    // it hands the other half of its partial to the thread of the same row
+    // and the other partial, and sums even + odd (the same order for both).
+    const int tid = threadIdx.x;     // 0..127: TMEM lane of S and of O'
+    const int hr = warp & 1;         // row half: tile rows 32 hr .. 32 hr + 31
+    const int hc = warp >> 1;        // 0: even partial, finishes queries [0, NQ/2); 1: odd, [NQ/2, NQ)
+    const int r = 32 * hr + lane;    // tile row
+    const int col0 = hc * C::C2;
     const uint32_t tlane = tmem + ((uint32_t)(32 * warp) << 16);
     float m_used[C::C2], lp[C::C2];
 #pragma unroll
@@ -319,45 +313,57 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
     // warps, so they take the same named barriers in the same order.
     bool ok = true;
     for (int t = 0; t < nt; ++t) {
-      const int sb = t & 1;
-      ok = bar_all(3, 128, mbar_wait_bounded(&s_full[sb], (t >> 1) & 1, abort_flag));
+      const int sb = t % NSB, pb = t & 1;
+      ok = bar_all(3, 128, mbar_wait_bounded(&s_full[sb], (t / NSB) & 1, abort_flag));
       if (!ok) break;
       tc::fence_after();
-      uint32_t sr[C::C2];
-      ld_s<NQ>(tlane + sb * NQ, sr);
-      tc::wait_ld();
-      tc::fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s_free[sb]);
       float x[C::C2];
+      {
+        uint32_t v[NQ / 16][16];
+#pragma unroll
+        for (int cb = 0; cb < NQ / 16; ++cb) tc::ld_32x32b_x16(tlane + sb * 2 * NQ + hc * NQ + cb * 16, v[cb]);
+        tc::wait_ld();
+        tc::fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_free[sb]);
+        // v holds queries [0, NQ); lo = [0, NQ/2), hi = [NQ/2, NQ) (compile-time indices)
+        float* xo = xs + ((size_t)hc * 64 + r) * C::C2;
+#pragma unroll
+        for (int c = 0; c < C::C2; ++c) {
+          const float lo = __uint_as_float(v[c / 16][c % 16]);
+          const float hi = __uint_as_float(v[(C::C2 + c) / 16][(C::C2 + c) % 16]);
+          xo[c] = hc == 0 ? hi : lo;
+        }
+        named_bar_sync(1, 128);
+        const float* xi = xs + ((size_t)(1 - hc) * 64 + r) * C::C2;
+#pragma unroll
+        for (int c = 0; c < C::C2; ++c) {
+          const float lo = __uint_as_float(v[c / 16][c % 16]);
+          const float hi = __uint_as_float(v[(C::C2 + c) / 16][(C::C2 + c) % 16]);
+          x[c] = hc == 0 ? lo + xi[c] : xi[c] + hi;
+        }
+      }
 #pragma unroll
       for (int c = 0; c < C::C2; ++c) {
-        x[c] = __uint_as_float(sr[c]);
         float v = x[c];
-        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
-        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
-        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
-        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
-        if ((lane & 15) == 0) red[(sb * 4 + warp) * NQ + col0 + c] = v;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+        if (lane == 0) red[(pb * 2 + hr) * NQ + col0 + c] = v;
       }
       named_bar_sync(1, 128);
       bool need_mine = false;
-      float a_c[C::C2];
 #pragma unroll
       for (int c = 0; c < C::C2; ++c) {
         const int col = col0 + c;
-        float tmax = red[(sb * 4) * NQ + col];
-#pragma unroll
-        for (int w2 = 1; w2 < 4; ++w2) tmax = fmaxf(tmax, red[(sb * 4 + w2) * NQ + col]);
-        const bool need = tmax > m_used[c] + kMuRescaleLog2;
-        a_c[c] = 1.f;
-        if (need) {
-          a_c[c] = exp2f(m_used[c] - tmax);
-          lp[c] *= a_c[c];
+        const float tmax = fmaxf(red[(pb * 2) * NQ + col], red[(pb * 2 + 1) * NQ + col]);
+        float a_c = 1.f;
+        if (tmax > m_used[c] + kMuRescaleLog2) {
+          a_c = exp2f(m_used[c] - tmax);
+          lp[c] *= a_c;
           m_used[c] = tmax;
           need_mine = true;
         }
-        if (warp == 0 && (lane & 15) == 0) alpha[sb * NQ + col] = a_c[c];
+        if (hr == 0 && lane == 0) alpha[pb * NQ + col] = a_c;
       }
       // any column of the tile raised its maximum (t > 0: O' holds earlier tiles)
       const bool any = !bar_all(2, 128, !need_mine);
@@ -373,30 +379,30 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
             tc::ld_32x32b_x16(ta, o);
             tc::wait_ld();
 #pragma unroll
-            for (int j = 0; j < 16; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha[sb * NQ + cb * 16 + j]);
+            for (int j = 0; j < 16; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * alpha[pb * NQ + cb * 16 + j]);
             tc::st_32x32b_x16(ta, o);
           }
         }
         tc::wait_st();
       }
-      // P buffer sb was last read by P.V of tile t-2
+      // P buffer pb was last read by P.V of tile t-2
       if (t >= 2) {
-        ok = bar_all(3, 128, mbar_wait_bounded(&o_done[sb], ((t - 2) >> 1) & 1, abort_flag));
+        ok = bar_all(3, 128, mbar_wait_bounded(&o_done[pb], ((t - 2) >> 1) & 1, abort_flag));
         if (!ok) break;
       }
-      uint8_t* pb = pt + sb * C::PBYTES;
+      uint8_t* pbuf = pt + pb * C::PBYTES;
 #pragma unroll
       for (int c = 0; c < C::C2; ++c) {
         const int col = col0 + c;
         const float pr = exp2f(x[c] - m_used[c]);
         lp[c] += pr;
-        store_bf16(reinterpret_cast<uint16_t*>(pb + col * 128 + ((((r >> 3) ^ (col & 7)) & 7) << 4) + (r & 7) * 2),
+        store_bf16(reinterpret_cast<uint16_t*>(pbuf + col * 128 + ((((r >> 3) ^ (col & 7)) & 7) << 4) + (r & 7) * 2),
                    pr);
       }
       fence_proxy_async_smem();
       tc::fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[sb]);
+      if (lane == 0) mbar_arrive(&p_full[pb]);
     }
     if (!ok) {
       if (lane == 0 && !*abort_flag) record_error(p.err, kDevErrWaitFull);
@@ -410,13 +416,11 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
 #pragma unroll
       for (int c = 0; c < C::C2; ++c) {
         float v = lp[c];
-        v += __shfl_xor_sync(0xffffffffu, v, 1);
-        v += __shfl_xor_sync(0xffffffffu, v, 2);
-        v += __shfl_xor_sync(0xffffffffu, v, 4);
-        v += __shfl_xor_sync(0xffffffffu, v, 8);
-        if ((lane & 15) == 0) {
-          lsum[warp * NQ + col0 + c] = v;
-          if (warp == 0) mfin[col0 + c] = m_used[c];
+#pragma unroll
+        for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) {
+          lsum[hr * NQ + col0 + c] = v;
+          if (hr == 0) mfin[col0 + c] = m_used[c];
         }
       }
       const bool all_ok = bar_all(1, 128, ok);
@@ -435,7 +439,7 @@ __global__ void __launch_bounds__(kMuThreads, NQ <= 32 ? 2 : 1) mu_attention_ker
         }
         if (tid < NQ) {
           part_u[(size_t)tid * part_stride] = mfin[tid];
-          part_u[(size_t)tid * part_stride + 1] = lsum[tid] + lsum[NQ + tid] + lsum[2 * NQ + tid] + lsum[3 * NQ + tid];
+          part_u[(size_t)tid * part_stride + 1] = lsum[tid] + lsum[NQ + tid];
         }
       }
     }
@@ -551,9 +555,9 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_slice_kernel(const __grid_co
         const int slot = trow[b0 + t];
         if (slot >= 0 && slot < p.capacity) {
           mbar_arrive_expect_tx(&full[sl], (uint32_t)(NCS * kMuBox));
-          for (int c = 0; c < NCS; ++c)
-            tc::tma_load_3d(ring + (sl * NCS + c) * kMuBox, &p.pool, 0, ((int)rank * NCS + c) * kRows, slot,
-                            &full[sl]);
+          for (int c = 0; c < NCS; c += p.cpb)  // boxes of cpb chunks
+            tc::tma_load_3d(ring + (sl * NCS + c) * kMuBox, p.cpb == 4 ? &p.pool4 : &p.pool2, 0,
+                            ((int)rank * NCS + c) * kRows, slot, &full[sl]);
         } else {
           record_error(p.err, kDevErrBounds);
           mbar_arrive(&full[sl]);
@@ -893,39 +897,41 @@ int encode3d(CUtensorMap* map, const void* ptr, uint64_t d0, uint64_t d1, uint64
   return r == CUDA_SUCCESS ? 0 : (int)r;
 }
 
-// Shared-memory plan of a launch: Q' chunks, the ring, two P tiles,
-// barriers, scratch. Returns the dynamic shared-memory bytes.
+// Shared-memory plan of a launch (one CTA per SM): Q' chunks, the score
+// ring, the value ring, two P tiles, barriers, scratch. Stages of four
+// chunks (one 32 KB box) where d allows and at least two score and two
+// value stages fit, else of two; about a third of the stages go to the
+// value ring. Returns the dynamic shared-memory bytes, -1 if no plan fits.
 int mu_smem_plan(MuParams& P, int nq, int d) {
-  const int qbytes = (d / 64) * nq * 128;
-  const int fixed = 2 * nq * 128 + 4096 + 1024;
   const int nc = d / 64;
-  // Two CTAs per SM streaming every tile twice (the second pass from L2)
-  // when the queries leave room for an 8-stage ring in half the SM; else one
-  // CTA per SM holding whole tiles from S to P.V (hold mode) when a tile and
-  // four chunks of lookahead fit; else one CTA per SM streaming twice.
-  // Two interleaved CTAs measured faster than one CTA holding its tiles.
-  int ns_full = ((kMuSmemBudget - qbytes - fixed) / kMuBox) & ~1;
-  if (ns_full > kMuMaxStages) ns_full = kMuMaxStages;
-  const int ns_half = ((kMuSmemHalf - qbytes - fixed) / kMuBox) & ~1;
-  int ns;
-  P.hold = 0;
-  if (ns_half >= 8) {
-    ns = ns_half;
-  } else if (ns_full >= nc + 4) {
-    ns = ns_full;
-    P.hold = 1;
-  } else {
-    ns = ns_full;
-  }
-  if (ns < 4) return -1;
-  P.ns = ns;
+  const int qbytes = nc * nq * 128;
+  const int pbytes = 2 * nq * 128;
   P.off_ring = (qbytes + 1023) / 1024 * 1024;
-  P.off_p = P.off_ring + ns * kMuBox;
-  P.off_bar = P.off_p + 2 * nq * 128;
-  const int nbars = 1 + 2 * ns + 9;  // q_full, full/empty rings, s_full/s_free/p_full/o_done pairs, drain
+  // misc: 16 B words + red[2][4][NQ] + alpha[2][NQ] + lsum[4][NQ] + mfin[NQ] + exchange [64][NQ]
+  const int misc = 16 + (8 + 2 + 4 + 1 + 64) * nq * 4;
+  const int chunks = (kMuSmemBudget - P.off_ring - pbytes - misc - 1024) / kMuBox;
+  P.cpb = 0;
+  for (int cpb : {4, 2}) {
+    if (nc % cpb) continue;
+    const int stages = chunks / cpb;
+    const int nsv = stages / 3 > 2 ? stages / 3 : 2;
+    int nss = stages - nsv;
+    if (nss > 16) nss = 16;
+    if (nss < 2) continue;
+    P.cpb = cpb;
+    P.ns = nss;
+    P.nsv = nsv;
+    break;
+  }
+  if (!P.cpb) return -1;
+  // two score buffers (2 NQ columns each) when tensor memory holds them next to O'
+  P.nsb = nq * (4 + nc / 2) <= 512 ? 2 : 1;
+  const int sb = P.cpb * kMuBox;
+  P.off_v = P.off_ring + P.ns * sb;
+  P.off_p = P.off_v + P.nsv * sb;
+  P.off_bar = P.off_p + pbytes;
+  const int nbars = 1 + 2 * P.ns + 2 * P.nsv + 9;  // q_full, two full/empty rings, s_full/s_free/p_full/o_done pairs, drain
   P.off_misc = (P.off_bar + nbars * 8 + 15) / 16 * 16;
-  // misc: 16 B words + red[2][4][NQ] + alpha[2][NQ] + lsum[4][NQ] + mfin[NQ]
-  const int misc = 16 + (8 + 2 + 4 + 1) * nq * 4;
   return P.off_misc + misc + 1024;
 }
 
@@ -956,7 +962,8 @@ int mu_slice_plan(MuParams& P, int nq, int wsl, int cl) {
   if (nslot > 8) nslot = 8;
   if (nslot < 3) return -1;
   P.ns = nslot;
-  P.hold = 1;
+  P.nsv = 0;
+  P.cpb = ncs % 4 == 0 && (cl * wsl / 64) % 4 == 0 ? 4 : 2;
   P.cl = cl;
   P.wsl = wsl;
   P.off_p = P.off_ring + nslot * tile;
@@ -1035,9 +1042,10 @@ int mu_prefill_query_tile(int nblk, int H, int d) {
   return 16;
 }
 
-int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity) {
-  // a slot is [d/64 chunks][R][64]: chunk c of a block is rows c*R .. c*R+R-1 of the view
-  return encode3d(map, pool, 64, (uint64_t)kRows * (d / 64), (uint64_t)capacity, 64);
+int encode_mu_pool_map(CUtensorMap* map, void* pool, int d, int capacity, int chunks_per_box) {
+  // a slot is [d/64 chunks][R][64]: chunk c of a block is rows c*R .. c*R+R-1
+  // of the view, and a box of chunks_per_box consecutive chunks is one copy
+  return encode3d(map, pool, 64, (uint64_t)kRows * (d / 64), (uint64_t)capacity, (uint32_t)(kRows * chunks_per_box));
 }
 
 MuDecodePlan mu_decode_plan(int H, int d) {

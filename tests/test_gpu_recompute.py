@@ -262,8 +262,9 @@ def test_mu_decode_at_model_widths(H, D, cluster, has_null, slices, monkeypatch)
     d = 256, 768 = 160M, 1024 = 410M, 2048 = 1.5B; the two-pass kernel
     stays where the exchange would not fit). H = 32 at d = 2048 takes two
     16-query tiles per item, H = 20 one 32-query tile. Contexts of 0, 1,
-    31, 33 and 70 blocks: no split, one short split, one split, a split
-    plus a one-block split, several splits with a ragged last."""
+    31, 33 and 70 blocks: no readable block, one short split, and one to
+    three splits with a ragged last (splits of at least 24 blocks, 32 with
+    column slices)."""
     d = H * D
     ctx = [0, 1, 31, 33, 70]
     monkeypatch.setenv("SMEM_MU_CLUSTERS", "1" if slices else "0")
@@ -281,7 +282,7 @@ def test_mu_decode_at_model_widths(H, D, cluster, has_null, slices, monkeypatch)
 @pytest.mark.parametrize("slices", [False, True])
 def test_mu_decode_sixteen_splits(slices, monkeypatch):
     """600 blocks at d = 256: 16 splits of 38 blocks, the last ragged; 300
-    blocks: 16 splits of 19 (two-pass) or 10 of 32 (column slices, clusters
+    blocks: 13 splits of 24 (two-pass) or 10 of 32 (column slices, clusters
     of one CTA)."""
     H, D = 4, 64
     ctx = [600, 300, 5]
