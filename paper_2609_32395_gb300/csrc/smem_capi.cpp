@@ -26,7 +26,7 @@ using smem::Layout;
 
 struct smem_cache {
   CUtensorMap pool_map{};     // decode kernel's view of the pool (device caches)
-  CUtensorMap pool_map_pf{};  // prefill kernel's view (whole 64-row tiles)
+  CUtensorMap pool_map_pf{};  // prefill kernel's view (a block's K and V rows of 64 columns per box)
   CUtensorMap pool_map_mu2{};  // memory-row view [C][d/64][R][64], two-chunk boxes (recompute caches)
   CUtensorMap pool_map_mu4{};  // the same, four-chunk boxes (when d/64 is a multiple of 4)
   smem_config cfg{};
@@ -484,7 +484,8 @@ int smem_cache_create(const smem_config* cfg, void* dev_buf, size_t dev_bytes, s
       er = smem::encode_pool_map(&c->pool_map, c->dev + L.off_pool, L.L, L.Hkv, L.D, L.capacity,
                                  smem::decode_stage_rows(L.D));
       if (er == 0)
-        er = smem::encode_pool_map(&c->pool_map_pf, c->dev + L.off_pool, L.L, L.Hkv, L.D, L.capacity, smem::kRows);
+        er = smem::encode_pool_map(&c->pool_map_pf, c->dev + L.off_pool, L.L, L.Hkv, L.D, L.capacity,
+                                 2 * smem::kRows);  // a block's K rows and V rows in one box
     }
     if (er != 0) {
       std::snprintf(g_detail, sizeof(g_detail), "tensor map encode failed (%d)", er);

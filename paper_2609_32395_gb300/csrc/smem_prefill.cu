@@ -43,6 +43,11 @@ struct Pf {
   static constexpr int BOX = 64 * (D < 64 ? D * 2 : 128);  // one [64 rows][box width] box
   static constexpr int TILE = BOXES * BOX;        // K or V of one block and head
   static constexpr int STAGE = 2 * TILE;
+  // A stage holds, per column box bx, the K box then the V box of the same
+  // columns (one TMA copy of 128 pool rows each): K box bx at bx * KVS, V
+  // box bx at bx * KVS + BOX. Fewer, larger copies keep the producer thread
+  // below its TMA instruction rate.
+  static constexpr int KVS = 2 * BOX;
   static constexpr int NS = D == 32 ? 8 : (D == 64 ? 5 : 4);  // ring stages (2 CTAs per SM fit at d_h <= 64)
   static constexpr int PBYTES = 64 * 64 * 2;      // P tile [64 queries][64 keys] bf16
   static constexpr int OFF_Q = 0;
@@ -65,15 +70,17 @@ struct Pf {
 
 // Shared-memory descriptors of the K-major Q/K tiles (k-th step of 16
 // columns) and of the MN-major V tile (k-th step of 16 rows).
+// `stride`: bytes from one column box to the next (BOX for the query tile,
+// KVS for a key tile in a stage).
 template <int D>
-__device__ __forceinline__ uint64_t qk_desc(uint32_t base, int k) {
+__device__ __forceinline__ uint64_t qk_desc(uint32_t base, int k, int stride) {
   if constexpr (D == 32) return tc::sdesc_sw64(base + k * 32, 16, 512);
-  else return tc::sdesc_sw128(base + (k >> 2) * Pf<D>::BOX + (k & 3) * 32, 16, 1024);
+  else return tc::sdesc_sw128(base + (k >> 2) * stride + (k & 3) * 32, 16, 1024);
 }
 template <int D>
 __device__ __forceinline__ uint64_t v_desc(uint32_t base, int k) {
-  if constexpr (D == 32) return tc::sdesc_sw64(base + k * 1024, Pf<D>::BOX, 512);
-  else return tc::sdesc_sw128(base + k * 2048, Pf<D>::BOX, 1024);
+  if constexpr (D == 32) return tc::sdesc_sw64(base + k * 1024, Pf<D>::KVS, 512);
+  else return tc::sdesc_sw128(base + k * 2048, Pf<D>::KVS, 1024);
 }
 
 // O columns of a softmax thread (its half of the row), read or written in TMEM.
@@ -109,7 +116,7 @@ __device__ __forceinline__ void st_o(uint32_t trow, const uint32_t (&o)[D / 2]) 
 constexpr float kRescaleLog2 = 8.0f;  // raise the running max when it grows by more than 2^8
 
 struct PrefillParams {
-  CUtensorMap pool;          // [C][L*H*2*R][D], box 64 x 64 rows
+  CUtensorMap pool;          // [C][L*H*2*R][D], box 64 columns x 128 rows (a block's K then V)
   CUtensorMap qs, ks, vs, qc;  // [b][H][D], box 64 x 1 x 64
   const int* table_row;
   const uint16_t* null_kv;
@@ -146,12 +153,12 @@ __device__ __forceinline__ void rot8(float* t, const float2* cs) {
 // swizzle) in place by one table row; one warp, then a proxy fence so that
 // the tensor cores see the new values.
 template <int D>
-__device__ void rotate_tile(uint8_t* tile, const float2* cs_row, int lane) {
+__device__ void rotate_tile(uint8_t* tile, const float2* cs_row, int lane, int stride) {
   constexpr int CH = D / 8;  // 16-byte chunks per row
   for (int i = lane; i < 64 * CH; i += 32) {
     const int r = i / CH, c = i % CH;
     uint8_t* ptr = D == 32 ? tile + r * 64 + ((c ^ ((r >> 1) & 3)) << 4)
-                           : tile + (c >> 3) * (64 * 128) + r * 128 + ((((c & 7) ^ (r & 7))) << 4);
+                           : tile + (c >> 3) * stride + r * 128 + ((((c & 7) ^ (r & 7))) << 4);
     float t[8];
     unpack8(*reinterpret_cast<const uint4*>(ptr), t);
     rot8(t, cs_row + c * 4);
@@ -332,13 +339,12 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           break;
         }
         uint8_t* kd = ring + st * C::STAGE;
-        uint8_t* vd = kd + C::TILE;
         if (sa) {
           mbar_arrive_expect_tx(&full[st], C::STAGE);
 #pragma unroll
           for (int bx = 0; bx < C::BOXES; ++bx) {
-            tc::tma_load_3d(kd + bx * C::BOX, &p.ks, bx * 64, h / (p.H / p.Hkv), 0, &full[st]);
-            tc::tma_load_3d(vd + bx * C::BOX, &p.vs, bx * 64, h / (p.H / p.Hkv), 0, &full[st]);
+            tc::tma_load_3d(kd + bx * C::KVS, &p.ks, bx * 64, h / (p.H / p.Hkv), 0, &full[st]);
+            tc::tma_load_3d(kd + bx * C::KVS + C::BOX, &p.vs, bx * 64, h / (p.H / p.Hkv), 0, &full[st]);
           }
         } else {
           const int slot = p.table_row[b0 + j];
@@ -349,10 +355,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
             mbar_arrive_expect_tx(&full[st], C::STAGE);
             const int y = ((p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2) * C::R;
 #pragma unroll
-            for (int bx = 0; bx < C::BOXES; ++bx) {
-              tc::tma_load_3d(kd + bx * C::BOX, &p.pool, bx * 64, y, slot, &full[st]);
-              tc::tma_load_3d(vd + bx * C::BOX, &p.pool, bx * 64, y + C::R, slot, &full[st]);
-            }
+            for (int bx = 0; bx < C::BOXES; ++bx)  // the K rows and then the V rows of these columns
+              tc::tma_load_3d(kd + bx * C::KVS, &p.pool, bx * 64, y, slot, &full[st]);
           }
         }
         ++issued;
@@ -376,7 +380,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       if (near0 + 32 + lane < b0 + nt) jv1 = p.bidx_row[near0 + 32 + lane];
       if (ok) {
         tc::fence_after();
-        rotate_tile<D>(qt, p.rope_tab + (size_t)p.rope_w * (D / 2), lane);
+        rotate_tile<D>(qt, p.rope_tab + (size_t)p.rope_w * (D / 2), lane, C::BOX);
       }
       const uint32_t qa = smem_u32(qt);
       for (int jj = 0; ok && jj <= nt; ++jj) {
@@ -391,13 +395,13 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
             const int o = b0 + jj - near0;
             const int j = __shfl_sync(0xffffffffu, o < 32 ? jv0 : jv1, o & 31);
             const int dk = max(0, p.rope_w - (p.q_blk - j));
-            if (dk > 0) rotate_tile<D>(ring + st * C::STAGE, p.rope_tab + (size_t)dk * (D / 2), lane);
+            if (dk > 0) rotate_tile<D>(ring + st * C::STAGE, p.rope_tab + (size_t)dk * (D / 2), lane, C::KVS);
           }
           if (lane == 0) {
             const uint32_t ka = smem_u32(ring + st * C::STAGE);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)
-              tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k), qk_desc<D>(ka, k), C::ID_QK, k > 0);
+              tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k, C::BOX), qk_desc<D>(ka, k, C::KVS), C::ID_QK, k > 0);
             tc::commit(&s_full[sb]);
           }
           __syncwarp();
@@ -409,7 +413,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           tc::fence_after();
           if (lane == 0) {
             const uint32_t pa = smem_u32(pt + pb * C::PBYTES);
-            const uint32_t va = smem_u32(ring + st * C::STAGE + C::TILE);
+            const uint32_t va = smem_u32(ring + st * C::STAGE + C::BOX);
 #pragma unroll
             for (int k = 0; k < 4; ++k)
               tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024), v_desc<D>(va, k), C::ID_PV,
@@ -446,7 +450,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           const uint32_t ka = smem_u32(ring + st * C::STAGE);
 #pragma unroll
           for (int k = 0; k < D / 16; ++k)
-            tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k), qk_desc<D>(ka, k), C::ID_QK, k > 0);
+            tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k, C::BOX), qk_desc<D>(ka, k, C::KVS), C::ID_QK, k > 0);
           tc::commit(&s_full[sb]);
         }
         if (jj >= 1) {  // O += P . V for tile jj-1
@@ -455,7 +459,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
           if (!ok) break;
           tc::fence_after();
           const uint32_t pa = smem_u32(pt + pb * C::PBYTES);
-          const uint32_t va = smem_u32(ring + st * C::STAGE + C::TILE);
+          const uint32_t va = smem_u32(ring + st * C::STAGE + C::BOX);
 #pragma unroll
           for (int k = 0; k < 4; ++k)
             tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024), v_desc<D>(va, k), C::ID_PV,
