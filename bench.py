@@ -1205,6 +1205,9 @@ def run_ours(args):
     if recompute:
         k = recompute["memory_row_kernel"]
         k["hbm_frac"] = k["achieved_gbs"] / peak
+        # DRAM bytes of one launch from the committed ncu summary (16-sequence
+        # capture, scaled by the memory rows read; null once the kernel changed)
+        k["traffic"] = profiled_traffic("mu_decode_410m.txt", k["rows_per_launch"])
         if rec_serve:
             for c in rec_serve:
                 c["hbm_frac"] = c["achieved_gbs"] / peak
