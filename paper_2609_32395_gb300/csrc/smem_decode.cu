@@ -544,10 +544,16 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
           break;
         }
         if (ch == 0) {
+          // the unit's queries in fp32, pre-scaled; rows of absent group members zeroed
           const uint16_t* qs = qarea + s * QN * D;
-          for (int i = lane; i < ng * (D / 8); i += 32) {
+          for (int i = lane; i < QN * (D / 8); i += 32) {
             float t[8];
-            unpack8(*reinterpret_cast<const uint4*>(qs + i * 8), t);
+            if (i < ng * (D / 8)) {
+              unpack8(*reinterpret_cast<const uint4*>(qs + i * 8), t);
+            } else {
+#pragma unroll
+              for (int e = 0; e < 8; ++e) t[e] = 0.f;
+            }
 #pragma unroll
             for (int e = 0; e < 8; ++e) qbuf[i * 8 + e] = t[e] * p.scale_log2;
           }
@@ -555,40 +561,59 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
         }
         const uint8_t* kb = ring + s * C::STAGE;
         const uint8_t* vb = kb + C::HALF;
-        // scores of this lane's row(s) against every query of the group
+        // scores of this lane's row(s) against every query of the group: one
+        // 8-column slice at a time, each query slice loaded once for all rows,
+        // QN x RPL independent accumulators interleaved
         float sc[QN][C::RPL];
 #pragma unroll
-        for (int h2 = 0; h2 < C::RPL; ++h2) {
-          const int r = C::RPL == 2 ? lane + 32 * h2 : rr;
-          float kr[C::QW];
+        for (int j = 0; j < QN; ++j)
 #pragma unroll
-          for (int j = 0; j < C::QW / 8; ++j)
-            unpack8(*reinterpret_cast<const uint4*>(kb + chunk_off<D>(r, hh * 8 + j)), &kr[j * 8]);
+          for (int h2 = 0; h2 < C::RPL; ++h2) sc[j][h2] = 0.f;
+#pragma unroll
+        for (int s8 = 0; s8 < C::QW / 8; ++s8) {
+          float kr[C::RPL][8];
+#pragma unroll
+          for (int h2 = 0; h2 < C::RPL; ++h2) {
+            const int r = C::RPL == 2 ? lane + 32 * h2 : rr;
+            unpack8(*reinterpret_cast<const uint4*>(kb + chunk_off<D>(r, hh * 8 + s8)), kr[h2]);
+          }
 #pragma unroll
           for (int j = 0; j < QN; ++j) {
-            float dot = 0.f;
-            if (j < ng) {
-              const float4* qv = reinterpret_cast<const float4*>(qbuf + j * D + hh * C::QW);
+            const float4* qv = reinterpret_cast<const float4*>(qbuf + j * D + hh * C::QW + s8 * 8);
+            const float4 qa = qv[0], qb = qv[1];
 #pragma unroll
-              for (int e4 = 0; e4 < C::QW / 4; ++e4) {
-                const float4 q4 = qv[e4];
-                dot = fmaf(q4.x, kr[4 * e4], dot);
-                dot = fmaf(q4.y, kr[4 * e4 + 1], dot);
-                dot = fmaf(q4.z, kr[4 * e4 + 2], dot);
-                dot = fmaf(q4.w, kr[4 * e4 + 3], dot);
-              }
+            for (int h2 = 0; h2 < C::RPL; ++h2) {
+              float dot = sc[j][h2];
+              dot = fmaf(qa.x, kr[h2][0], dot);
+              dot = fmaf(qa.y, kr[h2][1], dot);
+              dot = fmaf(qa.z, kr[h2][2], dot);
+              dot = fmaf(qa.w, kr[h2][3], dot);
+              dot = fmaf(qb.x, kr[h2][4], dot);
+              dot = fmaf(qb.y, kr[h2][5], dot);
+              dot = fmaf(qb.z, kr[h2][6], dot);
+              dot = fmaf(qb.w, kr[h2][7], dot);
+              sc[j][h2] = dot;
             }
-            if (C::LPR == 2) dot += __shfl_xor_sync(0xffffffffu, dot, 1);
-            sc[j][h2] = dot;
           }
         }
+        if (C::LPR == 2) {
+#pragma unroll
+          for (int j = 0; j < QN; ++j)
+#pragma unroll
+            for (int h2 = 0; h2 < C::RPL; ++h2) sc[j][h2] += __shfl_xor_sync(0xffffffffu, sc[j][h2], 1);
+        }
+        // per-query maxima over the stage's rows, the QN reductions interleaved
+        float gmx[QN];
+#pragma unroll
+        for (int j = 0; j < QN; ++j) gmx[j] = C::RPL == 2 ? fmaxf(sc[j][0], sc[j][C::RPL - 1]) : sc[j][0];
+#pragma unroll
+        for (int o = C::LPR; o < 32; o <<= 1)
+#pragma unroll
+          for (int j = 0; j < QN; ++j) gmx[j] = fmaxf(gmx[j], __shfl_xor_sync(0xffffffffu, gmx[j], o));
         float galpha[QN];
 #pragma unroll
         for (int j = 0; j < QN; ++j) {
-          float mx = C::RPL == 2 ? fmaxf(sc[j][0], sc[j][C::RPL - 1]) : sc[j][0];
-#pragma unroll
-          for (int o = C::LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-          const float m_new = fmaxf(gm[j], mx);
+          const float m_new = fmaxf(gm[j], gmx[j]);
           galpha[j] = exp2f(gm[j] - m_new);
           gm[j] = m_new;
           if (j < ng) {
