@@ -20,8 +20,12 @@
 // accumulates in fp32 with each lane owning 8 columns of a quarter of the
 // rows. A CA unit writes its split partial (m, l, acc[d_h]); the warp that
 // completes the last split of an (item, head) merges all splits in split
-// order (null row first). SA units read their <= 64 in-block rows straight
-// from global memory. No warp ever waits for another warp; every reduction
+// order (null row first). With grouped-query attention a CA unit serves the
+// 2 or 4 query heads that share a key/value head: the warp scores each stage
+// against all of them with warp-level tensor-core MMAs (the group as the
+// rows of a 16-row operand) and keeps P in registers for P.V, so the rows
+// stream once per group at a few dozen instructions per stage. SA units
+// read their <= 64 in-block rows straight from global memory. No warp ever waits for another warp; every reduction
 // order is fixed by the block count, so the same block set gives the same
 // bits whatever the slots or the edit history.
 #include <cuda.h>
@@ -127,6 +131,39 @@ __device__ __forceinline__ uint4 ld_nc16(const void* p) {
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                : "l"(p));
   return v;
+}
+
+// Warp-level tensor-core helpers of the grouped decode (PTX mma.sync /
+// ldmatrix). mma_16816: D[16x8] += A[16x16] B[16x8], bf16 in, fp32 out, the
+// A rows 8..15 zero (a1 = a3 = 0): a0/a2 = columns 2t.. / 2t+8.. of row g.
+__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+// The same keeping only row g of D (the rows 8..15 of a zero A are zero).
+__device__ __forceinline__ void mma_16816_acc2(float (&d)[2], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+  float z0 = 0.f, z1 = 0.f;
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(z0), "+f"(z1)
+      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+// Four 8x8 b16 matrices; lane l gives the 16-byte row address of row l%8 of
+// matrix l/8. Plain: thread (g, t) gets row g, columns 2t, 2t+1 of each
+// matrix; trans: rows 2t, 2t+1 of column g.
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t saddr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(saddr));
+}
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t saddr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(saddr));
 }
 
 __device__ __forceinline__ void store_bf16x8(uint16_t* dst, const float* v, float scale) {
@@ -523,17 +560,26 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     const DecodeItem& it = p.items[U.item];
     if constexpr (QN > 1) {
       // ---- grouped unit: the p.qn query heads U.h .. U.h+qn-1 read one
-      // key/value head; every chunk is scored against all of them (queries
-      // in shared memory, fp32, pre-scaled), so the rows stream once per group
+      // key/value head; the warp scores every stage against all of them on
+      // the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate): the
+      // group's queries are rows 0..qn-1 of a 16-row A operand (the other
+      // rows zero), K and V fragments come from the swizzled stage by
+      // ldmatrix, and P goes from the score accumulators straight into the
+      // A operand of O += P.V (bf16). Thread (gq = lane/4, tq = lane%4)
+      // holds query row gq: its scores of rows 2tq, 2tq+1 of every 8-row
+      // tile of the stage and its O columns 2tq, 2tq+1 of every 8 columns.
+      // The rows stream once per group; a stage costs 2 * 16 MMAs.
+      constexpr int KS = D / 16;        // k-steps of a score MMA chain
+      constexpr int NT = C::SROWS / 8;  // 8-row tiles of a stage
+      constexpr int ON = D / 8;         // 8-column tiles of O
       const int ng = p.qn;
-      float gm[QN], gl[QN], gacc[QN][8];
+      const int gq = lane >> 2, tq = lane & 3;
+      const bool real = gq < ng;
+      uint32_t qa[KS][2];  // A fragments of row gq: columns 16ks + 2tq (+8)
+      float o[ON][2];
+      float gmr = -INFINITY, glr = 0.f;  // running maximum, partial sum (this thread's rows)
 #pragma unroll
-      for (int j = 0; j < QN; ++j) {
-        gm[j] = -INFINITY;
-        gl[j] = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) gacc[j][e] = 0.f;
-      }
+      for (int on = 0; on < ON; ++on) o[on][0] = o[on][1] = 0.f;
       const int nch = U.nt * C::CHUNKS;
       for (int ch = 0; ch < nch; ++ch, ++k) {
         const int s = k % C::NS;
@@ -544,112 +590,67 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
           break;
         }
         if (ch == 0) {
-          // the unit's queries in fp32, pre-scaled; rows of absent group members zeroed
-          const uint16_t* qs = qarea + s * QN * D;
-          for (int i = lane; i < QN * (D / 8); i += 32) {
-            float t[8];
-            if (i < ng * (D / 8)) {
-              unpack8(*reinterpret_cast<const uint4*>(qs + i * 8), t);
-            } else {
+          const uint16_t* qs = qarea + s * QN * D + (real ? gq : 0) * D;
 #pragma unroll
-              for (int e = 0; e < 8; ++e) t[e] = 0.f;
-            }
-#pragma unroll
-            for (int e = 0; e < 8; ++e) qbuf[i * 8 + e] = t[e] * p.scale_log2;
+          for (int ks = 0; ks < KS; ++ks) {
+            qa[ks][0] = real ? *reinterpret_cast<const uint32_t*>(qs + 16 * ks + 2 * tq) : 0u;
+            qa[ks][1] = real ? *reinterpret_cast<const uint32_t*>(qs + 16 * ks + 8 + 2 * tq) : 0u;
           }
-          __syncwarp();
         }
         const uint8_t* kb = ring + s * C::STAGE;
         const uint8_t* vb = kb + C::HALF;
-        // scores of this lane's row(s) against every query of the group: one
-        // 8-column slice at a time, each query slice loaded once for all rows,
-        // QN x RPL independent accumulators interleaved
-        float sc[QN][C::RPL];
+        // S[q][r] = Q[q] . K[r]: one ldmatrix.x4 brings two k-steps of an 8-row tile
+        float sacc[NT][4];
 #pragma unroll
-        for (int j = 0; j < QN; ++j)
+        for (int nt = 0; nt < NT; ++nt) {
+          sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
 #pragma unroll
-          for (int h2 = 0; h2 < C::RPL; ++h2) sc[j][h2] = 0.f;
-#pragma unroll
-        for (int s8 = 0; s8 < C::QW / 8; ++s8) {
-          float kr[C::RPL][8];
-#pragma unroll
-          for (int h2 = 0; h2 < C::RPL; ++h2) {
-            const int r = C::RPL == 2 ? lane + 32 * h2 : rr;
-            unpack8(*reinterpret_cast<const uint4*>(kb + chunk_off<D>(r, hh * 8 + s8)), kr[h2]);
-          }
-#pragma unroll
-          for (int j = 0; j < QN; ++j) {
-            const float4* qv = reinterpret_cast<const float4*>(qbuf + j * D + hh * C::QW + s8 * 8);
-            const float4 qa = qv[0], qb = qv[1];
-#pragma unroll
-            for (int h2 = 0; h2 < C::RPL; ++h2) {
-              float dot = sc[j][h2];
-              dot = fmaf(qa.x, kr[h2][0], dot);
-              dot = fmaf(qa.y, kr[h2][1], dot);
-              dot = fmaf(qa.z, kr[h2][2], dot);
-              dot = fmaf(qa.w, kr[h2][3], dot);
-              dot = fmaf(qb.x, kr[h2][4], dot);
-              dot = fmaf(qb.y, kr[h2][5], dot);
-              dot = fmaf(qb.z, kr[h2][6], dot);
-              dot = fmaf(qb.w, kr[h2][7], dot);
-              sc[j][h2] = dot;
-            }
+          for (int kp = 0; kp < KS / 2; ++kp) {
+            uint32_t b[4];
+            ldsm_x4(b, smem_u32(kb + chunk_off<D>(8 * nt + (lane & 7), 4 * kp + (lane >> 3))));
+            mma_16816(sacc[nt], qa[2 * kp][0], qa[2 * kp][1], b[0], b[1]);
+            mma_16816(sacc[nt], qa[2 * kp + 1][0], qa[2 * kp + 1][1], b[2], b[3]);
           }
         }
-        if (C::LPR == 2) {
+        // online softmax of row gq over the stage (the quad of tq holds the row)
+        float mx = -INFINITY;
 #pragma unroll
-          for (int j = 0; j < QN; ++j)
-#pragma unroll
-            for (int h2 = 0; h2 < C::RPL; ++h2) sc[j][h2] += __shfl_xor_sync(0xffffffffu, sc[j][h2], 1);
+        for (int nt = 0; nt < NT; ++nt) {
+          sacc[nt][0] *= p.scale_log2;
+          sacc[nt][1] *= p.scale_log2;
+          mx = fmaxf(mx, fmaxf(sacc[nt][0], sacc[nt][1]));
         }
-        // per-query maxima over the stage's rows, the QN reductions interleaved
-        float gmx[QN];
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        const float m_new = fmaxf(gmr, mx);
+        const float alpha = exp2f(gmr - m_new);
+        gmr = m_new;
+        uint32_t pa[NT];  // bf16 P of row gq, rows 2tq, 2tq+1 of each 8-row tile
+        float ps = 0.f;
 #pragma unroll
-        for (int j = 0; j < QN; ++j) gmx[j] = C::RPL == 2 ? fmaxf(sc[j][0], sc[j][C::RPL - 1]) : sc[j][0];
+        for (int nt = 0; nt < NT; ++nt) {
+          const uint32_t w = real ? pack_bf16x2(exp2f(sacc[nt][0] - m_new), exp2f(sacc[nt][1] - m_new)) : 0u;
+          pa[nt] = w;
+          ps += bf16lo(w) + bf16hi(w);  // the sum of the P the MMA uses
+        }
+        glr = glr * alpha + ps;
 #pragma unroll
-        for (int o = C::LPR; o < 32; o <<= 1)
+        for (int on = 0; on < ON; ++on) {
+          o[on][0] *= alpha;
+          o[on][1] *= alpha;
+        }
+        // O[q][c] += P[q][r] V[r][c]: k-step = 16 rows (two score tiles), one
+        // ldmatrix.x4.trans brings two 8-column tiles of V
 #pragma unroll
-          for (int j = 0; j < QN; ++j) gmx[j] = fmaxf(gmx[j], __shfl_xor_sync(0xffffffffu, gmx[j], o));
-        float galpha[QN];
+        for (int kk = 0; kk < NT / 2; ++kk) {
 #pragma unroll
-        for (int j = 0; j < QN; ++j) {
-          const float m_new = fmaxf(gm[j], gmx[j]);
-          galpha[j] = exp2f(gm[j] - m_new);
-          gm[j] = m_new;
-          if (j < ng) {
-            if (C::RPL == 2) {
-              const float p0 = exp2f(sc[j][0] - m_new), p1 = exp2f(sc[j][C::RPL - 1] - m_new);
-              gl[j] = gl[j] * galpha[j] + p0 + p1;
-              pbuf[j * 64 + lane] = p0;
-              pbuf[j * 64 + lane + 32] = p1;
-            } else {
-              const float pr = exp2f(sc[j][0] - m_new);
-              gl[j] = gl[j] * galpha[j] + (hh == 0 ? pr : 0.f);
-              if (hh == 0) pbuf[j * 64 + rr] = pr;
-            }
+          for (int op = 0; op < ON / 2; ++op) {
+            uint32_t b[4];
+            ldsm_x4_trans(b, smem_u32(vb + chunk_off<D>(16 * kk + (lane & 7) + ((lane >> 3) & 1) * 8,
+                                                       2 * op + (lane >> 4))));
+            mma_16816_acc2(o[2 * op], pa[2 * kk], pa[2 * kk + 1], b[0], b[1]);
+            mma_16816_acc2(o[2 * op + 1], pa[2 * kk], pa[2 * kk + 1], b[2], b[3]);
           }
-#pragma unroll
-          for (int e = 0; e < 8; ++e) gacc[j][e] *= galpha[j];
-        }
-        __syncwarp();
-        // P.V: lane (g, c), rows g*RG .. g*RG+RG-1, columns c*8 .. c*8+7, every query
-        float pv[QN][8];
-#pragma unroll
-        for (int j = 0; j < QN; ++j) {
-          const float4 a = *reinterpret_cast<const float4*>(pbuf + j * 64 + g * RG);
-          const float4 b = *reinterpret_cast<const float4*>(pbuf + j * 64 + g * RG + 4);
-          pv[j][0] = a.x; pv[j][1] = a.y; pv[j][2] = a.z; pv[j][3] = a.w;
-          pv[j][4] = b.x; pv[j][5] = b.y; pv[j][6] = b.z; pv[j][7] = b.w;
-        }
-#pragma unroll
-        for (int i = 0; i < RG; ++i) {
-          const int r = g * RG + i;
-          float t[8];
-          unpack8(*reinterpret_cast<const uint4*>(vb + chunk_off<D>(r, c)), t);
-#pragma unroll
-          for (int j = 0; j < QN; ++j)
-#pragma unroll
-            for (int e = 0; e < 8; ++e) gacc[j][e] = fmaf(pv[j][i], t[e], gacc[j][e]);
         }
         __syncwarp();
         if (lane == 0) {
@@ -659,36 +660,33 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
         __syncwarp();
       }
       if (failed) break;
+      glr += __shfl_xor_sync(0xffffffffu, glr, 1);
+      glr += __shfl_xor_sync(0xffffffffu, glr, 2);
       const int nsplit = ceil_div(it.nblk, decode_split_blocks(it.nblk));
-      unsigned last = 0;  // bit j: this unit completed query j's last split
+      if (nsplit == 1 && !p.null_kv) {
+        if (real) {
+          const float inv = 1.f / glr;
+          uint16_t* dst = p.oca + ((size_t)U.item * p.H + U.h + gq) * D + 2 * tq;
 #pragma unroll
-      for (int j = 0; j < QN; ++j) {
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) gl[j] += __shfl_xor_sync(0xffffffffu, gl[j], o);
-#pragma unroll
-        for (int o = CPL; o < 32; o <<= 1)
-#pragma unroll
-          for (int e = 0; e < 8; ++e) gacc[j][e] += __shfl_xor_sync(0xffffffffu, gacc[j][e], o);
-        if (j >= ng) continue;
-        if (nsplit == 1 && !p.null_kv) {
-          if (g == 0) store_bf16x8(p.oca + ((size_t)U.item * p.H + U.h + j) * D + c * 8, gacc[j], 1.f / gl[j]);
-          continue;
+          for (int on = 0; on < ON; ++on)
+            *reinterpret_cast<uint32_t*>(dst + 8 * on) = pack_bf16x2(o[on][0] * inv, o[on][1] * inv);
         }
-        float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h + j) * (D + 4);
-        if (g == 0) {
-          *reinterpret_cast<float4*>(pp + 4 + c * 8) = make_float4(gacc[j][0], gacc[j][1], gacc[j][2], gacc[j][3]);
-          *reinterpret_cast<float4*>(pp + 8 + c * 8) = make_float4(gacc[j][4], gacc[j][5], gacc[j][6], gacc[j][7]);
-        }
-        if (lane == 0) {
-          pp[0] = gm[j];
-          pp[1] = gl[j];
+        continue;
+      }
+      if (real) {
+        float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h + gq) * (D + 4);
+#pragma unroll
+        for (int on = 0; on < ON; ++on)
+          *reinterpret_cast<float2*>(pp + 4 + 8 * on + 2 * tq) = make_float2(o[on][0], o[on][1]);
+        if (tq == 0) {
+          pp[0] = gmr;
+          pp[1] = glr;
         }
       }
-      if (nsplit == 1 && !p.null_kv) continue;
       __threadfence();
       // one ticket per query head, taken by lanes 0 .. ng-1 at once
       const bool mine = lane < ng && atomicAdd(&p.counters[U.item * p.H + U.h + lane], 1u) == (unsigned)(nsplit - 1);
-      last = __ballot_sync(0xffffffffu, mine);
+      const unsigned last = __ballot_sync(0xffffffffu, mine);
       for (int j = 0; j < ng; ++j) {
         if (!(last >> j & 1u)) continue;
         __threadfence();

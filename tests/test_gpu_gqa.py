@@ -55,11 +55,11 @@ def test_gqa_prefill_matches_oracle(Hkv, D, cluster_mode):
 
 
 @pytest.mark.parametrize("Hkv,rope,D,H", [(2, 0, 64, 8), (1, 0, 64, 8), (2, 15, 64, 8), (2, 0, 128, 4),
-                                          (4, 0, 128, 4), (2, 0, 32, 8), (4, 0, 64, 12)])
+                                          (4, 0, 128, 4), (2, 0, 32, 8), (4, 0, 64, 12), (4, 0, 64, 8)])
 def test_gqa_decode_consecutive_steps(Hkv, rope, D, H):
     """Groups of 4 (one grouped unit of four queries), 8 (two units), 2 at
-    d_h 128 and 32, 3 (one query per unit), and 1; with and without rotary
-    phases."""
+    d_h 128 and 64 (a unit of two in the four-query tile) and 4 at d_h 32, 3
+    (one query per unit), and 1; with and without rotary phases."""
     dc, nblks = _cache(Hkv, rope=rope, D=D, H=H)
     pos0 = [0, 30, 61, 5]
     for s, p in enumerate(pos0):
