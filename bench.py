@@ -437,7 +437,7 @@ def measure_decode_variant(steps, warmup, device, seqs, layers=None, window=None
     alg = [r * 4 * wl.Hkv * wl.D for r in rows for _ in range(wl.L)]  # each key/value row once
     out = {"window": win, "heads": wl.H, "kv_heads": wl.Hkv, "head_dim": wl.D, "pool_bytes": int(wl.cache.nbytes),
            "tok_per_s": steps * seqs / elapsed, "steps": steps,
-           "kernel_ms_mean": float(np.mean(kern_ms)),
+           "kernel_ms_mean": float(np.mean(kern_ms)), "rows_per_launch": float(np.mean(rows)),
            "achieved_gbs": sum(alg) / (sum(kern_ms) / 1e3) / 1e9}
     wl.cache.close()
     return out
@@ -1193,6 +1193,9 @@ def run_ours(args):
     if gqa:
         gqa["hbm_frac"] = gqa["achieved_gbs"] / peak
         gqa["workload"] = WORKLOAD["name"] + " with 4 key/value heads shared by groups of 4 query heads"
+        # DRAM bytes per launch from the committed ncu summary (32-sequence
+        # capture, scaled by the rows read; null once the kernel changed)
+        gqa["traffic"] = profiled_traffic("decode_gqa_410m.txt", gqa["rows_per_launch"])
         line["gqa"] = gqa
     if d32:
         d32["hbm_frac"] = d32["achieved_gbs"] / peak
