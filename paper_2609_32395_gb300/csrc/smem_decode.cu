@@ -188,16 +188,18 @@ __device__ __forceinline__ void rot8f(float* t, const float2* cs) {
 }
 
 // Issue side of one warp's chunk stream over dynamically fetched CA units.
-// Lane 0 only. Units come from a launch-wide atomic counter, one unit ahead
-// of the unit being issued; each fetched unit is pushed on the warp's unit
-// queue together with the stage that holds its first chunk.
+// Lane 0 only. Units come from a launch-wide atomic counter; the next unit is
+// fetched when the issue side reaches the end of the current one (still NS
+// chunks ahead of the warp's math), so a warp never holds a unit it will not
+// start soon -- with about one unit per warp, an early fetch let some warps
+// take two units while others had none. Each fetched unit is pushed on the
+// warp's unit queue together with the stage that holds its first chunk.
 struct Issue {
   int u;       // unit being issued (< 0: exhausted)
   int c;       // next chunk of that unit
   int nc;      // chunks of that unit
   int item, h, b0;
   int ybase;   // pool-map row of the unit's (layer, key/value head) K tile
-  int next_u;  // unit fetched for after this one
   int pushed;  // queue entries pushed
 };
 
@@ -218,7 +220,6 @@ __device__ __forceinline__ void issue_begin_unit(const DecodeParams& p, Issue& i
     is.h = U.h;
     is.b0 = U.b0;
     is.ybase = ((p.layer * p.Hkv + U.h / (p.H / p.Hkv)) * 2) * Dec<D>::R;
-    is.next_u = fetch_unit(p);
   } else {
     is.nc = 0;
   }
@@ -250,7 +251,7 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
     }
     if (qbytes) bulk_g2s(qslot, p.qc + (size_t)is.item * p.c_stride + (size_t)is.h * D, qbytes, bar);
   }
-  if (++is.c == is.nc) issue_begin_unit<D>(p, is, is.next_u, uq);
+  if (++is.c == is.nc) issue_begin_unit<D>(p, is, fetch_unit(p), uq);
   return true;
 }
 
@@ -520,15 +521,22 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
   const int wid = blockIdx.x * C::NW + warp;
   const int stride = gridDim.x * C::NW;
 
-  // prologue: start streaming the first CA units
+  // prologue: start streaming the first CA units. When there are fewer CA
+  // units than twice the warps, a warp with self-attention work takes its
+  // first CA unit only after that work, so that no CA unit waits behind it.
   Issue is;
   int issued = 0;
-  if (lane == 0) {
-    is.pushed = 0;
-    issue_begin_unit<D>(p, is, fetch_unit(p), uq);
-    for (int s = 0; s < C::NS; ++s)
-      if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * QN * D, &full[s], uq)) ++issued;
-  }
+  const long long n_ca = (long long)p.n_pairs * (p.H / p.qn);
+  const bool defer = (p.mode & 1) && wid < p.n_items * p.H && n_ca < 2LL * stride;
+  auto prologue = [&]() {
+    if (lane == 0) {
+      is.pushed = 0;
+      issue_begin_unit<D>(p, is, fetch_unit(p), uq);
+      for (int s = 0; s < C::NS; ++s)
+        if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * QN * D, &full[s], uq)) ++issued;
+    }
+  };
+  if (!defer) prologue();
 
   // self-attention units (static, while the first tiles are in flight)
   for (int u = wid; u < p.n_items * p.H; u += stride) {
@@ -538,6 +546,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     U.h = u - U.item * p.H;
     sa_unit<D, ROPE>(p, U, pbuf, lane);
   }
+  if (defer) prologue();
   __syncwarp();
 
   constexpr int CPL = D / 8;             // P.V column chunks
