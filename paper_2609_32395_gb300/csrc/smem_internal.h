@@ -36,13 +36,15 @@ struct Layout {
 
 // Split-K plan of the decode cross-attention: the number of memory blocks a
 // split reads, a function of the sequence's block count alone (so the same
-// block set always reduces in the same order). At least 16 blocks: a unit's
-// fixed costs (queries, partial, ticket, merge) stay small next to its rows
-// in batched decode; at most 32, so that a long context alone still gives
-// the warps of every SM work (1024 blocks: 64 splits, 4096: 128).
+// block set always reduces in the same order). Below 512 blocks, 16 blocks:
+// a unit's fixed costs (queries, partial, ticket, merge) stay small next to
+// its rows in batched decode. From 512 blocks on, ceil(nblk/64) within
+// [8, 32] -- 64 splits up to 2048 blocks, 128 at 4096 -- so that a long
+// context alone still gives the warps of every SM work.
 SMEM_HD inline int decode_split_blocks(int nblk) {
-  const int sb = (nblk + 127) / 128;
-  return sb < 16 ? 16 : (sb > 32 ? 32 : sb);
+  if (nblk < 512) return 16;
+  const int sb = (nblk + 63) / 64;
+  return sb < 8 ? 8 : (sb > 32 ? 32 : sb);
 }
 SMEM_HD inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
