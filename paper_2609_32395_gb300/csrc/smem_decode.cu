@@ -61,10 +61,9 @@ struct Dec {
   static constexpr int THREADS = NW * 32;
   static constexpr int LPR = D < 64 ? 1 : D / 64;  // lanes per row in the score phase
   static constexpr int OFF_BAR = NW * NS * STAGE;
-  static constexpr int OFF_P = OFF_BAR + NW * NS * 8;               // per warp: P of QN queries
-  static constexpr int OFF_Q = OFF_P + NW * QN * 64 * 4;            // per stage: the unit's queries
-  static constexpr int OFF_QB = OFF_Q + NW * NS * QN * D * 2;       // per warp: fp32 queries (QN > 1)
-  static constexpr int OFF_UQ = OFF_QB + (QN > 1 ? NW * QN * D * 4 : 0);  // per warp: unit queue
+  static constexpr int OFF_P = OFF_BAR + NW * NS * 8;               // per warp: P of 64 rows (fp32)
+  static constexpr int OFF_Q = OFF_P + NW * 64 * 4;                 // per stage: the unit's queries
+  static constexpr int OFF_UQ = OFF_Q + NW * NS * QN * D * 2;       // per warp: unit queue
   static constexpr int OFF_END = OFF_UQ + NW * kUnitQueue * 4;
   static constexpr int SMEM = OFF_END + 1024;      // + slack to align the base to 1 KB
 };
@@ -507,9 +506,8 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
   const int lane = threadIdx.x & 31;
   uint8_t* ring = base + warp * C::NS * C::STAGE;
   uint64_t* full = reinterpret_cast<uint64_t*>(base + C::OFF_BAR) + warp * C::NS;
-  float* pbuf = reinterpret_cast<float*>(base + C::OFF_P) + warp * QN * 64;
+  float* pbuf = reinterpret_cast<float*>(base + C::OFF_P) + warp * 64;
   uint16_t* qarea = reinterpret_cast<uint16_t*>(base + C::OFF_Q) + warp * C::NS * QN * D;
-  float* qbuf = reinterpret_cast<float*>(base + C::OFF_QB) + warp * QN * D;  // QN > 1 only
   int* uq = reinterpret_cast<int*>(base + C::OFF_UQ) + warp * kUnitQueue;
 
   if (lane == 0) {

@@ -188,8 +188,6 @@ int blas_gemm_sb(void* blas, bool ta, bool tb, int m, int n, int k, float alpha,
 constexpr int kMaxMuGroups = 512;   // groups (row set x query tile) per launch
 constexpr int kMuMaxSplits = 16;    // splits of one group's blocks
 constexpr int kMuSmemBudget = 220 * 1024;  // one CTA per SM
-constexpr int kMuSmemHalf = 110 * 1024;    // two CTAs per SM
-constexpr int kMuMaxStages = 32;           // ring stages of 8 KB
 // One group: NQ queries (rows n0.. of query set qg) that read the same row
 // set (the first nblk table blocks of `seq`), cut into nsplit units of
 // split_blks blocks; units of a group are consecutive from unit_begin.
