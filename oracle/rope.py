@@ -25,7 +25,7 @@ relative-phase shortcut.
 Readings (the paper does not fix them): the interleaved pair convention of
 RoFormer; phases in units of blocks for cross-attention and of tokens for
 self-attention, both with the same base; window W >= 1, W = None for the
-unsaturated ("direct extension") reading.
+unsaturated reading (phases carried on past the trained range).
 """
 from __future__ import annotations
 

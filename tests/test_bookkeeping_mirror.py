@@ -76,7 +76,7 @@ def test_random_stream_invariants():
 
 
 def test_delete_then_reappend_moves_slot():
-    """Config-1 edit: delete block 3 of 8, re-append it -> a different slot."""
+    """The tiny-cache edit: delete block 3 of 8, re-append it -> a different slot."""
     m = CacheMirror(16, 1, 16)
     for j in range(8):
         assert m.append(0, j) == (0, j)
