@@ -40,11 +40,12 @@ def test_recompute_layer_prefill_matches_oracle(D, H, has_null):
     assert smem.smem_check_device_error(lc.h) == smem.OK
 
 
-@pytest.mark.parametrize("H,D,nblk", [(12, 64, 256), (12, 64, 64), (16, 64, 40), (16, 128, 24)])
+@pytest.mark.parametrize("H,D,nblk", [(12, 64, 256), (12, 64, 64), (16, 64, 40), (16, 128, 24), (16, 32, 64)])
 def test_recompute_prefill_at_model_widths(H, D, nblk):
-    """d = 768 / 1024 / 2048 (the 160M / 410M / 1.5B reader widths): every
-    query-tile width of the kernel (64 queries per CTA at 256 blocks, 32 at
-    64 and 40, 16 at d = 2048)."""
+    """d = 768 / 1024 / 2048 (the 160M / 410M / 1.5B reader widths) and 512:
+    every query-tile width of the kernel (32 queries per CTA at d = 768 and
+    1024, 16 at d = 2048, 64 at d = 512, where two score buffers of 64
+    queries fit tensor memory)."""
     d = H * D
     model = LayerModel(1, d, seed=701 + d)
     lc = LayerCache(model, H, D, max_seqs=1, max_blocks=nblk + 4, capacity=nblk + 4, recompute=True)
@@ -191,10 +192,10 @@ def test_mu_decode_kernel_matches_oracle(has_null):
     assert smem.smem_check_device_error(lc.h) == smem.OK
 
 
-@pytest.mark.parametrize("H,D,nblk", [(4, 64, 7), (12, 64, 40), (16, 64, 20), (16, 128, 12)])
+@pytest.mark.parametrize("H,D,nblk", [(4, 64, 7), (12, 64, 40), (16, 64, 20), (16, 128, 12), (16, 32, 64)])
 def test_mu_prefill_kernel_matches_oracle(H, D, nblk):
     """The block form: H x 64 queries over one row set, every query-tile
-    width (64, 32, 16)."""
+    width (16 at 7 blocks or d = 2048, 32 at d = 768 / 1024, 64 at d = 512)."""
     from tests.gpu_helpers import MAX_ABS, MEAN_ABS
     d = H * D
     model = LayerModel(1, d, seed=1301 + d)
@@ -207,7 +208,9 @@ def test_mu_prefill_kernel_matches_oracle(H, D, nblk):
     got = op.float().cpu().numpy().astype(np.float64)
     _, mus = lc.memory(0, nblk)
     for h in range(H):
-        ref = _oracle_mu(qp[h].double().numpy(), list(mus), lc.nu)
+        q = qp[h].double().numpy()
+        # a few queries at a time keeps the oracle's broadcast rows small
+        ref = np.concatenate([_oracle_mu(q[i:i + 8], list(mus), lc.nu) for i in range(0, B_TOK, 8)])
         err = np.abs(got[h] - ref)
         assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (h, err.max(), err.mean())
 
