@@ -423,15 +423,12 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
   const float* pb = p.part + ((size_t)pd.pair_begin * p.H + pd.h) * (D + 4);
   const size_t ps = (size_t)p.H * (D + 4);
   constexpr int G = 16;  // splits whose loads are in flight together
-  // pass 1: the maximum over the null row and every split
+  // pass 1: the maximum over the null row and every split -- lane i reads
+  // splits i, i + 32, ... and the warp reduces (a maximum is order-free)
   float M = nscore;
-  for (int s0 = 0; s0 < pd.nsplit; s0 += G) {
-    float mv[G];
+  for (int s2 = lane; s2 < pd.nsplit; s2 += 32) M = fmaxf(M, __ldcg(pb + s2 * ps));
 #pragma unroll
-    for (int g = 0; g < G; ++g) mv[g] = s0 + g < pd.nsplit ? __ldcg(pb + (s0 + g) * ps) : -INFINITY;
-#pragma unroll
-    for (int g = 0; g < G; ++g) M = fmaxf(M, mv[g]);
-  }
+  for (int o = 1; o < 32; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
   float Lsum = 0.f, A[CPT];
 #pragma unroll
   for (int e = 0; e < CPT; ++e) A[e] = 0.f;
