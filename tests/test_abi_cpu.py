@@ -193,3 +193,24 @@ def test_recompute_workspace_covers_every_query_tile():
         assert w4 - w0 >= 4 * 32 * 16 * (d + 4) * 4  # 4 items x 32 query rows x 16 splits
     finally:
         smem.smem_cache_destroy(h)
+
+
+def test_memory_row_and_static_scratch_entry_points_need_a_device():
+    """Without a device the memory-row attention entry points and the
+    static-scratch decode refuse with SMEM_ERR_NO_DEVICE before touching any
+    argument; a NULL cache is SMEM_ERR_INVALID_ARG."""
+    import ctypes
+    L = smem.lib()
+    seq = (ctypes.c_int32 * 1)(0)
+    for recompute in (False, True):
+        h = smem.smem_cache_create(smem.make_config(1, 4, 64, 2, 8, 8, recompute_kv=recompute), None)
+        try:
+            assert L.smem_mu_decode(h, 1, seq, seq, None, None, None, 0, None) == smem.ERR_NO_DEVICE
+            assert L.smem_mu_prefill(h, 0, 1, None, None, None, 0, None) == smem.ERR_NO_DEVICE
+            assert L.smem_decode_static_scratch(h, 0, 1, seq, seq, seq, None, None, None, None, None, None,
+                                                None) == smem.ERR_NO_DEVICE
+        finally:
+            smem.smem_cache_destroy(h)
+    assert L.smem_mu_decode(None, 1, seq, seq, None, None, None, 0, None) == smem.ERR_INVALID_ARG
+    assert L.smem_mu_prefill(None, 0, 1, None, None, None, 0, None) == smem.ERR_INVALID_ARG
+    assert L.smem_mu_decode_plan(None, None, None, None) == smem.ERR_INVALID_ARG
