@@ -13,12 +13,14 @@
 // and after this kernel; this kernel streams every row once per layer (2d
 // bytes per row, half the materialized 4 H d_h) and keeps all queries that
 // share a row set in one CTA:
-//   S^T [64 rows][NQ queries] = mu_tile Q'^T   (M = 64, K = d)
+//   S^T [64 rows][NQ queries] = mu_tile Q'^T   (K = d)
 //   O'^T [d][NQ]             += mu_tile^T P^T  (M = 128 per column pair, K = 64)
-// both on the tensor cores (tcgen05, fp32 accumulators in TMEM). A decode
-// step puts the H heads of one sequence in one CTA (NQ = H rounded up to 16);
-// a one-block prefill puts NQ of the block's 64 queries of one head in a
-// CTA. The row tile is streamed twice -- once into a score ring for S,
+// both on the tensor cores (tcgen05, fp32 accumulators in TMEM); the scores
+// are issued as M = 128 MMAs over chunk pairs (see the kernel). A decode step
+// puts up to NQ heads of one sequence in one CTA (NQ = H rounded up to 16,
+// or tiles of heads when the accumulators would not fit); a one-block
+// prefill puts NQ of the block's 64 queries of one head in a CTA. The row
+// tile is streamed twice -- once into a score ring for S,
 // once into a value ring for P.V (the second pass normally hits L2) -- so
 // any d fits in shared memory; the two rings are separate so that value
 // chunks waiting for their tile's softmax never hold up the score stream
@@ -28,7 +30,8 @@
 // its partial (m, l, O'); a second kernel, one CTA per (group, 128 columns),
 // merges the splits in split order, null row first (the null row nu is just
 // one more d-wide row). Reduction orders depend only on the block count, so
-// outputs are bitwise independent of the edit path.
+// outputs are bitwise independent of the edit path. An opt-in decode variant
+// (mu_slice_kernel) splits d across a cluster and reads each tile once.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
