@@ -40,7 +40,7 @@
  *     cuBLAS handle (cuBLAS's own small device state, freed by
  *     smem_cache_destroy); the GEMM workspace there is the caller's too.
  *   - Supported shapes: block_tokens == rows_per_block == 64,
- *     head_dim 64 or 128 (SMEM_ERR_UNSUPPORTED otherwise).
+ *     head_dim 32, 64 or 128 (SMEM_ERR_UNSUPPORTED otherwise).
  *   - At head_dim 64 the one-block prefill runs one thread-block cluster per
  *     head when the device can hold all of them at once (checked at cache
  *     creation; with clusters smaller than 16 CTAs only up to 128 readable
@@ -83,7 +83,7 @@ enum {
 typedef struct smem_config {
     int32_t n_layers;           /* L >= 1                                      */
     int32_t n_heads;            /* H >= 1                                      */
-    int32_t head_dim;           /* d_h: 64 or 128                              */
+    int32_t head_dim;           /* d_h: 32, 64 or 128                          */
     int32_t block_tokens;       /* b: 64                                       */
     int32_t rows_per_block;     /* R: 64                                       */
     int32_t max_seqs;           /* sequence ids are 0 .. max_seqs-1            */
@@ -245,7 +245,13 @@ int smem_decode(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids
  *     SMEM_ERR_SCRATCH_LIMIT before anything is enqueued.
  *   - The first call on each device looks up the array's device address
  *     with that device current; make that first call before any stream
- *     capture on the device.
+ *     capture on the device. The address belongs to the device's current
+ *     context: a call made after that context changed (for instance after
+ *     cudaDeviceReset) looks it up again, so it too should come before any
+ *     capture.
+ *   - It runs the same kernel instance and split plan as smem_decode (the
+ *     grouped units of a grouped-query cache included), so its outputs are
+ *     bitwise equal to smem_decode's on the same cache state.
  *   - Every call on every cache of the process shares the one array, and it
  *     keeps the last call's contents: each call first clears the counters it
  *     needs at zero. Calls whose work overlaps on the GPU (different streams

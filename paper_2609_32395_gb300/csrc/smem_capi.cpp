@@ -786,7 +786,7 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     P.s_stride = P.c_stride = L.H * L.D;
     P.Hkv = L.Hkv;
     P.kv_stride = L.Hkv * L.D;
-    P.qn = 1;
+    P.qn = smem::decode_group_width(L.D, L.H / L.Hkv, L.rope_w != 0);  // the units smem_decode runs
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
     P.rope_tab = rope_tab(c);
     P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);
@@ -801,7 +801,7 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
       if (nblk[i0 + i]) pairs += smem::ceil_div(nblk[i0 + i], smem::decode_split_blocks(nblk[i0 + i]));
     }
     P.n_pairs = pairs;
-    const long long units = (long long)(pairs + n) * L.H;
+    const long long units = (long long)pairs * (L.H / P.qn) + (long long)n * L.H;
     const long long wpc = smem::decode_warps_per_cta();
     const int grid = (int)std::min<long long>((units + wpc - 1) / wpc, smem::decode_max_grid(L.D, c->num_sms));
     if (injected_failure(c)) return SMEM_ERR_CUDA;

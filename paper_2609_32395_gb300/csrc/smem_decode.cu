@@ -910,20 +910,37 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
 static __device__ __align__(256) unsigned char g_decode_static_scratch[SMEM_STATIC_SCRATCH_BYTES];
 
 int static_scratch_address(void** out) {
+  // The address belongs to the device's context: it is looked up once per
+  // (device, context) and looked up again when the current context changed
+  // (e.g. after cudaDeviceReset made a new primary context).
   constexpr int kMaxDevices = 64;
   static std::mutex mu;
   static void* addr[kMaxDevices] = {};
+  static CUcontext owner[kMaxDevices] = {};
+  static PFN_cuCtxGetCurrent_v4000 get_ctx = nullptr;
   int dev = -1;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return (int)e;
   if (dev < 0 || dev >= kMaxDevices) return (int)cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(mu);
-  if (!addr[dev]) {
+  if (!get_ctx) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &fn, 4000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return (int)cudaErrorNotSupported;
+    get_ctx = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(fn);
+  }
+  CUcontext ctx = nullptr;
+  if (get_ctx(&ctx) != CUDA_SUCCESS) return (int)cudaErrorDeviceUninitialized;
+  if (!addr[dev] || !ctx || ctx != owner[dev]) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_decode_static_scratch);  // this device is current
     if (e != cudaSuccess) return (int)e;
     if (!p) return (int)cudaErrorInvalidSymbol;
+    if (get_ctx(&ctx) != CUDA_SUCCESS || !ctx) return (int)cudaErrorDeviceUninitialized;
     addr[dev] = p;
+    owner[dev] = ctx;
   }
   *out = addr[dev];
   return 0;

@@ -199,12 +199,15 @@ def _replay_order(ops, seed):
     return out
 
 
-def test_churn_410m_replay_bitwise():
-    """32 sequences x 512 blocks (H = 16, d_h = 64): a seeded stream of 2000
-    edit / decode ops, a permuted replay reaching the same block set, and a
-    cache built directly from that set give bitwise-identical probe decodes;
-    the probe matches the oracle on sampled heads."""
-    seed, S, N0, H, D = 4, 32, 512, 16, 64
+@pytest.mark.parametrize("N0", [512, 4096])
+def test_churn_410m_replay_bitwise(N0):
+    """32 sequences x 512 or 4096 blocks (H = 16, d_h = 64, one physical
+    layer: 34 GB per cache at 4096): a seeded stream of 2000 edit / decode
+    ops, a permuted replay reaching the same block set, and a cache built
+    directly from that set give bitwise-identical probe decodes; the probe
+    matches the oracle on sampled heads. At 4096 blocks every probe item
+    reads on the long-context split plan."""
+    seed, S, H, D = 4, 32, 16, 64
     ops, live, fresh = _churn_ops(seed, S, N0, 2000)
     n_new = sum(1 for o in ops if o[0] == "app")  # slot headroom for every append
     pool_new = {}
