@@ -38,8 +38,16 @@ def _load():
         lib.oracle_reader_decode.argtypes = [ctypes.c_int] * 4 + [_ip, _dp, _dp, ctypes.c_int, _dp, _dp,
                                                                    ctypes.c_int32, ctypes.c_int] + [_dp] * 8
         lib.oracle_reader_decode.restype = ctypes.c_int
+        lib.oracle_set_threads.argtypes = [ctypes.c_int]
+        lib.oracle_set_threads.restype = ctypes.c_int
         _lib = lib
     return _lib
+
+
+def set_threads(n: int) -> int:
+    """Threads the oracle's per-head loops use (OpenMP); 0 keeps the current
+    setting. Returns the count in effect (1 when built without OpenMP)."""
+    return int(_load().oracle_set_threads(int(n)))
 
 
 def bf16_bits_to_f64(bits) -> np.ndarray:

@@ -23,12 +23,17 @@
  * Each attention is a softmax over its key list with scale 1/sqrt(d_h),
  * computed in two passes (maximum, then exponentials and sums) with the C
  * library's exp in fp64, loops in canonical order. An empty key list gives
- * a zero output. Nothing is blocked, fused or reordered beyond that.
+ * a zero output. Nothing is blocked, fused or reordered beyond that. Heads
+ * are independent: built with OpenMP, the per-head loops spread heads over
+ * threads, each head computed by one thread in the same order as alone.
  */
 #include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 #define ORACLE_ERR_DUPLICATE (-4)
 #define ORACLE_ERR_ALLOC (-12)
@@ -117,6 +122,53 @@ static long ca_rows(int H, int R, int D, int h, int n_sel, const int32_t *order,
     return n;
 }
 
+/* Threads of the per-head loops below (OpenMP when the library was built
+ * with it; each head is computed by one thread exactly as it would be
+ * alone, so the result does not depend on the thread count). Returns the
+ * thread count in effect. */
+int oracle_set_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+    return omp_get_max_threads();
+#else
+    (void)n;
+    return 1;
+#endif
+}
+
+/* The one-block pass of one head (its own row-pointer lists). */
+static int prefill_head(int h, int H, int D, int b, int R, int n_sel, const int32_t *order,
+                        const double *blocks_k, const double *blocks_v,
+                        int has_null, const double *k_null, const double *v_null, long nrows,
+                        const double *qs, const double *ks, const double *vs,
+                        const double *qc, double *osa, double *oca)
+{
+    const double scale = 1.0 / sqrt((double)D);
+    const double **kr, **vr;
+    int t, u, rc = 0;
+    kr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + b + 1));
+    vr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + b + 1));
+    if (!kr || !vr) { free(kr); free(vr); return ORACLE_ERR_ALLOC; }
+    /* self-attention inside the block: query t sees keys 0..t */
+    for (t = 0; t < b && rc == 0; ++t) {
+        for (u = 0; u <= t; ++u) {
+            kr[u] = ks + ((size_t)u * H + h) * D;
+            vr[u] = vs + ((size_t)u * H + h) * D;
+        }
+        rc = attend(D, scale, qs + ((size_t)t * H + h) * D, t + 1, kr, vr,
+                    osa + ((size_t)t * H + h) * D);
+    }
+    /* cross-attention into the rows of strictly earlier blocks */
+    ca_rows(H, R, D, h, n_sel, order, blocks_k, blocks_v, has_null, k_null, v_null, kr, vr);
+    for (t = 0; t < b && rc == 0; ++t)
+        rc = attend(D, scale, qc + ((size_t)t * H + h) * D, nrows, kr, vr,
+                    oca + ((size_t)t * H + h) * D);
+    free(kr);
+    free(vr);
+    return rc;
+}
+
 /*
  * One-block reader pass for one layer (block-skip serving, Sec. 3.1):
  *   qs, ks, vs, qc: [b][H][D] self-attention Q/K/V and cross-attention Q of
@@ -133,39 +185,57 @@ int oracle_reader_prefill(int H, int D, int b, int R,
                           const double *qs, const double *ks, const double *vs,
                           const double *qc, double *osa, double *oca)
 {
-    const double scale = 1.0 / sqrt((double)D);
-    int32_t *order = NULL;
-    const double **kr = NULL, **vr = NULL;
+    int32_t *order;
     long nrows;
-    int n_sel, h, t, u, rc = 0;
+    int n_sel, h, rc = 0;
 
     order = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n_blocks > 0 ? n_blocks : 1));
     if (!order) return ORACLE_ERR_ALLOC;
     n_sel = oracle_rowset(n_blocks, block_idx, q_idx, order);
     if (n_sel < 0) { free(order); return n_sel; }
     nrows = (long)n_sel * R + (has_null ? 1 : 0);
-    kr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + b + 1));
-    vr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + b + 1));
-    if (!kr || !vr) { rc = ORACLE_ERR_ALLOC; goto done; }
-
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
     for (h = 0; h < H; ++h) {
-        /* self-attention inside the block: query t sees keys 0..t */
-        for (t = 0; t < b && rc == 0; ++t) {
-            for (u = 0; u <= t; ++u) {
-                kr[u] = ks + ((size_t)u * H + h) * D;
-                vr[u] = vs + ((size_t)u * H + h) * D;
-            }
-            rc = attend(D, scale, qs + ((size_t)t * H + h) * D, t + 1, kr, vr,
-                        osa + ((size_t)t * H + h) * D);
+        int r = prefill_head(h, H, D, b, R, n_sel, order, blocks_k, blocks_v, has_null, k_null, v_null,
+                             nrows, qs, ks, vs, qc, osa, oca);
+        if (r) {
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+            rc = r;
         }
-        /* cross-attention into the rows of strictly earlier blocks */
-        ca_rows(H, R, D, h, n_sel, order, blocks_k, blocks_v, has_null, k_null, v_null, kr, vr);
-        for (t = 0; t < b && rc == 0; ++t)
-            rc = attend(D, scale, qc + ((size_t)t * H + h) * D, nrows, kr, vr,
-                        oca + ((size_t)t * H + h) * D);
     }
-done:
     free(order);
+    return rc;
+}
+
+/* The decode step of one head (its own row-pointer lists). */
+static int decode_head(int h, int H, int D, int R, int n_sel, const int32_t *order,
+                       const double *blocks_k, const double *blocks_v,
+                       int has_null, const double *k_null, const double *v_null, long nrows, int p,
+                       const double *kin, const double *vin,
+                       const double *qs, const double *k_new, const double *v_new,
+                       const double *qc, double *osa, double *oca)
+{
+    const double scale = 1.0 / sqrt((double)D);
+    const double **kr, **vr;
+    int u, rc;
+    kr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + p + 2));
+    vr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + p + 2));
+    if (!kr || !vr) { free(kr); free(vr); return ORACLE_ERR_ALLOC; }
+    for (u = 0; u < p; ++u) {
+        kr[u] = kin + ((size_t)u * H + h) * D;
+        vr[u] = vin + ((size_t)u * H + h) * D;
+    }
+    kr[p] = k_new + (size_t)h * D;
+    vr[p] = v_new + (size_t)h * D;
+    rc = attend(D, scale, qs + (size_t)h * D, p + 1, kr, vr, osa + (size_t)h * D);
+    if (rc == 0) {
+        ca_rows(H, R, D, h, n_sel, order, blocks_k, blocks_v, has_null, k_null, v_null, kr, vr);
+        rc = attend(D, scale, qc + (size_t)h * D, nrows, kr, vr, oca + (size_t)h * D);
+    }
     free(kr);
     free(vr);
     return rc;
@@ -188,36 +258,28 @@ int oracle_reader_decode(int H, int D, int R,
                          const double *qs, const double *k_new, const double *v_new,
                          const double *qc, double *osa, double *oca)
 {
-    const double scale = 1.0 / sqrt((double)D);
-    int32_t *order = NULL;
-    const double **kr = NULL, **vr = NULL;
+    int32_t *order;
     long nrows;
-    int n_sel, h, u, rc = 0;
+    int n_sel, h, rc = 0;
 
     order = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n_blocks > 0 ? n_blocks : 1));
     if (!order) return ORACLE_ERR_ALLOC;
     n_sel = oracle_rowset(n_blocks, block_idx, q_idx, order);
     if (n_sel < 0) { free(order); return n_sel; }
     nrows = (long)n_sel * R + (has_null ? 1 : 0);
-    kr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + p + 2));
-    vr = (const double **)malloc(sizeof(double *) * (size_t)(nrows + p + 2));
-    if (!kr || !vr) { rc = ORACLE_ERR_ALLOC; goto done; }
-
-    for (h = 0; h < H && rc == 0; ++h) {
-        for (u = 0; u < p; ++u) {
-            kr[u] = kin + ((size_t)u * H + h) * D;
-            vr[u] = vin + ((size_t)u * H + h) * D;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+    for (h = 0; h < H; ++h) {
+        int r = decode_head(h, H, D, R, n_sel, order, blocks_k, blocks_v, has_null, k_null, v_null, nrows,
+                            p, kin, vin, qs, k_new, v_new, qc, osa, oca);
+        if (r) {
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+            rc = r;
         }
-        kr[p] = k_new + (size_t)h * D;
-        vr[p] = v_new + (size_t)h * D;
-        rc = attend(D, scale, qs + (size_t)h * D, p + 1, kr, vr, osa + (size_t)h * D);
-        if (rc) break;
-        ca_rows(H, R, D, h, n_sel, order, blocks_k, blocks_v, has_null, k_null, v_null, kr, vr);
-        rc = attend(D, scale, qc + (size_t)h * D, nrows, kr, vr, oca + (size_t)h * D);
     }
-done:
     free(order);
-    free(kr);
-    free(vr);
     return rc;
 }
