@@ -34,6 +34,7 @@ WORKLOAD = dict(name="410M-shaped batched decode", L=24, H=16, D=64, seqs=64, ct
 R = 64
 B_TOK = 64
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0  # the nominal HBM3e bandwidth (context beside the measured copy peak)
 
 
 def parse_args():
@@ -50,6 +51,7 @@ def parse_args():
     ap.add_argument("--no-rope", action="store_true", help="skip the rotary-phase (RoPE composite) cells")
     ap.add_argument("--no-d32", action="store_true", help="skip the d_h = 32 decode cell")
     ap.add_argument("--no-gqa", action="store_true", help="skip the grouped-query decode cell")
+    ap.add_argument("--no-long", action="store_true", help="skip the bounded 1.5B long-context cells")
     ap.add_argument("--workload", default="decode", choices=["decode", "long"],
                     help="long: the 1.5B-shaped long-context cells (prefill latency, decode tok/s)")
     ap.add_argument("--long-batches", default="1,16", help="batches of the long-context cells")
@@ -394,7 +396,7 @@ def layer_decode_step(wl, stack, x, ws, mu, events=None):
     """One decode token for every sequence through all layers of the full
     reader layer (LayerNorm, projections, attention, FFN); a finished block
     is appended from synthetic memory rows through the layer's key/value
-    maps. Returns (our kernel launches, cuBLAS calls)."""
+    maps. Returns the number of kernel launches."""
     import torch
 
     from paper_2609_32395_gb300 import smem
@@ -407,17 +409,16 @@ def layer_decode_step(wl, stack, x, ws, mu, events=None):
                                       stack.sw[layer], x, ws)
     if events is not None:
         events[1].record(st)
-    ours, blas = 6 * wl.L, 6 * wl.L  # 3 LayerNorm, GELU, 2 attention; 6 GEMMs per layer
+    ours = 8 * wl.L  # per layer: 6 projections (LayerNorm, GELU, residual fused) and 2 attention launches
     wl.pos += 1
     for s in np.nonzero(wl.pos == B_TOK)[0]:
         smem.smem_append_block_rows(wl.h, int(s), int(wl.nblk[s]), mu, stack.sw, ws)
-        ours += 1
-        blas += 2 * wl.L
+        ours += 1 + 2 * wl.L  # key and value projections of every layer, then the table insert
         wl.new_used[s] += 1
         wl.nblk[s] += 1
         wl.pos[s] = 0
     wl.step_no += 1
-    return ours, blas
+    return ours
 
 
 def measure_layer_decode(wl, steps, warmup, device):
@@ -439,12 +440,11 @@ def measure_layer_decode(wl, steps, warmup, device):
         layer_decode_step(wl, stack, x, ws, mu)
     torch.cuda.synchronize()
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
-    rows, ours, blas = [], 0, 0
+    rows, ours = [], 0
     for i in range(steps):
         x.copy_(x0)
         rows.append(wl.rows_read())
-        o, b = layer_decode_step(wl, stack, x, ws, mu, events=ev[i])
-        ours, blas = ours + o, blas + b
+        ours += layer_decode_step(wl, stack, x, ws, mu, events=ev[i])
     torch.cuda.synchronize()
     if smem.smem_check_device_error(wl.h) != smem.OK:
         raise RuntimeError("device error recorded during the full-layer decode")
@@ -456,7 +456,7 @@ def measure_layer_decode(wl, steps, warmup, device):
     alg = kv + w + act
     return {"tok_per_s": wl.S / (step_ms / 1e3), "step_ms": step_ms, "step_ms_p50": float(np.median(ms)),
             "alg_bytes_per_step": alg, "weight_bytes_per_step": w, "kv_bytes_per_step": kv,
-            "achieved_gbs": alg / (step_ms / 1e3) / 1e9, "our_launches": ours, "cublas_calls": blas,
+            "achieved_gbs": alg / (step_ms / 1e3) / 1e9, "launches": ours,
             "timing": "CUDA events around the layer calls of each step (appends excluded), inputs resident"}
 
 
@@ -784,7 +784,7 @@ def measure_layer_serve(nblk, device, iters=30, flush_bytes=512 << 20, recompute
     out = {"context_blocks": nblk, "latency_ms": med, "latency_ms_min": lat[0], "alg_bytes": alg,
            "weight_bytes": w, "kv_bytes": kv, "achieved_gbs": alg / (med / 1e3) / 1e9,
            "flops": stack.flops_per_layer(B_TOK) * wl.L + wl.flops_per_launch() * wl.L,
-           "launches_per_serve": {"ours": 7 * wl.L, "cublas": 6 * wl.L}}
+           "launches_per_serve": 8 * wl.L}
     wl.cache.close()
     return out
 
@@ -794,137 +794,150 @@ LONG = dict(name="1.5B-shaped long cached context", L=24, H=16, D=128, contexts=
             seed=2)
 
 
-def run_long(args):
-    """One-block prefill latency and decode tok/s per context length at the
-    1.5B reader shape. Each batch builds one cache at the longest context;
-    shorter contexts read its block prefix (block-causal mask). Layers that
-    do not fit in HBM are emulated: the 24 logical layers cycle over the
-    physical layers that fit (per-layer working set >> L2)."""
+def long_batch_cells(batch, contexts, device, peak, bf16_peak, layers_cap=None, serve_iters=6, n_steps=8):
+    """Cells of one batch size: a cache at the longest context (1.5B reader
+    shape, shuffled slots) whose shorter contexts read its block prefix
+    (block-causal mask); decode tok/s and kernel HBM fraction per context and,
+    at batch 1, the 24-layer one-block serve latency and the prefill kernel's
+    HBM and tensor fractions. Layers that do not fit (or above `layers_cap`)
+    are emulated: the 24 logical layers cycle over the physical ones (each
+    physical layer's working set is far above L2)."""
     import torch
 
     import synth
+    from paper_2609_32395_gb300 import smem
+
+    W = LONG
+    H, D, L = W["H"], W["D"], W["L"]
+    nmax = max(contexts)
+    block_bytes = 2 * H * R * D * 2  # K and V of one layer
+    free, _ = torch.cuda.mem_get_info()
+    budget = free - (16 << 30)
+    l_phys = max(1, min(L, budget // (batch * (nmax + 8) * block_bytes)))
+    if layers_cap:
+        l_phys = min(l_phys, layers_cap)
+    l_phys = int(l_phys)
+    cap = batch * (nmax + 4)
+    cfg = smem.make_config(l_phys, H, D, batch, nmax + 4, cap,
+                           free_order=synth.slot_permutation(W["seed"] + batch, cap))
+    cache = smem.SmemCache(cfg, device=device)
+    for s in range(batch):
+        for b0 in range(0, nmax, 16):
+            ids = list(range(b0, min(nmax, b0 + 16)))
+            K, V = synth.block_rows_torch(W["seed"], s, ids, l_phys, H, R, D, device)
+            for i, j in enumerate(ids):
+                smem.smem_append_block(cache.h, s, j, K[i], V[i])
+            del K, V
+    shape = (batch, H, D)
+    dins = [synth.tensor_torch(W["seed"], k, shape, 0, 0, device=device)
+            for k in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
+    osa = torch.empty(shape, dtype=torch.bfloat16, device=device)
+    oca = torch.empty_like(osa)
+    pshape = (B_TOK, H, D)
+    pins = [synth.tensor_torch(W["seed"], k, pshape, 0, 0, device=device)
+            for k in (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+    posa = torch.empty(pshape, dtype=torch.bfloat16, device=device)
+    poca = torch.empty_like(posa)
+    seqs = np.arange(batch, dtype=np.int32)
+    st = torch.cuda.current_stream()
+    cells = []
+    for ctx in contexts:
+        qidx = np.full(batch, ctx, dtype=np.int32)
+        pos = np.zeros(batch, dtype=np.int32)
+        for _ in range(2):
+            for layer in range(L):
+                smem.smem_decode(cache.h, layer % l_phys, seqs, pos, qidx, *dins, osa, oca)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * L * n_steps)]
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        t0.record(st)
+        for i in range(n_steps):
+            for layer in range(L):
+                ev[2 * (i * L + layer)].record(st)
+                smem.smem_decode(cache.h, layer % l_phys, seqs, pos, qidx, *dins, osa, oca)
+                ev[2 * (i * L + layer) + 1].record(st)
+        t1.record(st)
+        torch.cuda.synchronize()
+        step_ms = t0.elapsed_time(t1) / n_steps
+        kms = float(np.mean([ev[2 * k].elapsed_time(ev[2 * k + 1]) for k in range(L * n_steps)]))
+        dec_bytes = batch * (ctx * R + 1) * 4 * H * D
+        cell = {"batch": batch, "context_blocks": ctx, "memory_rows": ctx * R,
+                "layers_physical": l_phys, "layers_logical": L,
+                "emulated": bool(l_phys < L),
+                "decode_tok_s": batch / (step_ms / 1e3), "decode_ms_per_step": step_ms,
+                "decode_kernel_ms": kms, "decode_gbs": dec_bytes / (kms / 1e3) / 1e9,
+                "decode_hbm_frac": dec_bytes / (kms / 1e3) / 1e9 / peak,
+                "decode_hbm_frac_nominal_8tbs": dec_bytes / (kms / 1e3) / 1e9 / NOMINAL_HBM_GBS}
+        if batch == 1:
+            # one-block cached serve: 24 prefill launches, graph-replayed, L2 flushed
+            def serve():
+                for layer in range(L):
+                    smem.smem_prefill_block(cache.h, 0, layer % l_phys, ctx, *pins, posa, poca)
+
+            serve()
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                serve()
+            flush = torch.empty(512 << 20, dtype=torch.uint8, device=device)
+            lat, kern = [], []
+            for i in range(serve_iters):
+                flush.zero_()
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(st)
+                g.replay()
+                b.record(st)
+                torch.cuda.synchronize()
+                lat.append(a.elapsed_time(b))
+            for i in range(serve_iters):
+                flush.zero_()
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(st)
+                smem.smem_prefill_block(cache.h, 0, i % l_phys, ctx, *pins, posa, poca)
+                b.record(st)
+                torch.cuda.synchronize()
+                kern.append(a.elapsed_time(b))
+            del g, flush
+            pf_bytes = ctx * R * 4 * H * D + 6 * B_TOK * H * D * 2
+            pf_flops = 4 * B_TOK * ctx * R * H * D + 4 * (B_TOK * (B_TOK + 1) // 2) * H * D
+            km = float(np.median(kern))
+            cell.update({"serve_latency_ms": float(np.median(lat)), "prefill_kernel_ms": km,
+                         "prefill_gbs": pf_bytes / (km / 1e3) / 1e9,
+                         "prefill_hbm_frac": pf_bytes / (km / 1e3) / 1e9 / peak,
+                         "prefill_tflops": pf_flops / (km / 1e3) / 1e12,
+                         "prefill_tensor_frac": pf_flops / (km / 1e3) / 1e12 / bf16_peak})
+        cells.append(cell)
+    if smem.smem_check_device_error(cache.h) != smem.OK:
+        raise RuntimeError("device error recorded")
+    cache.close()
+    cache.buf = None
+    torch.cuda.empty_cache()
+    return cells
+
+
+def run_long(args):
+    """One-block prefill latency and decode tok/s per context length at the
+    1.5B reader shape, every batch and context of the workload."""
+    import torch
+
     from paper_2609_32395_gb300 import smem
 
     torch.cuda.set_device(0)
     device = torch.device("cuda", 0)
     smem.lib()
     W = LONG
-    H, D, L = W["H"], W["D"], W["L"]
     contexts = [int(x) for x in args.long_contexts.split(",")]
     batches = [int(x) for x in args.long_batches.split(",")]
-    nmax = max(contexts)
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     bf16_peak = float(peaks.get("bf16_tflops", 1900.0))
-    block_bytes = 2 * H * R * D * 2  # K and V of one layer
     cells = []
     for batch in batches:
-        free, _ = torch.cuda.mem_get_info()
-        budget = free - (16 << 30)
-        l_phys = max(1, min(L, budget // (batch * (nmax + 8) * block_bytes)))
-        if args.long_layers:
-            l_phys = min(l_phys, args.long_layers)
-        cap = batch * (nmax + 4)
-        cfg = smem.make_config(int(l_phys), H, D, batch, nmax + 4, cap,
-                               free_order=synth.slot_permutation(W["seed"] + batch, cap))
-        cache = smem.SmemCache(cfg, device=device)
-        for s in range(batch):
-            for b0 in range(0, nmax, 16):
-                ids = list(range(b0, min(nmax, b0 + 16)))
-                K, V = synth.block_rows_torch(W["seed"], s, ids, int(l_phys), H, R, D, device)
-                for i, j in enumerate(ids):
-                    smem.smem_append_block(cache.h, s, j, K[i], V[i])
-                del K, V
-        shape = (batch, H, D)
-        dins = [synth.tensor_torch(W["seed"], k, shape, 0, 0, device=device)
-                for k in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
-        osa = torch.empty(shape, dtype=torch.bfloat16, device=device)
-        oca = torch.empty_like(osa)
-        pshape = (B_TOK, H, D)
-        pins = [synth.tensor_torch(W["seed"], k, pshape, 0, 0, device=device)
-                for k in (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
-        posa = torch.empty(pshape, dtype=torch.bfloat16, device=device)
-        poca = torch.empty_like(posa)
-        seqs = np.arange(batch, dtype=np.int32)
-        st = torch.cuda.current_stream()
-        for ctx in contexts:
-            qidx = np.full(batch, ctx, dtype=np.int32)
-            pos = np.zeros(batch, dtype=np.int32)
-
-            def step():
-                for layer in range(L):
-                    smem.smem_decode(cache.h, layer % int(l_phys), seqs, pos, qidx, *dins, osa, oca)
-
-            for _ in range(2):
-                step()
-            n_steps = 8
-            ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * L * n_steps)]
-            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            torch.cuda.synchronize()
-            t0.record(st)
-            for i in range(n_steps):
-                for layer in range(L):
-                    ev[2 * (i * L + layer)].record(st)
-                    smem.smem_decode(cache.h, layer % int(l_phys), seqs, pos, qidx, *dins, osa, oca)
-                    ev[2 * (i * L + layer) + 1].record(st)
-            t1.record(st)
-            torch.cuda.synchronize()
-            step_ms = t0.elapsed_time(t1) / n_steps
-            kms = float(np.mean([ev[2 * k].elapsed_time(ev[2 * k + 1]) for k in range(L * n_steps)]))
-            dec_bytes = batch * (ctx * R + 1) * 4 * H * D
-            cell = {"batch": batch, "context_blocks": ctx, "memory_rows": ctx * R,
-                    "layers_physical": int(l_phys), "layers_logical": L,
-                    "emulated": bool(l_phys < L),
-                    "decode_tok_s": batch / (step_ms / 1e3), "decode_ms_per_step": step_ms,
-                    "decode_kernel_ms": kms, "decode_gbs": dec_bytes / (kms / 1e3) / 1e9,
-                    "decode_hbm_frac": dec_bytes / (kms / 1e3) / 1e9 / peak}
-            if batch == 1:
-                # one-block cached serve: 24 prefill launches, graph-replayed, L2 flushed
-                def serve():
-                    for layer in range(L):
-                        smem.smem_prefill_block(cache.h, 0, layer % int(l_phys), ctx, *pins, posa, poca)
-
-                serve()
-                torch.cuda.synchronize()
-                g = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(g):
-                    serve()
-                flush = torch.empty(512 << 20, dtype=torch.uint8, device=device)
-                lat, kern = [], []
-                for i in range(6):
-                    flush.zero_()
-                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                    a.record(st)
-                    g.replay()
-                    b.record(st)
-                    torch.cuda.synchronize()
-                    lat.append(a.elapsed_time(b))
-                for i in range(6):
-                    flush.zero_()
-                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                    a.record(st)
-                    smem.smem_prefill_block(cache.h, 0, i % int(l_phys), ctx, *pins, posa, poca)
-                    b.record(st)
-                    torch.cuda.synchronize()
-                    kern.append(a.elapsed_time(b))
-                del g, flush
-                pf_bytes = ctx * R * 4 * H * D + 6 * B_TOK * H * D * 2
-                pf_flops = 4 * B_TOK * ctx * R * H * D + 4 * (B_TOK * (B_TOK + 1) // 2) * H * D
-                km = float(np.median(kern))
-                cell.update({"serve_latency_ms": float(np.median(lat)), "prefill_kernel_ms": km,
-                             "prefill_gbs": pf_bytes / (km / 1e3) / 1e9,
-                             "prefill_hbm_frac": pf_bytes / (km / 1e3) / 1e9 / peak,
-                             "prefill_tflops": pf_flops / (km / 1e3) / 1e12,
-                             "prefill_tensor_frac": pf_flops / (km / 1e3) / 1e12 / bf16_peak})
+        for cell in long_batch_cells(batch, contexts, device, peak, bf16_peak, layers_cap=args.long_layers):
             cells.append(cell)
             print(json.dumps(cell), file=sys.stderr, flush=True)
-        if smem.smem_check_device_error(cache.h) != smem.OK:
-            raise RuntimeError("device error recorded")
-        cache.close()
-        cache.buf = None
-        torch.cuda.empty_cache()
-    print(json.dumps({"workload": W["name"], "heads": H, "head_dim": D, "layers": L, "peak_hbm_gbs": peak,
-                      "peak_source": peak_src, "cells": cells}), flush=True)
+    print(json.dumps({"workload": W["name"], "heads": W["H"], "head_dim": W["D"], "layers": W["L"],
+                      "peak_hbm_gbs": peak, "peak_source": peak_src, "cells": cells}), flush=True)
 
 
 # ----------------------------------------------------------------------------- edit latency
@@ -1015,7 +1028,7 @@ class OracleDecodeSample:
                      for kind in (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
                 self.calls.append(dict(idx=np.arange(n), mk=f(rows[0]), mv=f(rows[1]), n=n, p=p, kin=f(kin),
                                        vin=f(vin), q=[f(x) for x in q], rows=n * R + p + 1))
-        self.desc = (f"fp64 C oracle, single thread: decode calls (all {H} heads, full contexts) of sequences "
+        self.desc = (f"fp64 C oracle: decode calls (all {H} heads, full contexts) of sequences "
                      f"0..{min(n_seqs, seqs) - 1} at layers {list(layers)}, repeated; time per memory row "
                      f"extrapolated to the workload's mean context and {self.L} layers per token")
 
@@ -1033,17 +1046,156 @@ class OracleDecodeSample:
         return 1.0 / (per_row * self.mean_rows * self.L)
 
 
-def oracle_baseline(seqs, budget_s=12.0):
+def _time_threads(fn, threads):
+    """Wall time of fn() with the oracle's per-head loops on `threads`."""
+    import oracle
+
+    used = oracle.set_threads(threads)
+    t0 = time.perf_counter()
+    fn()
+    return time.perf_counter() - t0, used
+
+
+def _oracle_block_rows(seed, seq, ids, layer, H, D, device):
+    """fp64 host copies [n][H][R][D] of memory rows from the seeded
+    generator (run on the device for speed; the values are the generator's,
+    bit for bit the numpy ones)."""
+    import synth
+
+    K, V = synth.block_rows_torch(seed, seq, list(ids), 1, H, R, D, device, layers=[layer])
+    return K[:, 0].double().cpu().numpy(), V[:, 0].double().cpu().numpy()
+
+
+def oracle_config_baselines(device, ncores):
+    """The fp64 oracle on every workload of the benchmark's configuration
+    list, single-threaded and with OpenMP over heads on `ncores` threads.
+    Configs 1 and 2 run in full; configs 3-5 on a stated sample, extrapolated
+    linearly in memory rows, heads and layers (labelled)."""
+    import oracle
+    import synth
+    from oracle.bookkeeping import CacheMirror
+
+    f = oracle.bf16_bits_to_f64
+    out = {}
+
+    def both(fn):
+        t1, _ = _time_threads(fn, 1)
+        tn, used = _time_threads(fn, ncores)
+        return t1, tn, used
+
+    # config 1: tiny reader (H 4, d_h 64, 8 blocks): one-block pass and a decode, in full
+    H, D, n = 4, 64, 8
+    mk, mv = _oracle_block_rows(0, 0, range(n), 0, H, D, device)
+    pin = [f(synth.tensor_np(0, k, (B_TOK, H, D), 0, 1)) for k in
+           (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+    t1, tn, used = both(lambda: oracle.reader_prefill(np.arange(n), mk, mv, n, *pin))
+    out["tiny"] = {"what": "one-block pass, H 4, d_h 64, 8 blocks (full)", "unit": "ms",
+                   "single_thread": 1e3 * t1, "openmp": 1e3 * tn, "threads": used}
+
+    # config 2: 160M one-block serve, 12 layers, 16 / 64 / 256 blocks; OpenMP
+    # in full, single thread in full at 16 / 64 blocks and on layers {0, 11}
+    # at 256 blocks (x6, labelled)
+    H, D, L = SERVE["H"], SERVE["D"], SERVE["L"]
+    cells = []
+    for nblk in SERVE["contexts"]:
+        t1 = tn = 0.0
+        single_layers = range(L) if nblk <= 64 else (0, L - 1)
+        for layer in range(L):
+            mk, mv = _oracle_block_rows(SERVE["seed"], 0, range(nblk), layer, H, D, device)
+            pin = [f(synth.tensor_np(SERVE["seed"], k, (B_TOK, H, D), layer, 0)) for k in
+                   (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+            fn = lambda: oracle.reader_prefill(np.arange(nblk), mk, mv, nblk, *pin)  # noqa: E731
+            if layer in single_layers:
+                t1 += _time_threads(fn, 1)[0]
+            b, used = _time_threads(fn, ncores)
+            tn += b
+        cell = {"context_blocks": nblk, "single_thread_ms": 1e3 * t1 * L / len(single_layers), "openmp_ms": 1e3 * tn}
+        if len(single_layers) < L:
+            cell["single_thread_extrapolated"] = f"layers {list(single_layers)} x {L / len(single_layers):g}"
+        cells.append(cell)
+    out["serve_160m"] = {"what": f"one-block serve, {L} layers, H {H}, d_h {D} (OpenMP: full)", "threads": used,
+                         "unit": "ms", "cells": cells}
+
+    # config 4: 1.5B long context; sample: layer 0 at 512 blocks (one-block
+    # pass: every head with OpenMP, heads 0-1 single-threaded; batch-1 decode:
+    # every head), extrapolated per memory row, head and layer to 24 layers
+    H, D, L, n = LONG["H"], LONG["D"], LONG["L"], 512
+    mk, mv = _oracle_block_rows(LONG["seed"], 0, range(n), 0, H, D, device)
+    pin = [f(synth.tensor_np(LONG["seed"], k, (B_TOK, H, D), 0, 0)) for k in
+           (synth.KIND_QS, synth.KIND_KS, synth.KIND_VS, synth.KIND_QC)]
+    dq = [f(synth.tensor_np(LONG["seed"], k, (1, H, D), 0, 0))[0] for k in
+          (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
+    mk2, mv2 = np.ascontiguousarray(mk[:, :2]), np.ascontiguousarray(mv[:, :2])
+    pin2 = [np.ascontiguousarray(x[:, :2]) for x in pin]
+    p1 = _time_threads(lambda: oracle.reader_prefill(np.arange(n), mk2, mv2, n, *pin2), 1)[0] * H / 2
+    pn, used = _time_threads(lambda: oracle.reader_prefill(np.arange(n), mk, mv, n, *pin), ncores)
+    d1, dn, _ = both(lambda: oracle.reader_decode(np.arange(n), mk, mv, n, 0, None, None, *dq))
+    cells = []
+    for ctx in LONG["contexts"]:
+        k = ctx / n * L
+        cells.append({"context_blocks": ctx, "serve_single_thread_ms": 1e3 * p1 * k, "serve_openmp_ms": 1e3 * pn * k,
+                      "decode_single_thread_tok_s": 1.0 / (d1 * k), "decode_openmp_tok_s": 1.0 / (dn * k)})
+    out["long_1p5b"] = {"what": f"H {H}, d_h {D}, {L} layers; sample: layer 0 at {n} blocks, one-block pass "
+                                f"(single thread: heads 0-1) and batch-1 decode; extrapolated per memory row, head "
+                                f"and layer", "extrapolated": True, "threads": used, "cells": cells}
+
+    # config 5: churn at the 410M shape; the oracle's bookkeeping mirror times its
+    # deletes, the attention oracle one sequence's decode at 4096 blocks (layer 0)
+    H, D = EDIT["H"], EDIT["D"]
+    cells = []
+    for ctx in EDIT["contexts"]:
+        m = CacheMirror(EDIT["seqs"] * (ctx + 8), EDIT["seqs"], ctx + 8)
+        for sq in range(EDIT["seqs"]):
+            for j in range(ctx):
+                m.append(sq, j)
+        rng = np.random.default_rng(ctx)
+        victims = [(int(rng.integers(0, EDIT["seqs"])), int(j)) for j in rng.choice(ctx, 200, replace=False)]
+        t0 = time.perf_counter()
+        for sq, j in victims:
+            m.delete(sq, j)
+        cells.append({"context_blocks": ctx, "mirror_delete_us": 1e6 * (time.perf_counter() - t0) / len(victims)})
+    n = max(EDIT["contexts"])
+    mk, mv = _oracle_block_rows(EDIT["seed"], 0, range(n), 0, H, D, device)
+    dq = [f(synth.tensor_np(EDIT["seed"], k, (1, H, D), 0, 0))[0] for k in
+          (synth.KIND_QDEC_S, synth.KIND_KNEW, synth.KIND_VNEW, synth.KIND_QDEC_C)]
+    d1, dn, used = both(lambda: oracle.reader_decode(np.arange(n), mk, mv, n, 0, None, None, *dq))
+    out["churn_410m"] = {"what": f"bookkeeping mirror deletes (32 sequences); decode of one sequence at {n} blocks, "
+                                 "one layer, all heads", "threads": used, "cells": cells,
+                         "decode_ms_single_thread": 1e3 * d1, "decode_ms_openmp": 1e3 * dn}
+    return out
+
+
+def oracle_baseline(seqs, device=None, budget_s=10.0, configs=True):
+    """The headline (config 3) oracle time, single-threaded and with OpenMP
+    over heads on every host core, plus the per-config table."""
+    import oracle
+
+    ncores = os.cpu_count() or 1
     samp = OracleDecodeSample(seqs)
-    secs = rows = 0.0
-    n = 0
-    while secs < budget_s or n < len(samp.calls):
-        t, r = samp.call(n)
-        secs += t
-        rows += r
-        n += 1
-    return {"value": samp.tok_per_s(secs, rows), "unit": "tok/s", "cores": 1, "kind": "oracle",
-            "sample": f"{samp.desc}; {n} calls, {secs:.1f} s"}
+
+    def timed(threads, budget):
+        used = oracle.set_threads(threads)
+        secs = rows = 0.0
+        n = 0
+        while secs < budget or n < len(samp.calls):
+            t, r = samp.call(n)
+            secs += t
+            rows += r
+            n += 1
+        return samp.tok_per_s(secs, rows), used, n, secs
+
+    v1, _, n1, s1 = timed(1, budget_s)
+    vn, used, nn, sn = timed(ncores, budget_s / 2)
+    desc = samp.desc.replace("single thread: ", "")
+    res = {"value": vn, "unit": "tok/s", "cores": used, "kind": "oracle",
+           "sample": f"{desc}; OpenMP over heads on {used} threads ({ncores} host cores); {nn} calls, "
+                     f"{sn:.1f} s; extrapolated",
+           "single_thread": {"value": v1, "unit": "tok/s", "cores": 1, "calls": n1, "seconds": s1},
+           "host_cores": ncores}
+    if configs and device is not None:
+        res["configs"] = oracle_config_baselines(device, ncores)
+    oracle.set_threads(ncores)
+    return res
 
 
 # ----------------------------------------------------------------------------- arms
@@ -1051,8 +1203,11 @@ def run_reference(args):
     ws, rank, _ = dist_env()
     if rank != 0:
         return
+    import oracle
+
     W = WORKLOAD
     samp = OracleDecodeSample(args.seqs)
+    used = oracle.set_threads(os.cpu_count() or 1)
     secs = rows = 0.0
     for i in range(args.warmup + args.steps):
         t, r = samp.call(i)
@@ -1066,8 +1221,8 @@ def run_reference(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": W["name"], "layers": W["L"], "heads": W["H"], "head_dim": W["D"],
                    "sequences": args.seqs, "context_blocks": [W["ctx_lo"], W["ctx_hi"]], "block": B_TOK},
-        "cpu_baseline": {"value": value, "unit": "tok/s", "cores": 1, "kind": "oracle",
-                         "sample": f"each step one call; {samp.desc}"},
+        "cpu_baseline": {"value": value, "unit": "tok/s", "cores": used, "kind": "oracle",
+                         "sample": f"each step one call; OpenMP over heads on {used} threads; {samp.desc}"},
         "e2e": {"value": value, "unit": "tok/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -1194,6 +1349,17 @@ def run_ours(args):
         if rope is not None:
             rope["serve"] = [measure_serve(n, device, rope_window=ROPE_WINDOW) for n in SERVE["contexts"]]
     edit = None if args.no_serve else [measure_edit_latency(n, device) for n in EDIT["contexts"]]
+    long_cells = None
+    if not args.no_long and rank == 0:
+        # the 1.5B long-context cells, bounded: batch 1 at 1024 and 4096 blocks
+        # and batch 16 at 1024, on two physical layers (24-layer emulated)
+        wl.cache.close()
+        wl.cache.buf = None
+        torch.cuda.empty_cache()
+        pk, _ = measured_peaks()
+        hbm, tf = float(pk.get("hbm_gbs", FALLBACK_HBM_GBS)), float(pk.get("bf16_tflops", 1900.0))
+        long_cells = long_batch_cells(1, [1024, 4096], device, hbm, tf, layers_cap=2)
+        long_cells += long_batch_cells(16, [1024], device, hbm, tf, layers_cap=2)
 
     if rank != 0:
         if ws > 1:
@@ -1206,7 +1372,7 @@ def run_ours(args):
     peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     units_launch = float(np.mean(rows))
     traffic = profiled_traffic("decode_410m.txt", units_launch)
-    cpu = None if args.no_cpu_baseline else oracle_baseline(args.seqs)
+    cpu = None if args.no_cpu_baseline else oracle_baseline(args.seqs, device)
     line = {
         "metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
@@ -1217,7 +1383,7 @@ def run_ours(args):
                    "l2": "inputs larger than L2 (pool of memory rows >> 129 MB); no flush",
                    "parallelism": f"independent sequences per GPU x{ws}"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": traffic,
+                     "frac": achieved / peak, "frac_nominal_8tbs": achieved / NOMINAL_HBM_GBS, "traffic": traffic,
                      "kernel": "decode_kernel<64> (split-K paged cross-attention + in-block self-attention)",
                      "peak_source": f"{peak_src} hbm_gbs", "kernel_ms_mean": float(np.mean(kern_ms)),
                      "alg_bytes_per_launch": float(np.mean(alg_bytes))},
@@ -1239,7 +1405,8 @@ def run_ours(args):
                          "cells": serve}
     if layer_dec or layer_serve:
         layer = {"what": "full reader layer: pre-LN self-attention, cross-attention and 4d GELU FFN "
-                         "branches with random-init bf16 weights (projections on cuBLAS)"}
+                         "branches with random-init bf16 weights (projections on the library's tcgen05 "
+                         "kernel, LayerNorm / residual / GELU fused)"}
         if layer_dec:
             layer_dec["hbm_frac"] = layer_dec["achieved_gbs"] / peak
             layer["decode"] = dict(workload=WORKLOAD["name"], unit="tok/s", steps=layer_steps, **layer_dec)
@@ -1279,6 +1446,12 @@ def run_ours(args):
     if edit:
         line["edit"] = {"workload": EDIT["name"], "unit": "us",
                         "note": "host = whole C ABI call; device = table-edit kernel; no row moves", "cells": edit}
+    if long_cells:
+        line["long"] = {"workload": LONG["name"], "heads": LONG["H"], "head_dim": LONG["D"], "layers": LONG["L"],
+                        "note": "24 logical layers cycled over 2 physical layers (24-layer emulated; each "
+                                "physical layer's K/V far above L2); fractions of the measured HBM copy peak and "
+                                "of the measured bf16 burst peak",
+                        "cells": long_cells}
     if e2e:
         line["e2e"] = e2e
     if cpu:

@@ -35,10 +35,8 @@
  *     as it was. No C++ exception crosses this interface.
  *   - The library allocates no device memory: the caller passes one device
  *     buffer of smem_cache_required_bytes() bytes to smem_cache_create and
- *     owns it; it must outlive the cache. The one exception is the
- *     reader-layer group at the end: its first call on a cache creates a
- *     cuBLAS handle (cuBLAS's own small device state, freed by
- *     smem_cache_destroy); the GEMM workspace there is the caller's too.
+ *     owns it; it must outlive the cache. The reader-layer calls at the end
+ *     take a caller-owned workspace as well.
  *   - Supported shapes: block_tokens == rows_per_block == 64,
  *     head_dim 32, 64 or 128 (SMEM_ERR_UNSUPPORTED otherwise).
  *   - At head_dim 64 the one-block prefill runs one thread-block cluster per
@@ -59,7 +57,7 @@
 extern "C" {
 #endif
 
-#define SMEM_ABI_VERSION 7
+#define SMEM_ABI_VERSION 8
 
 enum {
     SMEM_OK = 0,
@@ -274,9 +272,15 @@ int smem_decode_static_scratch(smem_cache *c, int32_t layer, int32_t nb, const i
  * layers) has per-layer keys mu W_kc and values mu W_vc; the null row is one
  * d-vector nu projected the same way. The attentions are those of
  * smem_prefill_block / smem_decode on the same cache; projections are bf16
- * GEMMs with fp32 accumulation (cuBLAS); intermediates LN outputs, q/k/v,
- * attention outputs and GELU outputs are rounded to bf16, the residual
- * stream stays fp32.
+ * products with fp32 accumulation on the library's tensor-core kernels
+ * (LayerNorm applied as the operand is loaded; residual add, GELU, rotary
+ * phases and in-block rows applied as results are stored); intermediates LN
+ * outputs, q/k/v, attention outputs and GELU outputs are rounded to bf16,
+ * the residual stream stays fp32. Every projection reduces in an order fixed
+ * by its shape and the device's SM count, so results are bitwise
+ * reproducible. Layer calls are issued with programmatic dependent launch:
+ * a projection may start loading its weights while the previous kernel on
+ * the stream finishes.
  *
  * Workspace: every call below takes a device buffer `ws` of at least
  * smem_layer_workspace_bytes(c, n_rows) bytes (256-byte aligned, the
@@ -406,6 +410,40 @@ const char *smem_last_error_detail(void);
  * callers can check that a failing call leaves the state unchanged.
  * n = 0 disables it. */
 int smem_debug_fail_after(smem_cache *c, int32_t n);
+
+/* Testing hook (failure detection without a GPU fault): stores `slot` into
+ * entry `pos` of the DEVICE copy of seq's table (pos < the table's length)
+ * without touching the host state. A value other than the host's slot
+ * corrupts the device table on purpose: a decode or prefill that meets a
+ * slot outside [0, capacity) skips that read and records the device error
+ * (smem_check_device_error then returns SMEM_ERR_DEVICE_FAULT). Writing the
+ * host's slot back (smem_get_table) restores the entry. */
+int smem_debug_set_table_entry(smem_cache *c, int32_t seq, int32_t pos, int32_t slot, void *stream);
+
+/* Testing hook: launches a kernel whose one wait (an mbarrier nothing ever
+ * arrives on) must give up after limit_ns nanoseconds (1 .. 1e9) and record
+ * the device error, exercising the bounded waits every kernel uses. The
+ * context stays usable; smem_check_device_error returns
+ * SMEM_ERR_DEVICE_FAULT and clears the word. */
+int smem_debug_wait_probe(smem_cache *c, long long limit_ns, void *stream);
+
+/* Testing hook: one projection on the reader layer's tensor-core kernel, as
+ * the layer calls use it (no counterpart in the paper; for kernel tests).
+ *   out[b][m][n] = epi(alpha * sum_k A'[b][m][k] W_b[k][n]),  b < batch
+ * A': bf16 A [M][lda] (+ b * a_bs elements); or, with ln_g != NULL, the fp32
+ * rows A [M][lda] normalised over K columns (LayerNorm, eps 1e-5, gain ln_g,
+ * bias ln_b [K] fp32) and rounded to bf16. W: bf16 [w_rows][w_cols]
+ * (row pitch w_cols); b_kmajor = 0: W_b[k][n] = W[k][n + b * w_boff];
+ * 1: W_b[k][n] = W[n][k + b * w_boff]. epi 0: bf16 store, 1: fp32 add into
+ * out, 2: GELU then bf16. Output column n of row m goes to out + b * o_bs +
+ * (n / col_group) * group_stride + m * ldo + n % col_group (col_group 0: N).
+ * N and K multiples of 32; device pointers 16-byte aligned. Uses the cache's
+ * device only for its error word. */
+int smem_debug_gemm(smem_cache *c, const void *A, int32_t lda, long long a_bs, const float *ln_g,
+                    const float *ln_b, const void *W, int32_t w_rows, int32_t w_cols, int32_t b_kmajor,
+                    int32_t w_boff, int32_t M, int32_t N, int32_t K, int32_t batch, int32_t epi, float alpha,
+                    void *out, int32_t ldo, long long o_bs, int32_t col_group, long long group_stride,
+                    void *stream);
 
 /* Static text of an error code. */
 const char *smem_strerror(int code);

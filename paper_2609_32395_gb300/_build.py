@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OBJ = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsmem.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["smem_capi.cpp", "smem_copy.cu", "smem_decode.cu", "smem_layer.cu", "smem_prefill.cu", "smem_recompute.cu"]
+SOURCES = ["smem_capi.cpp", "smem_copy.cu", "smem_decode.cu", "smem_gemm.cu", "smem_prefill.cu", "smem_recompute.cu"]
 HEADERS = ["smem_device.cuh", "smem_internal.h", "smem_tc.cuh"]
 
 
@@ -52,11 +52,16 @@ def up_to_date() -> bool:
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
+    """SMEM_DEBUG=1 in the environment builds the bounds-checking variant
+    (kernels check table, row and split indices and record an error instead
+    of touching memory out of range)."""
     if not force and up_to_date():
         return LIB
     nvcc = _nvcc()
     os.makedirs(OBJ, exist_ok=True)
     common = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", f"-I{INCLUDE}", f"-I{CSRC}"] + list(extra_flags)
+    if os.environ.get("SMEM_DEBUG", "0") not in ("", "0"):
+        common.append("-DSMEM_DEBUG=1")
 
     def compile_one(src):
         out = os.path.join(OBJ, os.path.splitext(src)[0] + ".o")
@@ -76,7 +81,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
                 print(log)
     tmp = LIB + f".tmp{os.getpid()}"
     cmd = [nvcc, "-shared", "-o", tmp] + [o for o, _ in results] + ARCH + [
-        "-cudart", "shared", "-lcublas", "-Xlinker", f"-rpath,{_cuda_lib_dir(nvcc)}"]
+        "-cudart", "shared", "-Xlinker", f"-rpath,{_cuda_lib_dir(nvcc)}"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -43,8 +43,6 @@ struct smem_cache {
   int fail_after = 0;                      // test hook: n-th next launch fails
   int pf_cluster_max = 0;                  // prefill cluster limit on this device (0: no clusters)
   smem::MuDecodePlan mu_plan{};            // recompute caches: decode kernel and query tile on this device
-  void* blas = nullptr;                    // cuBLAS handle of the reader-layer calls (created on first use)
-  ~smem_cache() { smem::blas_destroy(blas); }
 };
 
 namespace {
@@ -187,30 +185,23 @@ inline const uint16_t* null_kv(smem_cache* c) {
 }
 
 // Workspace of a reader-layer call over n rows (offsets from the caller's
-// 256-byte aligned buffer): cuBLAS workspace, then bf16 h [n][d], qkv
-// [n][3d], att [n][d], qc [n][d], fp32 f [n][4d], bf16 g [n][4d]; on a
-// recompute cache also bf16 q' and O' [n][H][d] and the split partials of
-// the memory-row attention.
+// 256-byte aligned buffer): bf16 qkv [n][3d], att [n][d], qc [n][d], g
+// [n][4d]; on a recompute cache also bf16 q' and O' [n][H][d] and the split
+// partials of the memory-row attention.
 struct LayerWs {
-  size_t blas, h, qkv, att, qc, f, g, qp, op, part, total;
+  size_t qkv, att, qc, g, qp, op, part, total;
 };
 
 LayerWs layer_ws(const Layout& L, int n) {
   const size_t d = (size_t)L.H * L.D;
   LayerWs w{};
   size_t off = 0;
-  w.blas = off;
-  off += smem::kBlasWorkspaceBytes;
-  w.h = off;
-  off = align_up(off + (size_t)n * d * 2, 256);
   w.qkv = off;
   off = align_up(off + (size_t)n * 3 * d * 2, 256);
   w.att = off;
   off = align_up(off + (size_t)n * d * 2, 256);
   w.qc = off;
   off = align_up(off + (size_t)n * d * 2, 256);
-  w.f = off;
-  off = align_up(off + (size_t)n * 4 * d * 4, 256);
   w.g = off;
   off = align_up(off + (size_t)n * 4 * d * 2, 256);
   w.qp = w.op = w.part = off;
@@ -228,20 +219,17 @@ LayerWs layer_ws(const Layout& L, int n) {
                                  n >= smem::kBlockTok ? (size_t)smem::kBlockTok * L.H : (size_t)0);
     off = align_up(off + rows * smem::kMuMaxSplits * (d + 4) * 4, 256);
   }
-  w.total = off;
+  w.total = std::max(off, (size_t)256);
   return w;
 }
 
 int layer_rows_max(const Layout& L) { return std::max(smem::kBlockTok, L.max_batch); }
 
-// Checks the workspace and binds cuBLAS to it and the stream (creating the
-// handle on first use).
-int layer_begin(smem_cache* c, void* ws, size_t ws_bytes, int n_rows, cudaStream_t st) {
+// Checks the workspace of a layer call.
+int layer_begin(smem_cache* c, void* ws, size_t ws_bytes, int n_rows) {
   if (!ws) return SMEM_ERR_INVALID_ARG;
   if (reinterpret_cast<uintptr_t>(ws) & 255u) return SMEM_ERR_ALIGN;
   if (ws_bytes < layer_ws(c->lay, n_rows).total) return SMEM_ERR_INVALID_ARG;
-  if (!c->blas && smem::blas_create(&c->blas, g_detail, sizeof(g_detail))) return SMEM_ERR_CUDA;
-  if (smem::blas_bind(c->blas, st, ws, smem::kBlasWorkspaceBytes, g_detail, sizeof(g_detail))) return SMEM_ERR_CUDA;
   return SMEM_OK;
 }
 
@@ -272,7 +260,36 @@ int cuda_rc(cudaError_t e, const char* what) {
   return SMEM_ERR_CUDA;
 }
 
-inline int blas_rc(int r) { return r ? SMEM_ERR_CUDA : SMEM_OK; }
+// A projection on the library's tensor-core kernel (error word of the cache).
+int gemm_rc(smem_cache* c, smem::GemmCall g, cudaStream_t st, const char* what) {
+  g.err = reinterpret_cast<int*>(c->dev + c->lay.off_err);
+  return cuda_rc(smem::launch_gemm(g, c->num_sms, st), what);
+}
+
+// Per-head projection of `rows` memory rows X [rows][d] by a key or value map
+// W [d][Hkv*D]: head h of the result, [rows][D] bf16, goes to
+// out + h * head_stride (the pool slot's or null row's layout).
+int project_heads(smem_cache* c, int rows, const void* X, const void* W, uint16_t* out, long long head_stride,
+                  cudaStream_t st) {
+  const Layout& L = c->lay;
+  const int d = L.H * L.D, kvd = L.Hkv * L.D;
+  smem::GemmCall g;
+  g.a = X;
+  g.lda = d;
+  g.w = W;
+  g.w_rows = d;
+  g.w_cols = kvd;
+  g.ldw = kvd;
+  g.M = rows;
+  g.N = kvd;
+  g.K = d;
+  g.out = out;
+  g.ldo = L.D;
+  g.col_group = L.D;
+  g.group_stride = head_stride;
+  return gemm_rc(c, g, st, "memory-row projection");
+}
+
 
 // One-block attention of one layer (arguments validated by the caller).
 // mode bit 0: self-attention, bit 1: cross-attention; tok_s, tok_c: token
@@ -309,6 +326,7 @@ int prefill_impl(smem_cache* c, int seq, int layer, int q_block_idx, const void*
     a.split_blks = nblk ? smem::prefill_split_blocks(nblk, c->lay.H, c->lay.D) : 1;
   a.n_splits = nblk ? smem::ceil_div(nblk, a.split_blks) : 0;
   a.capacity = c->lay.capacity;
+  a.max_blocks = c->lay.max_blocks;
   a.mode = mode;
   a.tok_s = tok_s;
   a.tok_c = tok_c;
@@ -387,6 +405,8 @@ int decode_impl(smem_cache* c, int layer, int nb, const int32_t* seq_ids, const 
     P.rope_tab = rope_tab(c);
     P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);
     P.rope_w = L.rope_w;
+    P.max_seqs = L.max_seqs;
+    P.part_pairs = (long long)L.max_batch * L.dec_max_splits;
     int pairs = 0;
     for (int i = 0; i < n; ++i) {
       const int s = seq_ids[i0 + i];
@@ -791,6 +811,8 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     P.rope_tab = rope_tab(c);
     P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);
     P.rope_w = L.rope_w;
+    P.max_seqs = L.max_seqs;
+    P.part_pairs = (long long)((SMEM_STATIC_SCRATCH_BYTES - 256 - ticket_bytes) / ((size_t)L.H * (L.D + 4) * 4));
     int pairs = 0;
     for (int i = 0; i < n; ++i) {
       P.items[i].seq = seq_ids[i0 + i];
@@ -843,7 +865,7 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
   if (c->fifo.empty()) return SMEM_ERR_POOL_FULL;
   DeviceGuard g(c->device);
   const cudaStream_t st = as_stream(stream);
-  int rc = layer_begin(c, ws, ws_bytes, 0, st);
+  int rc = layer_begin(c, ws, ws_bytes, 0);
   if (rc) return rc;
   if (injected_failure(c)) return SMEM_ERR_CUDA;
   const int32_t s = c->fifo.front();
@@ -855,10 +877,8 @@ int smem_append_block_rows(smem_cache* c, int32_t seq, int32_t block_idx, const 
     rc = cuda_rc(smem::launch_mu_tile(slot, static_cast<const uint16_t*>(mu), d, st), "append rows");
   for (int l = 0; l < L.L && !rc && !L.recompute; ++l)
     for (int kv = 0; kv < 2 && !rc; ++kv)
-      rc = blas_rc(smem::blas_project_heads(c->blas, smem::kRows, d, L.Hkv, L.D, static_cast<const uint16_t*>(mu),
-                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc), L.Hkv * L.D,
-                                            slot + ((size_t)l * L.Hkv * 2 + kv) * smem::kRows * L.D,
-                                            (long long)head_stride, g_detail, sizeof(g_detail)));
+      rc = project_heads(c, smem::kRows, mu, kv ? w[l].w_vc : w[l].w_kc,
+                         slot + ((size_t)l * L.Hkv * 2 + kv) * smem::kRows * L.D, (long long)head_stride, st);
   if (!rc) rc = cuda_rc(smem::launch_table_insert(table_row(c, seq), bidx_row(c, seq), pos, (int)ix.size(), s,
                                                           block_idx, st), "append rows");
   if (rc) return rc;
@@ -882,7 +902,7 @@ int smem_set_null_vector(smem_cache* c, const void* nu, const smem_layer_weights
     if (rc) return rc;
   }
   DeviceGuard g(c->device);
-  int rc = layer_begin(c, ws, ws_bytes, 0, as_stream(stream));
+  int rc = layer_begin(c, ws, ws_bytes, 0);
   if (rc) return rc;
   if (injected_failure(c)) return SMEM_ERR_CUDA;
   uint16_t* nk = reinterpret_cast<uint16_t*>(c->dev + L.off_null);
@@ -891,10 +911,8 @@ int smem_set_null_vector(smem_cache* c, const void* nu, const smem_layer_weights
     return cuda_rc(cudaMemcpyAsync(nk, nu, (size_t)d * 2, cudaMemcpyDeviceToDevice, as_stream(stream)), "null vector");
   for (int l = 0; l < L.L && !rc; ++l)
     for (int kv = 0; kv < 2 && !rc; ++kv)
-      rc = blas_rc(smem::blas_project_heads(c->blas, 1, d, L.Hkv, L.D, static_cast<const uint16_t*>(nu),
-                                            static_cast<const uint16_t*>(kv ? w[l].w_vc : w[l].w_kc), L.Hkv * L.D,
-                                            nk + ((size_t)l * L.Hkv * 2 + kv) * L.D, (long long)2 * L.D, g_detail,
-                                            sizeof(g_detail)));
+      rc = project_heads(c, 1, nu, kv ? w[l].w_vc : w[l].w_kc, nk + ((size_t)l * L.Hkv * 2 + kv) * L.D,
+                         (long long)2 * L.D, as_stream(stream));
   return rc;
 }
 
@@ -913,37 +931,61 @@ struct LayerRun {
   cudaStream_t st;
   int kvd() const { return c->lay.Hkv * c->lay.D; }  // key (or value) width of a token
   int w3() const { return d + 2 * kvd(); }            // q|k|v width of a token
-  uint16_t* h() const { return reinterpret_cast<uint16_t*>(ws + o.h); }
   uint16_t* qkv() const { return reinterpret_cast<uint16_t*>(ws + o.qkv); }
   uint16_t* att() const { return reinterpret_cast<uint16_t*>(ws + o.att); }
   uint16_t* qc() const { return reinterpret_cast<uint16_t*>(ws + o.qc); }
-  float* f() const { return reinterpret_cast<float*>(ws + o.f); }
   uint16_t* g() const { return reinterpret_cast<uint16_t*>(ws + o.g); }
-  int ln(const float* gain, const float* bias) {
-    return cuda_rc(smem::launch_layernorm(x, n, d, gain, bias, smem::kLayerNormEps, h(), st), "layernorm");
+  // out = [LN](A) W over this call's n tokens; A = the residual stream x
+  // (fp32, normalised with gain/bias) when gain is set, else bf16 [n][k]
+  smem::GemmCall proj(const void* A, const float* gain, const float* bias, const void* W, int cols, int k, void* out,
+                      int epi) const {
+    smem::GemmCall g;
+    g.a = gain ? static_cast<const void*>(x) : A;
+    g.lda = k;
+    g.ln_g = gain;
+    g.ln_b = bias;
+    g.w = W;
+    g.w_rows = k;
+    g.w_cols = cols;
+    g.ldw = cols;
+    g.M = n;
+    g.N = cols;
+    g.K = k;
+    g.epi = epi;
+    g.out = out;
+    g.ldo = cols;
+    g.pdl = true;
+    return g;
   }
-  int gemm(int cols, int k, const uint16_t* A, const void* W, void* C, bool f32, bool acc) {
-    return blas_rc(smem::blas_gemm(c->blas, n, cols, k, A, static_cast<const uint16_t*>(W), C, f32, acc, g_detail,
-                                   sizeof(g_detail)));
+  // qkv = LN1(x) W_qkv; for a one-block prefill (ib set) the key/value
+  // columns also become the block's in-block rows, and with rotary phases
+  // the query and key columns turn by the token's offset first
+  int qkv_proj(uint16_t* ib) {
+    smem::GemmCall g = proj(nullptr, w->ln1_g, w->ln1_b, w->w_qkv, w3(), d, qkv(), smem::kEpiBf16);
+    if (ib) {
+      g.ib = ib;
+      g.ib_col0 = d;
+      g.ib_kvd = kvd();
+      g.ib_D = c->lay.D;
+      if (c->lay.rope_w) {
+        g.rope_tab = rope_tab(c);
+        g.rope_cols = d + kvd();
+        g.rope_D = c->lay.D;
+      }
+    }
+    return gemm_rc(c, g, st, "qkv projection");
   }
-  // h1 = LN1(x); qkv = h1 W_qkv
-  int qkv_proj() {
-    int rc = ln(w->ln1_g, w->ln1_b);
-    return rc ? rc : gemm(w3(), d, h(), w->w_qkv, qkv(), false, false);
-  }
-  // x += att W_os; h2 = LN2(x); qc = h2 W_qc
+  // x += att W_os; qc = LN2(x) W_qc
   int after_sa() {
-    int rc = gemm(d, d, att(), w->w_os, x, true, true);
-    if (!rc) rc = ln(w->ln2_g, w->ln2_b);
-    return rc ? rc : gemm(d, d, h(), w->w_qc, qc(), false, false);
+    int rc = gemm_rc(c, proj(att(), nullptr, nullptr, w->w_os, d, d, x, smem::kEpiAddF32), st, "output projection");
+    return rc ? rc : gemm_rc(c, proj(nullptr, w->ln2_g, w->ln2_b, w->w_qc, d, d, qc(), smem::kEpiBf16), st,
+                             "cross-attention query projection");
   }
   // x += att W_oc; x += GELU(LN3(x) W_1) W_2
   int after_ca() {
-    int rc = gemm(d, d, att(), w->w_oc, x, true, true);
-    if (!rc) rc = ln(w->ln3_g, w->ln3_b);
-    if (!rc) rc = gemm(4 * d, d, h(), w->w_1, f(), true, false);
-    if (!rc) rc = cuda_rc(smem::launch_gelu(f(), g(), (long long)n * 4 * d, st), "gelu");
-    return rc ? rc : gemm(d, 4 * d, g(), w->w_2, x, true, true);
+    int rc = gemm_rc(c, proj(att(), nullptr, nullptr, w->w_oc, d, d, x, smem::kEpiAddF32), st, "output projection");
+    if (!rc) rc = gemm_rc(c, proj(nullptr, w->ln3_g, w->ln3_b, w->w_1, 4 * d, d, g(), smem::kEpiGeluBf16), st, "FFN");
+    return rc ? rc : gemm_rc(c, proj(g(), nullptr, nullptr, w->w_2, d, 4 * d, x, smem::kEpiAddF32), st, "FFN");
   }
 };
 
@@ -1036,16 +1078,48 @@ int mu_cross_attention(LayerRun& r, int layer, int nb, const int32_t* seq_ids, c
   uint16_t* op = reinterpret_cast<uint16_t*>(r.ws + r.o.op);
   const int nq = prefill ? smem::kBlockTok : nb;  // queries per head
   // q'[.][h][i] = scale sum_j qc[.][h][j] W_kc[i][h D + j]; prefill stores [h][q][d], decode [s][h][d]
-  int rc = blas_rc(smem::blas_gemm_sb(c->blas, true, false, d, nq, D, scale, wkc, d, D, r.qc(), d, D, qp,
-                                      prefill ? d : H * d, prefill ? (long long)smem::kBlockTok * d : d, H, g_detail,
-                                      sizeof(g_detail)));
+  smem::GemmCall g;
+  g.a = r.qc();
+  g.lda = d;
+  g.a_bs = D;
+  g.w = wkc;
+  g.w_rows = d;
+  g.w_cols = d;
+  g.ldw = d;
+  g.b_kmajor = 1;
+  g.w_boff = D;
+  g.M = nq;
+  g.N = d;
+  g.K = D;
+  g.batch = H;
+  g.alpha = scale;
+  g.out = qp;
+  g.ldo = prefill ? d : H * d;
+  g.o_bs = prefill ? (long long)smem::kBlockTok * d : d;
+  g.pdl = true;
+  int rc = gemm_rc(c, g, r.st, "memory-row query map");
   if (rc) return rc;
   rc = mu_attend(c, r.ws, r.o, prefill, nb, seq_ids, q_block_idx, seq, q_idx, qp, op, r.st);
   if (rc) return rc;
   // att[.][h][e] = sum_i O'[h-row][i] W_vc[i][h D + e]
-  return blas_rc(smem::blas_gemm_sb(c->blas, false, false, D, nq, d, 1.f, wvc, d, D, op,
-                                    prefill ? d : H * d, prefill ? (long long)smem::kBlockTok * d : d, r.att(), d, D,
-                                    H, g_detail, sizeof(g_detail)));
+  smem::GemmCall v;
+  v.a = op;
+  v.lda = prefill ? d : H * d;
+  v.a_bs = prefill ? (long long)smem::kBlockTok * d : d;
+  v.w = wvc;
+  v.w_rows = d;
+  v.w_cols = d;
+  v.ldw = d;
+  v.w_boff = D;
+  v.M = nq;
+  v.N = D;
+  v.K = d;
+  v.batch = H;
+  v.out = r.att();
+  v.ldo = d;
+  v.o_bs = D;
+  v.pdl = true;
+  return gemm_rc(c, v, r.st, "memory-row value map");
 }
 
 }  // namespace
@@ -1062,22 +1136,14 @@ int smem_reader_layer_prefill(smem_cache* c, int32_t seq, int32_t layer, int32_t
   DeviceGuard g(c->device);
   const cudaStream_t st = as_stream(stream);
   const int n = smem::kBlockTok;
-  rc = layer_begin(c, ws, ws_bytes, n, st);
+  rc = layer_begin(c, ws, ws_bytes, n);
   if (rc) return rc;
   const Layout& L = c->lay;
   LayerRun r{c, w, x, static_cast<uint8_t*>(ws), layer_ws(L, n), n, L.H * L.D, st};
   const int d = r.d, kvd = r.kvd(), w3 = r.w3();
-  rc = r.qkv_proj();
-  if (!rc && L.rope_w) {  // self-attention queries and keys turn by their in-block offsets
-    rc = cuda_rc(smem::launch_rope_rows(r.qkv(), r.qkv(), w3, w3, L.H, r.qkv() + d, r.qkv() + d, w3, w3, L.Hkv, n,
-                                        L.D, rope_tab(c), st),
-                 "rotary");
-  }
-  // the block's self-attention keys/values become its in-block rows (already turned)
-  if (!rc)
-    rc = cuda_rc(smem::launch_inblock_write(inblock_layer(c, seq, layer), r.qkv() + d, r.qkv() + d + kvd, n, L.Hkv,
-                                            L.D, st, w3),
-                 "in-block write");
+  // q|k|v of the block; its self-attention keys/values also become its
+  // in-block rows, queries and keys turned by their offsets with rotary phases
+  rc = r.qkv_proj(inblock_layer(c, seq, layer));
   if (!rc)
     rc = prefill_impl(c, seq, layer, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + d + kvd, r.qkv(), r.att(), r.att(),
                       1, w3, w3, st);
@@ -1103,12 +1169,12 @@ int smem_reader_layer_decode(smem_cache* c, int32_t layer, int32_t nb, const int
   if (rc) return rc;
   DeviceGuard g(c->device);
   const cudaStream_t st = as_stream(stream);
-  rc = layer_begin(c, ws, ws_bytes, nb, st);
+  rc = layer_begin(c, ws, ws_bytes, nb);
   if (rc) return rc;
   const Layout& L = c->lay;
   LayerRun r{c, w, x, static_cast<uint8_t*>(ws), layer_ws(L, nb), nb, L.H * L.D, st};
   const int d = r.d, kvd = r.kvd(), w3 = r.w3();
-  rc = r.qkv_proj();
+  rc = r.qkv_proj(nullptr);
   if (!rc)
     rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, r.qkv(), r.qkv() + d, r.qkv() + d + kvd, r.qkv(),
                      r.att(), r.att(), 1, w3, w3, st, w3);
@@ -1143,7 +1209,7 @@ int smem_mu_decode(smem_cache* c, int32_t nb, const int32_t* seq_ids, const int3
   }
   DeviceGuard g(c->device);
   const cudaStream_t st = as_stream(stream);
-  const int rc = layer_begin(c, ws, ws_bytes, nb, st);
+  const int rc = layer_begin(c, ws, ws_bytes, nb);
   if (rc) return rc;
   return mu_attend(c, static_cast<uint8_t*>(ws), layer_ws(c->lay, nb), false, nb, seq_ids, q_block_idx, 0, 0,
                    static_cast<const uint16_t*>(qp), static_cast<uint16_t*>(op), st);
@@ -1159,7 +1225,7 @@ int smem_mu_prefill(smem_cache* c, int32_t seq, int32_t q_block_idx, const void*
   if (!aligned16(qp) || !aligned16(op)) return SMEM_ERR_ALIGN;
   DeviceGuard g(c->device);
   const cudaStream_t st = as_stream(stream);
-  const int rc = layer_begin(c, ws, ws_bytes, smem::kBlockTok, st);
+  const int rc = layer_begin(c, ws, ws_bytes, smem::kBlockTok);
   if (rc) return rc;
   return mu_attend(c, static_cast<uint8_t*>(ws), layer_ws(c->lay, smem::kBlockTok), true, 0, nullptr, nullptr, seq,
                    q_block_idx, static_cast<const uint16_t*>(qp), static_cast<uint16_t*>(op), st);
@@ -1269,6 +1335,65 @@ int smem_mu_decode_plan(const smem_cache* c, int32_t* nq, int32_t* cluster, int3
   if (cluster) *cluster = c->mu_plan.cl;
   if (slice_cols) *slice_cols = c->mu_plan.wsl;
   return SMEM_OK;
+}
+
+int smem_debug_set_table_entry(smem_cache* c, int32_t seq, int32_t pos, int32_t slot, void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (seq < 0 || seq >= c->lay.max_seqs) return SMEM_ERR_NO_SUCH_SEQ;
+  if (pos < 0 || pos >= (int)c->idx[seq].size()) return SMEM_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  return cuda_rc(smem::launch_store_int(table_row(c, seq) + pos, slot, as_stream(stream)), "table entry");
+}
+
+int smem_debug_wait_probe(smem_cache* c, long long limit_ns, void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (limit_ns < 1 || limit_ns > 1000000000LL) return SMEM_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  return cuda_rc(smem::launch_wait_probe(reinterpret_cast<int*>(c->dev + c->lay.off_err),
+                                         (unsigned long long)limit_ns, as_stream(stream)),
+                 "wait probe");
+}
+
+int smem_debug_gemm(smem_cache* c, const void* A, int32_t lda, long long a_bs, const float* ln_g, const float* ln_b,
+                    const void* W, int32_t w_rows, int32_t w_cols, int32_t b_kmajor, int32_t w_boff, int32_t M,
+                    int32_t N, int32_t K, int32_t batch, int32_t epi, float alpha, void* out, int32_t ldo,
+                    long long o_bs, int32_t col_group, long long group_stride, void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (!A || !W || !out || (ln_g && !ln_b) || M < 1 || N < 32 || K < 32 || N % 32 || K % 32 || batch < 1 ||
+      epi < 0 || epi > 2 || lda < K || w_rows < 1 || w_cols < 1 || (b_kmajor != 0 && b_kmajor != 1) || w_boff < 0 ||
+      col_group < 0 || (col_group && col_group % 32) || lda % 8 || ldo % 8 || a_bs % 8 || o_bs % 8)
+    return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(A) || !aligned16(W) || !aligned16(out) || (ln_g && (!aligned16(ln_g) || !aligned16(ln_b))))
+    return SMEM_ERR_ALIGN;
+  DeviceGuard g(c->device);
+  smem::GemmCall gc;
+  gc.a = A;
+  gc.lda = lda;
+  gc.a_bs = a_bs;
+  gc.ln_g = ln_g;
+  gc.ln_b = ln_b;
+  gc.w = W;
+  gc.w_rows = w_rows;
+  gc.w_cols = w_cols;
+  gc.ldw = w_cols;
+  gc.b_kmajor = b_kmajor;
+  gc.w_boff = w_boff;
+  gc.M = M;
+  gc.N = N;
+  gc.K = K;
+  gc.batch = batch;
+  gc.epi = epi;
+  gc.alpha = alpha;
+  gc.out = out;
+  gc.ldo = ldo;
+  gc.o_bs = o_bs;
+  gc.col_group = col_group;
+  gc.group_stride = group_stride;
+  if (injected_failure(c)) return SMEM_ERR_CUDA;
+  return gemm_rc(c, gc, as_stream(stream), "projection");
 }
 
 int smem_abi_version(void) { return SMEM_ABI_VERSION; }

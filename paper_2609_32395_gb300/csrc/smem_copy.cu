@@ -223,6 +223,30 @@ cudaError_t launch_mu_tile(uint16_t* slot, const uint16_t* mu, int d, cudaStream
   return cudaGetLastError();
 }
 
+// Testing hooks (failure detection without a GPU fault): one int stored to
+// device memory; and a wait on an mbarrier that nothing ever arrives on,
+// which must give up after limit_ns and record the error.
+__global__ void store_int_kernel(int* p, int v) { *p = v; }
+
+__global__ void wait_probe_kernel(int* err, unsigned long long limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    if (!mbar_wait_bounded(&bar, 0, nullptr, limit_ns)) record_error(err, kDevErrWaitFull);
+  }
+}
+
+cudaError_t launch_store_int(int* p, int v, cudaStream_t st) {
+  store_int_kernel<<<1, 1, 0, st>>>(p, v);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_probe(int* err, unsigned long long limit_ns, cudaStream_t st) {
+  wait_probe_kernel<<<1, 32, 0, st>>>(err, limit_ns);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st) {
   const long long n16 = (long long)(bytes / 16);
   if (n16 == 0) return cudaSuccess;

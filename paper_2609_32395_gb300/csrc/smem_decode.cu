@@ -235,7 +235,11 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
   if (is.u < 0) return false;
   const int blk = is.b0 + is.c / C::CHUNKS;
   const int row0 = (is.c % C::CHUNKS) * C::SROWS;
-  const int slot = p.table[(size_t)p.items[is.item].seq * p.max_blocks + blk];
+  const DecodeItem& itm = p.items[is.item];
+  const bool in_range = SMEM_DCHECK(is.item < p.n_items && itm.seq >= 0 && itm.seq < p.max_seqs && blk >= 0 &&
+                                        blk < itm.nblk && itm.nblk <= p.max_blocks,
+                                    p.err);
+  const int slot = in_range ? p.table[(size_t)itm.seq * p.max_blocks + blk] : -1;
   const uint32_t qbytes = is.c == 0 ? p.qn * D * 2 : 0;  // the unit's qn query heads (contiguous)
   if (slot < 0 || slot >= p.capacity) {
     record_error(p.err, kDevErrBounds);
@@ -262,6 +266,10 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
   constexpr int LPR = Dec<D>::LPR;
   constexpr int RPP = 32 / LPR;  // rows per pass
   const DecodeItem& it = p.items[U.item];
+  if (!SMEM_DCHECK(U.item < p.n_items && it.seq >= 0 && it.seq < p.max_seqs && it.pos >= 0 && it.pos < kBlockTok &&
+                       it.nblk <= p.max_blocks,
+                   p.err))
+    return;
   const int n = it.pos + 1;
   const int grp = p.H / p.Hkv;  // query heads per key/value head (grouped-query attention)
   const int kvh = U.h / grp;
@@ -382,6 +390,8 @@ struct Pending {
 
 template <int D, bool ROPE>
 __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane) {
+  if (!SMEM_DCHECK(pd.item < p.n_items && pd.h < p.H && (long long)pd.pair_begin + pd.nsplit <= p.part_pairs, p.err))
+    return;
   constexpr int CPT = D / 32;  // columns per lane
   const size_t qoff = ((size_t)pd.item * p.H + pd.h) * D;
   const size_t qcoff = (size_t)pd.item * p.c_stride + (size_t)pd.h * D;
@@ -677,7 +687,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
         }
         continue;
       }
-      if (real) {
+      if (real && SMEM_DCHECK((long long)it.pair_begin + U.split < p.part_pairs, p.err)) {
         float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h + gq) * (D + 4);
 #pragma unroll
         for (int on = 0; on < ON; ++on)
@@ -869,12 +879,13 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     }
     settle<D, ROPE>(p, pend2, lane);
     announce(p, pend1, pend2, lane);
+    const bool part_in = SMEM_DCHECK((long long)it.pair_begin + U.split < p.part_pairs, p.err);
     float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h) * (D + 4);
-    if (g == 0) {
+    if (g == 0 && part_in) {
       *reinterpret_cast<float4*>(pp + 4 + c * 8) = make_float4(acc[0], acc[1], acc[2], acc[3]);
       *reinterpret_cast<float4*>(pp + 8 + c * 8) = make_float4(acc[4], acc[5], acc[6], acc[7]);
     }
-    if (lane == 0) {
+    if (lane == 0 && part_in) {
       pp[0] = m;
       pp[1] = l;
     }

@@ -41,6 +41,16 @@ enum DeviceError : int {
   kDevErrBounds = 4,      // an index failed a bounds check
 };
 
+// Bounds checks of the debug build (compiled with -DSMEM_DEBUG): an index
+// that fails records kDevErrBounds in the error word and the caller skips
+// the access; without the flag the condition is not evaluated. The checks
+// that guard pool reads (slot < capacity) are in every build.
+#ifdef SMEM_DEBUG
+#define SMEM_DCHECK(cond, err) ((cond) ? true : (::smem::record_error((err), ::smem::kDevErrBounds), false))
+#else
+#define SMEM_DCHECK(cond, err) true
+#endif
+
 // A wait gives up after this many nanoseconds of %globaltimer.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
 
@@ -53,6 +63,14 @@ __device__ __forceinline__ unsigned long long global_timer_ns() {
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
+
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start while the previous kernel on the stream finishes;
+// griddep_wait() blocks until that kernel has completed and its memory is
+// visible (a no-op without the launch attribute). griddep_launch() lets the
+// next such kernel start its own prologue.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 __device__ __forceinline__ void record_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
@@ -105,14 +123,15 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for the phase of `bar` with the given parity to complete. Returns
-// false when the limit runs out or *abort becomes non-zero.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+// false when the limit (nanoseconds) runs out or *abort becomes non-zero.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                                  unsigned long long limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_timer_ns();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (abort_flag && *abort_flag) return false;
-    if (global_timer_ns() - t0 > kWaitLimitNs) return false;
+    if (global_timer_ns() - t0 > limit_ns) return false;
   }
 }
 

@@ -109,6 +109,8 @@ struct DecodeParams {
   const float2* rope_tab;    // [kRopePhases][D/2] (cos, sin), or nullptr: no rotary phases
   const int* bidx;           // [max_seqs][max_blocks] block index of each table entry
   int rope_w;                // saturating window W
+  int max_seqs;              // rows of the device tables (bounds checks)
+  long long part_pairs;      // (item, split) pairs the partial buffer holds (bounds checks)
   DecodeItem items[kMaxDecodeItems];
 };
 
@@ -152,6 +154,9 @@ cudaError_t launch_rope_rows(const uint16_t* src_a, uint16_t* dst_a, int src_tok
 cudaError_t launch_null_write(uint16_t* null_kv, const uint16_t* k, const uint16_t* v, int L, int H, int D,
                               cudaStream_t st);
 cudaError_t launch_zero(void* p, size_t bytes, cudaStream_t st);
+// Testing hooks: store one int; a bounded wait that nothing completes.
+cudaError_t launch_store_int(int* p, int v, cudaStream_t st);
+cudaError_t launch_wait_probe(int* err, unsigned long long limit_ns, cudaStream_t st);
 // Memory rows of a recompute cache: mu [R][d] (d a multiple of 64) -> slot
 // [d/64][R][64], each 64-column chunk of the block contiguous (8 KB).
 cudaError_t launch_mu_tile(uint16_t* slot, const uint16_t* mu, int d, cudaStream_t st);
@@ -161,26 +166,77 @@ cudaError_t launch_table_insert(int* table_row, int* bidx_row, int pos, int n_ol
                                 cudaStream_t st);
 
 // ---------------------------------------------------------------------------
-// dense parts of the reader layer (LayerNorm, GELU, cuBLAS projections)
+// dense parts of the reader layer
 // ---------------------------------------------------------------------------
 constexpr float kLayerNormEps = 1e-5f;
-constexpr size_t kBlasWorkspaceBytes = (size_t)32 << 20;
-// h [n][d] bf16 = LayerNorm(x [n][d] fp32) * g + b.
-cudaError_t launch_layernorm(const float* x, int n, int d, const float* g, const float* b, float eps, uint16_t* h,
-                             cudaStream_t st);
-// out [n] bf16 = GELU(f [n] fp32), n a multiple of 4.
-cudaError_t launch_gelu(const float* f, uint16_t* out, long long n, cudaStream_t st);
-// An opaque cuBLAS handle; nonzero return = failure, message in `detail`.
-int blas_create(void** out, char* detail, size_t detail_len);
-void blas_destroy(void* blas);
-int blas_bind(void* blas, cudaStream_t st, void* ws, size_t ws_bytes, char* detail, size_t detail_len);
-int blas_gemm(void* blas, int m, int n, int k, const uint16_t* A, const uint16_t* W, void* C, bool c_f32,
-              bool accumulate, char* detail, size_t detail_len);
-int blas_project_heads(void* blas, int rows, int d, int H, int D, const uint16_t* X, const uint16_t* W, int ldw,
-                       uint16_t* out, long long head_stride, char* detail, size_t detail_len);
-int blas_gemm_sb(void* blas, bool ta, bool tb, int m, int n, int k, float alpha, const uint16_t* A, int lda,
-                 long long sA, const uint16_t* B, int ldb, long long sB, uint16_t* C, int ldc, long long sC, int batch,
-                 char* detail, size_t detail_len);
+
+// ---------------------------------------------------------------------------
+// projections on tcgen05 (smem_gemm.cu)
+// ---------------------------------------------------------------------------
+enum GemmEpilogue : int {
+  kEpiBf16 = 0,      // out (bf16) = alpha * acc
+  kEpiAddF32 = 1,    // out (fp32) += alpha * acc  (residual stream)
+  kEpiGeluBf16 = 2,  // out (bf16) = GELU(alpha * acc)
+};
+
+// One projection out[b][m][n] = epi(alpha * sum_k A[b][m][k] W_b[k][n]) for
+// b < batch (grid z). A: bf16 [M][lda] (+ b * a_bs), or with ln_g set the
+// fp32 residual stream [M][lda] normalised on the fly (LayerNorm over K
+// columns, gain ln_g, bias ln_b). W: the bf16 matrix [w_rows][w_cols] (row
+// pitch ldw elements); b_kmajor = 0: W is [K][N] (the batch's columns start
+// at b * w_boff); 1: W is [N][K] (the batch's K columns start at b * w_boff).
+// Output column n goes to out + b * o_bs + (n / col_group) * group_stride +
+// m * ldo + n % col_group (col_group 0: N). N and K multiples of 32.
+struct GemmCall {
+  const void* a = nullptr;
+  int lda = 0;
+  long long a_bs = 0;
+  const float* ln_g = nullptr;
+  const float* ln_b = nullptr;
+  const void* w = nullptr;
+  int w_rows = 0, w_cols = 0, ldw = 0;
+  int b_kmajor = 0;
+  int w_boff = 0;
+  int M = 0, N = 0, K = 0, batch = 1;
+  int epi = kEpiBf16;
+  float alpha = 1.f;
+  void* out = nullptr;
+  int ldo = 0;
+  long long o_bs = 0;
+  int col_group = 0;
+  long long group_stride = 0;
+  // q|k|v projection of a one-block prefill: columns [0, rope_cols) turned by
+  // the token's in-block offset (heads of rope_D columns); columns
+  // [ib_col0, ib_col0 + 2 ib_kvd) also stored as in-block rows [Hkv][2][b][ib_D]
+  const float2* rope_tab = nullptr;
+  int rope_cols = 0, rope_D = 0;
+  uint16_t* ib = nullptr;
+  int ib_col0 = 0, ib_kvd = 0, ib_D = 0;
+  int* err = nullptr;
+  bool pdl = false;  // programmatic dependent launch after the previous kernel
+};
+
+struct GemmParams {
+  CUtensorMap wmap;
+  const void* a;
+  const float* ln_g;
+  const float* ln_b;
+  void* out;
+  const float2* rope_tab;
+  uint16_t* ib;
+  long long a_bs, o_bs, group_stride;
+  int lda, ldo, M, N, K;
+  int ln, b_kmajor, w_boff, epi, col_group, ks, chunks;
+  int rope_cols, rope_D, ib_col0, ib_kvd, ib_D;
+  float alpha, eps;
+  int* err;
+};
+
+struct GemmPlan {
+  int bn, ks, ctas;
+};
+GemmPlan gemm_plan(int M, int N, int K, int batch, int num_sms);
+cudaError_t launch_gemm(const GemmCall& g, int num_sms, cudaStream_t st);
 
 // ---------------------------------------------------------------------------
 // cross-attention over memory rows (recompute-K/V caches)
@@ -264,6 +320,7 @@ struct PrefillArgs {
   int* err;
   long long slot_elems;
   int L, H, D, layer, nblk, split_blks, n_splits, capacity;
+  int max_blocks;             // table capacity of a sequence (bounds checks)
   int cluster;                // 1: cluster mode (one cluster of n_splits + 1 CTAs per head)
   const float2* rope_tab;     // rotary table or nullptr (Qs/Ks then arrive already turned by offset)
   const int* bidx_row;        // block index of each table entry of this sequence

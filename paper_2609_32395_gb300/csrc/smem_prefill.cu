@@ -126,7 +126,7 @@ struct PrefillParams {
   float* part;
   unsigned* counters;
   int* err;
-  int L, H, layer, nblk, split_blks, n_splits, capacity, max_splits;
+  int L, H, layer, nblk, split_blks, n_splits, capacity, max_splits, max_blocks;
   int Hkv;             // key/value heads (H / Hkv query heads share one)
   int mode;            // bit 0: in-block self-attention, bit 1: cross-attention
   int n_sa;            // self-attention CTAs of the cluster-free grid (0 or H)
@@ -301,6 +301,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   const bool work = nt > 0;
 
   if (threadIdx.x == 0) {
+    griddep_launch();
     mbar_init(q_full, 1);
     for (int s = 0; s < C::NS; ++s) {
       mbar_init(&full[s], 1);
@@ -322,6 +323,9 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   __syncthreads();
   tc::fence_after();
   const uint32_t tmem = *tslot;
+  // launched with programmatic dependent launch: everything above overlaps
+  // the previous kernel; every global read and write comes after this wait
+  griddep_wait();
 
   if (warp == 4) {
     // ------------------------------------------------------------ TMA producer
@@ -347,7 +351,9 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
             tc::tma_load_3d(kd + bx * C::KVS + C::BOX, &p.vs, bx * 64, h / (p.H / p.Hkv), 0, &full[st]);
           }
         } else {
-          const int slot = p.table_row[b0 + j];
+          const bool in_range =
+              SMEM_DCHECK(b0 + j >= 0 && b0 + j < p.nblk && p.nblk <= p.max_blocks && split < p.max_splits, p.err);
+          const int slot = in_range ? p.table_row[b0 + j] : -1;
           if (slot < 0 || slot >= p.capacity) {
             record_error(p.err, kDevErrBounds);
             mbar_arrive(&full[st]);
@@ -604,7 +610,8 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         pp[1] = ok ? lrow : 0.f;
       }
     }
-    if (!CL && ok && !direct) {
+    const bool part_ok = CL || SMEM_DCHECK(h < p.H && split < p.max_splits && p.n_splits <= p.max_splits, p.err);
+    if (!CL && ok && !direct && part_ok) {
       float* pp = p.part + (((size_t)h * p.max_splits + split) * C::B + r) * (D + 4);
 #pragma unroll
       for (int c = 0; c < D / 2; c += 4)
@@ -617,7 +624,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
     }
     // the four softmax warps agree on the outcome before the ticket
     const bool all_ok = bar_all(1, 128, ok);
-    if (!CL && all_ok && !direct) {
+    if (!CL && all_ok && !direct && part_ok) {
       if (threadIdx.x == 0) *ticket = atomicAdd(&p.counters[h], 1u);
       named_bar_sync(1, 128);
       if (*ticket == (unsigned)(p.n_splits - 1)) {
@@ -726,7 +733,18 @@ static cudaError_t launch_prefill_d(const PrefillParams& p, int grid, cudaStream
   using C = Pf<D>;
   cudaError_t e = ensure_smem_limit<1000 + D + (ROPE ? 1 : 0)>(prefill_kernel<D, false, ROPE>, C::SMEM);
   if (e != cudaSuccess) return e;
-  prefill_kernel<D, false, ROPE><<<grid, C::THREADS, C::SMEM, st>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(C::THREADS);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, prefill_kernel<D, false, ROPE>, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -748,13 +766,15 @@ static cudaError_t launch_prefill_cluster(const PrefillParams& p, cudaStream_t s
   cfg.blockDim = dim3(Pf<64>::THREADS);
   cfg.dynamicSmemBytes = Pf<64>::SMEM;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = cs;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   e = cudaLaunchKernelEx(&cfg, prefill_kernel<64, true, ROPE>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
@@ -858,6 +878,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   P.split_blks = a.split_blks;
   P.n_splits = (mode & 2) ? a.n_splits : 0;
   P.capacity = a.capacity;
+  P.max_blocks = a.max_blocks;
   P.max_splits = kPrefillMaxSplits;
   P.scale_log2 = a.scale_log2;
   P.n_sa = ((mode & 1) || ((mode & 2) && a.nblk == 0)) ? a.H : 0;

@@ -265,11 +265,14 @@ def test_churn_410m_replay_bitwise(N0):
     cfg = smem.make_config(1, H, D, S, max(fresh) + 8, total + 8, free_order=synth.slot_permutation(300, total + 8))
     c3 = smem.SmemCache(cfg, device="cuda")
     for s in range(S):
+        old = [j for j in sorted(live[s]) if j < N0]
+        for b0 in range(0, len(old), 64):  # original blocks, generated 64 at a time
+            ids = old[b0:b0 + 64]
+            K, V = synth.block_rows_torch(seed, s, ids, 1, H, R, D, "cuda")
+            for i, j in enumerate(ids):
+                smem.smem_append_block(c3.h, s, j, K[i], V[i])
         for j in sorted(live[s]):
-            if j < N0:
-                K, V = synth.block_rows_torch(seed, s, [j], 1, H, R, D, "cuda")
-                smem.smem_append_block(c3.h, s, j, K[0], V[0])
-            else:
+            if j >= N0:
                 K, V = new_block(s, j)
                 smem.smem_append_block(c3.h, s, j, K, V)
     osa = torch.empty(dshape, dtype=torch.bfloat16, device="cuda")
