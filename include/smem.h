@@ -429,21 +429,24 @@ int smem_debug_wait_probe(smem_cache *c, long long limit_ns, void *stream);
 
 /* Testing hook: one projection on the reader layer's tensor-core kernel, as
  * the layer calls use it (no counterpart in the paper; for kernel tests).
- *   out[b][m][n] = epi(alpha * sum_k A'[b][m][k] W_b[k][n]),  b < batch
- * A': bf16 A [M][lda] (+ b * a_bs elements); or, with ln_g != NULL, the fp32
- * rows A [M][lda] normalised over K columns (LayerNorm, eps 1e-5, gain ln_g,
- * bias ln_b [K] fp32) and rounded to bf16. W: bf16 [w_rows][w_cols]
- * (row pitch w_cols); b_kmajor = 0: W_b[k][n] = W[k][n + b * w_boff];
+ *   out[b][m][n] = epi(alpha * sum_k A[b][m][k] W_b[k][n]),  b < batch
+ * A: bf16 [M][lda] (+ b * a_bs elements). W: bf16 [w_rows][w_cols] (row
+ * pitch w_cols); b_kmajor = 0: W_b[k][n] = W[k][n + b * w_boff];
  * 1: W_b[k][n] = W[n][k + b * w_boff]. epi 0: bf16 store, 1: fp32 add into
  * out, 2: GELU then bf16. Output column n of row m goes to out + b * o_bs +
  * (n / col_group) * group_stride + m * ldo + n % col_group (col_group 0: N).
  * N and K multiples of 32; device pointers 16-byte aligned. Uses the cache's
  * device only for its error word. */
-int smem_debug_gemm(smem_cache *c, const void *A, int32_t lda, long long a_bs, const float *ln_g,
-                    const float *ln_b, const void *W, int32_t w_rows, int32_t w_cols, int32_t b_kmajor,
-                    int32_t w_boff, int32_t M, int32_t N, int32_t K, int32_t batch, int32_t epi, float alpha,
-                    void *out, int32_t ldo, long long o_bs, int32_t col_group, long long group_stride,
-                    void *stream);
+int smem_debug_gemm(smem_cache *c, const void *A, int32_t lda, long long a_bs, const void *W, int32_t w_rows,
+                    int32_t w_cols, int32_t b_kmajor, int32_t w_boff, int32_t M, int32_t N, int32_t K,
+                    int32_t batch, int32_t epi, float alpha, void *out, int32_t ldo, long long o_bs,
+                    int32_t col_group, long long group_stride, void *stream);
+
+/* Testing hook: the reader layer's LayerNorm kernel, h [n][d] bf16 =
+ * (x - mean) / sqrt(biased variance + 1e-5) * gain + bias per row of the fp32
+ * x [n][d] (d a multiple of 4); fp32 statistics, bf16 round-to-nearest-even. */
+int smem_debug_layernorm(smem_cache *c, const float *x, int32_t n, int32_t d, const float *gain, const float *bias,
+                         void *h, void *stream);
 
 /* Static text of an error code. */
 const char *smem_strerror(int code);

@@ -185,17 +185,19 @@ inline const uint16_t* null_kv(smem_cache* c) {
 }
 
 // Workspace of a reader-layer call over n rows (offsets from the caller's
-// 256-byte aligned buffer): bf16 qkv [n][3d], att [n][d], qc [n][d], g
-// [n][4d]; on a recompute cache also bf16 q' and O' [n][H][d] and the split
-// partials of the memory-row attention.
+// 256-byte aligned buffer): bf16 h [n][d] (LayerNorm output), qkv [n][3d],
+// att [n][d], qc [n][d], g [n][4d]; on a recompute cache also bf16 q' and O'
+// [n][H][d] and the split partials of the memory-row attention.
 struct LayerWs {
-  size_t qkv, att, qc, g, qp, op, part, total;
+  size_t h, qkv, att, qc, g, qp, op, part, total;
 };
 
 LayerWs layer_ws(const Layout& L, int n) {
   const size_t d = (size_t)L.H * L.D;
   LayerWs w{};
   size_t off = 0;
+  w.h = off;
+  off = align_up(off + (size_t)n * d * 2, 256);
   w.qkv = off;
   off = align_up(off + (size_t)n * 3 * d * 2, 256);
   w.att = off;
@@ -931,19 +933,20 @@ struct LayerRun {
   cudaStream_t st;
   int kvd() const { return c->lay.Hkv * c->lay.D; }  // key (or value) width of a token
   int w3() const { return d + 2 * kvd(); }            // q|k|v width of a token
+  uint16_t* h() const { return reinterpret_cast<uint16_t*>(ws + o.h); }
   uint16_t* qkv() const { return reinterpret_cast<uint16_t*>(ws + o.qkv); }
   uint16_t* att() const { return reinterpret_cast<uint16_t*>(ws + o.att); }
   uint16_t* qc() const { return reinterpret_cast<uint16_t*>(ws + o.qc); }
   uint16_t* g() const { return reinterpret_cast<uint16_t*>(ws + o.g); }
-  // out = [LN](A) W over this call's n tokens; A = the residual stream x
-  // (fp32, normalised with gain/bias) when gain is set, else bf16 [n][k]
-  smem::GemmCall proj(const void* A, const float* gain, const float* bias, const void* W, int cols, int k, void* out,
-                      int epi) const {
+  // h = LN(x) with this gain and bias (bf16)
+  int ln(const float* gain, const float* bias) {
+    return cuda_rc(smem::launch_layernorm(x, n, d, gain, bias, h(), true, st), "layernorm");
+  }
+  // out = A W over this call's n tokens (A bf16 [n][k])
+  smem::GemmCall proj(const void* A, const void* W, int cols, int k, void* out, int epi) const {
     smem::GemmCall g;
-    g.a = gain ? static_cast<const void*>(x) : A;
+    g.a = A;
     g.lda = k;
-    g.ln_g = gain;
-    g.ln_b = bias;
     g.w = W;
     g.w_rows = k;
     g.w_cols = cols;
@@ -961,7 +964,9 @@ struct LayerRun {
   // columns also become the block's in-block rows, and with rotary phases
   // the query and key columns turn by the token's offset first
   int qkv_proj(uint16_t* ib) {
-    smem::GemmCall g = proj(nullptr, w->ln1_g, w->ln1_b, w->w_qkv, w3(), d, qkv(), smem::kEpiBf16);
+    int rc = ln(w->ln1_g, w->ln1_b);
+    if (rc) return rc;
+    smem::GemmCall g = proj(h(), w->w_qkv, w3(), d, qkv(), smem::kEpiBf16);
     if (ib) {
       g.ib = ib;
       g.ib_col0 = d;
@@ -977,15 +982,16 @@ struct LayerRun {
   }
   // x += att W_os; qc = LN2(x) W_qc
   int after_sa() {
-    int rc = gemm_rc(c, proj(att(), nullptr, nullptr, w->w_os, d, d, x, smem::kEpiAddF32), st, "output projection");
-    return rc ? rc : gemm_rc(c, proj(nullptr, w->ln2_g, w->ln2_b, w->w_qc, d, d, qc(), smem::kEpiBf16), st,
-                             "cross-attention query projection");
+    int rc = gemm_rc(c, proj(att(), w->w_os, d, d, x, smem::kEpiAddF32), st, "output projection");
+    if (!rc) rc = ln(w->ln2_g, w->ln2_b);
+    return rc ? rc : gemm_rc(c, proj(h(), w->w_qc, d, d, qc(), smem::kEpiBf16), st, "cross-attention query projection");
   }
   // x += att W_oc; x += GELU(LN3(x) W_1) W_2
   int after_ca() {
-    int rc = gemm_rc(c, proj(att(), nullptr, nullptr, w->w_oc, d, d, x, smem::kEpiAddF32), st, "output projection");
-    if (!rc) rc = gemm_rc(c, proj(nullptr, w->ln3_g, w->ln3_b, w->w_1, 4 * d, d, g(), smem::kEpiGeluBf16), st, "FFN");
-    return rc ? rc : gemm_rc(c, proj(g(), nullptr, nullptr, w->w_2, d, 4 * d, x, smem::kEpiAddF32), st, "FFN");
+    int rc = gemm_rc(c, proj(att(), w->w_oc, d, d, x, smem::kEpiAddF32), st, "output projection");
+    if (!rc) rc = ln(w->ln3_g, w->ln3_b);
+    if (!rc) rc = gemm_rc(c, proj(h(), w->w_1, 4 * d, d, g(), smem::kEpiGeluBf16), st, "FFN");
+    return rc ? rc : gemm_rc(c, proj(g(), w->w_2, d, 4 * d, x, smem::kEpiAddF32), st, "FFN");
   }
 };
 
@@ -1356,25 +1362,23 @@ int smem_debug_wait_probe(smem_cache* c, long long limit_ns, void* stream) {
                  "wait probe");
 }
 
-int smem_debug_gemm(smem_cache* c, const void* A, int32_t lda, long long a_bs, const float* ln_g, const float* ln_b,
-                    const void* W, int32_t w_rows, int32_t w_cols, int32_t b_kmajor, int32_t w_boff, int32_t M,
-                    int32_t N, int32_t K, int32_t batch, int32_t epi, float alpha, void* out, int32_t ldo,
-                    long long o_bs, int32_t col_group, long long group_stride, void* stream) {
+int smem_debug_gemm(smem_cache* c, const void* A, int32_t lda, long long a_bs, const void* W, int32_t w_rows,
+                    int32_t w_cols, int32_t b_kmajor, int32_t w_boff, int32_t M, int32_t N, int32_t K, int32_t batch,
+                    int32_t epi, float alpha, void* out, int32_t ldo, long long o_bs, int32_t col_group,
+                    long long group_stride, void* stream) {
   if (!c) return SMEM_ERR_INVALID_ARG;
   if (!c->dev) return SMEM_ERR_NO_DEVICE;
-  if (!A || !W || !out || (ln_g && !ln_b) || M < 1 || N < 32 || K < 32 || N % 32 || K % 32 || batch < 1 ||
-      epi < 0 || epi > 2 || lda < K || w_rows < 1 || w_cols < 1 || (b_kmajor != 0 && b_kmajor != 1) || w_boff < 0 ||
-      col_group < 0 || (col_group && col_group % 32) || lda % 8 || ldo % 8 || a_bs % 8 || o_bs % 8)
+  if (!A || !W || !out || M < 1 || N < 32 || K < 32 || N % 32 || K % 32 || batch < 1 || epi < 0 || epi > 2 ||
+      lda < K || w_rows < 1 || w_cols < 1 || (b_kmajor != 0 && b_kmajor != 1) || w_boff < 0 || col_group < 0 ||
+      (col_group && col_group % 32) || lda % 8 || ldo % 8 || a_bs % 8 || o_bs % 8 || w_cols % 8 ||
+      (batch > 1 && a_bs < 1))
     return SMEM_ERR_INVALID_ARG;
-  if (!aligned16(A) || !aligned16(W) || !aligned16(out) || (ln_g && (!aligned16(ln_g) || !aligned16(ln_b))))
-    return SMEM_ERR_ALIGN;
+  if (!aligned16(A) || !aligned16(W) || !aligned16(out)) return SMEM_ERR_ALIGN;
   DeviceGuard g(c->device);
   smem::GemmCall gc;
   gc.a = A;
   gc.lda = lda;
   gc.a_bs = a_bs;
-  gc.ln_g = ln_g;
-  gc.ln_b = ln_b;
   gc.w = W;
   gc.w_rows = w_rows;
   gc.w_cols = w_cols;
@@ -1394,6 +1398,17 @@ int smem_debug_gemm(smem_cache* c, const void* A, int32_t lda, long long a_bs, c
   gc.group_stride = group_stride;
   if (injected_failure(c)) return SMEM_ERR_CUDA;
   return gemm_rc(c, gc, as_stream(stream), "projection");
+}
+
+int smem_debug_layernorm(smem_cache* c, const float* x, int32_t n, int32_t d, const float* gain, const float* bias,
+                         void* h, void* stream) {
+  if (!c) return SMEM_ERR_INVALID_ARG;
+  if (!c->dev) return SMEM_ERR_NO_DEVICE;
+  if (!x || !gain || !bias || !h || n < 1 || d < 4 || d % 4) return SMEM_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(gain) || !aligned16(bias) || !aligned16(h)) return SMEM_ERR_ALIGN;
+  DeviceGuard g(c->device);
+  return cuda_rc(smem::launch_layernorm(x, n, d, gain, bias, static_cast<uint16_t*>(h), false, as_stream(stream)),
+                 "layernorm");
 }
 
 int smem_abi_version(void) { return SMEM_ABI_VERSION; }

@@ -1,7 +1,7 @@
 // smem_gemm.cu -- the dense projections of the reader layer on tcgen05 tensor
-// cores (arXiv 2609.32395, Sec. 2 "Model", App. A "Reader": pre-LN residual
-// branches with Q/K/V/O maps and a 4d GELU FFN; memory rows projected to each
-// layer's keys and values).
+// cores, and its LayerNorm (arXiv 2609.32395, Sec. 2 "Model", App. A
+// "Reader": pre-LN residual branches with Q/K/V/O maps and a 4d GELU FFN;
+// memory rows projected to each layer's keys and values).
 //
 // out[m][n] = epilogue( alpha * sum_k A[m][k] W[k][n] ), bf16 operands, fp32
 // accumulation in tensor memory. The reader's shapes are skinny (64 query
@@ -9,34 +9,42 @@
 // 4d weights), so a projection streams its weights once and its time is set
 // by latency, not by math. The kernel is laid out for that:
 //
-//   * a CTA owns 128 rows (tokens) x BN output columns; MMA M = 128, N = BN
-//     (64 or 128), K = 16 per instruction, issued by one thread;
-//   * the K range is cut over a thread-block cluster of up to 8 CTAs: each
-//     accumulates its share of K in tensor memory, parks the fp32 partial in
-//     its shared memory, and every CTA then adds the partials of a slice of
-//     the rows over distributed shared memory in rank order (a fixed order:
-//     bitwise reproducible, no global workspace, no atomics);
-//   * weights arrive by TMA (128-byte swizzle) into a 4-stage ring; the first
-//     stages are requested before the kernel waits for the previous kernel
-//     (programmatic dependent launch), since weights do not depend on it;
-//   * the A operand is written into shared memory by six producer warps: the
-//     bf16 activations, or -- for the pre-LN projections -- LayerNorm of the
-//     fp32 residual stream computed on the fly. Row statistics come from the
-//     cluster: each CTA reduces its own K slice (mean and centred sum of
-//     squares, two passes), the slices are combined in rank order (the
-//     pairwise update of Chan, Golub and LeVeque), so no CTA reads more of a
-//     row than its slice;
+//   * a CTA of four warps owns 128 rows (tokens) x BN output columns; MMA
+//     M = 128, N = BN (64 or 128), K = 16 per instruction, issued by one
+//     thread; warp 0 issues the copies, warp 1 the MMAs, then all four read
+//     the accumulator (TMEM lanes 32w..32w+31) and run the epilogue;
+//   * both operands arrive by TMA (128-byte swizzle) into a 4-stage ring:
+//     weights as W[k][n] (MN-major boxes) or W[n][k] (K-major), activations as
+//     a [batch][M][K] view (rows and columns past M and K read as zero). The
+//     weight copies of the first stages are requested before the kernel waits
+//     for the previous kernel (programmatic dependent launch): weights never
+//     depend on it;
+//   * the K range is cut over a thread-block cluster of up to 8 CTAs when the
+//     output tiles alone would leave SMs idle: each CTA accumulates its share
+//     of K, parks the fp32 partial in its shared memory, and every CTA then
+//     adds the partials of a slice of the rows over distributed shared memory
+//     in rank order (a fixed order: bitwise reproducible, no global workspace,
+//     no atomics). The plan keeps every cluster in one wave (a GPC hosts only
+//     whole clusters);
 //   * epilogues: bf16 store (optionally into per-head column groups, the pool
 //     slot layout), fp32 residual add, GELU (x * Phi(x), erff) to bf16, and
 //     for the q|k|v projection of a one-block prefill the rotary turn of the
 //     query and key columns by token offset plus the copy of the key/value
 //     columns into the block's in-block rows.
+//
+// LayerNorm runs as its own small kernel (one warp per token, fp32 two-pass
+// moments, bf16 out), launched with programmatic dependent launch as well.
+// A form that normalised the fp32 rows inside the projection (per-slice
+// statistics combined across the cluster) measured slower: its producer
+// warps spent a few microseconds per phase, mostly waiting for instruction
+// fetch, against about one for this kernel.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstdlib>
 
 #include "smem_device.cuh"
 #include "smem_internal.h"
@@ -48,23 +56,29 @@ namespace {
 
 constexpr int kBM = 128;          // rows (tokens) per CTA
 constexpr int kNS = 4;            // ring stages
-constexpr int kThreads = 256;     // warp 0: weight TMA, warp 1: MMA + TMEM, warps 2-7: A producers
-constexpr int kAProd = 192;       // A-producer threads (warps 2-7); warps 4-7 also run the epilogue
+constexpr int kThreads = 128;     // warp 0: TMA, warp 1: TMEM + MMA; then all four: epilogue
 constexpr int kMaxCluster = 8;
+constexpr int kLnThreads = 256;   // LayerNorm: 8 warps, one token each
 
+// Shared memory: a ring of `ns` stages (ns <= kNS, sized per launch to the
+// K chunks a CTA streams, so that short projections leave room for the next
+// kernel's CTAs), then the barriers; the drained ring also parks the split
+// partials (ring_bytes covers them).
 template <int BN>
 struct Gm {
   static constexpr int A_BYTES = kBM * 128;  // [128 rows][64 k] bf16, 128-byte swizzle
   static constexpr int W_BYTES = BN * 128;   // [64 k][BN] as BN/64 boxes of 8 KB, or [BN][64 k]
   static constexpr int STAGE = A_BYTES + W_BYTES;
   static constexpr int PSTRIDE = BN + 4;     // floats per row of a parked partial
-  static constexpr int OFF_STAT = kNS * STAGE;          // [128] float2: (mean, M2) of this CTA's K slice
-  static constexpr int OFF_NORM = OFF_STAT + kBM * 8;   // [128] float2: (mean, rstd) of the whole row
-  static constexpr int OFF_BAR = OFF_NORM + kBM * 8;    // full_w[NS] | full_a[NS] | empty[NS] | acc
-  static constexpr int NBAR = 3 * kNS + 1;
-  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;   // TMEM slot, abort flag
-  static constexpr int SMEM = OFF_MISC + 16 + 1024;
+  static constexpr int NBAR = 2 * kNS + 1;   // full[NS] | empty[NS] | acc
+  static constexpr int MISC = NBAR * 8 + 16;  // barriers, TMEM slot, abort flag
+  static constexpr int SMEM_MAX = kNS * STAGE + MISC + 1024;
   static_assert(kBM * PSTRIDE * 4 <= kNS * STAGE, "partials fit in the ring");
+  // ring bytes of a launch: its stages, and at least the parked rows
+  static int ring_bytes(int ns, int mrows, int ks) {
+    const int r = ns * STAGE, pk = ks > 1 ? mrows * PSTRIDE * 4 : 0;
+    return ((r > pk ? r : pk) + 1023) / 1024 * 1024;
+  }
 };
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
@@ -94,12 +108,6 @@ __device__ __forceinline__ float4 ld_dsmem_f32x4(uint32_t addr) {
 __device__ __forceinline__ float bf16_round(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
 
 __device__ __forceinline__ float gelu_erf(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
-
-// Barrier over every thread of the cluster (or of the CTA without one).
-__device__ __forceinline__ void group_sync(int ks) {
-  if (ks > 1) tc::cluster_sync();
-  else __syncthreads();
-}
 
 // Epilogue of NV consecutive output columns col.. of row `row` (tile-local
 // row r for the rotary phase / in-block row); v holds alpha * accumulator.
@@ -170,26 +178,24 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
   const int c0 = (int)((long long)p.chunks * rank / ks);
   const int c1 = (int)((long long)p.chunks * (rank + 1) / ks);
   const int nch = c1 - c0;
-  uint64_t* full_w = reinterpret_cast<uint64_t*>(base + C::OFF_BAR);
-  uint64_t* full_a = full_w + kNS;
-  uint64_t* empty = full_a + kNS;
+  const int ns = p.ns;
+  uint64_t* full = reinterpret_cast<uint64_t*>(base + p.ring_bytes);
+  uint64_t* empty = full + kNS;
   uint64_t* acc_bar = empty + kNS;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(base + C::OFF_MISC);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::OFF_MISC + 4);
-  float2* stat = reinterpret_cast<float2*>(base + C::OFF_STAT);
-  float2* norm = reinterpret_cast<float2*>(base + C::OFF_NORM);
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(base + p.ring_bytes + C::NBAR * 8);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + p.ring_bytes + C::NBAR * 8 + 4);
 
   if (threadIdx.x == 0) {
     griddep_launch();  // the next kernel may start its own prologue
-    for (int s = 0; s < kNS; ++s) {
-      mbar_init(&full_w[s], 1);
-      mbar_init(&full_a[s], kAProd);
+    for (int s = 0; s < ns; ++s) {
+      mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
     mbar_init(acc_bar, 1);
     *abort_flag = 0;
     fence_mbar_init();
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.wmap)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.amap)) : "memory");
   }
   if (warp == 1) tc::alloc(tslot, BN);
   tc::fence_before();
@@ -197,195 +203,86 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
   tc::fence_after();
   const uint32_t tmem = *tslot;
 
-  auto load_w = [&](int i) {  // chunk i of this split into stage i % NS (thread 0 of warp 0)
-    const int st = i % kNS;
+  // chunk i of this split into stage i % NS (thread 0): weights and the A tile,
+  // both completing full[st]
+  auto load_w = [&](int i) {
+    const int st = i % ns;
     uint8_t* wb = base + st * C::STAGE + C::A_BYTES;
     const int k = (c0 + i) * 64;
-    mbar_arrive_expect_tx(&full_w[st], C::W_BYTES);
+    mbar_arrive_expect_tx(&full[st], C::W_BYTES + C::A_BYTES);
     if (p.b_kmajor) {
-      tma_load_2d(wb, &p.wmap, k + p.w_boff * bz, n0, &full_w[st]);
+      tma_load_2d(wb, &p.wmap, k + p.w_boff * bz, n0, &full[st]);
     } else {
 #pragma unroll
-      for (int j = 0; j < BN / 64; ++j) tma_load_2d(wb + j * 8192, &p.wmap, n0 + j * 64 + p.w_boff * bz, k, &full_w[st]);
+      for (int j = 0; j < BN / 64; ++j) tma_load_2d(wb + j * 8192, &p.wmap, n0 + j * 64 + p.w_boff * bz, k, &full[st]);
     }
   };
-  // weights do not depend on the previous kernel: request the first stages now
+  auto load_a = [&](int i) {
+    if (p.a_bmajor) tc::tma_load_3d(base + (i % ns) * C::STAGE, &p.amap, (c0 + i) * 64, bz, m0, &full[i % ns]);
+    else tc::tma_load_3d(base + (i % ns) * C::STAGE, &p.amap, (c0 + i) * 64, m0, bz, &full[i % ns]);
+  };
   int issued = 0;
-  if (warp == 0 && lane == 0)
-    for (; issued < min(kNS, nch); ++issued) load_w(issued);
-
-  const bool aprod = warp >= 2;
-  const int atid = threadIdx.x - 64;  // 0..191 for the A producers
+  if (threadIdx.x == 0)
+    for (; issued < min(ns, nch); ++issued) load_w(issued);  // weights do not depend on the previous kernel
   // everything below may read the previous kernel's outputs or write this
-  // kernel's (the split-K reduction runs on every thread)
+  // kernel's
   griddep_wait();
-  // ---- LayerNorm statistics of this CTA's K slice (two passes), per row
-  const int kb = min(c0 * 64, p.K), ke = min(c1 * 64, p.K);
-  if (p.ln && aprod) {
-    const float* xa = static_cast<const float*>(p.a) + (size_t)bz * p.a_bs;
-    const int n4 = (ke - kb) / 4;
-    for (int r = warp - 2; r < mrows; r += 6) {
-      const float4* xr = reinterpret_cast<const float4*>(xa + (size_t)(m0 + r) * p.lda + kb);
-      float s = 0.f;
-      for (int c = lane; c < n4; c += 32) {
-        const float4 v = xr[c];
-        s += (v.x + v.y) + (v.z + v.w);
-      }
-#pragma unroll
-      for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-      const float mean = n4 ? s / (float)(4 * n4) : 0.f;
-      float q = 0.f;
-      for (int c = lane; c < n4; c += 32) {
-        const float4 v = xr[c];
-        const float a = v.x - mean, b = v.y - mean, cc = v.z - mean, d = v.w - mean;
-        q += (a * a + b * b) + (cc * cc + d * d);
-      }
-#pragma unroll
-      for (int o = 16; o; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
-      if (lane == 0) stat[r] = make_float2(mean, q);
-    }
-  }
-  group_sync(ks);  // every split's statistics are visible in the cluster
-  if (p.ln && aprod) {
-    // combine the slices in rank order: counts, means and centred sums of squares
-    for (int r = atid; r < mrows; r += kAProd) {
-      float cnt = 0.f, mean = 0.f, m2 = 0.f;
-      for (int s = 0; s < ks; ++s) {
-        const int sb = min((int)((long long)p.chunks * s / ks) * 64, p.K);
-        const int se = min((int)((long long)p.chunks * (s + 1) / ks) * 64, p.K);
-        const float nb = (float)(se - sb);
-        if (nb == 0.f) continue;
-        float2 v;
-        if (ks > 1) {
-          const uint32_t ra = tc::dsmem_addr(smem_u32(&stat[r]), (uint32_t)s);
-          v = tc::ld_dsmem_f32x2(ra);
-        } else {
-          v = stat[r];
-        }
-        if (cnt == 0.f) {
-          cnt = nb;
-          mean = v.x;
-          m2 = v.y;
-        } else {
-          const float tot = cnt + nb, delta = v.x - mean;
-          mean = mean + delta * (nb / tot);
-          m2 = m2 + v.y + delta * delta * (cnt * nb / tot);
-          cnt = tot;
-        }
-      }
-      norm[r] = make_float2(mean, rsqrtf(m2 / (float)p.K + p.eps));
-    }
-    named_bar_sync(1, kAProd);
-  }
 
   bool ok = true;
-  if (warp == 0) {
-    // ------------------------------------------------------------ weight TMA
-    if (lane == 0) {
-      for (int i = issued; i < nch; ++i) {
-        const int st = i % kNS;
-        if (!mbar_wait_bounded(&empty[st], ((i / kNS) - 1) & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
-        load_w(i);
-        ++issued;
-      }
-      if (!ok) {
-        record_error(p.err, kDevErrWaitEmpty);
-        *abort_flag = 1;
-      }
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = tc::idesc_bf16(128, BN, 0, p.b_kmajor ? 0 : 1);
-      for (int i = 0; i < nch; ++i) {
-        const int st = i % kNS;
-        ok = mbar_wait_bounded(&full_w[st], (i / kNS) & 1, abort_flag) &&
-             mbar_wait_bounded(&full_a[st], (i / kNS) & 1, abort_flag);
-        if (!ok) break;
-        tc::fence_after();
-        const uint32_t aa = smem_u32(base + st * C::STAGE);
-        const uint32_t wa = aa + C::A_BYTES;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const uint64_t bd = p.b_kmajor ? tc::sdesc_sw128(wa + k * 32, 16, 1024)
-                                         : tc::sdesc_sw128(wa + k * 2048, 8192, 1024);
-          tc::mma_bf16(tmem, tc::sdesc_sw128(aa + k * 32, 16, 1024), bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
-        }
-        tc::commit(&empty[st]);
-      }
-      if (!ok) {
-        record_error(p.err, kDevErrWaitFull);
-        *abort_flag = 1;
-      }
-      tc::commit(acc_bar);  // arrives once every MMA issued above has completed
-    }
-  } else {
-    // ------------------------------------------------------------ A producers
-    const int j = atid & 7;  // 16-byte column group of the chunk this thread fills
-    for (int i = 0; i < nch && ok; ++i) {
-      const int st = i % kNS;
-      if (i >= kNS && !mbar_wait_bounded(&empty[st], ((i / kNS) - 1) & 1, abort_flag)) {
+  if (threadIdx.x == 0) {
+    // ------------------------------------------------------------ copies
+    for (int i = 0; i < issued; ++i) load_a(i);
+    for (int i = issued; i < nch; ++i) {
+      const int st = i % ns;
+      if (!mbar_wait_bounded(&empty[st], ((i / ns) - 1) & 1, abort_flag)) {
         ok = false;
         break;
       }
-      uint8_t* at = base + st * C::STAGE;
-      const int kc = (c0 + i) * 64 + j * 8;  // first column of this thread's group
-      const bool col_in = kc < p.K;
-      float g[8], bb[8];
-      if (p.ln && col_in) {
-        const float4 g0 = *reinterpret_cast<const float4*>(p.ln_g + kc);
-        const float4 g1 = *reinterpret_cast<const float4*>(p.ln_g + kc + 4);
-        const float4 b0 = *reinterpret_cast<const float4*>(p.ln_b + kc);
-        const float4 b1 = *reinterpret_cast<const float4*>(p.ln_b + kc + 4);
-        g[0] = g0.x, g[1] = g0.y, g[2] = g0.z, g[3] = g0.w, g[4] = g1.x, g[5] = g1.y, g[6] = g1.z, g[7] = g1.w;
-        bb[0] = b0.x, bb[1] = b0.y, bb[2] = b0.z, bb[3] = b0.w, bb[4] = b1.x, bb[5] = b1.y, bb[6] = b1.z, bb[7] = b1.w;
-      }
-      for (int r = atid >> 3; r < kBM; r += kAProd / 8) {
-        uint4 w = make_uint4(0u, 0u, 0u, 0u);
-        if (r < mrows && col_in) {
-          if (p.ln) {
-            const float* xr = static_cast<const float*>(p.a) + (size_t)bz * p.a_bs + (size_t)(m0 + r) * p.lda + kc;
-            const float4 v0 = *reinterpret_cast<const float4*>(xr);
-            const float4 v1 = *reinterpret_cast<const float4*>(xr + 4);
-            const float2 nr = norm[r];
-            const float x[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-            uint32_t h[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-              h[e] = pack_bf16x2((x[2 * e] - nr.x) * nr.y * g[2 * e] + bb[2 * e],
-                                 (x[2 * e + 1] - nr.x) * nr.y * g[2 * e + 1] + bb[2 * e + 1]);
-            w = make_uint4(h[0], h[1], h[2], h[3]);
-          } else {
-            w = *reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(p.a) + (size_t)bz * p.a_bs +
-                                                (size_t)(m0 + r) * p.lda + kc);
-          }
-        }
-        *reinterpret_cast<uint4*>(at + r * 128 + ((j ^ (r & 7)) << 4)) = w;
-      }
-      fence_proxy_async_smem();
-      mbar_arrive(&full_a[st]);
+      load_w(i);
+      load_a(i);
+      ++issued;
     }
     if (!ok) {
       record_error(p.err, kDevErrWaitEmpty);
       *abort_flag = 1;
     }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    const uint32_t idesc = tc::idesc_bf16(128, BN, 0, p.b_kmajor ? 0 : 1);
+    for (int i = 0; i < nch; ++i) {
+      const int st = i % ns;
+      ok = mbar_wait_bounded(&full[st], (i / ns) & 1, abort_flag);
+      if (!ok) break;
+      tc::fence_after();
+      const uint32_t aa = smem_u32(base + st * C::STAGE);
+      const uint32_t wa = aa + C::A_BYTES;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint64_t bd = p.b_kmajor ? tc::sdesc_sw128(wa + k * 32, 16, 1024)
+                                       : tc::sdesc_sw128(wa + k * 2048, 8192, 1024);
+        tc::mma_bf16(tmem, tc::sdesc_sw128(aa + k * 32, 16, 1024), bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
+      }
+      tc::commit(&empty[st]);
+    }
+    if (!ok) {
+      record_error(p.err, kDevErrWaitFull);
+      *abort_flag = 1;
+    }
+    tc::commit(acc_bar);  // arrives once every MMA issued above has completed
   }
+  __syncwarp();
 
-  // ---- epilogue: warps 4-7 read the accumulator rows (TMEM lanes 32(w-4)..)
+  // ---- epilogue: warp w reads the accumulator rows 32w.. (TMEM lanes 32w..)
   float* part = reinterpret_cast<float*>(base);  // the ring, free once every MMA completed
-  if (warp >= 4) {
-    const int q = warp - 4;
-    const int r = 32 * q + lane;
+  const int r = 32 * warp + lane;
+  if (32 * warp < mrows) {
     const bool done = mbar_wait_bounded(acc_bar, 0, nullptr);
     if (!done && lane == 0) record_error(p.err, kDevErrWaitMma);
     tc::fence_after();
 #pragma unroll 1
     for (int cb = 0; cb < BN / 32; ++cb) {
       uint32_t u[32];
-      ld_tmem_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(cb * 32), u);
+      ld_tmem_32x32b_x32(tmem + ((uint32_t)(32 * warp) << 16) + (uint32_t)(cb * 32), u);
       tc::wait_ld();
       const int col = n0 + cb * 32;
       if (r < mrows) {
@@ -401,8 +298,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
         }
       }
     }
-    tc::fence_before();
   }
+  tc::fence_before();
   if (ks > 1) {
     tc::cluster_sync();  // every split's partial rows are parked
     // rank s adds the partials of rows [s * rp, (s + 1) * rp) in rank order
@@ -410,19 +307,24 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     const int r0 = rank * rp, r1 = min(mrows, r0 + rp);
     constexpr int G4 = BN / 4;
     for (int it = threadIdx.x; it < (r1 - r0) * G4; it += kThreads) {
-      const int r = r0 + it / G4, c = (it % G4) * 4;
+      const int rr = r0 + it / G4, c = (it % G4) * 4;
       if (n0 + c >= p.N) continue;
-      const uint32_t la = smem_u32(part + r * C::PSTRIDE + c);
-      float4 s = ld_dsmem_f32x4(tc::dsmem_addr(la, 0));
-      for (int t = 1; t < ks; ++t) {
-        const float4 v = ld_dsmem_f32x4(tc::dsmem_addr(la, (uint32_t)t));
-        s.x += v.x;
-        s.y += v.y;
-        s.z += v.z;
-        s.w += v.w;
+      const uint32_t la = smem_u32(part + rr * C::PSTRIDE + c);
+      float4 pv[kMaxCluster];  // every split's partial is requested before the sum
+#pragma unroll
+      for (int t = 0; t < kMaxCluster; ++t)
+        pv[t] = t < ks ? ld_dsmem_f32x4(tc::dsmem_addr(la, (uint32_t)t)) : make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 s4 = pv[0];
+#pragma unroll
+      for (int t = 1; t < kMaxCluster; ++t) {
+        if (t >= ks) break;
+        s4.x += pv[t].x;
+        s4.y += pv[t].y;
+        s4.z += pv[t].z;
+        s4.w += pv[t].w;
       }
-      float v[4] = {s.x, s.y, s.z, s.w};
-      epilogue<4>(p, bz, m0 + r, n0 + c, v);
+      float v[4] = {s4.x, s4.y, s4.z, s4.w};
+      epilogue<4>(p, bz, m0 + rr, n0 + c, v);
     }
     tc::cluster_sync();  // no CTA leaves while a peer may still read its partials
   } else {
@@ -432,11 +334,65 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     tc::fence_after();
     tc::dealloc(tmem, BN);
   }
-  if (warp == 0 && lane == 0 && !ok) {
+  if (threadIdx.x == 0 && !ok) {
     // copies already requested land before the CTA exits (bounded)
-    for (int i = 0; i < issued; ++i) mbar_wait_bounded(&full_w[i % kNS], (i / kNS) & 1, nullptr);
+    for (int i = 0; i < issued; ++i) mbar_wait_bounded(&full[i % ns], (i / ns) & 1, nullptr);
   }
 }
+
+// h = LayerNorm(x) * g + b in fp32 (mean, then the biased variance of the
+// centred values), rounded to bf16. x [n][d] fp32, d a multiple of 4.
+__global__ void __launch_bounds__(kLnThreads) layernorm_kernel(const float* __restrict__ x, int n, int d,
+                                                                const float* __restrict__ g,
+                                                                const float* __restrict__ b, float eps,
+                                                                uint16_t* __restrict__ h) {
+  if (threadIdx.x == 0) griddep_launch();
+  griddep_wait();
+  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x * (kLnThreads / 32) + (threadIdx.x >> 5);
+  if (row >= n) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)row * d);
+  const int c4 = d / 4;
+  float s = 0.f;
+  for (int c = lane; c < c4; c += 32) {
+    const float4 v = xr[c];
+    s += (v.x + v.y) + (v.z + v.w);
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  const float mean = s / (float)d;
+  float q = 0.f;
+  for (int c = lane; c < c4; c += 32) {
+    const float4 v = xr[c];
+    const float a = v.x - mean, bb = v.y - mean, cc = v.z - mean, dd = v.w - mean;
+    q += (a * a + bb * bb) + (cc * cc + dd * dd);
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+  const float rstd = rsqrtf(q / (float)d + eps);
+  const float4* g4 = reinterpret_cast<const float4*>(g);
+  const float4* b4 = reinterpret_cast<const float4*>(b);
+  uint2* hr = reinterpret_cast<uint2*>(h + (size_t)row * d);
+  for (int c = lane; c < c4; c += 32) {
+    const float4 v = xr[c], gg = g4[c], bv = b4[c];
+    uint2 o;
+    o.x = pack_bf16x2((v.x - mean) * rstd * gg.x + bv.x, (v.y - mean) * rstd * gg.y + bv.y);
+    o.y = pack_bf16x2((v.z - mean) * rstd * gg.z + bv.z, (v.w - mean) * rstd * gg.w + bv.w);
+    hr[c] = o;
+  }
+}
+
+}  // namespace
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("SMEM_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
+
+namespace {
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -453,12 +409,15 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 template <int BN>
 cudaError_t launch_bn(GemmParams& p, int tiles_n, int mtiles, int batch, bool pdl, cudaStream_t st) {
   using C = Gm<BN>;
-  cudaError_t e = ensure_smem_limit<100 + BN>(gemm_kernel<BN>, C::SMEM);
+  cudaError_t e = ensure_smem_limit<100 + BN>(gemm_kernel<BN>, C::SMEM_MAX);
   if (e != cudaSuccess) return e;
+  const int per_cta = (p.chunks + p.ks - 1) / p.ks;  // K chunks of the longest split
+  p.ns = per_cta < kNS ? (per_cta > 1 ? per_cta : 1) : kNS;
+  p.ring_bytes = C::ring_bytes(p.ns, p.M < kBM ? p.M : kBM, p.ks);
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3((unsigned)(tiles_n * p.ks), (unsigned)mtiles, (unsigned)batch);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.dynamicSmemBytes = (size_t)p.ring_bytes + C::MISC + 1024;
   cfg.stream = st;
   cudaLaunchAttribute at[2];
   int na = 0;
@@ -469,7 +428,7 @@ cudaError_t launch_bn(GemmParams& p, int tiles_n, int mtiles, int batch, bool pd
     at[na].val.clusterDim.z = 1;
     ++na;
   }
-  if (pdl) {
+  if (pdl && pdl_enabled()) {
     at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     at[na].val.programmaticStreamSerializationAllowed = 1;
     ++na;
@@ -481,55 +440,168 @@ cudaError_t launch_bn(GemmParams& p, int tiles_n, int mtiles, int batch, bool pd
 
 }  // namespace
 
-// Tile and split plan of a projection: the widest N tile and the largest
-// cluster (<= 8 CTAs, at most one 64-column K chunk per CTA minimum) that
-// keep the grid within one wave of the device's SMs. A function of the shape
-// and the SM count only.
+// Clusters of `ks` CTAs of the BN = 64 / 128 kernel that the current device
+// holds at once (a GPC hosts only whole clusters), per device, looked up once.
+namespace {
+int max_active_clusters(int bn, int ks) {
+  constexpr int kMaxDev = 16;
+  static int table[kMaxDev][2][kMaxCluster + 1] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 0;
+  int& v = table[dev][bn == 128 ? 1 : 0][ks];
+  if (v) return v;
+  const void* fn = bn == 128 ? reinterpret_cast<const void*>(gemm_kernel<128>)
+                             : reinterpret_cast<const void*>(gemm_kernel<64>);
+  const int smem = bn == 128 ? Gm<128>::SMEM_MAX : Gm<64>::SMEM_MAX;
+  cudaError_t e = bn == 128 ? ensure_smem_limit<228>(gemm_kernel<128>, smem) : ensure_smem_limit<164>(gemm_kernel<64>, smem);
+  if (e != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)(ks * 64));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = (unsigned)ks;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = 1;
+  }
+  v = n;
+  return n;
+}
+}  // namespace
+
+// Tile and split plan of a projection: over BN in {128, 64} and clusters of
+// 1..8 CTAs (at least one 64-column K chunk per CTA), the most CTAs whose
+// clusters the device holds in one wave; ties keep the wider tile. A
+// function of the shape and the device only.
 GemmPlan gemm_plan(int M, int N, int K, int batch, int num_sms) {
+  (void)num_sms;
   const int chunks = (K + 63) / 64;
   const int mtiles = (M + kBM - 1) / kBM;
   GemmPlan best{128, 1, 0};
   for (int bn : {128, 64}) {
+    if (bn == 128 && N <= 64) continue;  // a 64-wide output needs no 128 tile
     const int tiles = (N + bn - 1) / bn * mtiles * batch;
-    int ks = tiles >= num_sms ? 1 : std::max(1, num_sms / tiles);
-    ks = std::min(ks, std::min(kMaxCluster, std::max(1, chunks)));
-    const int ctas = tiles * ks;
-    if (ctas > best.ctas) best = GemmPlan{bn, ks, ctas};
+    for (int ks = 1; ks <= std::min(kMaxCluster, chunks); ++ks) {
+      if (ks > 1 && tiles > max_active_clusters(bn, ks)) break;  // a second wave of clusters
+      if (ks == 1 && tiles > max_active_clusters(bn, 1) && best.ctas > 0) break;
+      const int ctas = tiles * ks;
+      if (ctas > best.ctas) best = GemmPlan{bn, ks, ctas};
+    }
   }
   return best;
+}
+
+namespace {
+// Tensor maps of recently used operands (bf16, 128-byte swizzle), keyed by
+// address, rank, extents, strides and box: a layer call reuses every layer's
+// weights and the same workspace buffers on every call.
+bool cached_map(CUtensorMap* out, const void* ptr, int rank, const uint64_t* dims, const uint64_t* strides,
+                const uint32_t* box) {
+  struct Entry {
+    const void* ptr;
+    int rank;
+    uint64_t dims[3], strides[2];
+    uint32_t box[3];
+    CUtensorMap map;
+  };
+  constexpr int kEntries = 96;
+  static thread_local Entry cache[kEntries];
+  static thread_local int used = 0, next = 0;
+  for (int i = 0; i < used; ++i) {
+    const Entry& e = cache[i];
+    bool same = e.ptr == ptr && e.rank == rank;
+    for (int k = 0; same && k < rank; ++k) same = e.dims[k] == dims[k] && e.box[k] == box[k];
+    for (int k = 0; same && k + 1 < rank; ++k) same = e.strides[k] == strides[k];
+    if (same) {
+      *out = e.map;
+      return true;
+    }
+  }
+  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+  if (!enc) return false;
+  Entry& e = cache[next];
+  cuuint64_t d[3], st[2];
+  cuuint32_t bx[3], es[3] = {1, 1, 1};
+  for (int k = 0; k < rank; ++k) {
+    d[k] = dims[k];
+    bx[k] = box[k];
+  }
+  for (int k = 0; k + 1 < rank; ++k) st[k] = strides[k];
+  if (enc(&e.map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(ptr), d, st, bx, es,
+          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return false;
+  e.ptr = ptr;
+  e.rank = rank;
+  for (int k = 0; k < 3; ++k) {
+    e.dims[k] = k < rank ? dims[k] : 0;
+    e.box[k] = k < rank ? box[k] : 0;
+  }
+  for (int k = 0; k < 2; ++k) e.strides[k] = k + 1 < rank ? strides[k] : 0;
+  *out = e.map;
+  next = (next + 1) % kEntries;
+  if (used < kEntries) ++used;
+  return true;
+}
+}  // namespace
+
+cudaError_t launch_layernorm(const float* x, int n, int d, const float* g, const float* b, uint16_t* h, bool pdl,
+                             cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)((n + kLnThreads / 32 - 1) / (kLnThreads / 32)));
+  cfg.blockDim = dim3(kLnThreads);
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = pdl && pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, layernorm_kernel, x, n, d, g, b, kLayerNormEps, h);
 }
 
 cudaError_t launch_gemm(const GemmCall& g, int num_sms, cudaStream_t st) {
   if (g.M <= 0 || g.N <= 0 || g.batch <= 0) return cudaSuccess;
   if (g.N % 32 || g.K % 32 || g.K <= 0) return cudaErrorInvalidValue;
-  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
-  if (!enc) return cudaErrorNotSupported;
+  if (!encode_fn()) return cudaErrorNotSupported;
   const GemmPlan pl = gemm_plan(g.M, g.N, g.K, g.batch, num_sms);
   static thread_local GemmParams p;
   p = GemmParams{};
-  const cuuint64_t dims[2] = {(cuuint64_t)g.w_cols, (cuuint64_t)g.w_rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)g.ldw * 2};
-  const cuuint32_t box[2] = {64u, g.b_kmajor ? (cuuint32_t)pl.bn : 64u};
-  const cuuint32_t estr[2] = {1, 1};
-  const CUresult r = enc(&p.wmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(g.w), dims, strides, box, estr,
-                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-  p.a = g.a;
-  p.ln_g = g.ln_g;
-  p.ln_b = g.ln_b;
+  const int boxy = g.b_kmajor ? pl.bn : 64;
+  {
+    const uint64_t dims[3] = {(uint64_t)g.w_cols, (uint64_t)g.w_rows, 1};
+    const uint64_t strides[2] = {(uint64_t)g.ldw * 2, (uint64_t)g.ldw * 2 * g.w_rows};
+    const uint32_t box[3] = {64u, (uint32_t)boxy, 1u};
+    if (!cached_map(&p.wmap, g.w, 2, dims, strides, box)) return cudaErrorInvalidValue;
+  }
+  // activations: a [batch][M][K] view, or [M][batch][K] when the batch
+  // stride is the smaller one (strides increase outward either way); rows
+  // and columns past M and K read as zero
+  {
+    const long long bs = g.batch > 1 ? g.a_bs : (long long)g.lda * g.M;
+    p.a_bmajor = g.batch > 1 && bs < g.lda ? 1 : 0;
+    const uint64_t dims[3] = {(uint64_t)g.K, (uint64_t)(p.a_bmajor ? g.batch : g.M),
+                              (uint64_t)(p.a_bmajor ? g.M : g.batch)};
+    const uint64_t strides[2] = {(uint64_t)(p.a_bmajor ? bs : g.lda) * 2, (uint64_t)(p.a_bmajor ? g.lda : bs) * 2};
+    const uint32_t box[3] = {64u, p.a_bmajor ? 1u : (uint32_t)kBM, p.a_bmajor ? (uint32_t)kBM : 1u};
+    if (!cached_map(&p.amap, g.a, 3, dims, strides, box)) return cudaErrorInvalidValue;
+  }
   p.out = g.out;
   p.rope_tab = g.rope_tab;
   p.ib = g.ib;
-  p.a_bs = g.a_bs;
   p.o_bs = g.o_bs;
   p.group_stride = g.group_stride;
-  p.lda = g.lda;
   p.ldo = g.ldo;
   p.M = g.M;
   p.N = g.N;
   p.K = g.K;
-  p.ln = g.ln_g != nullptr;
   p.b_kmajor = g.b_kmajor;
   p.w_boff = g.w_boff;
   p.epi = g.epi;
@@ -542,7 +614,6 @@ cudaError_t launch_gemm(const GemmCall& g, int num_sms, cudaStream_t st) {
   p.ib_kvd = g.ib_kvd;
   p.ib_D = g.ib_D;
   p.alpha = g.alpha;
-  p.eps = kLayerNormEps;
   p.err = g.err;
   const int tiles_n = (g.N + pl.bn - 1) / pl.bn;
   const int mtiles = (g.M + kBM - 1) / kBM;

@@ -180,19 +180,16 @@ enum GemmEpilogue : int {
 };
 
 // One projection out[b][m][n] = epi(alpha * sum_k A[b][m][k] W_b[k][n]) for
-// b < batch (grid z). A: bf16 [M][lda] (+ b * a_bs), or with ln_g set the
-// fp32 residual stream [M][lda] normalised on the fly (LayerNorm over K
-// columns, gain ln_g, bias ln_b). W: the bf16 matrix [w_rows][w_cols] (row
-// pitch ldw elements); b_kmajor = 0: W is [K][N] (the batch's columns start
-// at b * w_boff); 1: W is [N][K] (the batch's K columns start at b * w_boff).
-// Output column n goes to out + b * o_bs + (n / col_group) * group_stride +
-// m * ldo + n % col_group (col_group 0: N). N and K multiples of 32.
+// b < batch (grid z). A: bf16 [M][lda] (+ b * a_bs). W: the bf16 matrix
+// [w_rows][w_cols] (row pitch ldw elements); b_kmajor = 0: W is [K][N] (the
+// batch's columns start at b * w_boff); 1: W is [N][K] (the batch's K
+// columns start at b * w_boff). Output column n goes to out + b * o_bs +
+// (n / col_group) * group_stride + m * ldo + n % col_group (col_group 0: N).
+// N and K multiples of 32.
 struct GemmCall {
   const void* a = nullptr;
   int lda = 0;
   long long a_bs = 0;
-  const float* ln_g = nullptr;
-  const float* ln_b = nullptr;
   const void* w = nullptr;
   int w_rows = 0, w_cols = 0, ldw = 0;
   int b_kmajor = 0;
@@ -218,19 +215,28 @@ struct GemmCall {
 
 struct GemmParams {
   CUtensorMap wmap;
-  const void* a;
-  const float* ln_g;
-  const float* ln_b;
+  CUtensorMap amap;  // bf16 A as [batch][M][K] (a_bmajor: [M][batch][K]), boxes of 64 columns x 128 rows
   void* out;
   const float2* rope_tab;
   uint16_t* ib;
-  long long a_bs, o_bs, group_stride;
-  int lda, ldo, M, N, K;
-  int ln, b_kmajor, w_boff, epi, col_group, ks, chunks;
+  long long o_bs, group_stride;
+  int ldo, M, N, K;
+  int b_kmajor, w_boff, epi, col_group, ks, chunks, a_bmajor;
+  int ns, ring_bytes;  // ring stages of this launch and their bytes (set by the launcher)
   int rope_cols, rope_D, ib_col0, ib_kvd, ib_D;
-  float alpha, eps;
+  float alpha;
   int* err;
 };
+
+// h [n][d] bf16 = LayerNorm(x [n][d] fp32) * g + b (programmatic dependent
+// launch when `pdl`).
+cudaError_t launch_layernorm(const float* x, int n, int d, const float* g, const float* b, uint16_t* h, bool pdl,
+                             cudaStream_t st);
+
+// Programmatic dependent launch for the layer path's projections and the
+// one-block prefill: on unless the environment variable SMEM_PDL is "0"
+// (read once per process).
+bool pdl_enabled();
 
 struct GemmPlan {
   int bn, ks, ctas;

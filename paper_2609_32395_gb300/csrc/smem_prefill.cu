@@ -742,7 +742,7 @@ static cudaError_t launch_prefill_d(const PrefillParams& p, int grid, cudaStream
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
   e = cudaLaunchKernelEx(&cfg, prefill_kernel<D, false, ROPE>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
@@ -774,7 +774,7 @@ static cudaError_t launch_prefill_cluster(const PrefillParams& p, cudaStream_t s
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;
   e = cudaLaunchKernelEx(&cfg, prefill_kernel<64, true, ROPE>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

@@ -9,8 +9,8 @@
 //   sum_r p_r (mu_r W_vc,h) = (sum_r p_r mu_r) W_vc,h
 // and the layer's cross-attention is an attention of d-wide queries q'_h
 // over the d-wide rows mu_r whose output O'_h = sum_r p_r mu_r is mapped by
-// W_vc,h afterwards. The two small per-head maps run as cuBLAS GEMMs before
-// and after this kernel; this kernel streams every row once per layer (2d
+// W_vc,h afterwards. The two small per-head maps run on the projection
+// kernel (smem_gemm.cu) before and after this one; this kernel streams every row once per layer (2d
 // bytes per row, half the materialized 4 H d_h) and keeps all queries that
 // share a row set in one CTA:
 //   S^T [64 rows][NQ queries] = mu_tile Q'^T   (K = d)

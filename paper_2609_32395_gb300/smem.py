@@ -35,7 +35,8 @@ EXPORTED = [
     "smem_cache_required_bytes", "smem_cache_create", "smem_cache_destroy", "smem_set_null_row",
     "smem_append_block", "smem_delete_block", "smem_release_seq", "smem_write_inblock", "smem_prefill_block",
     "smem_decode", "smem_decode_static_scratch", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table",
-    "smem_check_device_error", "smem_debug_gemm", "smem_debug_set_table_entry", "smem_debug_wait_probe",
+    "smem_check_device_error", "smem_debug_gemm", "smem_debug_layernorm", "smem_debug_set_table_entry",
+    "smem_debug_wait_probe",
     "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
     "smem_layer_workspace_bytes", "smem_append_block_rows", "smem_set_null_vector", "smem_reader_layer_prefill",
     "smem_reader_layer_decode", "smem_mu_decode", "smem_mu_prefill", "smem_share_block", "smem_slot_refs",
@@ -125,9 +126,10 @@ def lib():
             "smem_mu_decode_plan": (ctypes.c_int, [_vp, _i32p, _i32p, _i32p]),
             "smem_debug_set_table_entry": (ctypes.c_int, [_vp, _i32, _i32, _i32, _vp]),
             "smem_debug_wait_probe": (ctypes.c_int, [_vp, ctypes.c_longlong, _vp]),
-            "smem_debug_gemm": (ctypes.c_int, [_vp, _vp, _i32, ctypes.c_longlong, _vp, _vp, _vp, _i32, _i32, _i32,
-                                               _i32, _i32, _i32, _i32, _i32, _i32, ctypes.c_float, _vp, _i32,
-                                               ctypes.c_longlong, _i32, ctypes.c_longlong, _vp]),
+            "smem_debug_gemm": (ctypes.c_int, [_vp, _vp, _i32, ctypes.c_longlong, _vp, _i32, _i32, _i32, _i32, _i32,
+                                               _i32, _i32, _i32, _i32, ctypes.c_float, _vp, _i32, ctypes.c_longlong,
+                                               _i32, ctypes.c_longlong, _vp]),
+            "smem_debug_layernorm": (ctypes.c_int, [_vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -320,14 +322,21 @@ def smem_debug_wait_probe(h, limit_ns, stream=None):
     _check(lib().smem_debug_wait_probe(h, int(limit_ns), _stream(stream)), "smem_debug_wait_probe")
 
 
-def smem_debug_gemm(h, A, lda, W, b_kmajor, M, N, K, out, ldo, a_bs=0, ln_g=None, ln_b=None, w_boff=0, batch=1,
-                    epi=0, alpha=1.0, o_bs=0, col_group=0, group_stride=0, stream=None):
+def smem_debug_gemm(h, A, lda, W, b_kmajor, M, N, K, out, ldo, a_bs=0, w_boff=0, batch=1, epi=0, alpha=1.0,
+                    o_bs=0, col_group=0, group_stride=0, stream=None):
     """Testing hook: one projection on the reader layer's tensor-core kernel
     (see include/smem.h); W's shape is taken from the tensor."""
     w_rows, w_cols = int(W.shape[0]), int(W.shape[1])
-    return _check(lib().smem_debug_gemm(h, _ptr(A), lda, a_bs, _ptr(ln_g), _ptr(ln_b), _ptr(W), w_rows, w_cols,
-                                        b_kmajor, w_boff, M, N, K, batch, epi, float(alpha), _ptr(out), ldo, o_bs,
-                                        col_group, group_stride, _stream(stream)), "smem_debug_gemm")
+    return _check(lib().smem_debug_gemm(h, _ptr(A), lda, a_bs, _ptr(W), w_rows, w_cols, b_kmajor, w_boff, M, N, K,
+                                        batch, epi, float(alpha), _ptr(out), ldo, o_bs, col_group, group_stride,
+                                        _stream(stream)), "smem_debug_gemm")
+
+
+def smem_debug_layernorm(h, x, gain, bias, out, stream=None):
+    """Testing hook: the reader layer's LayerNorm kernel on x [n][d] fp32."""
+    n, d = int(x.shape[0]), int(x.shape[1])
+    return _check(lib().smem_debug_layernorm(h, _ptr(x), n, d, _ptr(gain), _ptr(bias), _ptr(out), _stream(stream)),
+                  "smem_debug_layernorm")
 
 
 def smem_abi_version() -> int:

@@ -131,8 +131,8 @@ def test_layer_entry_points_on_a_bookkeeping_cache():
         w0 = smem.smem_layer_workspace_bytes(h, 0)
         w64 = smem.smem_layer_workspace_bytes(h, 64)
         assert w0 == 256  # the memory-row projections need no scratch (a nominal minimum)
-        # qkv (bf16 3d), att and qc (bf16 d each), g (bf16 4d) per row
-        assert w64 == 64 * (3 * d * 2 + 2 * d * 2 + 4 * d * 2)
+        # h (LayerNorm output, bf16 d), qkv (bf16 3d), att and qc (bf16 d each), g (bf16 4d) per row
+        assert w64 == 64 * (d * 2 + 3 * d * 2 + 2 * d * 2 + 4 * d * 2)
         assert smem.smem_layer_workspace_bytes(h, 65) == 0      # above max(b, max_decode_batch)
         assert smem.smem_layer_workspace_bytes(h, -1) == 0
         w = [smem.SmemLayerWeights()] * 2
