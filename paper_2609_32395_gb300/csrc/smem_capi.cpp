@@ -758,6 +758,7 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     const std::vector<int32_t>& ix = c->idx[s];
     nblk[i] = (int)(std::lower_bound(ix.begin(), ix.end(), q_block_idx[i]) - ix.begin());
   }
+  const int qn = smem::decode_group_width(L.D, L.H / L.Hkv, L.rope_w != 0);  // the units smem_decode runs
   // scratch layout per launch: [256 B scheduler words][tickets][partials]
   const size_t ticket_bytes = align_up((size_t)std::min(nb, smem::kMaxDecodeItems) * L.H * 4, 256);
   size_t need = 0;
@@ -808,7 +809,7 @@ int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const i
     P.s_stride = P.c_stride = L.H * L.D;
     P.Hkv = L.Hkv;
     P.kv_stride = L.Hkv * L.D;
-    P.qn = smem::decode_group_width(L.D, L.H / L.Hkv, L.rope_w != 0);  // the units smem_decode runs
+    P.qn = qn;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)L.D));
     P.rope_tab = rope_tab(c);
     P.bidx = reinterpret_cast<const int*>(c->dev + L.off_bidx);

@@ -22,9 +22,10 @@
 // completes the last split of an (item, head) merges all splits in split
 // order (null row first). With grouped-query attention a CA unit serves the
 // 2 or 4 query heads that share a key/value head: the warp scores each stage
-// against all of them with warp-level tensor-core MMAs (the group as the
-// rows of a 16-row operand) and keeps P in registers for P.V, so the rows
-// stream once per group at a few dozen instructions per stage. SA units
+// against all of them with warp-level tensor-core MMAs (the stage's keys as
+// the 16 rows, the group's queries as the columns), transposes P in
+// registers (movmatrix) into the operand of O^T += V^T P^T, so the rows
+// stream once per group at 16 MMAs per stage. SA units
 // read their <= 64 in-block rows straight from global memory. No warp ever waits for another warp; every reduction
 // order is fixed by the block count, so the same block set gives the same
 // bits whatever the slots or the edit history.
@@ -150,6 +151,20 @@ __device__ __forceinline__ void mma_16816_acc2(float (&d)[2], uint32_t a0, uint3
       "{%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(z0), "+f"(z1)
       : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+// D[16x8] += A[16x16] B[16x8] with every A row used (keys as rows).
+__device__ __forceinline__ void mma_16816_full(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// Transpose of an 8x8 b16 matrix held as (row lane/4, columns 2(lane%4) ..+1).
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
 }
 // Four 8x8 b16 matrices; lane l gives the 16-byte row address of row l%8 of
 // matrix l/8. Plain: thread (g, t) gets row g, columns 2t, 2t+1 of each
@@ -575,25 +590,26 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     if constexpr (QN > 1) {
       // ---- grouped unit: the p.qn query heads U.h .. U.h+qn-1 read one
       // key/value head; the warp scores every stage against all of them on
-      // the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate): the
-      // group's queries are rows 0..qn-1 of a 16-row A operand (the other
-      // rows zero), K and V fragments come from the swizzled stage by
-      // ldmatrix, and P goes from the score accumulators straight into the
-      // A operand of O += P.V (bf16). Thread (gq = lane/4, tq = lane%4)
-      // holds query row gq: its scores of rows 2tq, 2tq+1 of every 8-row
-      // tile of the stage and its O columns 2tq, 2tq+1 of every 8 columns.
-      // The rows stream once per group; a stage costs 2 * 16 MMAs.
-      constexpr int KS = D / 16;        // k-steps of a score MMA chain
-      constexpr int NT = C::SROWS / 8;  // 8-row tiles of a stage
-      constexpr int ON = D / 8;         // 8-column tiles of O
+      // the tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate) with
+      // the stage's keys as the 16 rows and the group's queries as the 8
+      // columns (query columns >= qn are zero):
+      //   S^T[key][q] = K[key][:] . Q[q][:]     (A = K by ldmatrix, B = Q)
+      //   O^T[c][q]  += V^T[c][key] P^T[key][q] (A = V^T by ldmatrix.trans)
+      // P^T's fragments come from the score accumulators by one movmatrix
+      // transpose per 8x8 tile. Thread (g = lane/4, t = lane%4) holds keys g,
+      // g+8 of every 16-key tile and columns c = g, g+8 of every 16-column
+      // tile, for queries 2t, 2t+1. A stage costs 16 MMAs at every head
+      // width; the rows stream once per group.
+      constexpr int MT = C::SROWS / 16;  // 16-key tiles of a stage
+      constexpr int KS = D / 16;         // k-steps of the score MMAs
+      constexpr int DT = D / 16;         // 16-column tiles of O^T
       const int ng = p.qn;
       const int gq = lane >> 2, tq = lane & 3;
-      const bool real = gq < ng;
-      uint32_t qa[KS][2];  // A fragments of row gq: columns 16ks + 2tq (+8)
-      float o[ON][2];
-      float gmr = -INFINITY, glr = 0.f;  // running maximum, partial sum (this thread's rows)
+      uint32_t qb[KS][2];  // B fragments: query gq, columns 16ks + 2tq (+8)
+      float o[DT][4];      // O^T: columns 16dt + gq (+8) x queries 2tq, 2tq+1
+      float gm[2] = {-INFINITY, -INFINITY}, gl[2] = {0.f, 0.f};  // per query column 2tq + e
 #pragma unroll
-      for (int on = 0; on < ON; ++on) o[on][0] = o[on][1] = 0.f;
+      for (int dt = 0; dt < DT; ++dt) o[dt][0] = o[dt][1] = o[dt][2] = o[dt][3] = 0.f;
       const int nch = U.nt * C::CHUNKS;
       for (int ch = 0; ch < nch; ++ch, ++k) {
         const int s = k % C::NS;
@@ -604,68 +620,79 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
           break;
         }
         if (ch == 0) {
+          const bool real = gq < ng;
           const uint16_t* qs = qarea + s * QN * D + (real ? gq : 0) * D;
 #pragma unroll
           for (int ks = 0; ks < KS; ++ks) {
-            qa[ks][0] = real ? *reinterpret_cast<const uint32_t*>(qs + 16 * ks + 2 * tq) : 0u;
-            qa[ks][1] = real ? *reinterpret_cast<const uint32_t*>(qs + 16 * ks + 8 + 2 * tq) : 0u;
+            qb[ks][0] = real ? *reinterpret_cast<const uint32_t*>(qs + 16 * ks + 2 * tq) : 0u;
+            qb[ks][1] = real ? *reinterpret_cast<const uint32_t*>(qs + 16 * ks + 8 + 2 * tq) : 0u;
           }
         }
         const uint8_t* kb = ring + s * C::STAGE;
         const uint8_t* vb = kb + C::HALF;
-        // S[q][r] = Q[q] . K[r]: one ldmatrix.x4 brings two k-steps of an 8-row tile
-        float sacc[NT][4];
+        // S^T per 16-key tile: keys as A rows (lane l addresses key 16mt +
+        // l%8 + 8((l/8)%2), columns 16ks + 8(l/16) ..)
+        float sacc[MT][4];
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
+        for (int mt = 0; mt < MT; ++mt) {
+          sacc[mt][0] = sacc[mt][1] = sacc[mt][2] = sacc[mt][3] = 0.f;
 #pragma unroll
-          for (int kp = 0; kp < KS / 2; ++kp) {
-            uint32_t b[4];
-            ldsm_x4(b, smem_u32(kb + chunk_off<D>(8 * nt + (lane & 7), 4 * kp + (lane >> 3))));
-            mma_16816(sacc[nt], qa[2 * kp][0], qa[2 * kp][1], b[0], b[1]);
-            mma_16816(sacc[nt], qa[2 * kp + 1][0], qa[2 * kp + 1][1], b[2], b[3]);
+          for (int ks = 0; ks < KS; ++ks) {
+            uint32_t a[4];
+            ldsm_x4(a, smem_u32(kb + chunk_off<D>(16 * mt + (lane & 7) + 8 * ((lane >> 3) & 1), 2 * ks + (lane >> 4))));
+            mma_16816_full(sacc[mt], a, qb[ks][0], qb[ks][1]);
           }
         }
-        // online softmax of row gq over the stage (the quad of tq holds the row)
-        float mx = -INFINITY;
+        // online softmax per query column (2tq + e): maximum over the keys of
+        // this thread, then over the 8 threads of the column (lanes tq + 4j)
+        float mx[2] = {-INFINITY, -INFINITY};
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          sacc[nt][0] *= p.scale_log2;
-          sacc[nt][1] *= p.scale_log2;
-          mx = fmaxf(mx, fmaxf(sacc[nt][0], sacc[nt][1]));
-        }
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-        const float m_new = fmaxf(gmr, mx);
-        const float alpha = exp2f(gmr - m_new);
-        gmr = m_new;
-        uint32_t pa[NT];  // bf16 P of row gq, rows 2tq, 2tq+1 of each 8-row tile
-        float ps = 0.f;
+        for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          const uint32_t w = real ? pack_bf16x2(exp2f(sacc[nt][0] - m_new), exp2f(sacc[nt][1] - m_new)) : 0u;
-          pa[nt] = w;
-          ps += bf16lo(w) + bf16hi(w);  // the sum of the P the MMA uses
-        }
-        glr = glr * alpha + ps;
-#pragma unroll
-        for (int on = 0; on < ON; ++on) {
-          o[on][0] *= alpha;
-          o[on][1] *= alpha;
-        }
-        // O[q][c] += P[q][r] V[r][c]: k-step = 16 rows (two score tiles), one
-        // ldmatrix.x4.trans brings two 8-column tiles of V
-#pragma unroll
-        for (int kk = 0; kk < NT / 2; ++kk) {
-#pragma unroll
-          for (int op = 0; op < ON / 2; ++op) {
-            uint32_t b[4];
-            ldsm_x4_trans(b, smem_u32(vb + chunk_off<D>(16 * kk + (lane & 7) + ((lane >> 3) & 1) * 8,
-                                                       2 * op + (lane >> 4))));
-            mma_16816_acc2(o[2 * op], pa[2 * kk], pa[2 * kk + 1], b[0], b[1]);
-            mma_16816_acc2(o[2 * op + 1], pa[2 * kk], pa[2 * kk + 1], b[2], b[3]);
+          for (int e = 0; e < 4; ++e) {
+            sacc[mt][e] *= p.scale_log2;
+            mx[e & 1] = fmaxf(mx[e & 1], sacc[mt][e]);
           }
+        float alpha[2], mn[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+#pragma unroll
+          for (int off = 4; off < 32; off <<= 1) mx[e] = fmaxf(mx[e], __shfl_xor_sync(0xffffffffu, mx[e], off));
+          mn[e] = fmaxf(gm[e], mx[e]);
+          alpha[e] = exp2f(gm[e] - mn[e]);
+          gm[e] = mn[e];
         }
+        // P (bf16) and its transpose into the B fragments of P^T
+        uint32_t pb[MT][2];
+        float ps[2] = {0.f, 0.f};
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+          const uint32_t top = pack_bf16x2(exp2f(sacc[mt][0] - mn[0]), exp2f(sacc[mt][1] - mn[1]));  // key gq
+          const uint32_t bot = pack_bf16x2(exp2f(sacc[mt][2] - mn[0]), exp2f(sacc[mt][3] - mn[1]));  // key gq + 8
+          ps[0] += bf16lo(top) + bf16lo(bot);  // the sums of the P the MMAs use
+          ps[1] += bf16hi(top) + bf16hi(bot);
+          pb[mt][0] = movmatrix_trans(top);
+          pb[mt][1] = movmatrix_trans(bot);
+        }
+#pragma unroll
+        for (int e = 0; e < 2; ++e) gl[e] = gl[e] * alpha[e] + ps[e];
+#pragma unroll
+        for (int dt = 0; dt < DT; ++dt) {
+          o[dt][0] *= alpha[0];
+          o[dt][1] *= alpha[1];
+          o[dt][2] *= alpha[0];
+          o[dt][3] *= alpha[1];
+        }
+        // O^T += V^T P^T: A = V^T tiles by ldmatrix.trans (lane l addresses
+        // key 16kk + l%8 + 8(l/16), columns 16dt + 8((l/8)%2) ..)
+#pragma unroll
+        for (int dt = 0; dt < DT; ++dt)
+#pragma unroll
+          for (int kk = 0; kk < MT; ++kk) {
+            uint32_t a[4];
+            ldsm_x4_trans(a, smem_u32(vb + chunk_off<D>(16 * kk + (lane & 7) + 8 * (lane >> 4), 2 * dt + ((lane >> 3) & 1))));
+            mma_16816_full(o[dt], a, pb[kk][0], pb[kk][1]);
+          }
         __syncwarp();
         if (lane == 0) {
           fence_proxy_async_smem();
@@ -674,29 +701,42 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
         __syncwarp();
       }
       if (failed) break;
-      glr += __shfl_xor_sync(0xffffffffu, glr, 1);
-      glr += __shfl_xor_sync(0xffffffffu, glr, 2);
+      // column sums over the 8 threads of each query column
+#pragma unroll
+      for (int e = 0; e < 2; ++e)
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) gl[e] += __shfl_xor_sync(0xffffffffu, gl[e], off);
       const int nsplit = ceil_div(it.nblk, decode_split_blocks(it.nblk));
-      if (nsplit == 1 && !p.null_kv) {
-        if (real) {
-          const float inv = 1.f / glr;
-          uint16_t* dst = p.oca + ((size_t)U.item * p.H + U.h + gq) * D + 2 * tq;
+      const bool direct = nsplit == 1 && !p.null_kv;
+      const bool part_in = direct || SMEM_DCHECK((long long)it.pair_begin + U.split < p.part_pairs, p.err);
 #pragma unroll
-          for (int on = 0; on < ON; ++on)
-            *reinterpret_cast<uint32_t*>(dst + 8 * on) = pack_bf16x2(o[on][0] * inv, o[on][1] * inv);
-        }
-        continue;
-      }
-      if (real && SMEM_DCHECK((long long)it.pair_begin + U.split < p.part_pairs, p.err)) {
-        float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h + gq) * (D + 4);
+      for (int e = 0; e < 2; ++e) {
+        const int q = 2 * tq + e;
+        if (q >= ng || !part_in) continue;
+        if (direct) {
+          const float inv = 1.f / gl[e];
+          uint16_t* dst = p.oca + ((size_t)U.item * p.H + U.h + q) * D + gq;
 #pragma unroll
-        for (int on = 0; on < ON; ++on)
-          *reinterpret_cast<float2*>(pp + 4 + 8 * on + 2 * tq) = make_float2(o[on][0], o[on][1]);
-        if (tq == 0) {
-          pp[0] = gmr;
-          pp[1] = glr;
+          for (int dt = 0; dt < DT; ++dt) {
+            const __nv_bfloat16 b0 = __float2bfloat16_rn(o[dt][e] * inv);
+            const __nv_bfloat16 b1 = __float2bfloat16_rn(o[dt][2 + e] * inv);
+            dst[16 * dt] = *reinterpret_cast<const uint16_t*>(&b0);
+            dst[16 * dt + 8] = *reinterpret_cast<const uint16_t*>(&b1);
+          }
+        } else {
+          float* pp = p.part + ((size_t)(it.pair_begin + U.split) * p.H + U.h + q) * (D + 4);
+#pragma unroll
+          for (int dt = 0; dt < DT; ++dt) {
+            pp[4 + 16 * dt + gq] = o[dt][e];
+            pp[4 + 16 * dt + 8 + gq] = o[dt][2 + e];
+          }
+          if (gq == 0) {
+            pp[0] = gm[e];
+            pp[1] = gl[e];
+          }
         }
       }
+      if (direct) continue;
       __threadfence();
       // one ticket per query head, taken by lanes 0 .. ng-1 at once
       const bool mine = lane < ng && atomicAdd(&p.counters[U.item * p.H + U.h + lane], 1u) == (unsigned)(nsplit - 1);

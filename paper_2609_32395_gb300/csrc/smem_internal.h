@@ -40,7 +40,10 @@ struct Layout {
 // a unit's fixed costs (queries, partial, ticket, merge) stay small next to
 // its rows in batched decode. From 512 blocks on, ceil(nblk/64) within
 // [8, 32] -- 64 splits up to 2048 blocks, 128 at 4096 -- so that a long
-// context alone still gives the warps of every SM work.
+// context alone still gives the warps of every SM work. (Grouped-query
+// units use the same plan: splits qn times shorter, for more units per warp,
+// measured slower -- 13.9k against 18.2k tok/s at 4 key/value heads -- their
+// per-unit partials, tickets and merges cost more than the shorter tail.)
 SMEM_HD inline int decode_split_blocks(int nblk) {
   if (nblk < 512) return 16;
   const int sb = (nblk + 63) / 64;
