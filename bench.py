@@ -322,53 +322,30 @@ class DecodeWorkload:
         return launches
 
     def _step_host(self, host_inputs, host_outputs, host_blocks):
-        """One step with every layer's inputs copied in from pinned host memory
-        and its outputs copied out, the copies on a second stream overlapped
-        with the decode of the neighbouring layers: layer l+1's inputs come in
-        while layer l runs, layer l's outputs go out while layer l+1 runs (two
-        output buffers). The step ends when its last copy has landed."""
+        """One step through the library's host-buffer decode call: every
+        layer's inputs come from pinned host memory and its outputs go back
+        to it through smem_decode_host, the copies on a copy stream of their
+        own, ordered by the library against the decode of the neighbouring
+        layers (two staging halves). The step ends when its last copy has
+        landed."""
         import torch
 
         from paper_2609_32395_gb300 import smem
 
         if not hasattr(self, "copy_stream"):
             self.copy_stream = torch.cuda.Stream()
-            self.out2 = (torch.empty_like(self.osa), torch.empty_like(self.oca))
-            self.cev = [[torch.cuda.Event() for _ in range(self.L)] for _ in range(3)]
+            self.stage = torch.empty(smem.smem_decode_host_stage_bytes(self.h, self.S), dtype=torch.uint8,
+                                     device=self.osa.device)
         st = torch.cuda.current_stream()
         cs = self.copy_stream
-        ev_in, ev_out, ev_read = self.cev
         k = self.step_no % self.n_sets
-        outs = ((self.osa, self.oca), self.out2)
-        cs.wait_stream(st)
-
-        def load(layer):
-            with torch.cuda.stream(cs):
-                for dst, src in zip(self.inputs[k][layer], host_inputs[k][layer]):
-                    dst.copy_(src, non_blocking=True)
-                ev_in[layer].record(cs)
-
-        load(0)
-        launches = 0
+        pos, nblk = self.pos.astype(np.int32), self.nblk.astype(np.int32)
         for layer in range(self.L):
-            if layer + 1 < self.L:
-                load(layer + 1)
-            st.wait_event(ev_in[layer])
-            if layer >= 2:
-                st.wait_event(ev_read[layer - 2])  # this output buffer's last contents are on the host
-            osa, oca = outs[layer & 1]
-            qs, kn, vn, qc = self.inputs[k][layer]
-            smem.smem_decode(self.h, layer, self.seq_ids, self.pos.astype(np.int32), self.nblk.astype(np.int32),
-                             qs, kn, vn, qc, osa, oca)
-            launches += 1
-            ev_out[layer].record(st)
-            with torch.cuda.stream(cs):
-                cs.wait_event(ev_out[layer])
-                host_outputs[0][layer].copy_(osa, non_blocking=True)
-                host_outputs[1][layer].copy_(oca, non_blocking=True)
-                ev_read[layer].record(cs)
+            qs, kn, vn, qc = host_inputs[k][layer]
+            smem.smem_decode_host(self.h, layer, self.seq_ids, pos, nblk, qs, kn, vn, qc, host_outputs[0][layer],
+                                  host_outputs[1][layer], self.stage, stream=st, copy_stream=cs)
         st.wait_stream(cs)
-        return launches + self._advance(host_blocks)
+        return self.L + self._advance(host_blocks)
 
 
 class LayerStack:

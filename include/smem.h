@@ -222,6 +222,29 @@ int smem_decode(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids
                 const int32_t *q_block_idx, const void *qs, const void *k_new, const void *v_new,
                 const void *qc, void *osa, void *oca, void *stream);
 
+/* The decode step of smem_decode with HOST inputs and outputs (a serving
+ * loop whose tokens live on the host): qs, k_new, v_new, qc are host bf16
+ * arrays [nb][..][d_h] (k_new, v_new with n_kv_heads heads), osa, oca host
+ * bf16 [nb][H][d_h] receiving the results. The call copies the inputs into
+ * one half of the caller's device staging buffer `stage` (256-byte aligned,
+ * at least smem_decode_host_stage_bytes(c, nb) bytes; consecutive calls
+ * alternate between its two halves), runs the decode step on `stream`, and
+ * copies the outputs back -- all asynchronous. With copy_stream NULL the
+ * copies run on `stream`; with another stream they run there, ordered by
+ * events against the decode, so that one call's copies overlap the
+ * neighbouring calls' decode steps (a half is reused only after its
+ * previous outputs have left). The host arrays must stay valid until the
+ * stream(s) have drained and should be pinned (pageable memory makes the
+ * copies synchronous); the outputs are on the host once copy_stream (or
+ * stream) has drained. The first call creates the cache's ordering events
+ * (destroyed with the cache); no device memory is allocated.
+ * The paper has no counterpart. */
+size_t smem_decode_host_stage_bytes(const smem_cache *c, int32_t nb);
+int smem_decode_host(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids, const int32_t *pos,
+                     const int32_t *q_block_idx, const void *qs, const void *k_new, const void *v_new,
+                     const void *qc, void *osa, void *oca, void *stage, size_t stage_bytes, void *stream,
+                     void *copy_stream);
+
 /* Bytes of the library's fixed device scratch used by
  * smem_decode_static_scratch (16 MiB; held on every GPU that loads the
  * library, for the life of the process). */

@@ -43,6 +43,19 @@ struct smem_cache {
   int fail_after = 0;                      // test hook: n-th next launch fails
   int pf_cluster_max = 0;                  // prefill cluster limit on this device (0: no clusters)
   smem::MuDecodePlan mu_plan{};            // recompute caches: decode kernel and query tile on this device
+  // smem_decode_host: which half of the caller's staging buffer the next
+  // call uses, and per half the events ordering its copies and its decode
+  unsigned host_calls = 0;
+  cudaEvent_t ev_in[2]{}, ev_out[2]{}, ev_free[2]{};
+  bool ev_made = false;
+  ~smem_cache() {
+    if (ev_made)
+      for (int i = 0; i < 2; ++i) {
+        cudaEventDestroy(ev_in[i]);
+        cudaEventDestroy(ev_out[i]);
+        cudaEventDestroy(ev_free[i]);
+      }
+  }
 };
 
 namespace {
@@ -726,6 +739,83 @@ int smem_decode(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids
   const int tok = c->lay.H * c->lay.D;
   return decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, qs, k_new, v_new, qc, osa, oca, 3, tok, tok,
                      as_stream(stream), c->lay.Hkv * c->lay.D);
+}
+
+namespace {
+// Staging half of smem_decode_host for nb items: qs, k_new, v_new, qc, osa,
+// oca, each 256-byte aligned.
+struct HostStage {
+  size_t qs, kn, vn, qc, osa, oca, half;
+};
+HostStage host_stage(const Layout& L, int nb) {
+  HostStage h{};
+  const size_t q = align_up((size_t)nb * L.H * L.D * 2, 256), kv = align_up((size_t)nb * L.Hkv * L.D * 2, 256);
+  h.qs = 0;
+  h.kn = q;
+  h.vn = h.kn + kv;
+  h.qc = h.vn + kv;
+  h.osa = h.qc + q;
+  h.oca = h.osa + q;
+  h.half = h.oca + q;
+  return h;
+}
+}  // namespace
+
+size_t smem_decode_host_stage_bytes(const smem_cache* c, int32_t nb) {
+  if (!c || nb < 1 || nb > c->lay.max_batch) return 0;
+  return 2 * host_stage(c->lay, nb).half;
+}
+
+int smem_decode_host(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,
+                     const int32_t* q_block_idx, const void* qs, const void* k_new, const void* v_new, const void* qc,
+                     void* osa, void* oca, void* stage, size_t stage_bytes, void* stream, void* copy_stream) {
+  int rc = check_decode_args(c, layer, nb, seq_ids, pos, q_block_idx);
+  if (rc) return rc;
+  if (c->lay.recompute) return SMEM_ERR_UNSUPPORTED;
+  const void* ptrs[7] = {qs, k_new, v_new, qc, osa, oca, stage};
+  for (const void* p : ptrs)
+    if (!p) return SMEM_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(stage) & 255u) return SMEM_ERR_ALIGN;
+  const Layout& L = c->lay;
+  const HostStage hs = host_stage(L, nb);
+  if (stage_bytes < 2 * hs.half) return SMEM_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  if (!c->ev_made) {
+    for (int i = 0; i < 2 && !rc; ++i)
+      rc = cuda_rc(cudaEventCreateWithFlags(&c->ev_in[i], cudaEventDisableTiming), "event") ||
+           cuda_rc(cudaEventCreateWithFlags(&c->ev_out[i], cudaEventDisableTiming), "event") ||
+           cuda_rc(cudaEventCreateWithFlags(&c->ev_free[i], cudaEventDisableTiming), "event");
+    if (rc) return SMEM_ERR_CUDA;
+    c->ev_made = true;
+  }
+  const cudaStream_t st = as_stream(stream);
+  const cudaStream_t cs = copy_stream ? as_stream(copy_stream) : st;
+  const int half = (int)(c->host_calls & 1u);
+  uint8_t* b = static_cast<uint8_t*>(stage) + (size_t)half * hs.half;
+  const size_t qb = (size_t)nb * L.H * L.D * 2, kvb = (size_t)nb * L.Hkv * L.D * 2;
+  // inputs in on the copy stream once this half's previous outputs are out
+  cudaError_t e = cudaSuccess;
+  if (cs != st && c->host_calls >= 2) e = cudaStreamWaitEvent(cs, c->ev_free[half], 0);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.qs, qs, qb, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.kn, k_new, kvb, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.vn, v_new, kvb, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.qc, qc, qb, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess && cs != st) e = cudaEventRecord(c->ev_in[half], cs);
+  if (e == cudaSuccess && cs != st) e = cudaStreamWaitEvent(st, c->ev_in[half], 0);
+  if (e != cudaSuccess) return cuda_rc(e, "host decode inputs");
+  const int tok = L.H * L.D;
+  rc = decode_impl(c, layer, nb, seq_ids, pos, q_block_idx, b + hs.qs, b + hs.kn, b + hs.vn, b + hs.qc, b + hs.osa,
+                   b + hs.oca, 3, tok, tok, st, L.Hkv * L.D);
+  if (rc) return rc;
+  // outputs out on the copy stream after the decode
+  if (cs != st) e = cudaEventRecord(c->ev_out[half], st);
+  if (e == cudaSuccess && cs != st) e = cudaStreamWaitEvent(cs, c->ev_out[half], 0);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(osa, b + hs.osa, qb, cudaMemcpyDeviceToHost, cs);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(oca, b + hs.oca, qb, cudaMemcpyDeviceToHost, cs);
+  if (e == cudaSuccess && cs != st) e = cudaEventRecord(c->ev_free[half], cs);
+  if (e != cudaSuccess) return cuda_rc(e, "host decode outputs");
+  ++c->host_calls;
+  return SMEM_OK;
 }
 
 int smem_decode_static_scratch(smem_cache* c, int32_t layer, int32_t nb, const int32_t* seq_ids, const int32_t* pos,

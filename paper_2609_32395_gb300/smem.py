@@ -34,7 +34,7 @@ STATIC_SCRATCH_BYTES = 16 << 20
 EXPORTED = [
     "smem_cache_required_bytes", "smem_cache_create", "smem_cache_destroy", "smem_set_null_row",
     "smem_append_block", "smem_delete_block", "smem_release_seq", "smem_write_inblock", "smem_prefill_block",
-    "smem_decode", "smem_decode_static_scratch", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table",
+    "smem_decode", "smem_decode_static_scratch", "smem_decode_host", "smem_decode_host_stage_bytes", "smem_get_table", "smem_get_free_fifo", "smem_get_device_table",
     "smem_check_device_error", "smem_debug_gemm", "smem_debug_layernorm", "smem_debug_set_table_entry",
     "smem_debug_wait_probe",
     "smem_free_slots", "smem_last_error_detail", "smem_debug_fail_after", "smem_strerror", "smem_abi_version",
@@ -124,6 +124,9 @@ def lib():
             "smem_share_block": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32, _vp, _i32p]),
             "smem_slot_refs": (ctypes.c_int, [_vp, _i32, _i32p]),
             "smem_mu_decode_plan": (ctypes.c_int, [_vp, _i32p, _i32p, _i32p]),
+            "smem_decode_host_stage_bytes": (ctypes.c_size_t, [_vp, _i32]),
+            "smem_decode_host": (ctypes.c_int, [_vp, _i32, _i32, _i32p, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _vp,
+                                                _vp, ctypes.c_size_t, _vp, _vp]),
             "smem_debug_set_table_entry": (ctypes.c_int, [_vp, _i32, _i32, _i32, _vp]),
             "smem_debug_wait_probe": (ctypes.c_int, [_vp, ctypes.c_longlong, _vp]),
             "smem_debug_gemm": (ctypes.c_int, [_vp, _vp, _i32, ctypes.c_longlong, _vp, _i32, _i32, _i32, _i32, _i32,
@@ -266,6 +269,23 @@ def smem_decode_static_scratch(h, layer, seq_ids, pos, q_block_idx, qs, k_new, v
     return _check(lib().smem_decode_static_scratch(h, layer, len(s), sp, pp, qp, _ptr(qs), _ptr(k_new), _ptr(v_new),
                                                    _ptr(qc), _ptr(osa), _ptr(oca), _stream(stream)),
                   "smem_decode_static_scratch")
+
+
+def smem_decode_host_stage_bytes(h, nb) -> int:
+    return int(lib().smem_decode_host_stage_bytes(h, nb))
+
+
+def smem_decode_host(h, layer, seq_ids, pos, q_block_idx, qs, k_new, v_new, qc, osa, oca, stage, stream=None,
+                     copy_stream=None):
+    """smem_decode with host (pinned) input/output tensors and a device
+    staging buffer; asynchronous (see include/smem.h)."""
+    s, sp = _i32arr(seq_ids)
+    p_, pp = _i32arr(pos)
+    q, qp = _i32arr(q_block_idx)
+    cs = None if copy_stream is None else _stream(copy_stream)
+    return _check(lib().smem_decode_host(h, layer, len(s), sp, pp, qp, _ptr(qs), _ptr(k_new), _ptr(v_new), _ptr(qc),
+                                         _ptr(osa), _ptr(oca), _ptr(stage), stage.numel() * stage.element_size(),
+                                         _stream(stream), cs), "smem_decode_host")
 
 
 def smem_get_table(h, seq):
