@@ -386,7 +386,7 @@ def layer_decode_step(wl, stack, x, ws, mu, events=None):
                                       stack.sw[layer], x, ws)
     if events is not None:
         events[1].record(st)
-    ours = 8 * wl.L  # per layer: 6 projections (LayerNorm, GELU, residual fused) and 2 attention launches
+    ours = 11 * wl.L  # per layer: 3 LayerNorm, 6 projections (GELU, residual fused) and 2 attention launches
     wl.pos += 1
     for s in np.nonzero(wl.pos == B_TOK)[0]:
         smem.smem_append_block_rows(wl.h, int(s), int(wl.nblk[s]), mu, stack.sw, ws)
@@ -761,7 +761,7 @@ def measure_layer_serve(nblk, device, iters=30, flush_bytes=512 << 20, recompute
     out = {"context_blocks": nblk, "latency_ms": med, "latency_ms_min": lat[0], "alg_bytes": alg,
            "weight_bytes": w, "kv_bytes": kv, "achieved_gbs": alg / (med / 1e3) / 1e9,
            "flops": stack.flops_per_layer(B_TOK) * wl.L + wl.flops_per_launch() * wl.L,
-           "launches_per_serve": 8 * wl.L}
+           "launches_per_serve": (14 if recompute else 11) * wl.L}
     wl.cache.close()
     return out
 
