@@ -18,11 +18,14 @@
 // base-2 online softmax, and write P as bf16 into a swizzled smem tile. The
 // running maximum is raised only when a row's maximum grows by more than 2^8
 // (then that row of O is rescaled in TMEM); otherwise the stale maximum keeps
-// every P <= 256, and O and l stay consistent with it. QK^T of tile j+1
-// overlaps the softmax of tile j. A split writes its partial (m, l, O) and the
-// CTA that completes the last split of a head merges all splits in split
-// order (null row first). The in-block SA is one masked tile per head on the
-// same machinery. Reduction orders depend only on the block count.
+// every P <= 256, and O and l stay consistent with it. The MMA warp issues
+// QK^T two tiles ahead of P.V, so a score tile is in TMEM a whole softmax
+// pass before it is read. A split writes its partial (m, l, O) and the CTA
+// that completes the last split of a head merges all splits in split order
+// (null row first); in cluster mode the partials stay in shared memory and
+// the cluster merges them over DSMEM. The in-block SA is one masked tile per
+// head on the same machinery. Reduction orders depend only on the block
+// count.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -67,6 +70,8 @@ struct Pf {
   static constexpr int PART_BYTES = B * (D + 4) * 4;          // one split's partial rows
   static constexpr int MERGE_SPR = NS * STAGE / PART_BYTES;   // split partials staged per round
 };
+
+static_assert(2 * (Pf<64>::SMEM + 1024) <= 228 * 1024, "two d_h = 64 CTAs per SM");
 
 // Shared-memory descriptors of the K-major Q/K tiles (k-th step of 16
 // columns) and of the MN-major V tile (k-th step of 16 rows).
@@ -114,6 +119,16 @@ __device__ __forceinline__ void st_o(uint32_t trow, const uint32_t (&o)[D / 2]) 
 }
 
 constexpr float kRescaleLog2 = 8.0f;  // raise the running max when it grows by more than 2^8
+
+// 2^x by the hardware's approximate base-2 exponential (PTX ex2.approx.ftz:
+// relative error near 2^-22, subnormal results flushed to zero). The
+// arguments here are at most kRescaleLog2 and the results are rounded to
+// bf16 for the P.V product.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 struct PrefillParams {
   CUtensorMap pool;          // [C][L*H*2*R][D], box 64 columns x 128 rows (a block's K then V)
@@ -193,69 +208,56 @@ __device__ __forceinline__ float null_dot(const PrefillParams& p, const uint16_t
 
 // Cluster mode (d_h = 64): one cluster of n_splits + 1 CTAs per head, rank 0
 // the in-block SA tile and rank k the split k-1. Each split CTA parks its
-// partial rows (m, l, O) in its own shared memory; after a cluster barrier
-// every CTA merges a slice of the 64 rows by reading the others' partials
-// over distributed shared memory, in split order (null row first).
-template <int D, bool ROPE>
+// partial rows (m, l, O) in its own shared memory, and rank 0 parks the null
+// row as a partial of its own (m = its score, l = 1, O = its value row);
+// after a cluster barrier every CTA merges a slice of the 64 rows, one row
+// per warp, summing in rank order (null row first). Lane s fetches rank s's
+// (m, l) and the warp shares them by shuffles; every lane fetches its columns
+// of every rank's O; all remote loads of a row go out in one batch. A warp
+// arrives on the closing cluster barrier once it has consumed the last remote
+// values it reads (a relaxed arrival: the values are in registers by then, so
+// it need not wait for the warp's output stores), and the caller waits on it:
+// no CTA leaves while another still reads its shared memory.
+template <int D>
 __device__ void cluster_merge(const PrefillParams& p, int h, uint32_t rank, uint32_t cs, uint32_t stage_saddr,
                               int warp, int lane) {
   constexpr int CPL = D / 32;  // columns per lane
-  const int ns = (int)cs - 1;
   const int rp = (kBlockTok + (int)cs - 1) / (int)cs;
   const int r0 = (int)rank * rp, r1 = min(kBlockTok, r0 + rp);
+  if (r0 + warp >= r1) tc::cluster_arrive_relaxed();  // no row for this warp
   for (int row = r0 + warp; row < r1; row += 6) {
-    const size_t qoff = ((size_t)row * p.H + h) * D;
-    const size_t qcoff = (size_t)row * p.tok_c + (size_t)h * D;
-    float nscore = -INFINITY;
-    if (p.null_kv) {
-      const uint16_t* kn = p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D;
-      float dot = null_dot<ROPE>(p, p.qc_ptr + qcoff, kn, lane * CPL, CPL);
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-      nscore = dot * p.scale_log2;
-    }
     const uint32_t row_saddr = stage_saddr + (uint32_t)(row * (D + 4) * 4);
-    float ms[kPrefillMaxSplits], ls[kPrefillMaxSplits];
+    const float2 mlv = lane < (int)cs ? tc::ld_dsmem_f32x2(tc::dsmem_addr(row_saddr, (uint32_t)lane))
+                                      : make_float2(-INFINITY, 0.f);
+    float2 ov[kPrefillMaxSplits][CPL / 2];
 #pragma unroll
     for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) {
-      const float2 v = s2 < ns ? tc::ld_dsmem_f32x2(tc::dsmem_addr(row_saddr, (uint32_t)(s2 + 1)))
-                               : make_float2(-INFINITY, 0.f);
-      ms[s2] = v.x;
-      ls[s2] = v.y;
-    }
-    float M = nscore;
+      const uint32_t ra = s2 < (int)cs ? tc::dsmem_addr(row_saddr, (uint32_t)s2) : 0u;
 #pragma unroll
-    for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) M = fmaxf(M, ms[s2]);
+      for (int e = 0; e < CPL / 2; ++e)
+        ov[s2][e] = s2 < (int)cs ? tc::ld_dsmem_f32x2(ra + 16 + (lane * CPL + 2 * e) * 4) : make_float2(0.f, 0.f);
+    }
+    float M = mlv.x;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float fl = exp2f(mlv.x - M);  // lane s: rank s's factor
     float Lsum = 0.f, A[CPL];
 #pragma unroll
     for (int e = 0; e < CPL; ++e) A[e] = 0.f;
-    if (p.null_kv) {
-      const float f = exp2f(nscore - M);
-      Lsum = f;
-      const uint16_t* vn = p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D + D;
-#pragma unroll
-      for (int e = 0; e < CPL; ++e) A[e] = f * bf16lo(vn[lane * CPL + e]);
-    }
-    float2 ov[kPrefillMaxSplits][CPL / 2];
-#pragma unroll
-    for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2)
-#pragma unroll
-      for (int e = 0; e < CPL / 2; ++e)
-        ov[s2][e] = s2 < ns ? tc::ld_dsmem_f32x2(
-                                  tc::dsmem_addr(row_saddr + 16 + (lane * CPL + 2 * e) * 4, (uint32_t)(s2 + 1)))
-                            : make_float2(0.f, 0.f);
 #pragma unroll
     for (int s2 = 0; s2 < kPrefillMaxSplits; ++s2) {
-      if (s2 >= ns) break;
-      const float f = exp2f(ms[s2] - M);
-      Lsum = fmaf(f, ls[s2], Lsum);
+      if (s2 >= (int)cs) break;
+      const float f = __shfl_sync(0xffffffffu, fl, s2);
+      Lsum = fmaf(f, __shfl_sync(0xffffffffu, mlv.y, s2), Lsum);
 #pragma unroll
       for (int e = 0; e < CPL / 2; ++e) {
         A[2 * e] = fmaf(f, ov[s2][e].x, A[2 * e]);
         A[2 * e + 1] = fmaf(f, ov[s2][e].y, A[2 * e + 1]);
       }
     }
+    if (row + 6 >= r1) tc::cluster_arrive_relaxed();  // this warp's last remote values are consumed
     const float inv = 1.f / Lsum;
+    const size_t qoff = ((size_t)row * p.H + h) * D;
     uint32_t* o32 = reinterpret_cast<uint32_t*>(p.oca + qoff) + lane * (CPL / 2);
 #pragma unroll
     for (int e = 0; e < CPL / 2; ++e) o32[e] = pack_bf16x2(A[2 * e] * inv, A[2 * e + 1] * inv);
@@ -372,115 +374,95 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         for (int j = 0; j < issued; ++j) mbar_wait_bounded(&full[j % C::NS], (j / C::NS) & 1, nullptr);
       }
     }
-  } else if (warp == 5 && ROPE && !sa) {
-    // ------------------------------------------- MMA issuer, rotary phases (CA)
-    // The whole warp runs the loop: it turns the query tile by W once and the
-    // key tile of every near block j (the last W table entries) by
-    // W - (i - j), so that each score sees the relative phase min(i - j, W);
-    // lane 0 issues the MMAs.
+  } else if (warp == 5) {
+    // ------------------------------------------------------------- MMA issuer
+    // The whole warp runs the loop, so control flow and descriptors stay
+    // warp-uniform; one elected lane issues the MMAs. QK^T runs two tiles
+    // ahead of P.V: S[j%2] is refilled with tile j+2 as soon as the softmax
+    // warps have read tile j out of it (s_free), so every score tile is ready
+    // a whole softmax pass before it is needed. With rotary phases the warp
+    // turns the query tile by W once and the key tile of every near block j
+    // (the last W table entries) by W - (i - j), so that each score sees the
+    // relative phase min(i - j, W).
     if (work) {
+      const bool leader = tc::elect_one();
+      const bool rot = ROPE && !sa;
       bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(q_full, 0, abort_flag));
-      const int near0 = max(b0, p.nblk - p.rope_w);
-      int jv0 = 0, jv1 = 0;
-      if (near0 + lane < b0 + nt) jv0 = p.bidx_row[near0 + lane];
-      if (near0 + 32 + lane < b0 + nt) jv1 = p.bidx_row[near0 + 32 + lane];
-      if (ok) {
-        tc::fence_after();
-        rotate_tile<D>(qt, p.rope_tab + (size_t)p.rope_w * (D / 2), lane, C::BOX);
+      int near0 = 0, jv0 = 0, jv1 = 0;
+      if (rot) {
+        near0 = max(b0, p.nblk - p.rope_w);
+        if (near0 + lane < b0 + nt) jv0 = p.bidx_row[near0 + lane];
+        if (near0 + 32 + lane < b0 + nt) jv1 = p.bidx_row[near0 + 32 + lane];
+        if (ok) {
+          tc::fence_after();
+          rotate_tile<D>(qt, p.rope_tab + (size_t)p.rope_w * (D / 2), lane, C::BOX);
+        }
       }
       const uint32_t qa = smem_u32(qt);
-      for (int jj = 0; ok && jj <= nt; ++jj) {
-        if (jj < nt) {  // S[jj%2] = Q . K^T
-          const int st = jj % C::NS, sb = jj & 1;
-          ok = __all_sync(0xffffffffu, mbar_wait_bounded(&full[st], (jj / C::NS) & 1, abort_flag));
-          if (ok && jj >= 2)
-            ok = __all_sync(0xffffffffu, mbar_wait_bounded(&s_free[sb], ((jj >> 1) - 1) & 1, abort_flag));
-          if (!ok) break;
-          tc::fence_after();
-          if (b0 + jj >= near0) {
-            const int o = b0 + jj - near0;
-            const int j = __shfl_sync(0xffffffffu, o < 32 ? jv0 : jv1, o & 31);
-            const int dk = max(0, p.rope_w - (p.q_blk - j));
-            if (dk > 0) rotate_tile<D>(ring + st * C::STAGE, p.rope_tab + (size_t)dk * (D / 2), lane, C::KVS);
-          }
-          if (lane == 0) {
-            const uint32_t ka = smem_u32(ring + st * C::STAGE);
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k)
-              tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k, C::BOX), qk_desc<D>(ka, k, C::KVS), C::ID_QK, k > 0);
-            tc::commit(&s_full[sb]);
-          }
-          __syncwarp();
+      // S[j%2] = Q . K_j^T
+      auto issue_qk = [&](int j) -> bool {
+        const int st = j % C::NS, sb = j & 1;
+        bool r = __all_sync(0xffffffffu, mbar_wait_bounded(&full[st], (j / C::NS) & 1, abort_flag));
+        if (r && j >= 2) r = __all_sync(0xffffffffu, mbar_wait_bounded(&s_free[sb], ((j >> 1) - 1) & 1, abort_flag));
+        if (!r) return false;
+        tc::fence_after();
+        if (rot && b0 + j >= near0) {
+          const int o = b0 + j - near0;
+          const int jb = __shfl_sync(0xffffffffu, o < 32 ? jv0 : jv1, o & 31);
+          const int dk = max(0, p.rope_w - (p.q_blk - jb));
+          if (dk > 0) rotate_tile<D>(ring + st * C::STAGE, p.rope_tab + (size_t)dk * (D / 2), lane, C::KVS);
         }
-        if (jj >= 1) {  // O += P . V for tile jj-1
-          const int j = jj - 1, st = j % C::NS, pb = j & 1;
-          ok = __all_sync(0xffffffffu, mbar_wait_bounded(&p_full[pb], (j >> 1) & 1, abort_flag));
-          if (!ok) break;
-          tc::fence_after();
-          if (lane == 0) {
-            const uint32_t pa = smem_u32(pt + pb * C::PBYTES);
-            const uint32_t va = smem_u32(ring + st * C::STAGE + C::BOX);
+        const uint32_t ka = smem_u32(ring + st * C::STAGE);
+        uint64_t ad[D / 16], bd[D / 16];
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-              tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024), v_desc<D>(va, k), C::ID_PV,
-                           (j > 0 || k > 0));
-            tc::commit(&empty[st]);
-            tc::commit(&o_done[pb]);
-          }
-          __syncwarp();
+        for (int k = 0; k < D / 16; ++k) {
+          ad[k] = qk_desc<D>(qa, k, C::BOX);
+          bd[k] = qk_desc<D>(ka, k, C::KVS);
         }
+        if (leader) {
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) tc::mma_bf16(tmem + 64 * sb, ad[k], bd[k], C::ID_QK, k > 0);
+          tc::commit(&s_full[sb]);
+        }
+        __syncwarp();
+        return true;
+      };
+      if (ok) tc::fence_after();
+      for (int j = 0; ok && j < min(2, nt); ++j) ok = issue_qk(j);
+      for (int j = 0; ok && j < nt; ++j) {
+        if (j + 2 < nt && !(ok = issue_qk(j + 2))) break;
+        // O += P_j . V_j
+        const int st = j % C::NS, pb = j & 1;
+        ok = __all_sync(0xffffffffu, mbar_wait_bounded(&p_full[pb], (j >> 1) & 1, abort_flag));
+        if (!ok) break;
+        tc::fence_after();
+        const uint32_t pa = smem_u32(pt + pb * C::PBYTES);
+        const uint32_t va = smem_u32(ring + st * C::STAGE + C::BOX);
+        uint64_t ad[4], bd[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          ad[k] = tc::sdesc_sw128(pa + k * 32, 16, 1024);
+          bd[k] = v_desc<D>(va, k);
+        }
+        if (leader) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) tc::mma_bf16(tmem + C::COL_O, ad[k], bd[k], C::ID_PV, (j > 0 || k > 0));
+          tc::commit(&empty[st]);
+          tc::commit(&o_done[pb]);
+        }
+        __syncwarp();
       }
       if (!ok) {
-        if (lane == 0 && !*abort_flag) record_error(p.err, kDevErrWaitMma);
+        if (leader && !*abort_flag) record_error(p.err, kDevErrWaitMma);
+        __syncwarp();
         *abort_flag = 1;
       }
-      if (lane == 0) {
+      // all issued MMAs complete before the CTA can release TMEM
+      if (leader) {
         tc::commit(drain);
         mbar_wait_bounded(drain, 0, nullptr);
       }
       __syncwarp();
-    }
-  } else if (warp == 5) {
-    // ------------------------------------------------------------- MMA issuer
-    if (lane == 0 && work) {
-      bool ok = mbar_wait_bounded(q_full, 0, abort_flag);
-      tc::fence_after();
-      const uint32_t qa = smem_u32(qt);
-      for (int jj = 0; ok && jj <= nt; ++jj) {
-        if (jj < nt) {  // S[jj%2] = Q . K^T
-          const int st = jj % C::NS, sb = jj & 1;
-          ok = mbar_wait_bounded(&full[st], (jj / C::NS) & 1, abort_flag);
-          if (ok && jj >= 2) ok = mbar_wait_bounded(&s_free[sb], ((jj >> 1) - 1) & 1, abort_flag);
-          if (!ok) break;
-          tc::fence_after();
-          const uint32_t ka = smem_u32(ring + st * C::STAGE);
-#pragma unroll
-          for (int k = 0; k < D / 16; ++k)
-            tc::mma_bf16(tmem + 64 * sb, qk_desc<D>(qa, k, C::BOX), qk_desc<D>(ka, k, C::KVS), C::ID_QK, k > 0);
-          tc::commit(&s_full[sb]);
-        }
-        if (jj >= 1) {  // O += P . V for tile jj-1
-          const int j = jj - 1, st = j % C::NS, pb = j & 1;
-          ok = mbar_wait_bounded(&p_full[pb], (j >> 1) & 1, abort_flag);
-          if (!ok) break;
-          tc::fence_after();
-          const uint32_t pa = smem_u32(pt + pb * C::PBYTES);
-          const uint32_t va = smem_u32(ring + st * C::STAGE + C::BOX);
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            tc::mma_bf16(tmem + C::COL_O, tc::sdesc_sw128(pa + k * 32, 16, 1024), v_desc<D>(va, k), C::ID_PV,
-                         (j > 0 || k > 0));
-          tc::commit(&empty[st]);
-          tc::commit(&o_done[pb]);
-        }
-      }
-      if (!ok) {
-        if (!*abort_flag) record_error(p.err, kDevErrWaitMma);
-        *abort_flag = 1;
-      }
-      // all issued MMAs complete before the CTA can release TMEM
-      tc::commit(drain);
-      mbar_wait_bounded(drain, 0, nullptr);
     }
   } else {
     // ---------------------------------------------------------- softmax warps
@@ -501,13 +483,24 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_free[sb]);
       float x[32];
-      float tmax = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        const int u = hf * 32 + c;
-        x[c] = (!sa || u <= r) ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
-        tmax = fmaxf(tmax, x[c]);
+      for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(sr[c]);
+      if (sa) {  // causal mask of the in-block tile
+#pragma unroll
+        for (int c = 0; c < 32; ++c)
+          if (hf * 32 + c > r) x[c] = -INFINITY;
       }
+      // row maximum of the raw scores as a tree; the base-2 scale is
+      // positive and rounding is monotone, so the scaled maximum equals the
+      // maximum of the scaled scores
+      float t[16];
+#pragma unroll
+      for (int c = 0; c < 16; ++c) t[c] = fmaxf(x[c], x[c + 16]);
+#pragma unroll
+      for (int w2 = 8; w2 >= 1; w2 >>= 1)
+#pragma unroll
+        for (int c = 0; c < w2; ++c) t[c] = fmaxf(t[c], t[c + w2]);
+      float tmax = t[0] * p.scale_log2;
       tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 16));
       const float m_new = fmaxf(m_used, tmax);
       const bool need = m_new > m_used + kRescaleLog2;
@@ -531,13 +524,19 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
         l *= exp2f(m_used - m_new);
         m_used = m_new;
       }
+      // P = 2^(s * scale - m): one FMA and one ex2 per score; the row sum
+      // in four independent partial sums
       uint32_t pk[16];
+      float la[4] = {0.f, 0.f, 0.f, 0.f};
+      const float nm = -m_used;
 #pragma unroll
       for (int c = 0; c < 32; c += 2) {
-        const float p0 = exp2f(x[c] - m_used), p1 = exp2f(x[c + 1] - m_used);
-        l += p0 + p1;
+        const float p0 = ex2_approx(fmaf(x[c], p.scale_log2, nm));
+        const float p1 = ex2_approx(fmaf(x[c + 1], p.scale_log2, nm));
+        la[(c >> 1) & 3] += p0 + p1;
         pk[c >> 1] = pack_bf16x2(p0, p1);
       }
+      l += (la[0] + la[1]) + (la[2] + la[3]);
       // P buffer sb was last read by P.V of tile j-2
       if (j >= 2) {
         ok = __all_sync(0xffffffffu, mbar_wait_bounded(&o_done[sb], ((j - 2) >> 1) & 1, abort_flag));
@@ -598,16 +597,40 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       for (int c = 0; c < D / 2; c += 8)
         *reinterpret_cast<uint4*>(out + c) = vn ? *reinterpret_cast<const uint4*>(vn + c) : make_uint4(0, 0, 0, 0);
     }
-    if (CL && !sa) {
-      // park this split's partial rows in shared memory for the cluster merge
-      float* pp = reinterpret_cast<float*>(ring) + (size_t)r * (D + 4);
+    if constexpr (CL) {
+      if (p.n_splits > 0) {
+        // park this thread's half row of the CTA's partial in the (idle) K/V
+        // ring for the cluster merge: rank 0 the null row (m = its score,
+        // l = 1, O = its value row; m = -inf, l = 0, O = 0 without one), a
+        // split its (m, l, O)
+        float pm = -INFINITY, pl = 0.f, v[D / 2];
+        if (sa) {
+          const uint16_t* kn = p.null_kv
+                                   ? p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D
+                                   : nullptr;
+          if (kn) {
+            float dot = null_dot<ROPE>(p, p.qc_ptr + (size_t)r * p.tok_c + (size_t)h * D, kn, col0, D / 2);
+            dot += __shfl_xor_sync(0xffffffffu, dot, 16);
+            pm = dot * p.scale_log2;
+            pl = 1.f;
+          }
 #pragma unroll
-      for (int c = 0; c < D / 2; c += 4)
-        *reinterpret_cast<float4*>(pp + 4 + col0 + c) =
-            ok ? make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]) : make_float4(0.f, 0.f, 0.f, 0.f);
-      if (hf == 0) {
-        pp[0] = ok ? m_used : -INFINITY;
-        pp[1] = ok ? lrow : 0.f;
+          for (int c = 0; c < D / 2; ++c) v[c] = kn ? bf16lo(kn[D + col0 + c]) : 0.f;
+        } else {
+          const bool have = ok && work;
+          pm = have ? m_used : -INFINITY;
+          pl = have ? lrow : 0.f;
+#pragma unroll
+          for (int c = 0; c < D / 2; ++c) v[c] = have ? o[c] : 0.f;
+        }
+        float* pp = reinterpret_cast<float*>(ring) + (size_t)r * (D + 4);
+#pragma unroll
+        for (int c = 0; c < D / 2; c += 4)
+          *reinterpret_cast<float4*>(pp + 4 + col0 + c) = make_float4(v[c], v[c + 1], v[c + 2], v[c + 3]);
+        if (hf == 0) {
+          pp[0] = pm;
+          pp[1] = pl;
+        }
       }
     }
     const bool part_ok = CL || SMEM_DCHECK(h < p.H && split < p.max_splits && p.n_splits <= p.max_splits, p.err);
@@ -713,15 +736,17 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       }
     }
   }
-  tc::fence_before();
-  __syncthreads();
   if constexpr (CL) {
     if (p.n_splits > 0) {
-      tc::cluster_sync();  // every split's partial rows are parked
-      cluster_merge<D, ROPE>(p, h, crank, cs, smem_u32(ring), warp, lane);
-      tc::cluster_sync();  // no CTA leaves while others read its shared memory
+      __syncwarp();
+      tc::cluster_sync();  // every partial row of the cluster is parked
+      cluster_merge<D>(p, h, crank, cs, smem_u32(ring), warp, lane);
+      __syncwarp();
+      tc::cluster_wait();  // no CTA leaves while another still reads its shared memory
     }
   }
+  tc::fence_before();
+  __syncthreads();
   if (warp == 4) {
     tc::fence_after();
     tc::dealloc(tmem, C::TMEM_COLS);

@@ -61,6 +61,14 @@ __device__ __forceinline__ void commit(uint64_t* bar) {
                : "memory");
 }
 
+// True in one lane of a converged warp (the same lane on every call); the
+// rest of the warp computes the same warp-uniform operands alongside it.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t r;
+  asm volatile("{\n\t.reg .pred p;\n\telect.sync _|p, 0xffffffff;\n\tselp.u32 %0, 1, 0, p;\n\t}" : "=r"(r));
+  return r != 0;
+}
+
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -182,6 +190,16 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+
+// The two halves of a cluster barrier, for work between a thread's arrival
+// and its wait (warp-uniform: every lane of a warp executes both). The
+// arrival is relaxed: it orders none of the thread's earlier memory
+// operations, so it does not wait for its outstanding stores; callers
+// publish what others need through a fence or an mbarrier of their own.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
 // Address of the same shared-memory offset in CTA `rank` of the cluster.
 __device__ __forceinline__ uint32_t dsmem_addr(uint32_t local_saddr, uint32_t rank) {
