@@ -302,6 +302,13 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
   const int nt = sa ? ((p.mode & 1) ? 1 : 0) : min(p.split_blks, p.nblk - b0);
   const bool work = nt > 0;
 
+  if (threadIdx.x == 128) {
+    // the tensor maps are kernel parameters, not the previous kernel's output
+    const CUtensorMap* maps[5] = {&p.pool, &p.qs, &p.ks, &p.vs, &p.qc};
+#pragma unroll
+    for (int i = 0; i < 5; ++i)
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(maps[i])) : "memory");
+  }
   if (threadIdx.x == 0) {
     griddep_launch();
     mbar_init(q_full, 1);
@@ -646,7 +653,7 @@ __global__ void __launch_bounds__(Pf<D>::THREADS, Pf<D>::MIN_CTAS) prefill_kerne
       __threadfence();
     }
     // the four softmax warps agree on the outcome before the ticket
-    const bool all_ok = bar_all(1, 128, ok);
+    const bool all_ok = CL || bar_all(1, 128, ok);  // the ticket merge only
     if (!CL && all_ok && !direct && part_ok) {
       if (threadIdx.x == 0) *ticket = atomicAdd(&p.counters[h], 1u);
       named_bar_sync(1, 128);
