@@ -9,8 +9,8 @@
 //
 // Work decomposition. A work unit is (item, split, head) for CA -- a split is
 // a run of consecutive table blocks whose length depends only on the block
-// count -- or (item, head) for SA. Units are dealt round-robin to worker
-// warps; every warp of a CTA is an independent worker with its own ring of
+// count -- or (item, head) for SA. CA units are handed out by a launch-wide
+// atomic counter; every warp of a CTA is an independent worker with its own ring of
 // shared-memory stages. A stage holds 32 rows (d_h = 64) or 16 rows
 // (d_h = 128) of K and of V of one head -- 8 KB -- loaded by tensor TMA with
 // the 128-byte swizzle, so that a lane can read a whole K row without bank
@@ -25,8 +25,10 @@
 // against all of them with warp-level tensor-core MMAs (the stage's keys as
 // the 16 rows, the group's queries as the columns), transposes P in
 // registers (movmatrix) into the operand of O^T += V^T P^T, so the rows
-// stream once per group at 16 MMAs per stage. SA units
-// read their <= 64 in-block rows straight from global memory. No warp ever waits for another warp; every reduction
+// stream once per group at 16 MMAs per stage. SA units read their <= 64
+// in-block rows straight from global memory (every load of a unit in flight
+// at once) and come from a second counter once a warp's CA stream has ended,
+// so they fill the launch's tail. No warp ever waits for another warp; every reduction
 // order is fixed by the block count, so the same block set gives the same
 // bits whatever the slots or the edit history.
 #include <cuda.h>
@@ -297,42 +299,81 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
   // with rotary phases the new token's query and key turn by its offset p
   const float2* rp = ROPE ? p.rope_tab + (size_t)it.pos * (D / 2) + hh * (QW / 2) : nullptr;
   if (p.mode & 1) {
+    constexpr int NP = kBlockTok / RPP;  // score passes
+    constexpr int NJ = QW / 8;           // 16-byte loads per row slice
+    constexpr int KB = NP * NJ <= 16 ? NP : 1;  // passes whose key rows load in one batch
+    // P.V: lane (g, c) owns column chunk c of rows g*RG .. g*RG+RG-1
+    constexpr int CPL = D / 8;        // column chunks
+    constexpr int G = 32 / CPL;       // row groups
+    constexpr int RG = kBlockTok / G; // rows per group
+    constexpr int VB = RG < 16 ? RG : 16;  // value rows per batch of loads
+    const int g = lane / CPL, c = lane % CPL;
+    // None of the unit's loads depends on another: the query slice, the first
+    // batch of key rows and (without rotary phases, whose tables need the
+    // registers) the first batch of value rows all go out before the first
+    // product, so the unit pays one memory round trip, not three.
+    uint4 qw[NJ], kw[KB][NJ], vw[VB];
+    auto load_keys = [&](int k0) {
+#pragma unroll
+      for (int kb = 0; kb < KB; ++kb) {
+        const int r = (k0 + kb) * RPP + lane / LPR;
+        const uint16_t* row = r == it.pos ? p.k_new + koff : ib + (size_t)r * D;
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) kw[kb][j] = r < n ? ld_nc16(row + hh * QW + j * 8) : make_uint4(0u, 0u, 0u, 0u);
+      }
+    };
+    auto load_values = [&](int i0) {
+#pragma unroll
+      for (int i = 0; i < VB; ++i) {
+        const int r = g * RG + i0 + i;
+        const uint16_t* row = r == it.pos ? p.v_new + koff : ib + (size_t)kBlockTok * D + (size_t)r * D;
+        vw[i] = r < n ? ld_nc16(row + c * 8) : make_uint4(0u, 0u, 0u, 0u);
+      }
+    };
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) qw[j] = ld_nc16(p.qs + soff + hh * QW + j * 8);
+    load_keys(0);
+    if (!ROPE) load_values(0);
     float q[QW];
 #pragma unroll
-    for (int j = 0; j < QW / 8; ++j) {
+    for (int j = 0; j < NJ; ++j) {
       float t[8];
-      unpack8(ld_nc16(p.qs + soff + hh * QW + j * 8), t);
+      unpack8(qw[j], t);
       if (ROPE) rot8f(t, rp + j * 4);
 #pragma unroll
       for (int e = 0; e < 8; ++e) q[j * 8 + e] = t[e] * p.scale_log2;
     }
     // scores of rows lane/LPR + k*RPP
-    float s[kBlockTok / RPP];
+    float s[NP];
     float mx = -INFINITY;
 #pragma unroll
-    for (int k = 0; k < kBlockTok / RPP; ++k) {
-      const int r = k * RPP + lane / LPR;
-      float dot = 0.f;
-      if (r < n) {
-        const uint16_t* row = r == it.pos ? p.k_new + koff : ib + (size_t)r * D;
+    for (int k0 = 0; k0 < NP; k0 += KB) {
+      if (k0 > 0) load_keys(k0);
 #pragma unroll
-        for (int j = 0; j < QW / 8; ++j) {
-          float t[8];
-          unpack8(ld_nc16(row + hh * QW + j * 8), t);
-          if (ROPE && r == it.pos) rot8f(t, rp + j * 4);  // stored rows are already turned
+      for (int kb = 0; kb < KB; ++kb) {
+        const int k = k0 + kb;
+        const int r = k * RPP + lane / LPR;
+        float dot = 0.f;
+        if (r < n) {
 #pragma unroll
-          for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
+          for (int j = 0; j < NJ; ++j) {
+            float t[8];
+            unpack8(kw[kb][j], t);
+            if (ROPE && r == it.pos) rot8f(t, rp + j * 4);  // stored rows are already turned
+#pragma unroll
+            for (int e = 0; e < 8; ++e) dot = fmaf(q[j * 8 + e], t[e], dot);
+          }
         }
+        if (LPR == 2) dot += __shfl_xor_sync(0xffffffffu, dot, 1);
+        s[k] = r < n ? dot : -INFINITY;
+        mx = fmaxf(mx, s[k]);
       }
-      if (LPR == 2) dot += __shfl_xor_sync(0xffffffffu, dot, 1);
-      s[k] = r < n ? dot : -INFINITY;
-      mx = fmaxf(mx, s[k]);
     }
 #pragma unroll
     for (int o = LPR; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     float l = 0.f;
 #pragma unroll
-    for (int k = 0; k < kBlockTok / RPP; ++k) {
+    for (int k = 0; k < NP; ++k) {
       const int r = k * RPP + lane / LPR;
       const float pr = r < n ? exp2f(s[k] - mx) : 0.f;
       if (hh == 0) {
@@ -343,23 +384,23 @@ __device__ void sa_unit(const DecodeParams& p, const Unit& U, float* pbuf, int l
     __syncwarp();
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    // P.V: lane (g, c) owns column chunk c of rows g*RG .. g*RG+RG-1
-    constexpr int CPL = D / 8;        // column chunks
-    constexpr int G = 32 / CPL;       // row groups
-    constexpr int RG = kBlockTok / G; // rows per group
-    const int g = lane / CPL, c = lane % CPL;
     float acc[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-    for (int i = 0; i < RG; ++i) {
-      const int r = g * RG + i;
-      if (r < n) {
-        const float pr = pbuf[r];
-        const uint16_t* row = r == it.pos ? p.v_new + koff : ib + (size_t)kBlockTok * D + (size_t)r * D;
-        float t[8];
-        unpack8(ld_nc16(row + c * 8), t);
+    // products in row order, VB value rows per batch of loads
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[e] = fmaf(pr, t[e], acc[e]);
+    for (int i0 = 0; i0 < RG; i0 += VB) {
+      if (i0 > 0 || ROPE) load_values(i0);
+#pragma unroll
+      for (int i = 0; i < VB; ++i) {
+        const int r = g * RG + i0 + i;
+        if (r < n) {
+          const float pr = pbuf[r];
+          float t[8];
+          unpack8(vw[i], t);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[e] = fmaf(pr, t[e], acc[e]);
+        }
       }
     }
 #pragma unroll
@@ -498,6 +539,100 @@ __device__ void merge_splits(const DecodeParams& p, const Pending& pd, int lane)
   if (lane == 0) p.counters[pd.item * p.H + pd.h] = 0u;
 }
 
+// The merges of a grouped unit's query heads h0 + j (bit j of `heads`: the
+// heads whose last ticket this warp holds), all at once: lanes
+// j*LPH .. j*LPH+LPH-1 serve head h0 + j with CPL columns each, so every
+// head's loads go out together instead of one head's after another's. Per
+// head the arithmetic is merge_splits' (the null-row score, the maximum over
+// it and the splits, then the weighted sums with the null row first and the
+// splits in split order).
+template <int D, bool ROPE, int QN>
+__device__ void merge_group(const DecodeParams& p, int item, int h0, unsigned heads, int nsplit, int pair_begin,
+                            int lane) {
+  constexpr int LPH = 32 / QN;  // lanes per query head
+  constexpr int CPL = D / LPH;  // columns per lane (4 or 8)
+  constexpr int GB = 8;         // splits whose loads are in flight together
+  static_assert(CPL % 4 == 0, "whole float4 column groups per lane");
+  const int j = lane / LPH, li = lane % LPH, c0 = li * CPL;
+  const bool act = ((heads >> j) & 1u) &&
+                   SMEM_DCHECK(item < p.n_items && h0 + j < p.H && (long long)pair_begin + nsplit <= p.part_pairs,
+                               p.err);
+  const int h = act ? h0 + j : h0;  // idle lanes address a valid head and load nothing
+  const uint16_t* kn = p.null_kv ? p.null_kv + ((size_t)p.layer * p.Hkv + h / (p.H / p.Hkv)) * 2 * D : nullptr;
+  float nscore = -INFINITY;
+  if (kn) {
+    float qv[CPL];
+#pragma unroll
+    for (int e = 0; e < CPL; ++e) qv[e] = act ? bf16lo(p.qc[(size_t)item * p.c_stride + (size_t)h * D + c0 + e]) : 0.f;
+    if (ROPE) {
+      // the null row's key phase is max(0, i - W): the query turns by min(i, W)
+      const float2* cs = p.rope_tab + (size_t)min(p.items[item].qblk, p.rope_w) * (D / 2) + c0 / 2;
+#pragma unroll
+      for (int e = 0; e < CPL; e += 2) {
+        const float2 c = cs[e / 2];
+        const float x0 = qv[e], x1 = qv[e + 1];
+        qv[e] = x0 * c.x - x1 * c.y;
+        qv[e + 1] = x0 * c.y + x1 * c.x;
+      }
+    }
+    float dot = 0.f;
+#pragma unroll
+    for (int e = 0; e < CPL; ++e) dot = fmaf(qv[e] * p.scale_log2, act ? bf16lo(kn[c0 + e]) : 0.f, dot);
+#pragma unroll
+    for (int o = 1; o < LPH; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+    nscore = dot;
+  }
+  const float* pb = p.part + ((size_t)pair_begin * p.H + h) * (D + 4);
+  const size_t ps = (size_t)p.H * (D + 4);
+  float M = nscore;
+  if (act)
+    for (int s2 = li; s2 < nsplit; s2 += LPH) M = fmaxf(M, __ldcg(pb + s2 * ps));
+#pragma unroll
+  for (int o = 1; o < LPH; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  float Lsum = 0.f, A[CPL];
+#pragma unroll
+  for (int e = 0; e < CPL; ++e) A[e] = 0.f;
+  if (kn && act) {
+    const float f = exp2f(nscore - M);
+    Lsum = f;
+#pragma unroll
+    for (int e = 0; e < CPL; ++e) A[e] = f * bf16lo(kn[D + c0 + e]);
+  }
+  for (int s0 = 0; s0 < nsplit; s0 += GB) {
+    float2 ml[GB];
+    float4 av[GB][CPL / 4];
+#pragma unroll
+    for (int g = 0; g < GB; ++g) {
+      const bool in = act && s0 + g < nsplit;
+      const float* ps2 = pb + (size_t)(s0 + g) * ps;
+      ml[g] = in ? __ldcg(reinterpret_cast<const float2*>(ps2)) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+      for (int e = 0; e < CPL / 4; ++e)
+        av[g][e] = in ? __ldcg(reinterpret_cast<const float4*>(ps2 + 4 + c0) + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int g = 0; g < GB; ++g) {
+      if (s0 + g >= nsplit) break;
+      const float f = exp2f(ml[g].x - M);
+      Lsum = fmaf(f, ml[g].y, Lsum);
+#pragma unroll
+      for (int e = 0; e < CPL / 4; ++e) {
+        A[4 * e] = fmaf(f, av[g][e].x, A[4 * e]);
+        A[4 * e + 1] = fmaf(f, av[g][e].y, A[4 * e + 1]);
+        A[4 * e + 2] = fmaf(f, av[g][e].z, A[4 * e + 2]);
+        A[4 * e + 3] = fmaf(f, av[g][e].w, A[4 * e + 3]);
+      }
+    }
+  }
+  if (act) {
+    const float inv = 1.f / Lsum;
+    uint32_t* o32 = reinterpret_cast<uint32_t*>(p.oca + ((size_t)item * p.H + h) * D + c0);
+#pragma unroll
+    for (int e = 0; e < CPL; e += 2) o32[e / 2] = pack_bf16x2(A[e] * inv, A[e + 1] * inv);
+    if (li == 0) p.counters[item * p.H + h] = 0u;
+  }
+}
+
 // pend2: read its ticket; the warp that completed the last split merges.
 template <int D, bool ROPE>
 __device__ __forceinline__ void settle(const DecodeParams& p, Pending& pd, int lane) {
@@ -538,35 +673,18 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
   }
   __syncthreads();
 
-  const int wid = blockIdx.x * C::NW + warp;
-  const int stride = gridDim.x * C::NW;
 
-  // prologue: start streaming the first CA units. When there are fewer CA
-  // units than twice the warps, a warp with self-attention work takes its
-  // first CA unit only after that work, so that no CA unit waits behind it.
+  // prologue: start streaming the first CA units. Every warp begins with
+  // cross-attention; the self-attention units come after a warp's stream has
+  // ended (below).
   Issue is;
   int issued = 0;
-  const long long n_ca = (long long)p.n_pairs * (p.H / p.qn);
-  const bool defer = (p.mode & 1) && wid < p.n_items * p.H && n_ca < 2LL * stride;
-  auto prologue = [&]() {
-    if (lane == 0) {
-      is.pushed = 0;
-      issue_begin_unit<D>(p, is, fetch_unit(p), uq);
-      for (int s = 0; s < C::NS; ++s)
-        if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * QN * D, &full[s], uq)) ++issued;
-    }
-  };
-  if (!defer) prologue();
-
-  // self-attention units (static, while the first tiles are in flight)
-  for (int u = wid; u < p.n_items * p.H; u += stride) {
-    Unit U;
-    U.sa = 1;
-    U.item = u / p.H;
-    U.h = u - U.item * p.H;
-    sa_unit<D, ROPE>(p, U, pbuf, lane);
+  if (lane == 0) {
+    is.pushed = 0;
+    issue_begin_unit<D>(p, is, fetch_unit(p), uq);
+    for (int s = 0; s < C::NS; ++s)
+      if (issue_next<D>(p, is, ring + s * C::STAGE, qarea + s * QN * D, &full[s], uq)) ++issued;
   }
-  if (defer) prologue();
   __syncwarp();
 
   constexpr int CPL = D / 8;             // P.V column chunks
@@ -741,16 +859,9 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
       // one ticket per query head, taken by lanes 0 .. ng-1 at once
       const bool mine = lane < ng && atomicAdd(&p.counters[U.item * p.H + U.h + lane], 1u) == (unsigned)(nsplit - 1);
       const unsigned last = __ballot_sync(0xffffffffu, mine);
-      for (int j = 0; j < ng; ++j) {
-        if (!(last >> j & 1u)) continue;
+      if (last) {
         __threadfence();
-        Pending pd;
-        pd.valid = 1;
-        pd.item = U.item;
-        pd.h = U.h + j;
-        pd.nsplit = nsplit;
-        pd.pair_begin = it.pair_begin;
-        merge_splits<D, ROPE>(p, pd, lane);
+        merge_group<D, ROPE, QN>(p, U.item, U.h, last, nsplit, it.pair_begin, lane);
       }
       continue;
     }
@@ -940,6 +1051,25 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     settle<D, ROPE>(p, pend2, lane);
     announce(p, pend1, pend2, lane);
     settle<D, ROPE>(p, pend2, lane);
+    // Self-attention units (in-block rows, read from global memory), fetched
+    // from their own counter once the warp's cross-attention stream has
+    // ended: they fill the launch's tail instead of holding every warp's
+    // first stage behind a memory system still busy with the ring
+    // prologues. They read no row and write no output that a cross-attention
+    // unit of the launch uses.
+    const int n_sa = p.n_items * p.H;
+    while (true) {
+      int v = 0;
+      if (lane == 0) v = (int)min(atomicAdd(p.sched + 2, 1ull), (unsigned long long)n_sa);
+      v = __shfl_sync(0xffffffffu, v, 0);
+      if (v >= n_sa) break;
+      Unit U;
+      U.sa = 1;
+      U.item = v / p.H;
+      U.h = v - U.item * p.H;
+      U.split = U.b0 = U.nt = 0;
+      sa_unit<D, ROPE>(p, U, pbuf, lane);
+    }
   }
   if (lane == 0) {
     if (failed) {
@@ -951,6 +1081,7 @@ __global__ void __launch_bounds__(Dec<D>::THREADS, 1) decode_kernel(const __grid
     if (done == (unsigned long long)gridDim.x * C::NW - 1) {
       p.sched[0] = 0ull;
       p.sched[1] = 0ull;
+      p.sched[2] = 0ull;  // next self-attention unit
     }
   }
 }
