@@ -228,9 +228,12 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __gri
     // Polls two queues: the P.V of the oldest tile whose P is ready (value
     // stage by stage, a column pair per MMA), and the next score stage
     // (landed, and for a tile's first stage its S buffer free). Neither
-    // blocks the other.
-    if (lane == 0 && nt > 0) {
-      bool ok = mbar_wait_bounded(q_full, 0, abort_flag);
+    // blocks the other. The whole warp runs the loop -- lane 0's poll results
+    // are shared, control flow and descriptors stay warp-uniform -- and one
+    // elected lane issues the MMAs and commits.
+    if (nt > 0) {
+      const bool leader = tc::elect_one();
+      bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(q_full, 0, abort_flag));
       tc::fence_after();
       const uint32_t qa = smem_u32(qt);
       const uint32_t sa = smem_u32(sring);
@@ -239,59 +242,87 @@ __global__ void __launch_bounds__(kMuThreads, 1) mu_attention_kernel(const __gri
       unsigned long long t_last = global_timer_ns();
       while (ok && tP < nt) {
         bool prog = false;
-        if (tP < kS / SPT && (kV % SPT != 0 || mbar_test_wait(&p_full[tP & 1], (tP >> 1) & 1))) {
+        if (tP < kS / SPT) {
           const int st = kV % nsv;
-          if (mbar_test_wait(&full_v[st], (kV / nsv) & 1)) {
+          bool go = lane == 0 && (kV % SPT != 0 || mbar_test_wait(&p_full[tP & 1], (tP >> 1) & 1)) &&
+                    mbar_test_wait(&full_v[st], (kV / nsv) & 1);
+          go = __shfl_sync(0xffffffffu, go, 0);
+          if (go) {
             tc::fence_after();
             const uint32_t a0 = va + st * SB;
             const uint32_t b = smem_u32(pt + (tP & 1) * C::PBYTES);
             for (int q = 0; q < cpb / 2; ++q) {
               const int cp = (kV % SPT) * (cpb / 2) + q;  // column pair of the row
+              uint64_t ad[4], bd[4];
 #pragma unroll
-              for (int kk = 0; kk < 4; ++kk)
-                tc::mma_bf16(tmem + colO + cp * NQ, tc::sdesc_sw128(a0 + 2 * q * kMuBox + kk * 2048, kMuBox, 1024),
-                             tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_PV, (tP > 0 || kk > 0));
+              for (int kk = 0; kk < 4; ++kk) {
+                ad[kk] = tc::sdesc_sw128(a0 + 2 * q * kMuBox + kk * 2048, kMuBox, 1024);
+                bd[kk] = tc::sdesc_sw128(b + kk * 32, 16, 1024);
+              }
+              if (leader) {
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                  tc::mma_bf16(tmem + colO + cp * NQ, ad[kk], bd[kk], C::ID_PV, (tP > 0 || kk > 0));
+              }
             }
-            tc::commit(&empty_v[st]);
+            if (leader) {
+              tc::commit(&empty_v[st]);
+              if ((kV + 1) % SPT == 0) tc::commit(&o_done[tP & 1]);
+            }
+            __syncwarp();
             ++kV;
-            if (kV % SPT == 0) {
-              tc::commit(&o_done[tP & 1]);
-              ++tP;
-            }
+            if (kV % SPT == 0) ++tP;
             prog = true;
           }
         }
         if (kS < total) {
           const int t = kS / SPT, j = kS % SPT, sb = t % NSB, st = kS % nss;
-          const bool sfree = j > 0 || t < NSB || mbar_test_wait(&s_free[sb], ((t / NSB) - 1) & 1);
-          if (sfree && mbar_test_wait(&full_s[st], (kS / nss) & 1)) {
+          bool go = lane == 0 && (j > 0 || t < NSB || mbar_test_wait(&s_free[sb], ((t / NSB) - 1) & 1)) &&
+                    mbar_test_wait(&full_s[st], (kS / nss) & 1);
+          go = __shfl_sync(0xffffffffu, go, 0);
+          if (go) {
             tc::fence_after();
             for (int q = 0; q < cpb / 2; ++q) {
               const int c = j * cpb + 2 * q;  // even chunk of the pair
               const uint32_t a = sa + st * SB + 2 * q * kMuBox, b = qa + c * C::PBYTES;
+              uint64_t ad[4], bd[4];
 #pragma unroll
-              for (int kk = 0; kk < 4; ++kk)
-                tc::mma_bf16(tmem + (uint32_t)(sb * 2 * NQ), tc::sdesc_sw128(a + kk * 32, 16, 1024),
-                             tc::sdesc_sw128(b + kk * 32, 16, 1024), C::ID_S2, (c | kk) > 0);
+              for (int kk = 0; kk < 4; ++kk) {
+                ad[kk] = tc::sdesc_sw128(a + kk * 32, 16, 1024);
+                bd[kk] = tc::sdesc_sw128(b + kk * 32, 16, 1024);
+              }
+              if (leader) {
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                  tc::mma_bf16(tmem + (uint32_t)(sb * 2 * NQ), ad[kk], bd[kk], C::ID_S2, (c | kk) > 0);
+              }
             }
-            tc::commit(&empty_s[st]);
+            if (leader) {
+              tc::commit(&empty_s[st]);
+              if (j == SPT - 1) tc::commit(&s_full[sb]);
+            }
+            __syncwarp();
             ++kS;
-            if (j == SPT - 1) tc::commit(&s_full[sb]);
             prog = true;
           }
         }
         if (prog) {
           t_last = global_timer_ns();
-        } else if (*abort_flag || global_timer_ns() - t_last > kWaitLimitNs) {
-          ok = false;
+        } else {
+          const bool give_up = lane == 0 && (*abort_flag || global_timer_ns() - t_last > kWaitLimitNs);
+          if (__shfl_sync(0xffffffffu, give_up, 0)) ok = false;
         }
       }
       if (!ok) {
-        if (!*abort_flag) record_error(p.err, kDevErrWaitMma);
+        if (leader && !*abort_flag) record_error(p.err, kDevErrWaitMma);
+        __syncwarp();
         *abort_flag = 1;
       }
-      tc::commit(drain);
-      mbar_wait_bounded(drain, 0, nullptr);
+      if (leader) {
+        tc::commit(drain);
+        mbar_wait_bounded(drain, 0, nullptr);
+      }
+      __syncwarp();
     }
   } else {
     // ---------------------------------------------------------- softmax warps
