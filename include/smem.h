@@ -39,13 +39,14 @@
  *     take a caller-owned workspace as well.
  *   - Supported shapes: block_tokens == rows_per_block == 64,
  *     head_dim 32, 64 or 128 (SMEM_ERR_UNSUPPORTED otherwise).
- *   - At head_dim 64 the one-block prefill runs one thread-block cluster per
- *     head when the device can hold all of them at once (checked at cache
- *     creation; with clusters smaller than 16 CTAs only up to 128 readable
- *     blocks); the environment variable
+ *   - At head_dim 64 the one-block prefill's split plan depends only on the
+ *     readable block count and the head count (at most 15 splits); it runs
+ *     one thread-block cluster of splits + 1 CTAs per head when the device
+ *     can hold all of them at once (checked at cache creation), else on the
+ *     cluster-free kernel with the same splits. The environment variable
  *     SMEM_PREFILL_CLUSTERS=0, read at creation, selects the cluster-free
- *     kernel instead. Both are deterministic; their split plans (hence
- *     rounding) differ.
+ *     kernel. Both merge the same partials in the same order: the outputs
+ *     are bitwise equal in either mode, on any device.
  */
 #ifndef SMEM_H
 #define SMEM_H

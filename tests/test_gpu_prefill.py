@@ -79,6 +79,33 @@ def test_160m_shape_one_layer(nblk, cluster_mode):
     assert smem.smem_check_device_error(dc.h) == smem.OK
 
 
+@pytest.mark.parametrize("nblk,has_null,rope", [(1, False, 0), (7, True, 0), (64, True, 0), (256, False, 0),
+                                                (40, True, 15)])
+def test_cluster_and_cluster_free_bitwise_equal(nblk, has_null, rope, monkeypatch):
+    """At d_h = 64 the split plan depends on the block and head counts alone;
+    the cluster kernel and the cluster-free one (a device that cannot hold
+    the clusters) merge the same partials in the same order, null row
+    first, so the same block set gives the same bits in either mode."""
+    outs = []
+    for clusters in (True, False):
+        if clusters:
+            monkeypatch.delenv("SMEM_PREFILL_CLUSTERS", raising=False)
+        else:
+            monkeypatch.setenv("SMEM_PREFILL_CLUSTERS", "0")
+        dc = DeviceCache(L=1, H=12, D=64, max_seqs=1, max_blocks=nblk + 2, capacity=nblk + 2, seed=71,
+                         has_null=has_null, rope_window=rope)
+        for j in range(nblk):
+            dc.append(0, j)
+        ins, osa, oca = dc.prefill(0, 0, nblk + 1)
+        if clusters and nblk <= 64 and not rope:
+            ref_sa, ref_ca = dc.oracle_prefill(0, 0, nblk + 1, *ins)
+            assert_close(out_f64(osa), ref_sa, "osa")
+            assert_close(out_f64(oca), ref_ca, "oca")
+        outs.append((osa.view(torch.int16).clone(), oca.view(torch.int16).clone()))
+    assert torch.equal(outs[0][0], outs[1][0])
+    assert torch.equal(outs[0][1], outs[1][1])
+
+
 @pytest.mark.parametrize("D", [32, 64, 128])
 def test_path_independence_bitwise(D):
     outs = []
