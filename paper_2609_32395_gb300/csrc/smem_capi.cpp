@@ -335,14 +335,10 @@ int prefill_impl(smem_cache* c, int seq, int layer, int q_block_idx, const void*
   a.layer = layer;
   a.nblk = nblk;
   if (c->lay.D == 64) {
-    // One split plan per (block count, head count), whatever the device: at
-    // most 15 splits, and a cluster of splits + 1 CTAs per head fitting one
-    // wave of two CTAs on each of a GB300's 152 SMs. It runs as clusters
-    // where the device holds one such cluster per head, else on the
-    // cluster-free kernel with the same splits; both merge the same partials
-    // in the same order (null row first), so the outputs carry the same bits.
-    const int ns_max = std::max(1, std::min(15, 304 / c->lay.H - 1));
-    a.split_blks = nblk ? smem::prefill_cluster_split_blocks(nblk, ns_max + 1) : 1;
+    // one split plan per (block count, head count), whatever the device; it
+    // runs as clusters where the device holds one cluster of splits + 1 CTAs
+    // per head, else on the cluster-free kernel with the same splits (same bits)
+    a.split_blks = nblk ? smem::prefill_split_blocks_d64(nblk, c->lay.H) : 1;
     a.n_splits = nblk ? smem::ceil_div(nblk, a.split_blks) : 0;
     a.cluster = c->pf_cluster_max >= a.n_splits + 1 && a.n_splits >= 1 ? 1 : 0;
   } else {

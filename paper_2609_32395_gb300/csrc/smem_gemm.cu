@@ -246,29 +246,37 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
       record_error(p.err, kDevErrWaitEmpty);
       *abort_flag = 1;
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
+    // The whole warp runs the loop (warp-uniform control flow and
+    // descriptors); one elected lane issues the MMAs and commits.
+    const bool leader = tc::elect_one();
     const uint32_t idesc = tc::idesc_bf16(128, BN, 0, p.b_kmajor ? 0 : 1);
     for (int i = 0; i < nch; ++i) {
       const int st = i % ns;
-      ok = mbar_wait_bounded(&full[st], (i / ns) & 1, abort_flag);
+      ok = __all_sync(0xffffffffu, mbar_wait_bounded(&full[st], (i / ns) & 1, abort_flag));
       if (!ok) break;
       tc::fence_after();
       const uint32_t aa = smem_u32(base + st * C::STAGE);
       const uint32_t wa = aa + C::A_BYTES;
+      uint64_t ad[4], bd[4];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
-        const uint64_t bd = p.b_kmajor ? tc::sdesc_sw128(wa + k * 32, 16, 1024)
-                                       : tc::sdesc_sw128(wa + k * 2048, 8192, 1024);
-        tc::mma_bf16(tmem, tc::sdesc_sw128(aa + k * 32, 16, 1024), bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
+        ad[k] = tc::sdesc_sw128(aa + k * 32, 16, 1024);
+        bd[k] = p.b_kmajor ? tc::sdesc_sw128(wa + k * 32, 16, 1024) : tc::sdesc_sw128(wa + k * 2048, 8192, 1024);
       }
-      tc::commit(&empty[st]);
+      if (leader) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) tc::mma_bf16(tmem, ad[k], bd[k], idesc, (i > 0 || k > 0) ? 1u : 0u);
+        tc::commit(&empty[st]);
+      }
+      __syncwarp();
     }
     if (!ok) {
-      record_error(p.err, kDevErrWaitFull);
+      if (leader) record_error(p.err, kDevErrWaitFull);
       *abort_flag = 1;
     }
-    tc::commit(acc_bar);  // arrives once every MMA issued above has completed
+    if (leader) tc::commit(acc_bar);  // arrives once every MMA issued above has completed
   }
   __syncwarp();
 

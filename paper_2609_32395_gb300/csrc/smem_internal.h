@@ -51,11 +51,11 @@ SMEM_HD inline int decode_split_blocks(int nblk) {
 }
 SMEM_HD inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
-// Split plan of the one-block prefill cross-attention, a function of the
-// block count and the cache's fixed head count and head dimension alone: the
-// cross-attention CTAs fit one wave on a GB300 (152 SMs; two CTAs per SM at
-// d_h = 64, one at 128), at most kPrefillMaxSplits splits per head, at least
-// two blocks per split.
+// Split plan of the one-block prefill cross-attention at d_h = 32 and 128
+// (d_h = 64: prefill_split_blocks_d64), a function of the block count and the
+// cache's fixed head count and head dimension alone: the cross-attention CTAs
+// fit one wave on a GB300 (152 SMs; two CTAs per SM at d_h = 32, one at 128),
+// at most kPrefillMaxSplits splits per head, at least two blocks per split.
 constexpr int kPrefillMaxSplits = 16;
 SMEM_HD inline int prefill_split_blocks(int nblk, int H, int D) {
   const int target = D <= 64 ? 304 : 152;
@@ -93,7 +93,7 @@ struct DecodeParams {
   const uint16_t* null_kv;   // [L][H][2][D] or nullptr
   float* part;               // [pair][H][D + 4]: m, l, pad, pad, acc[D]
   unsigned* counters;        // [max_batch][H] split tickets, zero between launches
-  unsigned long long* sched; // [2]: next CA unit, warps finished; zero between launches
+  unsigned long long* sched; // [3]: next CA unit, warps finished, next SA unit; zero between launches
   int* err;                  // device error word
   const uint16_t* qs;        // [nb][H][D]
   const uint16_t* k_new;
@@ -343,16 +343,16 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);
 // Largest cluster size (<= 16) with one cluster per head resident at once on
 // the current device for the d_h = 64 prefill; 0 if cluster mode is unavailable.
 int prefill_cluster_max(int H, int D);
-// Cluster mode removes the global split merge. With clusters of 16 it wins at
-// every context length; with smaller clusters (fewer splits than the
-// cluster-free plan) only while the launch is latency-bound.
-constexpr int kPrefillClusterMaxBlocks = 128;
-SMEM_HD inline bool prefill_use_clusters(int nblk, int cs_max) {
-  return cs_max >= 2 && (cs_max >= 16 || nblk <= kPrefillClusterMaxBlocks);
-}
-// Split plan of the cluster mode: blocks per split for a cluster limit cs_max.
-SMEM_HD inline int prefill_cluster_split_blocks(int nblk, int cs_max) {
-  int ns = cs_max - 1;
+// Split plan of the d_h = 64 prefill, a function of the block count and the
+// head count alone: at most 15 splits, at least two blocks per split, and a
+// cluster of splits + 1 CTAs per head within one wave of two CTAs on each of
+// a GB300's 152 SMs. The launch runs it as clusters where the device holds
+// one such cluster per head and on the cluster-free kernel otherwise; both
+// merge the same partials in the same order, so the bits do not depend on
+// the device.
+SMEM_HD inline int prefill_split_blocks_d64(int nblk, int H) {
+  int ns = 304 / H - 1;
+  if (ns > 15) ns = 15;
   if (ns > (nblk + 1) / 2) ns = (nblk + 1) / 2;
   if (ns < 1) ns = 1;
   return (nblk + ns - 1) / ns;
