@@ -44,8 +44,20 @@ def _inputs():
     return files
 
 
-def up_to_date() -> bool:
+def _flavor(extra_flags=()) -> str:
+    # what, besides the sources, decides the library's contents
+    debug = os.environ.get("SMEM_DEBUG", "0") not in ("", "0")
+    return " ".join(["debug" if debug else "release"] + list(extra_flags))
+
+
+def up_to_date(extra_flags=()) -> bool:
     if not os.path.exists(LIB):
+        return False
+    try:
+        with open(LIB + ".flavor") as f:
+            if f.read().strip() != _flavor(extra_flags):
+                return False  # built with other flags (e.g. the bounds-checking variant)
+    except OSError:
         return False
     t = os.path.getmtime(LIB)
     return all(os.path.getmtime(f) <= t for f in _inputs())
@@ -55,7 +67,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
     """SMEM_DEBUG=1 in the environment builds the bounds-checking variant
     (kernels check table, row and split indices and record an error instead
     of touching memory out of range)."""
-    if not force and up_to_date():
+    if not force and up_to_date(extra_flags):
         return LIB
     nvcc = _nvcc()
     os.makedirs(OBJ, exist_ok=True)
@@ -86,6 +98,8 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
     os.replace(tmp, LIB)
+    with open(LIB + ".flavor", "w") as f:
+        f.write(_flavor(extra_flags) + "\n")
     return LIB
 
 
