@@ -51,7 +51,11 @@ struct Pf {
   // box bx at bx * KVS + BOX. Fewer, larger copies keep the producer thread
   // below its TMA instruction rate.
   static constexpr int KVS = 2 * BOX;
-  static constexpr int NS = D == 32 ? 8 : (D == 64 ? 5 : 4);  // ring stages (2 CTAs per SM fit at d_h <= 64)
+  // ring stages: two CTAs per SM at d_h <= 64; at d_h = 128 one CTA per SM
+  // whose six 32 KB stages keep ~190 KB of copies in flight (four measured
+  // 74% of HBM over a long context, six 97%: the stream is bound by bytes
+  // in flight times the load latency)
+  static constexpr int NS = D == 32 ? 8 : (D == 64 ? 5 : 6);
   static constexpr int PBYTES = 64 * 64 * 2;      // P tile [64 queries][64 keys] bf16
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_RING = TILE;
@@ -72,6 +76,7 @@ struct Pf {
 };
 
 static_assert(2 * (Pf<64>::SMEM + 1024) <= 228 * 1024, "two d_h = 64 CTAs per SM");
+static_assert(Pf<128>::SMEM <= 227 * 1024, "one d_h = 128 CTA per SM");
 
 // Shared-memory descriptors of the K-major Q/K tiles (k-th step of 16
 // columns) and of the MN-major V tile (k-th step of 16 rows).
