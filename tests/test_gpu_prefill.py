@@ -7,7 +7,7 @@ import torch
 
 import synth
 from paper_2609_32395_gb300 import smem
-from tests.gpu_helpers import DeviceCache, assert_close, out_f64
+from tests.gpu_helpers import DeviceCache, assert_close, out_f64, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -131,6 +131,63 @@ def test_path_independence_bitwise(D):
         outs.append((osa.view(torch.int16).clone(), oca.view(torch.int16).clone()))
     for o in outs[1:]:
         assert torch.equal(o[0], outs[0][0]) and torch.equal(o[1], outs[0][1])
+
+
+def test_prefills_interleaved_with_edits_without_host_sync():
+    """Prefills are launched with programmatic dependent launch, so a launch
+    may begin while the previous kernel still runs. Appends, deletes and
+    prefills enqueued back to back with no host synchronisation must give,
+    output for output, the bits of the same calls each followed by a full
+    synchronisation (every read of the pool and the block table sees every
+    edit enqueued before it)."""
+    def run(sync):
+        dc = DeviceCache(L=2, H=12, D=64, max_seqs=1, max_blocks=64, capacity=80, seed=91, has_null=True,
+                         free_order=synth.slot_permutation(17, 80))
+        outs = []
+
+        def pf(layer, q_idx, tag):
+            qs, ks, vs, qc = [to_dev(x) for x in dc.prefill_inputs(layer, tag)]
+            osa = torch.empty((64, 12, 64), dtype=torch.bfloat16, device="cuda")
+            oca = torch.empty_like(osa)
+            smem.smem_prefill_block(dc.h, 0, layer, q_idx, qs, ks, vs, qc, osa, oca)
+            outs.append((osa, oca))
+            if sync:
+                torch.cuda.synchronize()
+
+        def edit(fn, *a):
+            fn(*a)
+            if sync:
+                torch.cuda.synchronize()
+
+        for j in range(40):
+            edit(dc.append, 0, j)
+        pf(0, 40, 0)
+        pf(1, 40, 1)
+        pf(0, 40, 2)
+        edit(dc.delete, 0, 7)
+        pf(0, 40, 3)
+        pf(1, 40, 4)
+        edit(dc.append, 0, 7)
+        edit(dc.append, 0, 45)
+        pf(0, 50, 5)
+        pf(1, 50, 6)
+        pf(0, 50, 7)
+        torch.cuda.synchronize()
+        assert smem.smem_check_device_error(dc.h) == smem.OK
+        return dc, [(a.view(torch.int16).clone(), b.view(torch.int16).clone()) for a, b in outs]
+
+    dc, fast = run(False)
+    _, slow = run(True)
+    assert len(fast) == len(slow)
+    for i, (f, s2) in enumerate(zip(fast, slow)):
+        assert torch.equal(f[0], s2[0]) and torch.equal(f[1], s2[1]), f"prefill {i}"
+    # the last prefill against the oracle (the final block set: 0..39 and 45)
+    ins = dc.prefill_inputs(0, 7)
+    ref_sa, ref_ca = dc.oracle_prefill(0, 0, 50, *ins)
+    got_sa = out_f64(fast[-1][0].view(torch.bfloat16))
+    got_ca = out_f64(fast[-1][1].view(torch.bfloat16))
+    assert_close(got_sa, ref_sa, "osa")
+    assert_close(got_ca, ref_ca, "oca")
 
 
 def test_prefill_ks_feed_decode():
