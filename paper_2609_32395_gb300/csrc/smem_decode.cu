@@ -217,7 +217,20 @@ struct Issue {
   int item, h, b0;
   int ybase;   // pool-map row of the unit's (layer, key/value head) K tile
   int pushed;  // queue entries pushed
+  int slot;    // pool slot of the block being issued
+  int slot_next;  // the unit's next block's slot, loaded a block ahead (-1: none or out of range)
 };
+
+// Table entry `blk` of a stream's item, or -1 when the index is out of range
+// (recorded in the bounds-checking build). The load is issued here and its
+// value is used a block later, so its latency stays off the warp's path.
+__device__ __forceinline__ int table_slot(const DecodeParams& p, int item, int blk) {
+  const DecodeItem& itm = p.items[item];
+  const bool in_range = SMEM_DCHECK(item < p.n_items && itm.seq >= 0 && itm.seq < p.max_seqs && blk >= 0 &&
+                                        blk < itm.nblk && itm.nblk <= p.max_blocks,
+                                    p.err);
+  return in_range ? p.table[(size_t)itm.seq * p.max_blocks + blk] : -1;
+}
 
 __device__ __forceinline__ int fetch_unit(const DecodeParams& p) {
   const unsigned long long u = atomicAdd(p.sched, 1ull);
@@ -236,6 +249,7 @@ __device__ __forceinline__ void issue_begin_unit(const DecodeParams& p, Issue& i
     is.h = U.h;
     is.b0 = U.b0;
     is.ybase = ((p.layer * p.Hkv + U.h / (p.H / p.Hkv)) * 2) * Dec<D>::R;
+    is.slot_next = table_slot(p, U.item, U.b0);  // used when the unit's first chunk is issued
   } else {
     is.nc = 0;
   }
@@ -250,13 +264,14 @@ __device__ __forceinline__ bool issue_next(const DecodeParams& p, Issue& is, uin
                                            uint64_t* bar, int* uq) {
   using C = Dec<D>;
   if (is.u < 0) return false;
-  const int blk = is.b0 + is.c / C::CHUNKS;
   const int row0 = (is.c % C::CHUNKS) * C::SROWS;
-  const DecodeItem& itm = p.items[is.item];
-  const bool in_range = SMEM_DCHECK(is.item < p.n_items && itm.seq >= 0 && itm.seq < p.max_seqs && blk >= 0 &&
-                                        blk < itm.nblk && itm.nblk <= p.max_blocks,
-                                    p.err);
-  const int slot = in_range ? p.table[(size_t)itm.seq * p.max_blocks + blk] : -1;
+  if (is.c % C::CHUNKS == 0) {
+    // a new block: its slot was loaded a block ago; load the next block's now
+    is.slot = is.slot_next;
+    const int nxt = is.c / C::CHUNKS + 1;  // the unit's next block (relative)
+    is.slot_next = nxt * C::CHUNKS < is.nc ? table_slot(p, is.item, is.b0 + nxt) : -1;
+  }
+  const int slot = is.slot;
   const uint32_t qbytes = is.c == 0 ? p.qn * D * 2 : 0;  // the unit's qn query heads (contiguous)
   if (slot < 0 || slot >= p.capacity) {
     record_error(p.err, kDevErrBounds);
