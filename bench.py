@@ -326,8 +326,10 @@ class DecodeWorkload:
         layer's inputs come from pinned host memory and its outputs go back
         to it through smem_decode_host, the copies on a copy stream of their
         own, ordered by the library against the decode of the neighbouring
-        layers (two staging halves). The step ends when its last copy has
-        landed."""
+        layers (two staging halves). The rows of a block that completes with
+        this step's token come from the host on the same copy stream while
+        the step's layers decode (they do not depend on them); the append
+        follows the step. The step ends when its last copy has landed."""
         import torch
 
         from paper_2609_32395_gb300 import smem
@@ -340,12 +342,19 @@ class DecodeWorkload:
         cs = self.copy_stream
         k = self.step_no % self.n_sets
         pos, nblk = self.pos.astype(np.int32), self.nblk.astype(np.int32)
+        completing = np.nonzero(self.pos + 1 == B_TOK)[0] if host_blocks is not None else []
         for layer in range(self.L):
             qs, kn, vn, qc = host_inputs[k][layer]
             smem.smem_decode_host(self.h, layer, self.seq_ids, pos, nblk, qs, kn, vn, qc, host_outputs[0][layer],
                                   host_outputs[1][layer], self.stage, stream=st, copy_stream=cs)
+            if layer == min(2, self.L - 1) and len(completing):
+                with torch.cuda.stream(cs):  # after the first layers' input copies
+                    for s in completing:
+                        u = self.new_used[s]
+                        self.new_K[s][u].copy_(host_blocks[0], non_blocking=True)
+                        self.new_V[s][u].copy_(host_blocks[1], non_blocking=True)
         st.wait_stream(cs)
-        return self.L + self._advance(host_blocks)
+        return self.L + self._advance(None)
 
 
 class LayerStack:

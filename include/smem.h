@@ -231,14 +231,17 @@ int smem_decode(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids
  * at least smem_decode_host_stage_bytes(c, nb) bytes; consecutive calls
  * alternate between its two halves), runs the decode step on `stream`, and
  * copies the outputs back -- all asynchronous. With copy_stream NULL the
- * copies run on `stream`; with another stream they run there, ordered by
+ * copies run on `stream`; with another stream the outputs come back on it
+ * and the inputs go in on a stream of the library's own, all ordered by
  * events against the decode, so that one call's copies overlap the
- * neighbouring calls' decode steps (a half is reused only after its
- * previous outputs have left). The host arrays must stay valid until the
- * stream(s) have drained and should be pinned (pageable memory makes the
- * copies synchronous); the outputs are on the host once copy_stream (or
- * stream) has drained. The first call creates the cache's ordering events
- * (destroyed with the cache); no device memory is allocated.
+ * neighbouring calls' decode steps and no call's inputs wait behind the
+ * previous call's outputs (a half is reused only after its previous outputs
+ * have left). The host arrays must stay valid until the stream(s) have
+ * drained and should be pinned (pageable memory makes the copies
+ * synchronous); the outputs are on the host, and every input has been
+ * read, once copy_stream (or stream) has drained. The first such call
+ * creates the cache's ordering events and input stream (destroyed with the
+ * cache); no device memory is allocated.
  * The paper has no counterpart. */
 size_t smem_decode_host_stage_bytes(const smem_cache *c, int32_t nb);
 int smem_decode_host(smem_cache *c, int32_t layer, int32_t nb, const int32_t *seq_ids, const int32_t *pos,

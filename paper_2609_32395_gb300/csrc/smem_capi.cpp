@@ -48,6 +48,10 @@ struct smem_cache {
   unsigned host_calls = 0;
   cudaEvent_t ev_in[2]{}, ev_out[2]{}, ev_free[2]{};
   bool ev_made = false;
+  // smem_decode_host's input copies (with a separate copy stream): on a
+  // stream of their own, so a layer's inputs do not queue behind the
+  // previous layer's outputs, which wait for its decode
+  cudaStream_t in_stream = nullptr;
   ~smem_cache() {
     if (ev_made)
       for (int i = 0; i < 2; ++i) {
@@ -55,6 +59,7 @@ struct smem_cache {
         cudaEventDestroy(ev_out[i]);
         cudaEventDestroy(ev_free[i]);
       }
+    if (in_stream) cudaStreamDestroy(in_stream);
   }
 };
 
@@ -796,17 +801,22 @@ int smem_decode_host(smem_cache* c, int32_t layer, int32_t nb, const int32_t* se
   }
   const cudaStream_t st = as_stream(stream);
   const cudaStream_t cs = copy_stream ? as_stream(copy_stream) : st;
+  if (cs != st && !c->in_stream &&
+      cuda_rc(cudaStreamCreateWithFlags(&c->in_stream, cudaStreamNonBlocking), "input stream"))
+    return SMEM_ERR_CUDA;
+  // inputs: on the library's input stream (outputs on the copy stream)
+  const cudaStream_t is = cs != st ? c->in_stream : st;
   const int half = (int)(c->host_calls & 1u);
   uint8_t* b = static_cast<uint8_t*>(stage) + (size_t)half * hs.half;
   const size_t qb = (size_t)nb * L.H * L.D * 2, kvb = (size_t)nb * L.Hkv * L.D * 2;
-  // inputs in on the copy stream once this half's previous outputs are out
+  // inputs in once this half's previous outputs are out
   cudaError_t e = cudaSuccess;
-  if (cs != st && c->host_calls >= 2) e = cudaStreamWaitEvent(cs, c->ev_free[half], 0);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.qs, qs, qb, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.kn, k_new, kvb, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.vn, v_new, kvb, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.qc, qc, qb, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess && cs != st) e = cudaEventRecord(c->ev_in[half], cs);
+  if (cs != st && c->host_calls >= 2) e = cudaStreamWaitEvent(is, c->ev_free[half], 0);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.qs, qs, qb, cudaMemcpyHostToDevice, is);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.kn, k_new, kvb, cudaMemcpyHostToDevice, is);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.vn, v_new, kvb, cudaMemcpyHostToDevice, is);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + hs.qc, qc, qb, cudaMemcpyHostToDevice, is);
+  if (e == cudaSuccess && cs != st) e = cudaEventRecord(c->ev_in[half], is);
   if (e == cudaSuccess && cs != st) e = cudaStreamWaitEvent(st, c->ev_in[half], 0);
   if (e != cudaSuccess) return cuda_rc(e, "host decode inputs");
   const int tok = L.H * L.D;
